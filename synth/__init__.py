@@ -1,0 +1,145 @@
+"""Seeded synthetic inputs shared by the oracle and the CUDA path.
+
+Holds none of the search method's arithmetic: it draws Gaussian-mixture
+vectors and N(0, 1/fan_in) encoder weights from the Philox4x32-10 generator
+(Salmon et al., SC'11) implemented in ``synth.c``, and names the workloads.
+
+The workloads stand in for the paper's BigANN (uint8, 128-d) and Deep1B
+(fp32, 96-d) benchmarks (paper Sec. 4.1, Table "datasets_all"), which are not
+available here: same dimensionality and value type, mixture-of-Gaussians
+structure, sizes from 1e5 to 1e9.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass, field
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB = None
+
+# Philox keys of the four independent draws
+SEED_DATA = 1
+SEED_QUERIES = 2
+SEED_ENCODER = 3
+SEED_KMEANS = 4
+STREAM_W1 = 1
+STREAM_W2 = 2
+
+
+def lib():
+    global _LIB
+    if _LIB is None:
+        path = os.path.join(_HERE, "libsynth.so")
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} missing: run __graft_entry__.build() first")
+        L = ctypes.CDLL(path)
+        L.synth_philox4x32_10.argtypes = [ctypes.POINTER(ctypes.c_uint32)] * 3
+        L.synth_mixture.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int,
+                                    ctypes.c_int, ctypes.c_double, ctypes.c_int64, ctypes.c_int64,
+                                    ctypes.c_void_p, ctypes.c_int]
+        L.synth_components.argtypes = [ctypes.c_uint64, ctypes.c_int, ctypes.c_int64,
+                                       ctypes.c_int64, ctypes.c_void_p]
+        L.synth_normal.argtypes = [ctypes.c_uint64, ctypes.c_uint32, ctypes.c_int64,
+                                   ctypes.c_double, ctypes.c_void_p]
+        _LIB = L
+    return _LIB
+
+
+def philox4x32_10(ctr, key):
+    c = (ctypes.c_uint32 * 4)(*ctr)
+    k = (ctypes.c_uint32 * 2)(*key)
+    o = (ctypes.c_uint32 * 4)()
+    lib().synth_philox4x32_10(c, k, o)
+    return [int(v) for v in o]
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    n: int            # base vectors
+    dim: int          # D
+    dtype: str        # "u8" or "f32"
+    mixture: int      # M components
+    sigma: float
+    nq: int           # queries
+    hidden: int       # H
+    bits: int         # b
+    k_max: int        # centroids per bucket
+    t: int            # target cluster capacity
+    probe: tuple = (8,)
+    clusters: tuple = (32,)
+    k: int = 10
+    notes: str = ""
+
+    @property
+    def dtype_code(self) -> int:
+        return 0 if self.dtype == "u8" else 1
+
+    @property
+    def row_bytes(self) -> int:
+        return self.dim * (1 if self.dtype == "u8" else 4)
+
+    @property
+    def in_scale(self) -> float:
+        return 1.0 / 255.0 if self.dtype == "u8" else 1.0
+
+
+WORKLOADS = {
+    # 1e5 uint8 x 128, 256 components: the small case the oracle finishes in seconds
+    "tiny": Workload("tiny", 100_000, 128, "u8", 256, 18.0, 1000, 256, 16, 4, 32,
+                     probe=(8,), clusters=(32,)),
+    # 1e7 uint8 x 128, b = 20
+    "u8-10m": Workload("u8-10m", 10_000_000, 128, "u8", 256, 18.0, 10_000, 512, 20, 8, 64,
+                       probe=(4, 16, 64), clusters=(32, 128)),
+    # 1e7 fp32 x 96, L2-normalised, b = 20
+    "f32-10m": Workload("f32-10m", 10_000_000, 96, "f32", 1024, 0.3, 10_000, 384, 20, 8, 64,
+                        probe=(8, 32), clusters=(64,)),
+    # 1e8 uint8 x 128, b = 24
+    "u8-100m": Workload("u8-100m", 100_000_000, 128, "u8", 4096, 18.0, 10_000, 512, 24, 16, 64),
+    # 1e9 uint8 x 128, b = 24
+    "u8-1b": Workload("u8-1b", 1_000_000_000, 128, "u8", 16384, 18.0, 10_000, 512, 24, 16, 64),
+}
+
+
+def mixture(w: Workload, seed_rows: int, row0: int, n: int, nthreads: int | None = None,
+            seed_centres: int = SEED_DATA) -> np.ndarray:
+    """Rows [row0, row0+n) of the workload's mixture (centres from seed_centres)."""
+    nthreads = nthreads or os.cpu_count() or 1
+    out = np.empty((n, w.dim), dtype=np.uint8 if w.dtype == "u8" else np.float32)
+    rc = lib().synth_mixture(w.dtype_code, seed_rows, seed_centres, w.mixture, w.dim, w.sigma,
+                             row0, n, out.ctypes.data, nthreads)
+    if rc != 0:
+        raise RuntimeError("synth_mixture failed")
+    return out
+
+
+def base(w: Workload, n: int | None = None, nthreads: int | None = None) -> np.ndarray:
+    return mixture(w, SEED_DATA, 0, w.n if n is None else n, nthreads)
+
+
+def queries(w: Workload, nq: int | None = None, nthreads: int | None = None) -> np.ndarray:
+    return mixture(w, SEED_QUERIES, 0, w.nq if nq is None else nq, nthreads)
+
+
+def components(w: Workload, seed_rows: int, row0: int, n: int) -> np.ndarray:
+    out = np.empty(n, dtype=np.int32)
+    lib().synth_components(seed_rows, w.mixture, row0, n, out.ctypes.data)
+    return out
+
+
+def normal(seed: int, stream: int, n: int, scale: float) -> np.ndarray:
+    out = np.empty(n, dtype=np.float32)
+    lib().synth_normal(seed, stream, n, scale, out.ctypes.data)
+    return out
+
+
+def encoder_weights(w: Workload, seed: int = SEED_ENCODER):
+    """Seeded encoder D -> H (ReLU) -> b with N(0, 1/fan_in) weights, zero biases.
+
+    Returns (W1 [H x D], b1 [H], W2 [b x H], b2 [b]) as fp32 arrays."""
+    W1 = normal(seed, STREAM_W1, w.hidden * w.dim, 1.0 / np.sqrt(w.dim)).reshape(w.hidden, w.dim)
+    W2 = normal(seed, STREAM_W2, w.bits * w.hidden, 1.0 / np.sqrt(w.hidden)).reshape(w.bits, w.hidden)
+    return W1, np.zeros(w.hidden, np.float32), W2, np.zeros(w.bits, np.float32)

@@ -1,0 +1,120 @@
+"""Whole oracle search. With every bucket probed, every cluster kept, the gate
+off and early stopping off, the method must return the exact k nearest
+neighbours (the problem statement of Sec. 3.1); plus budget invariants and the
+Recall@k definition of Sec. 4.4 on the 1e5 workload."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from paper_2608_15438_gb300.builder import build_index, config
+
+
+def exact_knn(base, qs, k):
+    if base.dtype == np.uint8:
+        b = base.astype(np.float64)
+        q = qs.astype(np.float64)
+    else:
+        b = base.astype(np.float64)
+        q = qs.astype(np.float64)
+    d = (q * q).sum(1)[:, None] + (b * b).sum(1)[None, :] - 2.0 * q @ b.T
+    if base.dtype == np.uint8:
+        d = np.rint(d)
+    ids = np.empty((len(qs), k), np.int64)
+    dd = np.empty((len(qs), k))
+    for i in range(len(qs)):
+        o = np.lexsort((np.arange(len(b)), d[i]))[:k]
+        ids[i], dd[i] = o, d[i][o]
+    return ids, dd
+
+
+def recall_at_k(found, truth, k):
+    """Sec. 4.4: |R ∩ G| / min(k, |G|), by unique ids, averaged over queries."""
+    r = []
+    for f, g in zip(found, truth):
+        g = set(int(v) for v in g[:k] if v >= 0)
+        f = set(int(v) for v in f[:k] if v >= 0)
+        r.append(len(f & g) / min(k, len(g)) if g else 1.0)
+    return float(np.mean(r))
+
+
+@pytest.mark.parametrize("dtype", ["u8", "f32"])
+def test_exhaustive_budget_is_exact_knn(tmp_path, dtype):
+    w = synth.WORKLOADS["tiny" if dtype == "u8" else "f32-10m"]
+    n, nq, b = 20000, 40, 8
+    base = synth.base(w, n)
+    qs = synth.queries(w, nq)
+    W1, b1, W2, b2 = synth.encoder_weights(w)
+    path = str(tmp_path / "ex.nrix")
+    info = build_index(config(w.dtype, w.dim, w.hidden, b, w.k_max, 16), base,
+                       (W1, b1, W2[:b], b2[:b]), path)
+    ix = oracle.Index(path)
+    p = oracle.params(t_low=0)
+    ids, d, st = ix.search(qs, 10, 1 << b, info["n_clusters"], p)
+    gi, gd = exact_knn(base, qs, 10)
+    if dtype == "u8":
+        assert np.array_equal(ids, gi)
+        assert np.array_equal(d, gd.astype(np.float32))
+    else:
+        assert np.allclose(d, gd, rtol=1e-5, atol=1e-6)
+        # ids agree wherever the distance order is unambiguous
+        gaps = np.diff(gd, axis=1)
+        sure = np.ones_like(gi, bool)
+        sure[:, :-1] &= gaps > 1e-5
+        sure[:, 1:] &= gaps > 1e-5
+        assert np.array_equal(ids[sure], gi[sure])
+    assert np.all(st[:, 0] == n)
+
+
+def test_recall_definition():
+    truth = np.array([[1, 2, 3], [4, 5, -1]])
+    found = np.array([[3, 9, 1], [5, 7, 8]])
+    assert recall_at_k(found, truth, 3) == pytest.approx((2 / 3 + 1 / 2) / 2)
+
+
+def test_tiny_invariants(tiny_index):
+    ix = oracle.Index(tiny_index["path"])
+    qs = tiny_index["queries"][:200]
+    cl_off = ix.cl_off().astype(np.int64)
+    bkt = ix.bkt_off().astype(np.int64)
+    tau = ix.tau()
+    lg = ix.encode(qs)
+    P, C, k = 32, 16, 10
+    p = oracle.params()
+    ids, d, st = ix.search(qs, k, P, C, p, logits=lg)
+    _, _, st_off = ix.search(qs, k, P, C, oracle.params(t_low=0), logits=lg)
+    for i in range(len(qs)):
+        # sorted by (dist, id), ids unique
+        valid = ids[i] >= 0
+        assert np.all(np.diff(d[i][valid]) >= 0)
+        assert len(set(ids[i][valid].tolist())) == valid.sum()
+        codes, _, _ = oracle.probe_list(lg[i], tau, P, p)
+        L, dL, ndir = ix.cluster_list(lg[i], codes, C, p)
+        assert len(L) - ndir <= C and st[i, 2] == len(L) and st[i, 3] == len(codes) == P
+        total = int((cl_off[L + 1] - cl_off[L]).sum())
+        assert st[i, 0] <= total and st_off[i, 0] == total
+        assert st[i, 0] <= st[i, 1] * p.round_size
+        assert st_off[i, 0] >= st[i, 0]
+        # every returned id lies in a cluster of L
+        rows = set()
+        idmap = None
+        for c in L:
+            rows.update(range(cl_off[c], cl_off[c + 1]))
+        if idmap is None:
+            idmap = ix.ids()
+        member_ids = set(int(idmap[r]) for r in rows)
+        assert set(ids[i][valid].tolist()) <= member_ids
+        # every cluster of a probed bucket is accounted for
+        allc = set()
+        for u in codes:
+            allc.update(range(bkt[u], bkt[u + 1]))
+        assert set(L.tolist()) <= allc
+
+
+def test_tiny_recall_grows_with_budget(tiny_index):
+    ix = oracle.Index(tiny_index["path"])
+    qs = tiny_index["queries"][:300]
+    gi, _ = exact_knn(tiny_index["base"], qs, 10)
+    p = oracle.params()
+    r = [recall_at_k(ix.search(qs, 10, P, C, p)[0], gi, 10) for P, C in [(4, 8), (32, 64), (256, 512)]]
+    assert r[0] < r[1] < r[2] and r[2] > 0.9
