@@ -1,0 +1,435 @@
+"""Benchmark of the NeuRoute batched query path on GB300.
+
+One step = one nr_search call over the workload's whole query batch (encode,
+route, select, refine) with the index and the queries resident in HBM.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload u8-10m]
+                  [--P 64 --C 128 --t-low 4] [--impl neuroute|reference] [--sweep]
+
+Prints one JSON line (rank 0). Metric: queries per second at the workload's
+Recall@10 ~ 0.90 operating point, plus the refinement kernel's achieved HBM
+bandwidth against the measured copy bandwidth of this GPU.
+Multi-GPU (torchrun): every rank is an independent replica with the full
+index and its own query batch (weak scaling, no data-path collective).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+# operating points (P, C, t_low) with Recall@10 in [0.88, 0.92], from `--sweep`
+OPERATING_POINTS = {
+    "tiny": (128, 256, 4),
+    "u8-10m": (256, 1024, 0),
+    "f32-10m": (256, 512, 4),
+}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="u8-10m")
+    ap.add_argument("--P", type=int, default=None)
+    ap.add_argument("--C", type=int, default=None)
+    ap.add_argument("--t-low", type=int, default=None)
+    ap.add_argument("--k", type=int, default=10)
+    ap.add_argument("--nq", type=int, default=None)
+    ap.add_argument("--impl", default="neuroute", choices=["neuroute", "reference"])
+    ap.add_argument("--sweep", action="store_true")
+    ap.add_argument("--index", default=None, help="reuse an index file")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() in ("active", "1", "yes"):
+                        reasons.add(n)
+            os.remove(self.path)
+        except Exception:
+            pass
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+def index_path(w):
+    """Index file named by a digest of everything that determines its bytes."""
+    h = hashlib.sha256(repr(w).encode())
+    for f in ("synth/synth.c", "paper_2608_15438_gb300/builder/nrbuild.cpp"):
+        h.update(open(os.path.join(ROOT, f), "rb").read())
+    return os.path.join(tempfile.gettempdir(), f"neuroute_{w.name}_{h.hexdigest()[:16]}.nrix")
+
+
+def build_or_load_index(w, path, rank, world):
+    import synth
+    from paper_2608_15438_gb300.builder import build_index, config
+
+    if rank == 0 and not os.path.exists(path):
+        base = synth.base(w)
+        info = build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t), base,
+                           synth.encoder_weights(w), path + ".tmp")
+        os.replace(path + ".tmp", path)
+        del base
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+    return path
+
+
+def ground_truth(torch, base_t, q_t, k, dtype):
+    """Exact k-NN by brute force on the GPU (torch fp32 matmul; exact for uint8
+    data, whose dot products and norms are integers below 2^24)."""
+    nb = base_t.shape[0]
+    bf = base_t.float()
+    bn = (bf * bf).sum(1)
+    out = []
+    step = max(1, int(2e9 // max(nb, 1)))
+    for i in range(0, q_t.shape[0], step):
+        qf = q_t[i:i + step].float()
+        d = (qf * qf).sum(1, keepdim=True) + bn[None, :] - 2.0 * (qf @ bf.T)
+        out.append(torch.topk(d, k, dim=1, largest=False).indices.cpu())
+        del d
+    return torch.cat(out).numpy()
+
+
+def recall_at(found, truth, k=10):
+    r = []
+    for f, g in zip(found, truth):
+        g = set(int(v) for v in g[:k])
+        f = set(int(v) for v in f[:k] if v >= 0)
+        r.append(len(f & g) / min(k, len(g)))
+    return float(np.mean(r))
+
+
+def traffic_from_profile(workload, P, C):
+    """Per-launch DRAM bytes of the refine kernel from a committed ncu summary,
+    valid only while the kernel source is unchanged since the capture."""
+    path = os.path.join(ROOT, "profiles", "refine_traffic.json")
+    try:
+        rec = json.load(open(path))
+        src = open(os.path.join(ROOT, "paper_2608_15438_gb300", "csrc", "nr_refine.cu"), "rb").read()
+        if rec.get("nr_refine_sha256") != hashlib.sha256(src).hexdigest():
+            return None
+        e = rec.get("captures", {}).get(f"{workload}/P{P}/C{C}")
+        return None if e is None else e.get("bytes_per_launch")
+    except Exception:
+        return None
+
+
+def cpu_baseline(w, path, queries, k, P, C, t_low, seconds, truth=None):
+    import oracle
+
+    orc = oracle.Index(path)
+    p = oracle.params(t_low=t_low)
+    cores = os.cpu_count() or 1
+    n = 16
+    t = time.perf_counter()
+    orc.search(queries[:n], k, P, C, p, nthreads=cores)
+    dt = max(time.perf_counter() - t, 1e-6)
+    n2 = int(min(len(queries), max(n, n * seconds / dt)))
+    t = time.perf_counter()
+    ids, _, _ = orc.search(queries[:n2], k, P, C, p, nthreads=cores)
+    dt2 = time.perf_counter() - t
+    res = {"value": n2 / dt2, "unit": "queries/s", "cores": cores, "kind": "oracle",
+           "sample": f"first {n2} of {len(queries)} queries of {w.name}, P={P} C={C} t_low={t_low}, "
+                     f"{cores} threads, {dt2:.1f} s"}
+    orc.close()
+    return res, ids
+
+
+def run_reference(args, w, rank, world):
+    """The oracle timed on the host cores (the CPU reference arm)."""
+    if rank != 0:
+        return 0
+    import synth
+
+    P, C, t_low = op_point(args, w)
+    path = args.index or index_path(w)
+    build_or_load_index(w, path, 0, 1)
+    nq = args.nq or w.nq
+    qs = synth.queries(w, nq)
+    import oracle
+
+    orc = oracle.Index(path)
+    p = oracle.params(t_low=t_low)
+    cores = os.cpu_count() or 1
+    n = 16
+    t = time.perf_counter()
+    orc.search(qs[:n], args.k, P, C, p, nthreads=cores)
+    dt = max(time.perf_counter() - t, 1e-6)
+    per_step = max(8.0, 120.0 / max(1, args.steps + args.warmup))
+    ns = int(min(nq, max(n, n * per_step / dt)))
+    for _ in range(args.warmup):
+        orc.search(qs[:ns], args.k, P, C, p, nthreads=cores)
+    times = []
+    for _ in range(args.steps):
+        t = time.perf_counter()
+        orc.search(qs[:ns], args.k, P, C, p, nthreads=cores)
+        times.append(time.perf_counter() - t)
+    tot = sum(times)
+    v = ns * args.steps / tot
+    line = {"impl": "reference", "metric": "QPS at Recall@10~0.90 (batched query path)", "value": v,
+            "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
+            "config": {"workload": w.name, "nq_per_step": ns, "P": P, "C": C, "t_low": t_low, "k": args.k},
+            "cpu_baseline": {"value": v, "unit": "queries/s", "cores": cores, "kind": "oracle",
+                             "sample": f"first {ns} of {nq} queries per step"},
+            "e2e": {"value": v, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def op_point(args, w):
+    P, C, t_low = OPERATING_POINTS.get(w.name, (64, 128, 4))
+    return (args.P or P, args.C or C, t_low if args.t_low is None else args.t_low)
+
+
+def main():
+    args = parse()
+    import synth
+
+    w = synth.WORKLOADS[args.workload]
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("gloo" if args.impl == "reference" else "nccl")
+    if args.impl == "reference":
+        rc = run_reference(args, w, rank, world)
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.destroy_process_group()
+        return rc
+
+    import torch
+
+    import __graft_entry__
+
+    __graft_entry__.build()
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    P, C, t_low = op_point(args, w)
+    k = args.k
+    path = args.index or index_path(w)
+    t0 = time.time()
+    build_or_load_index(w, path, rank, world)
+    t_build = time.time() - t0
+    ix = nr.Index(path, local)
+    nq = args.nq or w.nq
+    # each rank searches its own batch of the query distribution
+    qs = synth.mixture(w, synth.SEED_QUERIES, rank * nq, nq)
+    dq = torch.from_numpy(qs).to(dev)
+    ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    dd = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    # ground truth (outside any timed region)
+    base_np = synth.base(w)
+    base_t = torch.from_numpy(base_np).to(dev)
+    del base_np
+    truth = ground_truth(torch, base_t, dq, k, w.dtype)
+    del base_t
+    torch.cuda.empty_cache()
+
+    if args.sweep:
+        rows = []
+        for Pp in (16, 64, 256, 1024, 2048):
+            for Cc in (64, 256, 1024, 4096):
+                if Pp * ix.k_max > 16384:
+                    continue
+                for tl in (4, 0):
+                    ix.set_params(t_low=tl)
+                    ix.search(dq, k, Pp, Cc, out=(ids, dd))
+                    torch.cuda.synchronize()
+                    t = time.perf_counter()
+                    ix.search(dq, k, Pp, Cc, out=(ids, dd))
+                    torch.cuda.synchronize()
+                    el = time.perf_counter() - t
+                    st = ix.last_stats()
+                    rows.append({"P": Pp, "C": Cc, "t_low": tl, "recall": recall_at(ids.cpu().numpy(), truth, k),
+                                 "qps": nq / el, "cand_per_q": st.candidates / nq})
+                    print(json.dumps(rows[-1]), flush=True)
+        return 0
+
+    ix.set_params(t_low=t_low)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    for _ in range(max(3, args.warmup)):
+        ix.search(dq, k, P, C, out=(ids, dd), stream=stream)
+    torch.cuda.synchronize()
+    rec = recall_at(ids.cpu().numpy(), truth, k)
+    st = ix.last_stats()
+    ix.enable_timing(True)
+    launches0 = ix.kernel_launches()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    refine_ms = []
+    stage_ms = {"encode": 0.0, "route": 0.0, "select": 0.0, "refine": 0.0}
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(torch.cuda.current_device() if "CUDA_VISIBLE_DEVICES" not in os.environ else local) as clk:
+        for i in range(args.steps):
+            flush.random_(0, 255)  # evict L2 (129 MB) between timed steps
+            ev[i][0].record(stream)
+            ix.search(dq, k, P, C, out=(ids, dd), stream=stream)
+            ev[i][1].record(stream)
+            tm = ix.last_timing()
+            refine_ms.append(tm["refine"])
+            for kk in stage_ms:
+                stage_ms[kk] += tm[kk]
+        torch.cuda.synchronize()
+    launches = ix.kernel_launches() - launches0
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    tot_ms = sum(step_ms)
+    if world > 1:
+        import torch.distributed as dist
+
+        t = torch.tensor([tot_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        tot_ms = float(t.item())
+        dist.barrier()
+    value = nq * args.steps * world / (tot_ms / 1e3)
+
+    # end to end through the host-buffer entry point (copies inside the timed region)
+    hq = torch.from_numpy(qs).pin_memory()
+    hid = torch.empty((nq, k), dtype=torch.int64).pin_memory()
+    hd = torch.empty((nq, k), dtype=torch.float32).pin_memory()
+    ix.search_host(hq, k, P, C, out=(hid, hd))
+    e2e_t = []
+    for _ in range(args.steps):
+        flush.random_(0, 255)
+        torch.cuda.synchronize()
+        t = time.perf_counter()
+        ix.search_host(hq, k, P, C, out=(hid, hd))
+        e2e_t.append(time.perf_counter() - t)
+    e2e_v = nq * args.steps * world / sum(e2e_t)
+
+    cand = st.candidates
+    row_bytes = w.row_bytes
+    refine_avg_ms = sum(refine_ms) / len(refine_ms)
+    achieved = cand * row_bytes / (refine_avg_ms / 1e3) / 1e9
+    peaks, peak_src = measured_peaks()
+    traffic = traffic_from_profile(w.name, P, C)
+    out = {
+        "metric": "QPS at Recall@10~0.90 (batched query path); refine-scan HBM GB/s",
+        "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
+        "warmup": max(3, args.warmup), "ms_per_step": tot_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
+        "config": {"workload": w.name, "N": w.n, "D": w.dim, "nq": nq, "k": k, "bits": w.bits,
+                   "hidden": w.hidden, "K_max": w.k_max, "P": P, "C": C, "t_low": t_low,
+                   "round": 256, "recall_at_10": rec, "cand_per_query": cand / nq,
+                   "l2": "flushed between timed steps (256 MB write)",
+                   "parallelism": f"replicas x{world} (queries sharded, no collective)"},
+        "roofline": {"kernel": "nr_refine", "bound": "hbm", "achieved": achieved,
+                     "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
+                     "frac": achieved / peaks.get("hbm_gbs"), "peak_source": peak_src,
+                     "traffic": traffic,
+                     "algorithmic_bytes_per_launch": cand * row_bytes,
+                     "avg_launch_ms": refine_avg_ms},
+        "stage_ms_per_step": {kk: v / args.steps for kk, v in stage_ms.items()},
+        "e2e": {"value": e2e_v, "unit": "queries/s", "h2d_bytes_per_step": nq * row_bytes,
+                "d2h_bytes_per_step": nq * k * 12},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+        "index_build_s": t_build,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cb, _ = cpu_baseline(w, path, qs, k, P, C, t_low, args.cpu_seconds)
+        out["cpu_baseline"] = cb
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    ix.close()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,186 @@
+/*
+ * neuroute.h -- C ABI of the GB300 (sm_103a) NeuRoute batched query path.
+ *
+ * NeuRoute (arxiv 2608.15438) answers approximate k-nearest-neighbour queries
+ * (problem statement: Sec. 3.1) from a bucketised index built on learned
+ * binary codes. One search call runs, for every query, on the GPU:
+ *   encode    l = E(q): MLP D -> H (ReLU) -> b logits               (Sec. 3.2.1)
+ *   binarise  a_j = [l_j >= tau_j], base code u0 = sum_j a_j 2^j    (Eq. 10)
+ *   probe     flip sets F ranked by summed deviation
+ *             delta_j = |l_j - tau_j| -> probe codes u0 XOR F      (Sec. 3.2.3, Algorithm 1)
+ *   lookup    code -> clusters -> rows through two CSR levels      (Sec. 3.3)
+ *   select    singleton buckets to C^dir; centroid distances, gate
+ *             theta = d_min + M(d_min), top-C -> C^cent            (Sec. 3.4.2, Algorithm 2)
+ *   refine    exact squared L2 of the rows of C^dir U C^cent into a
+ *             top-k, heap-quality early stop in fixed rounds      (Sec. 3.4, Algorithm 2)
+ *
+ * Conventions for every call
+ *  - Pointers named d_* are DEVICE pointers on the index's device, row-major
+ *    and contiguous; h_* are host pointers. The caller owns them.
+ *  - `stream` is a cudaStream_t (NULL = the legacy default stream). Calls
+ *    enqueue work on it and return; outputs are valid once the stream has
+ *    synchronised. Argument and allocation errors are returned synchronously
+ *    and enqueue nothing.
+ *  - Device-side range checks never trap: a bad index in the file sets a
+ *    device flag that the next call (or nr_last_stats) reports as
+ *    NR_ERR_DEVICE_CHECK.
+ *  - One handle is not safe for concurrent calls (it owns one workspace).
+ *  - Float arithmetic that decides an integer (bits, probe order, the gate,
+ *    top-C, top-k membership) uses a fixed operation order, so results are
+ *    bit-identical to a sequential CPU evaluation fed the same logits.
+ *
+ * Index file (little-endian), written by the package's builder:
+ *   header 256 B: "NRIXv001", u32 version=1, u32 dtype (0 uint8, 1 fp32),
+ *     u64 N, u32 D, H, b, K_max, t, u32 0, u64 n_clusters, f32 in_scale,
+ *     u32 0, u64 section offsets[10], u64 file size
+ *   sections (256-byte aligned): W1 f32[H][D], b1 f32[H], W2 f32[b][H],
+ *     b2 f32[b], tau f32[b], bkt_off u32[2^b + 1] (code -> cluster range),
+ *     cl_off u32[n_clusters + 1] (cluster -> row range), cent f32[n_clusters][b],
+ *     ids u32[N] (original id of each stored row), vec (uint8|fp32)[N][D]
+ *     stored in (code, cluster, id) order.
+ */
+#ifndef NEUROUTE_H
+#define NEUROUTE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct nr_index nr_index; /* opaque, owned by the library */
+
+typedef enum {
+  NR_OK = 0,
+  NR_ERR_INVALID_ARG = -1,  /* a bad argument or an unsupported size */
+  NR_ERR_IO = -2,           /* the index file cannot be opened or read */
+  NR_ERR_FORMAT = -3,       /* the index file is malformed or truncated */
+  NR_ERR_OOM = -4,          /* device or host allocation failed */
+  NR_ERR_CUDA = -5,         /* a CUDA runtime call failed */
+  NR_ERR_DEVICE_CHECK = -6  /* a kernel found an out-of-range index in the file */
+} nr_status;
+
+/* Query-time knobs. Defaults from nr_params_default().
+ * Algorithm 1 filters (off by default): only the l_sel least-certain bits may
+ * flip; |F| <= r_max; summed deviation <= s_max.
+ * Gate of Algorithm 2: theta = d_min + M(d_min) with M(x) = gate_m0 + gate_m1 * x
+ * (fp32 fmaf); gate_m0 = +inf turns the gate off.
+ * Early stop (Sec. 3.4.2), counted in refinement rounds of round_size
+ * candidates: after round t, "updates" = top-k members not present before the
+ * round, "front updates" = those within the first ceil(alpha_front * k) slots;
+ * the round is low quality iff updates < u_min and front updates < f_min; the
+ * search stops once the top-k is full, t >= r_min and t_low consecutive rounds
+ * were low quality (t_low = 0: never stop early). */
+typedef struct {
+  int l_sel;          /* <= 0: all b bits */
+  int r_max;          /* <= 0: unbounded */
+  float s_max;        /* +inf: off */
+  float gate_m0;      /* +inf: gate off */
+  float gate_m1;
+  int round_size;     /* power of two in [32, 4096]; default 256 */
+  int t_low;          /* default 4 */
+  int u_min;          /* default 1 */
+  int f_min;          /* default 1 */
+  int r_min;          /* default 1 */
+  float alpha_front;  /* in [0, 1]; default 0.5 */
+} nr_params;
+
+/* Per-search statistics (sums over the queries of the last search call). */
+typedef struct {
+  int64_t nq;
+  int64_t candidates; /* rows given an exact distance (rows of completed rounds) */
+  int64_t rounds;     /* refinement rounds run */
+  int64_t clusters;   /* |C^dir U C^cent| */
+  int64_t probes;     /* probe codes generated */
+} nr_stats;
+
+/* Status name, static storage. */
+const char *nr_status_string(nr_status s);
+
+/* Fill *p with the defaults above. */
+nr_status nr_params_default(nr_params *p);
+
+/* Load an index file into device memory on `device` (CUDA ordinal).
+ * Errors: NR_ERR_IO, NR_ERR_FORMAT (bad magic, sizes, truncation; b must be in
+ * [1, 24]; a row must be a multiple of 16 bytes and at most 1024 bytes),
+ * NR_ERR_OOM, NR_ERR_CUDA. On success *out owns all device memory of the
+ * index; release it with nr_index_free. */
+nr_status nr_index_load(const char *path, int device, nr_index **out);
+
+/* Release the index and its workspace. NULL is a no-op. */
+void nr_index_free(nr_index *ix);
+
+/* info[0..7] = N, D, H, b, n_clusters, dtype (0 uint8, 1 fp32), K_max, t */
+nr_status nr_index_info(const nr_index *ix, int64_t *info);
+
+/* Validate and set the query-time knobs (p = NULL restores the defaults).
+ * NR_ERR_INVALID_ARG if a field is out of range. */
+nr_status nr_set_params(nr_index *ix, const nr_params *p);
+
+/* Encoder forward (Sec. 3.2.1): d_x [nq x D] (uint8 or fp32, the index dtype)
+ * -> d_logits [nq x b] fp32. h = ReLU(W1 (in_scale x) + b1), l = W2 h + b2;
+ * operands fp16, accumulation fp32 (logits agree with an exact evaluation to
+ * about 1e-3 of their norm). nq = 0 is a no-op. */
+nr_status nr_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits, void *stream);
+
+/* Probe codes (Eq. 10 and Algorithm 1) from d_logits [nq x b]:
+ * d_codes [nq x probe_budget] u32 receives, per query, the codes of the first
+ * min(probe_budget, #admissible flip sets) flip sets in ascending
+ * (cost, |F|, rank mask) order, the base code first; d_nprobe [nq] their count.
+ * Unused slots are set to 0xFFFFFFFF. 1 <= probe_budget <= 4096. */
+nr_status nr_route(nr_index *ix, const float *d_logits, int64_t nq, int probe_budget,
+                   uint32_t *d_codes, int32_t *d_nprobe, void *stream);
+
+/* Ordered cluster list C^dir U C^cent (Sec. 3.4.2) from d_logits:
+ * d_clusters [nq x (probe_budget + cluster_budget)] int32 cluster indices sorted
+ * by (centroid distance, cluster index), -1 padded; d_ncl [nq] their count.
+ * Limits: 1 <= cluster_budget <= 4096; probe_budget * K_max <= 16384. */
+nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int probe_budget,
+                            int cluster_budget, int32_t *d_clusters, int32_t *d_ncl,
+                            void *stream);
+
+/* Whole query path: d_queries [nq x D] (index dtype) -> d_out_ids [nq x k]
+ * int64 original ids and d_out_dists [nq x k] fp32 squared L2 distances, each
+ * row sorted by (distance, id), padded with (-1, +inf) when fewer than k rows
+ * were scored. For uint8 indexes distances are the exact integer sums.
+ * 1 <= k <= 256, 1 <= probe_budget <= 4096, 1 <= cluster_budget <= 4096,
+ * probe_budget * K_max <= 16384. The library's workspace grows on demand. */
+nr_status nr_search(nr_index *ix, const void *d_queries, int64_t nq, int k, int probe_budget,
+                    int cluster_budget, int64_t *d_out_ids, float *d_out_dists, void *stream);
+
+/* As nr_search, with the logits supplied by the caller (d_logits [nq x b]);
+ * the encoder is not run. */
+nr_status nr_search_logits(nr_index *ix, const void *d_queries, const float *d_logits, int64_t nq,
+                           int k, int probe_budget, int cluster_budget, int64_t *d_out_ids,
+                           float *d_out_dists, void *stream);
+
+/* As nr_search with HOST buffers: h_queries [nq x D] is copied to the device,
+ * the search runs, and h_out_ids / h_out_dists are copied back; the call
+ * returns after the stream has synchronised. Pinned host memory gives full
+ * copy bandwidth; pageable memory works. */
+nr_status nr_search_host(nr_index *ix, const void *h_queries, int64_t nq, int k, int probe_budget,
+                         int cluster_budget, int64_t *h_out_ids, float *h_out_dists,
+                         void *stream);
+
+/* Per-query statistics of the last search call: d_stats [nq x 4] int64 =
+ * (candidates, rounds, clusters, probes). Enqueued on `stream`. */
+nr_status nr_query_stats(nr_index *ix, int64_t *d_stats, int64_t nq, void *stream);
+
+/* Sums over the last search call (synchronises the device). Also returns
+ * NR_ERR_DEVICE_CHECK if a kernel has flagged bad index data since load. */
+nr_status nr_last_stats(nr_index *ix, nr_stats *out);
+
+/* Kernel time in milliseconds of the stages of the last search call
+ * (ms[0..3] = encode, route, select, refine) measured with CUDA events on the
+ * launch stream; enable with nr_enable_timing(ix, 1). Synchronises. */
+nr_status nr_enable_timing(nr_index *ix, int on);
+nr_status nr_last_timing(nr_index *ix, float *ms);
+
+/* Number of kernels the library launched since load (all entry points). */
+int64_t nr_kernel_launches(const nr_index *ix);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* NEUROUTE_H */

@@ -1,0 +1,593 @@
+// C ABI of the query path: index loading, argument checks, workspace and the
+// launch sequence encode -> route -> select -> refine (see neuroute.h).
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <cmath>
+#include <new>
+#include <vector>
+
+#include "neuroute.h"
+#include "nr_internal.cuh"
+
+namespace {
+
+constexpr int kMaxProbe = 4096;
+constexpr int kMaxClusterBudget = 4096;
+constexpr int kMaxSelect = 16384;  // probe_budget * K_max
+constexpr int kMaxTopK = 256;
+constexpr size_t kChunkBudget = (size_t)4 << 30;  // workspace bytes per query chunk
+
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+nr_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return NR_OK;
+  if (e == cudaErrorMemoryAllocation) return NR_ERR_OOM;
+  return NR_ERR_CUDA;
+}
+
+uint32_t rd32(const unsigned char *h, int o) {
+  uint32_t v;
+  memcpy(&v, h + o, 4);
+  return v;
+}
+uint64_t rd64(const unsigned char *h, int o) {
+  uint64_t v;
+  memcpy(&v, h + o, 8);
+  return v;
+}
+
+size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Per-chunk workspace layout of a search over qc queries.
+struct Layout {
+  size_t logits, codes, nprobe, L, nL, seg, slen, total;
+};
+Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
+  Layout l;
+  size_t o = 0;
+  const size_t Lmax = (size_t)P + (size_t)C;
+  l.logits = o; o = align256(o + (size_t)qc * ix->b * 4);
+  l.codes = o;  o = align256(o + (size_t)qc * P * 4);
+  l.nprobe = o; o = align256(o + (size_t)qc * 4);
+  l.L = o;      o = align256(o + (size_t)qc * Lmax * 4);
+  l.nL = o;     o = align256(o + (size_t)qc * 4);
+  l.seg = o;    o = align256(o + (size_t)qc * Lmax * sizeof(nr_seg));
+  l.slen = o;   o = align256(o + (size_t)qc * 4);
+  l.total = o;
+  return l;
+}
+
+nr_status ensure_ws(nr_index *ix, size_t bytes) {
+  if (bytes <= ix->ws_cap) return NR_OK;
+  if (ix->ws) {
+    cudaFree(ix->ws);
+    ix->ws = nullptr;
+    ix->ws_cap = 0;
+    ix->d_stats = nullptr;
+  }
+  size_t want = bytes + bytes / 4;
+  if (cudaMalloc(&ix->ws, want) != cudaSuccess) {
+    cudaGetLastError();
+    if (cudaMalloc(&ix->ws, bytes) != cudaSuccess) {
+      cudaGetLastError();
+      ix->ws = nullptr;
+      return NR_ERR_OOM;
+    }
+    want = bytes;
+  }
+  ix->ws_cap = want;
+  return NR_OK;
+}
+
+struct TimedStage {
+  int stage;  // 0 encode, 1 route, 2 select, 3 refine; -1 unused
+  cudaEvent_t a, b;
+};
+
+nr_status check_params(const nr_params *p) {
+  if (!(p->round_size >= 32 && p->round_size <= 4096 && (p->round_size & (p->round_size - 1)) == 0))
+    return NR_ERR_INVALID_ARG;
+  if (p->t_low < 0 || p->r_min < 0 || p->u_min < 0 || p->f_min < 0) return NR_ERR_INVALID_ARG;
+  if (!(p->alpha_front >= 0.0f && p->alpha_front <= 1.0f)) return NR_ERR_INVALID_ARG;
+  if (std::isnan(p->s_max) || std::isnan(p->gate_m0) || std::isnan(p->gate_m1)) return NR_ERR_INVALID_ARG;
+  return NR_OK;
+}
+
+}  // namespace
+
+// Host-side extras of an index: the per-cluster "bucket holds one cluster"
+// table used by K3, stage timers, and the device staging buffer of
+// nr_search_host.
+struct nr_index_ext {
+  uint8_t *single = nullptr;
+  std::vector<TimedStage> timers;
+  void *io = nullptr;
+  size_t io_cap = 0;
+};
+
+// The extension lives right after the index object (allocated together).
+struct nr_index_full {
+  nr_index ix;
+  nr_index_ext ext;
+};
+
+static nr_index_ext *ext_of(nr_index *ix) { return &reinterpret_cast<nr_index_full *>(ix)->ext; }
+
+const uint8_t *nr_single_table(nr_index *ix) { return ext_of(ix)->single; }
+
+extern "C" {
+
+const char *nr_status_string(nr_status s) {
+  switch (s) {
+    case NR_OK: return "NR_OK";
+    case NR_ERR_INVALID_ARG: return "NR_ERR_INVALID_ARG";
+    case NR_ERR_IO: return "NR_ERR_IO";
+    case NR_ERR_FORMAT: return "NR_ERR_FORMAT";
+    case NR_ERR_OOM: return "NR_ERR_OOM";
+    case NR_ERR_CUDA: return "NR_ERR_CUDA";
+    case NR_ERR_DEVICE_CHECK: return "NR_ERR_DEVICE_CHECK";
+  }
+  return "NR_ERR_UNKNOWN";
+}
+
+nr_status nr_params_default(nr_params *p) {
+  if (!p) return NR_ERR_INVALID_ARG;
+  p->l_sel = 0;
+  p->r_max = 0;
+  p->s_max = INFINITY;
+  p->gate_m0 = INFINITY;
+  p->gate_m1 = 0.0f;
+  p->round_size = 256;
+  p->t_low = 4;
+  p->u_min = 1;
+  p->f_min = 1;
+  p->r_min = 1;
+  p->alpha_front = 0.5f;
+  return NR_OK;
+}
+
+void nr_index_free(nr_index *ix) {
+  if (!ix) return;
+  DeviceGuard g(ix->device);
+  nr_index_ext *e = ext_of(ix);
+  for (auto &t : e->timers) {
+    cudaEventDestroy(t.a);
+    cudaEventDestroy(t.b);
+  }
+  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->bkt_off,
+                  ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->single, e->io};
+  for (void *p : ptrs)
+    if (p) cudaFree(p);
+  delete reinterpret_cast<nr_index_full *>(ix);
+}
+
+nr_status nr_index_load(const char *path, int device, nr_index **out) {
+  if (!path || !out) return NR_ERR_INVALID_ARG;
+  *out = nullptr;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess) {
+    cudaGetLastError();
+    return NR_ERR_CUDA;
+  }
+  if (device < 0 || device >= ndev) return NR_ERR_INVALID_ARG;
+  FILE *f = fopen(path, "rb");
+  if (!f) return NR_ERR_IO;
+  unsigned char h[256];
+  if (fread(h, 1, 256, f) != 256) {
+    fclose(f);
+    return NR_ERR_FORMAT;
+  }
+  if (fseeko(f, 0, SEEK_END) != 0) {
+    fclose(f);
+    return NR_ERR_IO;
+  }
+  const uint64_t fsize = (uint64_t)ftello(f);
+  if (memcmp(h, "NRIXv001", 8) != 0 || rd32(h, 8) != 1) {
+    fclose(f);
+    return NR_ERR_FORMAT;
+  }
+  auto *full = new (std::nothrow) nr_index_full();
+  if (!full) {
+    fclose(f);
+    return NR_ERR_OOM;
+  }
+  nr_index *ix = &full->ix;
+  ix->device = device;
+  ix->dtype = (int)rd32(h, 12);
+  ix->N = (int64_t)rd64(h, 16);
+  ix->D = (int)rd32(h, 24);
+  ix->H = (int)rd32(h, 28);
+  ix->b = (int)rd32(h, 32);
+  ix->K_max = (int)rd32(h, 36);
+  ix->t = (int)rd32(h, 40);
+  ix->n_cl = (int64_t)rd64(h, 48);
+  memcpy(&ix->in_scale, h + 56, 4);
+  nr_params_default(&ix->params);
+  uint64_t off[10];
+  for (int i = 0; i < 10; ++i) off[i] = rd64(h, 64 + 8 * i);
+  const size_t esz = ix->dtype == 0 ? 1 : 4;
+  ix->row_bytes = (int64_t)ix->D * (int64_t)esz;
+  auto bad = [&](nr_status st) {
+    fclose(f);
+    nr_index_free(ix);
+    return st;
+  };
+  if ((ix->dtype != 0 && ix->dtype != 1) || ix->b < 1 || ix->b > 24 || ix->D < 1 || ix->H < 1 ||
+      ix->H > 4096 || ix->N < 1 || ix->N >= (int64_t)0xFFFFFFFFll || ix->n_cl < 1 ||
+      ix->n_cl >= (int64_t)0xFFFFFFFFll || ix->row_bytes % 16 != 0 || ix->row_bytes > 1024 ||
+      ix->K_max < 0)
+    return bad(NR_ERR_FORMAT);
+  const uint64_t nb = ((uint64_t)1 << ix->b) + 1;
+  const uint64_t sz[10] = {(uint64_t)ix->H * ix->D * 4, (uint64_t)ix->H * 4,
+                           (uint64_t)ix->b * ix->H * 4, (uint64_t)ix->b * 4,
+                           (uint64_t)ix->b * 4,         nb * 4,
+                           (uint64_t)(ix->n_cl + 1) * 4, (uint64_t)ix->n_cl * ix->b * 4,
+                           (uint64_t)ix->N * 4,         (uint64_t)ix->N * ix->D * esz};
+  for (int i = 0; i < 10; ++i)
+    if (off[i] < 256 || off[i] + sz[i] > fsize) return bad(NR_ERR_FORMAT);
+  // host copies of the small sections
+  std::vector<float> W1((size_t)ix->H * ix->D), b1(ix->H), W2((size_t)ix->b * ix->H), b2(ix->b),
+      tau(ix->b);
+  std::vector<uint32_t> bkt(nb);
+  auto rd = [&](int i, void *dst) {
+    return fseeko(f, (off_t)off[i], SEEK_SET) == 0 && fread(dst, 1, sz[i], f) == sz[i];
+  };
+  if (!rd(0, W1.data()) || !rd(1, b1.data()) || !rd(2, W2.data()) || !rd(3, b2.data()) ||
+      !rd(4, tau.data()) || !rd(5, bkt.data()))
+    return bad(NR_ERR_IO);
+  // clusters per bucket: K_max from the header, else from the directory
+  int kmax_dir = 1;
+  std::vector<uint8_t> single((size_t)ix->n_cl, 0);
+  for (uint64_t u = 0; u + 1 < nb; ++u) {
+    if (bkt[u + 1] >= bkt[u]) {
+      const uint32_t n = bkt[u + 1] - bkt[u];
+      if ((int64_t)n > kmax_dir && n <= 65536) kmax_dir = (int)n;
+      if (n == 1 && bkt[u] < (uint64_t)ix->n_cl) single[bkt[u]] = 1;
+    }
+  }
+  if (ix->K_max < 1) ix->K_max = kmax_dir;
+  DeviceGuard g(device);
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return bad(NR_ERR_CUDA);
+  ix->num_sms = prop.multiProcessorCount;
+  std::vector<float> W1T((size_t)ix->D * ix->H);
+  for (int u = 0; u < ix->H; ++u)
+    for (int j = 0; j < ix->D; ++j) W1T[(size_t)j * ix->H + u] = W1[(size_t)u * ix->D + j];
+  auto up = [&](void **dptr, const void *src, size_t bytes) -> nr_status {
+    if (cudaMalloc(dptr, bytes > 0 ? bytes : 16) != cudaSuccess) {
+      cudaGetLastError();
+      *dptr = nullptr;
+      return NR_ERR_OOM;
+    }
+    if (src && bytes && cudaMemcpy(*dptr, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess)
+      return NR_ERR_CUDA;
+    return NR_OK;
+  };
+  nr_status st;
+  if ((st = up((void **)&ix->W1, W1.data(), sz[0])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->b1, b1.data(), sz[1])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->W2, W2.data(), sz[2])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->b2, b2.data(), sz[3])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->tau, tau.data(), sz[4])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->W1T, W1T.data(), sz[0])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->bkt_off, bkt.data(), sz[5])) != NR_OK) return bad(st);
+  if ((st = up((void **)&ext_of(ix)->single, single.data(), single.size())) != NR_OK) return bad(st);
+  if ((st = up((void **)&ix->d_err, nullptr, 16)) != NR_OK) return bad(st);
+  if (cudaMemset(ix->d_err, 0, 16) != cudaSuccess) return bad(NR_ERR_CUDA);
+  // large sections streamed through a pinned staging buffer
+  const size_t stage_bytes = (size_t)64 << 20;
+  void *stage = nullptr;
+  if (cudaMallocHost(&stage, stage_bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return bad(NR_ERR_OOM);
+  }
+  auto stream_up = [&](int i, void **dptr) -> nr_status {
+    if (cudaMalloc(dptr, sz[i] > 0 ? sz[i] : 16) != cudaSuccess) {
+      cudaGetLastError();
+      *dptr = nullptr;
+      return NR_ERR_OOM;
+    }
+    if (fseeko(f, (off_t)off[i], SEEK_SET) != 0) return NR_ERR_IO;
+    for (uint64_t done = 0; done < sz[i];) {
+      const size_t n = (size_t)((sz[i] - done) < stage_bytes ? (sz[i] - done) : stage_bytes);
+      if (fread(stage, 1, n, f) != n) return NR_ERR_IO;
+      if (cudaMemcpy((char *)*dptr + done, stage, n, cudaMemcpyHostToDevice) != cudaSuccess)
+        return NR_ERR_CUDA;
+      done += n;
+    }
+    return NR_OK;
+  };
+  st = stream_up(6, (void **)&ix->cl_off);
+  if (st == NR_OK) st = stream_up(7, (void **)&ix->cent);
+  if (st == NR_OK) st = stream_up(8, (void **)&ix->ids);
+  if (st == NR_OK) st = stream_up(9, &ix->vec);
+  cudaFreeHost(stage);
+  if (st != NR_OK) return bad(st);
+  fclose(f);
+  *out = ix;
+  return NR_OK;
+}
+
+nr_status nr_index_info(const nr_index *ix, int64_t *info) {
+  if (!ix || !info) return NR_ERR_INVALID_ARG;
+  info[0] = ix->N;
+  info[1] = ix->D;
+  info[2] = ix->H;
+  info[3] = ix->b;
+  info[4] = ix->n_cl;
+  info[5] = ix->dtype;
+  info[6] = ix->K_max;
+  info[7] = ix->t;
+  return NR_OK;
+}
+
+nr_status nr_set_params(nr_index *ix, const nr_params *p) {
+  if (!ix) return NR_ERR_INVALID_ARG;
+  nr_params d;
+  nr_params_default(&d);
+  if (!p) p = &d;
+  nr_status st = check_params(p);
+  if (st != NR_OK) return st;
+  ix->params = *p;
+  return NR_OK;
+}
+
+nr_status nr_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits, void *stream) {
+  if (!ix || nq < 0) return NR_ERR_INVALID_ARG;
+  if (nq == 0) return NR_OK;
+  if (!d_x || !d_logits) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  return cuda_status(nr_launch_encode(ix, d_x, nq, d_logits, (cudaStream_t)stream));
+}
+
+nr_status nr_route(nr_index *ix, const float *d_logits, int64_t nq, int probe_budget,
+                   uint32_t *d_codes, int32_t *d_nprobe, void *stream) {
+  if (!ix || nq < 0 || probe_budget < 1 || probe_budget > kMaxProbe) return NR_ERR_INVALID_ARG;
+  if (nq == 0) return NR_OK;
+  if (!d_logits || !d_codes || !d_nprobe || nq > (int64_t)1 << 30) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  return cuda_status(nr_launch_route(ix, d_logits, nq, probe_budget, d_codes, d_nprobe,
+                                     (cudaStream_t)stream));
+}
+
+static nr_status check_budgets(const nr_index *ix, int64_t nq, int k, int P, int C) {
+  if (nq < 0 || P < 1 || P > kMaxProbe || C < 1 || C > kMaxClusterBudget) return NR_ERR_INVALID_ARG;
+  if ((int64_t)P * ix->K_max > kMaxSelect) return NR_ERR_INVALID_ARG;
+  if (k < 1 || k > kMaxTopK || nq > ((int64_t)1 << 31) - 1) return NR_ERR_INVALID_ARG;
+  return NR_OK;
+}
+
+nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int probe_budget,
+                            int cluster_budget, int32_t *d_clusters, int32_t *d_ncl,
+                            void *stream) {
+  if (!ix) return NR_ERR_INVALID_ARG;
+  nr_status st = check_budgets(ix, nq, 1, probe_budget, cluster_budget);
+  if (st != NR_OK) return st;
+  if (nq == 0) return NR_OK;
+  if (!d_logits || !d_clusters || !d_ncl) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  const int P = probe_budget, C = cluster_budget;
+  Layout l = chunk_layout(ix, nq, P, C);
+  if ((st = ensure_ws(ix, l.total)) != NR_OK) return st;
+  char *w = (char *)ix->ws;
+  cudaError_t e = nr_launch_route(ix, d_logits, nq, P, (uint32_t *)(w + l.codes),
+                                  (int32_t *)(w + l.nprobe), s);
+  if (e == cudaSuccess)
+    e = nr_launch_select(ix, d_logits, (uint32_t *)(w + l.codes), (int32_t *)(w + l.nprobe), nq,
+                         P, C, d_clusters, d_ncl, (nr_seg *)(w + l.seg), (uint32_t *)(w + l.slen),
+                         nullptr, s);
+  return cuda_status(e);
+}
+
+static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logits_in, int64_t nq,
+                             int k, int P, int C, int64_t *d_ids, float *d_d, cudaStream_t s) {
+  nr_status st = check_budgets(ix, nq, k, P, C);
+  if (st != NR_OK) return st;
+  // workspace: [per-query stats][query counter][per-chunk buffers]
+  const size_t stats_off = 0;
+  const size_t cnt_off = align256(stats_off + (size_t)nq * 4 * 8);
+  const size_t chunk_off = align256(cnt_off + 16);
+  Layout one = chunk_layout(ix, 1, P, C);
+  int64_t qc = (int64_t)(kChunkBudget / (one.total > 0 ? one.total : 1));
+  if (qc < 1) qc = 1;
+  if (qc > nq) qc = nq;
+  Layout l = chunk_layout(ix, qc, P, C);
+  if ((st = ensure_ws(ix, chunk_off + l.total)) != NR_OK) return st;
+  char *w = (char *)ix->ws;
+  int64_t *stats = (int64_t *)(w + stats_off);
+  ix->d_stats = stats;
+  ix->last_nq = nq;
+  unsigned int *counter = (unsigned int *)(w + cnt_off);
+  char *cw = w + chunk_off;
+  nr_index_ext *ex = ext_of(ix);
+  size_t tslot = 0;
+  auto tstart = [&](int stage) -> size_t {
+    if (!ix->timing) return 0;
+    if (tslot >= ex->timers.size()) {
+      TimedStage t{stage, nullptr, nullptr};
+      cudaEventCreate(&t.a);
+      cudaEventCreate(&t.b);
+      ex->timers.push_back(t);
+    }
+    ex->timers[tslot].stage = stage;
+    cudaEventRecord(ex->timers[tslot].a, s);
+    return tslot;
+  };
+  auto tend = [&](size_t slot) {
+    if (!ix->timing) return;
+    cudaEventRecord(ex->timers[slot].b, s);
+    ++tslot;
+  };
+  cudaError_t e = cudaSuccess;
+  const int64_t RB = ix->row_bytes;
+  for (int64_t q0 = 0; q0 < nq && e == cudaSuccess; q0 += qc) {
+    const int64_t n = (nq - q0) < qc ? (nq - q0) : qc;
+    const void *qp = (const char *)d_q + q0 * RB;
+    const float *lg = d_logits_in ? d_logits_in + q0 * ix->b : (const float *)(cw + l.logits);
+    size_t ev;
+    if (!d_logits_in) {
+      ev = tstart(0);
+      e = nr_launch_encode(ix, qp, n, (float *)(cw + l.logits), s);
+      tend(ev);
+      if (e != cudaSuccess) break;
+    }
+    ev = tstart(1);
+    e = nr_launch_route(ix, lg, n, P, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), s);
+    tend(ev);
+    if (e != cudaSuccess) break;
+    ev = tstart(2);
+    e = nr_launch_select(ix, lg, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), n, P, C,
+                         (int32_t *)(cw + l.L), (int32_t *)(cw + l.nL), (nr_seg *)(cw + l.seg),
+                         (uint32_t *)(cw + l.slen), stats + q0 * 4, s);
+    tend(ev);
+    if (e != cudaSuccess) break;
+    ev = tstart(3);
+    e = nr_launch_refine(ix, qp, n, k, P + C, (nr_seg *)(cw + l.seg), (int32_t *)(cw + l.nL),
+                         (uint32_t *)(cw + l.slen), d_ids + q0 * k, d_d + q0 * k, stats + q0 * 4,
+                         counter, s);
+    tend(ev);
+  }
+  ix->timed_last = ix->timing;
+  for (size_t i = tslot; i < ex->timers.size(); ++i) ex->timers[i].stage = -1;
+  return cuda_status(e);
+}
+
+nr_status nr_search(nr_index *ix, const void *d_queries, int64_t nq, int k, int probe_budget,
+                    int cluster_budget, int64_t *d_out_ids, float *d_out_dists, void *stream) {
+  if (!ix) return NR_ERR_INVALID_ARG;
+  if (nq > 0 && (!d_queries || !d_out_ids || !d_out_dists)) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  if (nq == 0) return check_budgets(ix, nq, k, probe_budget, cluster_budget);
+  return search_impl(ix, d_queries, nullptr, nq, k, probe_budget, cluster_budget, d_out_ids,
+                     d_out_dists, (cudaStream_t)stream);
+}
+
+nr_status nr_search_logits(nr_index *ix, const void *d_queries, const float *d_logits, int64_t nq,
+                           int k, int probe_budget, int cluster_budget, int64_t *d_out_ids,
+                           float *d_out_dists, void *stream) {
+  if (!ix) return NR_ERR_INVALID_ARG;
+  if (nq > 0 && (!d_queries || !d_logits || !d_out_ids || !d_out_dists)) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  if (nq == 0) return check_budgets(ix, nq, k, probe_budget, cluster_budget);
+  return search_impl(ix, d_queries, d_logits, nq, k, probe_budget, cluster_budget, d_out_ids,
+                     d_out_dists, (cudaStream_t)stream);
+}
+
+nr_status nr_search_host(nr_index *ix, const void *h_queries, int64_t nq, int k, int probe_budget,
+                         int cluster_budget, int64_t *h_out_ids, float *h_out_dists,
+                         void *stream) {
+  if (!ix) return NR_ERR_INVALID_ARG;
+  nr_status st = check_budgets(ix, nq, k, probe_budget, cluster_budget);
+  if (st != NR_OK) return st;
+  if (nq == 0) return NR_OK;
+  if (!h_queries || !h_out_ids || !h_out_dists) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  // device staging for the inputs and outputs, kept by the index and grown on demand
+  const size_t qb = align256((size_t)nq * ix->row_bytes);
+  const size_t ib = align256((size_t)nq * k * 8);
+  const size_t db = align256((size_t)nq * k * 4);
+  nr_index_ext *ex = ext_of(ix);
+  if (ex->io_cap < qb + ib + db) {
+    if (ex->io) cudaFree(ex->io);
+    ex->io = nullptr;
+    ex->io_cap = 0;
+    if (cudaMalloc(&ex->io, qb + ib + db) != cudaSuccess) {
+      cudaGetLastError();
+      ex->io = nullptr;
+      return NR_ERR_OOM;
+    }
+    ex->io_cap = qb + ib + db;
+  }
+  char *d = (char *)ex->io;
+  cudaError_t e = cudaMemcpyAsync(d, h_queries, (size_t)nq * ix->row_bytes, cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) {
+    st = search_impl(ix, d, nullptr, nq, k, probe_budget, cluster_budget, (int64_t *)(d + qb),
+                     (float *)(d + qb + ib), s);
+    if (st == NR_OK) {
+      e = cudaMemcpyAsync(h_out_ids, d + qb, (size_t)nq * k * 8, cudaMemcpyDeviceToHost, s);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(h_out_dists, d + qb + ib, (size_t)nq * k * 4, cudaMemcpyDeviceToHost, s);
+    }
+  }
+  const cudaError_t e2 = cudaStreamSynchronize(s);
+  if (st != NR_OK) return st;
+  if (e == cudaSuccess) e = e2;
+  return cuda_status(e);
+}
+
+nr_status nr_query_stats(nr_index *ix, int64_t *d_stats, int64_t nq, void *stream) {
+  if (!ix || nq < 0 || nq > ix->last_nq || (nq > 0 && (!d_stats || !ix->d_stats)))
+    return NR_ERR_INVALID_ARG;
+  if (nq == 0) return NR_OK;
+  DeviceGuard g(ix->device);
+  return cuda_status(cudaMemcpyAsync(d_stats, ix->d_stats, (size_t)nq * 4 * 8,
+                                     cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
+}
+
+nr_status nr_last_stats(nr_index *ix, nr_stats *out) {
+  if (!ix || !out) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  memset(out, 0, sizeof(*out));
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_status(e);
+  out->nq = ix->last_nq;
+  if (ix->last_nq > 0 && ix->d_stats) {
+    std::vector<int64_t> h((size_t)ix->last_nq * 4);
+    e = cudaMemcpy(h.data(), ix->d_stats, h.size() * 8, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_status(e);
+    for (int64_t i = 0; i < ix->last_nq; ++i) {
+      out->candidates += h[(size_t)i * 4 + 0];
+      out->rounds += h[(size_t)i * 4 + 1];
+      out->clusters += h[(size_t)i * 4 + 2];
+      out->probes += h[(size_t)i * 4 + 3];
+    }
+  }
+  int flag = 0;
+  e = cudaMemcpy(&flag, ix->d_err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_status(e);
+  if (flag != 0) {
+    cudaMemset(ix->d_err, 0, sizeof(int));
+    return NR_ERR_DEVICE_CHECK;
+  }
+  return NR_OK;
+}
+
+nr_status nr_enable_timing(nr_index *ix, int on) {
+  if (!ix) return NR_ERR_INVALID_ARG;
+  ix->timing = on != 0;
+  return NR_OK;
+}
+
+nr_status nr_last_timing(nr_index *ix, float *ms) {
+  if (!ix || !ms) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  for (int i = 0; i < 4; ++i) ms[i] = 0.0f;
+  if (!ix->timed_last) return NR_OK;
+  for (auto &t : ext_of(ix)->timers) {
+    if (t.stage < 0) continue;
+    if (cudaEventSynchronize(t.b) != cudaSuccess) return NR_ERR_CUDA;
+    float v = 0.0f;
+    if (cudaEventElapsedTime(&v, t.a, t.b) != cudaSuccess) return NR_ERR_CUDA;
+    ms[t.stage] += v;
+  }
+  return NR_OK;
+}
+
+int64_t nr_kernel_launches(const nr_index *ix) { return ix ? ix->launches : 0; }
+
+}  // extern "C"

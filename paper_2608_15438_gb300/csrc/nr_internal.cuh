@@ -1,0 +1,66 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "neuroute.h"
+
+// Device-side check codes (first one wins; the host maps any to NR_ERR_DEVICE_CHECK)
+enum : int {
+  NR_DEV_OK = 0,
+  NR_DEV_BAD_BUCKET = 1,   // bkt_off range reversed or past n_clusters
+  NR_DEV_BAD_CLUSTER = 2,  // cl_off range reversed or past N
+  NR_DEV_TOO_MANY = 3,     // a bucket holds more than K_max clusters
+  NR_DEV_BAD_CODE = 4      // a probe code >= 2^b
+};
+
+struct nr_index {
+  int device = 0;
+  int dtype = 0;  // 0 uint8, 1 fp32
+  int64_t N = 0;
+  int D = 0, H = 0, b = 0, K_max = 0, t = 0;
+  int64_t n_cl = 0;
+  float in_scale = 1.0f;
+  int64_t row_bytes = 0;
+  // device arrays
+  float *W1 = nullptr, *b1 = nullptr, *W2 = nullptr, *b2 = nullptr, *tau = nullptr;
+  float *cent = nullptr;
+  float *W1T = nullptr;  // [D][H]
+  uint32_t *bkt_off = nullptr, *cl_off = nullptr, *ids = nullptr;
+  void *vec = nullptr;
+  int *d_err = nullptr;
+  nr_params params{};
+  // workspace (grows on demand)
+  void *ws = nullptr;
+  size_t ws_cap = 0;
+  int64_t last_nq = 0;
+  int64_t *d_stats = nullptr;  // into ws, [last_nq x 4]
+  bool timing = false;
+  bool timed_last = false;
+  cudaEvent_t ev[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
+  int64_t launches = 0;
+  int num_sms = 0;
+};
+
+// Per-query refinement segment: rows [row0, row0 + len) of cluster L[i]
+// start at stream position pos.
+struct nr_seg {
+  uint32_t row0;
+  uint32_t pos;
+};
+
+// kernel launchers (each returns cudaGetLastError() after the launch)
+cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
+                             cudaStream_t s);
+cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
+                            uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s);
+size_t nr_select_smem_bytes(int P, int C, int K_max);
+cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t *d_codes,
+                             const int32_t *d_nprobe, int64_t nq, int P, int C, int32_t *d_L,
+                             int32_t *d_nL, nr_seg *d_seg, uint32_t *d_slen, int64_t *d_stats,
+                             cudaStream_t s);
+cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, int Lmax,
+                             const nr_seg *d_seg, const int32_t *d_nL, const uint32_t *d_slen,
+                             int64_t *d_ids, float *d_dists, int64_t *d_stats,
+                             unsigned int *d_counter, cudaStream_t s);

@@ -1,0 +1,226 @@
+"""ctypes binding of libneuroute.so: the same entry points as
+include/neuroute.h, argument marshalling only. Device buffers are torch CUDA
+tensors (used for memory and streams only); every step of the search runs in
+the library's kernels. There is no fallback: if the library is missing or a
+call fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libneuroute.so")
+_LIB = None
+
+NR_OK = 0
+STATUS = {0: "NR_OK", -1: "NR_ERR_INVALID_ARG", -2: "NR_ERR_IO", -3: "NR_ERR_FORMAT",
+          -4: "NR_ERR_OOM", -5: "NR_ERR_CUDA", -6: "NR_ERR_DEVICE_CHECK"}
+
+EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_free",
+           "nr_index_info", "nr_set_params", "nr_encode", "nr_route", "nr_debug_clusters",
+           "nr_search", "nr_search_logits", "nr_search_host", "nr_query_stats", "nr_last_stats",
+           "nr_enable_timing", "nr_last_timing", "nr_kernel_launches"]
+
+
+class NRError(RuntimeError):
+    def __init__(self, call, status):
+        super().__init__(f"{call} failed: {STATUS.get(status, status)}")
+        self.status = status
+
+
+class Params(ctypes.Structure):
+    _fields_ = [("l_sel", ctypes.c_int), ("r_max", ctypes.c_int), ("s_max", ctypes.c_float),
+                ("gate_m0", ctypes.c_float), ("gate_m1", ctypes.c_float),
+                ("round_size", ctypes.c_int), ("t_low", ctypes.c_int), ("u_min", ctypes.c_int),
+                ("f_min", ctypes.c_int), ("r_min", ctypes.c_int), ("alpha_front", ctypes.c_float)]
+
+
+class Stats(ctypes.Structure):
+    _fields_ = [("nq", ctypes.c_int64), ("candidates", ctypes.c_int64), ("rounds", ctypes.c_int64),
+                ("clusters", ctypes.c_int64), ("probes", ctypes.c_int64)]
+
+
+def lib():
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} missing: run __graft_entry__.build() first")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+        L.nr_status_string.argtypes = [i32]
+        L.nr_status_string.restype = ctypes.c_char_p
+        L.nr_params_default.argtypes = [ctypes.POINTER(Params)]
+        L.nr_index_load.argtypes = [ctypes.c_char_p, i32, ctypes.POINTER(vp)]
+        L.nr_index_free.argtypes = [vp]
+        L.nr_index_free.restype = None
+        L.nr_index_info.argtypes = [vp, vp]
+        L.nr_set_params.argtypes = [vp, ctypes.POINTER(Params)]
+        L.nr_encode.argtypes = [vp, vp, i64, vp, vp]
+        L.nr_route.argtypes = [vp, vp, i64, i32, vp, vp, vp]
+        L.nr_debug_clusters.argtypes = [vp, vp, i64, i32, i32, vp, vp, vp]
+        L.nr_search.argtypes = [vp, vp, i64, i32, i32, i32, vp, vp, vp]
+        L.nr_search_logits.argtypes = [vp, vp, vp, i64, i32, i32, i32, vp, vp, vp]
+        L.nr_search_host.argtypes = [vp, vp, i64, i32, i32, i32, vp, vp, vp]
+        L.nr_query_stats.argtypes = [vp, vp, i64, vp]
+        L.nr_last_stats.argtypes = [vp, ctypes.POINTER(Stats)]
+        L.nr_enable_timing.argtypes = [vp, i32]
+        L.nr_last_timing.argtypes = [vp, vp]
+        L.nr_kernel_launches.argtypes = [vp]
+        L.nr_kernel_launches.restype = i64
+        for name in EXPORTS:
+            if name not in ("nr_status_string", "nr_index_free", "nr_kernel_launches"):
+                getattr(L, name).restype = i32
+        _LIB = L
+    return _LIB
+
+
+def _check(call, st):
+    if st != NR_OK:
+        raise NRError(call, st)
+
+
+def params(**kw) -> Params:
+    p = Params()
+    lib().nr_params_default(ctypes.byref(p))
+    for k, v in kw.items():
+        if not hasattr(p, k):
+            raise KeyError(k)
+        setattr(p, k, v)
+    return p
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+class Index:
+    """A loaded index on one GPU."""
+
+    def __init__(self, path: str, device: int = 0):
+        h = ctypes.c_void_p()
+        _check("nr_index_load", lib().nr_index_load(path.encode(), device, ctypes.byref(h)))
+        self.h = h
+        self.device = device
+        info = np.zeros(8, np.int64)
+        lib().nr_index_info(h, info.ctypes.data)
+        (self.N, self.D, self.H, self.b, self.n_clusters, self.dtype_code, self.k_max,
+         self.t) = (int(v) for v in info)
+
+    def close(self):
+        if self.h:
+            lib().nr_index_free(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    @property
+    def row_bytes(self):
+        return self.D * (1 if self.dtype_code == 0 else 4)
+
+    def set_params(self, p: Params | None = None, **kw):
+        if p is None:
+            p = params(**kw)
+        _check("nr_set_params", lib().nr_set_params(self.h, ctypes.byref(p)))
+        return p
+
+    def _dev(self):
+        import torch
+
+        return torch.device("cuda", self.device)
+
+    def encode(self, x, stream=None):
+        import torch
+
+        out = torch.empty((x.shape[0], self.b), dtype=torch.float32, device=self._dev())
+        _check("nr_encode", lib().nr_encode(self.h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)))
+        return out
+
+    def route(self, logits, P, stream=None):
+        import torch
+
+        nq = logits.shape[0]
+        codes = torch.empty((nq, P), dtype=torch.int32, device=self._dev())
+        nprobe = torch.empty(nq, dtype=torch.int32, device=self._dev())
+        _check("nr_route", lib().nr_route(self.h, _ptr(logits), nq, P, _ptr(codes), _ptr(nprobe),
+                                          _stream(stream)))
+        return codes, nprobe
+
+    def debug_clusters(self, logits, P, C, stream=None):
+        import torch
+
+        nq = logits.shape[0]
+        cl = torch.empty((nq, P + C), dtype=torch.int32, device=self._dev())
+        ncl = torch.empty(nq, dtype=torch.int32, device=self._dev())
+        _check("nr_debug_clusters", lib().nr_debug_clusters(self.h, _ptr(logits), nq, P, C, _ptr(cl),
+                                                            _ptr(ncl), _stream(stream)))
+        return cl, ncl
+
+    def _outputs(self, nq, k):
+        import torch
+
+        return (torch.empty((nq, k), dtype=torch.int64, device=self._dev()),
+                torch.empty((nq, k), dtype=torch.float32, device=self._dev()))
+
+    def search(self, queries, k, P, C, out=None, stream=None):
+        nq = queries.shape[0]
+        ids, d = out if out is not None else self._outputs(nq, k)
+        _check("nr_search", lib().nr_search(self.h, _ptr(queries), nq, k, P, C, _ptr(ids), _ptr(d),
+                                            _stream(stream)))
+        return ids, d
+
+    def search_logits(self, queries, logits, k, P, C, out=None, stream=None):
+        nq = queries.shape[0]
+        ids, d = out if out is not None else self._outputs(nq, k)
+        _check("nr_search_logits", lib().nr_search_logits(self.h, _ptr(queries), _ptr(logits), nq, k,
+                                                          P, C, _ptr(ids), _ptr(d), _stream(stream)))
+        return ids, d
+
+    def search_host(self, queries, k, P, C, out=None, stream=None):
+        """queries, and the outputs, are host tensors (pinned for full bandwidth)."""
+        import torch
+
+        nq = queries.shape[0]
+        if out is None:
+            out = (torch.empty((nq, k), dtype=torch.int64), torch.empty((nq, k), dtype=torch.float32))
+        ids, d = out
+        _check("nr_search_host", lib().nr_search_host(self.h, _ptr(queries), nq, k, P, C, _ptr(ids),
+                                                      _ptr(d), _stream(stream)))
+        return ids, d
+
+    def query_stats(self, nq, stream=None):
+        import torch
+
+        st = torch.empty((nq, 4), dtype=torch.int64, device=self._dev())
+        _check("nr_query_stats", lib().nr_query_stats(self.h, _ptr(st), nq, _stream(stream)))
+        return st
+
+    def last_stats(self) -> Stats:
+        s = Stats()
+        _check("nr_last_stats", lib().nr_last_stats(self.h, ctypes.byref(s)))
+        return s
+
+    def enable_timing(self, on=True):
+        _check("nr_enable_timing", lib().nr_enable_timing(self.h, 1 if on else 0))
+
+    def last_timing(self):
+        ms = np.zeros(4, np.float32)
+        _check("nr_last_timing", lib().nr_last_timing(self.h, ms.ctypes.data))
+        return {"encode": float(ms[0]), "route": float(ms[1]), "select": float(ms[2]),
+                "refine": float(ms[3])}
+
+    def kernel_launches(self) -> int:
+        return int(lib().nr_kernel_launches(self.h))

@@ -1,0 +1,272 @@
+"""GPU query path (through the C ABI) against the oracle, element by element.
+
+Integer and index results must be bit-identical when the GPU is fed the
+oracle's logits: probe codes (Algorithm 1), cluster lists (Algorithm 2's
+centroid stage), top-k ids and uint8 distances; fp32 distances are compared
+exactly too (both sides evaluate the same sequential fmaf chain), which is
+stricter than the 1e-5 relative tolerance allowed for them. Encoder logits
+are compared normwise within 1e-2 of the oracle's double-precision forward.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from gpu_util import build_small, need_cuda, recall
+from nrix_writer import write_nrix
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def torch():
+    return need_cuda()
+
+
+@pytest.fixture(scope="module")
+def tiny(torch, tiny_index):
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    ix = nr.Index(tiny_index["path"], 0)
+    orc = oracle.Index(tiny_index["path"])
+    qs = tiny_index["queries"]
+    lg = orc.encode(qs)
+    return {"ix": ix, "orc": orc, "q": qs, "lg": lg, "dq": torch.from_numpy(qs).cuda(),
+            "dl": torch.from_numpy(lg).cuda(), "base": tiny_index["base"]}
+
+
+@pytest.mark.parametrize("P", [1, 2, 8, 64, 500, 4096])
+def test_route_codes_bit_exact(tiny, torch, P):
+    codes, nprobe = tiny["ix"].route(tiny["dl"], P)
+    codes = codes.cpu().numpy().view(np.uint32)
+    nprobe = nprobe.cpu().numpy()
+    tau = tiny["orc"].tau()
+    p = oracle.params()
+    for i in range(0, len(tiny["q"]), 7 if P >= 500 else 1):
+        exp, _, _ = oracle.probe_list(tiny["lg"][i], tau, P, p)
+        assert nprobe[i] == len(exp)
+        assert np.array_equal(codes[i, : len(exp)], exp), i
+        assert np.all(codes[i, len(exp):] == 0xFFFFFFFF)
+
+
+@pytest.mark.parametrize("kw", [dict(l_sel=6), dict(r_max=2), dict(s_max=0.05),
+                                dict(l_sel=9, r_max=3, s_max=0.2)])
+def test_route_filters_bit_exact(tiny, torch, kw):
+    ix = tiny["ix"]
+    ix.set_params(**kw)
+    try:
+        codes, nprobe = ix.route(tiny["dl"], 300)
+    finally:
+        ix.set_params()
+    codes = codes.cpu().numpy().view(np.uint32)
+    tau = tiny["orc"].tau()
+    p = oracle.params(**kw)
+    for i in range(0, len(tiny["q"]), 3):
+        exp, _, _ = oracle.probe_list(tiny["lg"][i], tau, 300, p)
+        assert int(nprobe[i]) == len(exp)
+        assert np.array_equal(codes[i, : len(exp)], exp)
+
+
+def test_route_b4_hand_order(torch, tmp_path):
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    # a 4-bit index whose only purpose is to carry tau = 0 (vectors unused)
+    bkt = np.zeros(17, np.uint32)
+    bkt[1:] = 1
+    path = str(tmp_path / "b4.nrix")
+    write_nrix(path, np.zeros((1, 16), np.uint8), [0], bkt, [0, 1], np.zeros((1, 4)), np.zeros(4),
+               np.zeros((2, 16)), np.zeros(2), np.zeros((4, 2)), np.zeros(4))
+    ix = nr.Index(path, 0)
+    lg = torch.tensor([[0.375, -0.125, 0.5, -0.25]], dtype=torch.float32, device="cuda")
+    codes, n = ix.route(lg, 16)
+    assert [f"{c:X}" for c in codes.cpu().numpy().view(np.uint32)[0]] == list("57D4F16C39E0B28A")
+
+
+@pytest.mark.parametrize("P,C", [(1, 1), (8, 32), (64, 16), (256, 1000), (1024, 4096)])
+@pytest.mark.parametrize("gate", [(float("inf"), 0.0), (2.0, 0.5), (0.0, 0.0)])
+def test_cluster_list_bit_exact(tiny, torch, P, C, gate):
+    ix, orc = tiny["ix"], tiny["orc"]
+    ix.set_params(gate_m0=gate[0], gate_m1=gate[1])
+    try:
+        cl, ncl = ix.debug_clusters(tiny["dl"], P, C)
+    finally:
+        ix.set_params()
+    cl, ncl = cl.cpu().numpy(), ncl.cpu().numpy()
+    tau = orc.tau()
+    p = oracle.params(gate_m0=gate[0], gate_m1=gate[1])
+    for i in range(0, len(tiny["q"]), 5):
+        codes, _, _ = oracle.probe_list(tiny["lg"][i], tau, P, p)
+        L, _, _ = orc.cluster_list(tiny["lg"][i], codes, C, p)
+        assert ncl[i] == len(L), i
+        assert np.array_equal(cl[i, : len(L)], L), i
+        assert np.all(cl[i, len(L):] == -1)
+
+
+CASES = [dict(k=10, P=8, C=32), dict(k=10, P=128, C=256), dict(k=1, P=16, C=8),
+         dict(k=100, P=64, C=64), dict(k=256, P=32, C=512), dict(k=10, P=512, C=2048, t_low=0),
+         dict(k=10, P=64, C=128, round_size=32, t_low=1), dict(k=7, P=64, C=128, round_size=1024),
+         dict(k=10, P=64, C=128, round_size=64, t_low=2, u_min=3, f_min=2, alpha_front=0.7, r_min=3),
+         dict(k=10, P=64, C=64, gate_m0=1.0, gate_m1=0.25)]
+
+
+@pytest.mark.parametrize("case", CASES, ids=[str(i) for i in range(len(CASES))])
+def test_search_logits_bit_exact_u8(tiny, torch, case):
+    case = dict(case)
+    k, P, C = case.pop("k"), case.pop("P"), case.pop("C")
+    ix, orc = tiny["ix"], tiny["orc"]
+    ix.set_params(**case)
+    try:
+        ids, d = ix.search_logits(tiny["dq"], tiny["dl"], k, P, C)
+        st = ix.query_stats(len(tiny["q"]))
+        torch.cuda.synchronize()
+        tot = ix.last_stats()
+    finally:
+        ix.set_params()
+    ids_o, d_o, st_o = orc.search(tiny["q"], k, P, C, oracle.params(**case), logits=tiny["lg"])
+    assert np.array_equal(ids.cpu().numpy(), ids_o)
+    assert np.array_equal(d.cpu().numpy(), d_o)
+    assert np.array_equal(st.cpu().numpy(), st_o)
+    assert tot.candidates == st_o[:, 0].sum() and tot.nq == len(tiny["q"])
+
+
+@pytest.fixture(scope="module")
+def f32small(torch, tmp_path_factory):
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, base, info = build_small(tmp_path_factory.mktemp("f32"), "f32-10m", n=60000, bits=14,
+                                   k_max=8, t=32, name="f32")
+    w = synth.WORKLOADS["f32-10m"]
+    qs = synth.queries(w, 500)
+    orc = oracle.Index(path)
+    lg = orc.encode(qs)
+    return {"ix": nr.Index(path, 0), "orc": orc, "q": qs, "lg": lg, "base": base,
+            "dq": torch.from_numpy(qs).cuda(), "dl": torch.from_numpy(lg).cuda()}
+
+
+@pytest.mark.parametrize("k,P,C,extra", [(10, 8, 64, {}), (10, 32, 64, {}), (50, 128, 256, {"t_low": 0}),
+                                         (10, 64, 64, {"round_size": 128, "t_low": 2})])
+def test_search_logits_fp32(f32small, torch, k, P, C, extra):
+    ix, orc = f32small["ix"], f32small["orc"]
+    ix.set_params(**extra)
+    try:
+        ids, d = ix.search_logits(f32small["dq"], f32small["dl"], k, P, C)
+        torch.cuda.synchronize()
+    finally:
+        ix.set_params()
+    ids_o, d_o, _ = orc.search(f32small["q"], k, P, C, oracle.params(**extra), logits=f32small["lg"])
+    d = d.cpu().numpy()
+    fin = np.isfinite(d_o)
+    assert np.array_equal(np.isfinite(d), fin)
+    assert np.all(np.abs(d[fin] - d_o[fin]) <= 1e-5 * np.abs(d_o[fin]))
+    assert np.array_equal(ids.cpu().numpy(), ids_o)
+
+
+def test_encoder_logits_within_tolerance(tiny, f32small, torch):
+    for ctx in (tiny, f32small):
+        lg = ctx["ix"].encode(ctx["dq"]).cpu().numpy().astype(np.float64)
+        ref = ctx["lg"].astype(np.float64)
+        err = np.abs(lg - ref).max(1)
+        assert np.all(err <= 1e-2 * np.abs(ref).max(1))
+
+
+def test_end_to_end_recall_matches_oracle(tiny, torch):
+    from test_oracle_search import exact_knn
+
+    ix, orc = tiny["ix"], tiny["orc"]
+    gi, _ = exact_knn(tiny["base"], tiny["q"], 10)
+    for P, C in [(8, 32), (64, 128)]:
+        ids, _ = ix.search(tiny["dq"], 10, P, C)
+        ids_o, _, _ = orc.search(tiny["q"], 10, P, C, oracle.params())
+        r_g, r_o = recall(ids.cpu().numpy(), gi), recall(ids_o, gi)
+        assert abs(r_g - r_o) <= 0.002, (P, C, r_g, r_o)
+
+
+def test_host_buffers_equal_device_path(tiny, torch):
+    ix = tiny["ix"]
+    ids, d = ix.search(tiny["dq"], 10, 32, 64)
+    hq = torch.from_numpy(tiny["q"]).pin_memory()
+    hi, hd = ix.search_host(hq, 10, 32, 64)
+    assert torch.equal(hi, ids.cpu()) and torch.equal(hd, d.cpu())
+
+
+def test_empty_and_ragged_batches(tiny, torch):
+    ix, orc = tiny["ix"], tiny["orc"]
+    for nq in (0, 1, 3, 255, 257):
+        ids, d = ix.search_logits(tiny["dq"][:nq], tiny["dl"][:nq], 10, 16, 32)
+        ids_o, d_o, _ = orc.search(tiny["q"][:nq], 10, 16, 32, oracle.params(), logits=tiny["lg"][:nq])
+        assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
+
+
+def test_more_k_than_candidates_pads(tiny, torch):
+    ix, orc = tiny["ix"], tiny["orc"]
+    ids, d = ix.search_logits(tiny["dq"][:50], tiny["dl"][:50], 256, 1, 1)
+    ids_o, d_o, _ = orc.search(tiny["q"][:50], 256, 1, 1, oracle.params(), logits=tiny["lg"][:50])
+    ids = ids.cpu().numpy()
+    assert np.array_equal(ids, ids_o) and np.array_equal(d.cpu().numpy(), d_o)
+    assert (ids == -1).any()
+
+
+def test_invalid_arguments_are_rejected(tiny, torch):
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    ix = tiny["ix"]
+    for k, P, C in [(0, 8, 8), (257, 8, 8), (10, 0, 8), (10, 4097, 8), (10, 8, 0), (10, 8, 4097)]:
+        with pytest.raises(nr.NRError) as e:
+            ix.search(tiny["dq"][:4], k, P, C)
+        assert e.value.status == -1
+    with pytest.raises(nr.NRError):
+        ix.set_params(round_size=100)
+    with pytest.raises(nr.NRError):
+        ix.set_params(alpha_front=1.5)
+
+
+def test_malformed_files(torch, tmp_path):
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    with pytest.raises(nr.NRError) as e:
+        nr.Index(str(tmp_path / "missing.nrix"), 0)
+    assert e.value.status == -2
+    bkt = np.zeros(17, np.uint32)
+    bkt[1:] = 1
+    args = (np.zeros((1, 16), np.uint8), [0], bkt, [0, 1], np.zeros((1, 4)), np.zeros(4),
+            np.zeros((2, 16)), np.zeros(2), np.zeros((4, 2)), np.zeros(4))
+    path = str(tmp_path / "trunc.nrix")
+    write_nrix(path, *args, truncate_to=300)
+    with pytest.raises(nr.NRError) as e:
+        nr.Index(path, 0)
+    assert e.value.status == -3
+    path = str(tmp_path / "rows.nrix")  # a 4-byte row is not a multiple of 16 bytes
+    write_nrix(path, np.zeros((1, 4), np.uint8), *args[1:])
+    with pytest.raises(nr.NRError) as e:
+        nr.Index(path, 0)
+    assert e.value.status == -3
+
+
+def test_out_of_range_directory_is_flagged_not_faulted(torch, tmp_path):
+    """bkt_off pointing past the cluster table and a reversed cl_off range are
+    reported as NR_ERR_DEVICE_CHECK; the kernels skip the bad ranges."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    b = 3
+    bkt = np.array([0, 1, 3, 3, 9, 4, 4, 4, 4], np.uint32)  # code 3 -> [3, 9) past n_cl = 4
+    cl_off = np.array([0, 2, 1, 4, 5], np.uint32)           # cluster 1 reversed
+    vec = np.arange(5 * 16, dtype=np.uint8).reshape(5, 16)
+    path = str(tmp_path / "bad.nrix")
+    write_nrix(path, vec, np.arange(5), bkt, cl_off, np.zeros((4, b)), np.zeros(b),
+               np.zeros((2, 16)), np.zeros(2), np.zeros((b, 2)), np.zeros(b), K_max=8)
+    ix = nr.Index(path, 0)
+    q = torch.zeros((4, 16), dtype=torch.uint8, device="cuda")
+    lg = torch.tensor([[1, 1, -1], [-1, 1, -1], [1, -1, 1], [1, 1, 1]], dtype=torch.float32,
+                      device="cuda")
+    ids, d = ix.search_logits(q, lg, 5, 8, 8)
+    torch.cuda.synchronize()
+    with pytest.raises(nr.NRError) as e:
+        ix.last_stats()
+    assert e.value.status == -6
+    assert ix.last_stats().nq == 4  # the flag is cleared once reported
+    # the context is still usable and results are deterministic; clusters 0 and 2
+    # overlap in this file, so row 1 (id 1) is scored twice
+    ids2, _ = ix.search_logits(q, lg, 5, 8, 8)
+    torch.cuda.synchronize()
+    assert torch.equal(ids, ids2)
+    assert ids.cpu().tolist()[0] == [0, 1, 1, 2, 3]
