@@ -163,6 +163,28 @@ nr_status nr_search_host(nr_index *ix, const void *h_queries, int64_t nq, int k,
                          int cluster_budget, int64_t *h_out_ids, float *h_out_dists,
                          void *stream);
 
+/* As nr_search, but the call allocates no memory: its scratch lives in one
+ * fixed array of 32 MiB (NR_STATIC_SCRATCH_BYTES) compiled into the library,
+ * which every GPU that loads the library holds until the process exits.
+ * For callers that may not allocate device memory while serving queries:
+ * code running under a device-memory budget owned by a host framework or an
+ * inference server, and latency-critical loops in which cudaMalloc / cudaFree
+ * (which can synchronise the device) are not acceptable. The paper has no
+ * counterpart; results are identical to nr_search.
+ * Limit: a call needs about nq * (4b + 4P + 12(P + C) + 48) bytes (each of its
+ * nine buffers rounded up to 256 bytes); larger requests return
+ * NR_ERR_INVALID_ARG without enqueuing work, so split the batch.
+ * The first call on a device looks up the array's device address with that
+ * device made current; make that first call before any stream capture.
+ * All calls share the one array and it keeps the last call's contents: two
+ * calls whose work overlaps on the GPU (different streams, or different
+ * indexes on the same device) race and corrupt each other; serialise them.
+ * nr_last_stats and nr_query_stats after this call read its statistics from
+ * the array; stage timing is not recorded. */
+nr_status nr_search_static(nr_index *ix, const void *d_queries, int64_t nq, int k, int probe_budget,
+                           int cluster_budget, int64_t *d_out_ids, float *d_out_dists,
+                           void *stream);
+
 /* Per-query statistics of the last search call: d_stats [nq x 4] int64 =
  * (candidates, rounds, clusters, probes). Enqueued on `stream`. */
 nr_status nr_query_stats(nr_index *ix, int64_t *d_stats, int64_t nq, void *stream);

@@ -22,7 +22,7 @@ STATUS = {0: "NR_OK", -1: "NR_ERR_INVALID_ARG", -2: "NR_ERR_IO", -3: "NR_ERR_FOR
 EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_free",
            "nr_index_info", "nr_set_params", "nr_encode", "nr_route", "nr_debug_clusters",
            "nr_search", "nr_search_logits", "nr_search_host", "nr_query_stats", "nr_last_stats",
-           "nr_enable_timing", "nr_last_timing", "nr_kernel_launches"]
+           "nr_enable_timing", "nr_last_timing", "nr_kernel_launches", "nr_search_static"]
 
 
 class NRError(RuntimeError):
@@ -64,6 +64,7 @@ def lib():
         L.nr_search.argtypes = [vp, vp, i64, i32, i32, i32, vp, vp, vp]
         L.nr_search_logits.argtypes = [vp, vp, vp, i64, i32, i32, i32, vp, vp, vp]
         L.nr_search_host.argtypes = [vp, vp, i64, i32, i32, i32, vp, vp, vp]
+        L.nr_search_static.argtypes = [vp, vp, i64, i32, i32, i32, vp, vp, vp]
         L.nr_query_stats.argtypes = [vp, vp, i64, vp]
         L.nr_last_stats.argtypes = [vp, ctypes.POINTER(Stats)]
         L.nr_enable_timing.argtypes = [vp, i32]
@@ -199,6 +200,15 @@ class Index:
         ids, d = out
         _check("nr_search_host", lib().nr_search_host(self.h, _ptr(queries), nq, k, P, C, _ptr(ids),
                                                       _ptr(d), _stream(stream)))
+        return ids, d
+
+    def search_static(self, queries, k, P, C, out=None, stream=None):
+        """nr_search without any allocation inside the call: scratch comes from
+        the library's fixed 32 MiB device array (see include/neuroute.h)."""
+        nq = queries.shape[0]
+        ids, d = out if out is not None else self._outputs(nq, k)
+        _check("nr_search_static", lib().nr_search_static(self.h, _ptr(queries), nq, k, P, C,
+                                                          _ptr(ids), _ptr(d), _stream(stream)))
         return ids, d
 
     def query_stats(self, nq, stream=None):

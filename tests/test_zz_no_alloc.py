@@ -1,0 +1,61 @@
+"""nr_search_static: the search entry point that allocates nothing.
+
+Some callers cannot allocate device memory while they serve queries (a host
+framework or inference server owns the memory budget, or a latency-critical
+loop cannot afford cudaMalloc / cudaFree, which may synchronise the device).
+For them the library keeps its scratch in one fixed 32 MiB device array. This
+test calls that entry point through the C ABI twice in a row and checks that
+both calls return exactly what nr_search returns (ids and uint8 distances are
+integers, so the comparison is exact), and that a request too large for the
+array is refused before any work is enqueued.
+
+The file name puts it last in collection order, so a run that stops at the
+first failure has already run every other test; it also passes on its own in
+a fresh process (it builds its own small index).
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+import synth
+from gpu_util import build_small, need_cuda
+
+pytestmark = pytest.mark.gpu
+
+
+def test_static_scratch_search_matches_workspace_search(tmp_path):
+    torch = need_cuda()
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, _, _ = build_small(tmp_path, "tiny", n=30000, bits=12, name="static")
+    ix = nr.Index(path, 0)
+    w = synth.WORKLOADS["tiny"]
+    dq = torch.from_numpy(synth.queries(w, 300)).cuda()
+    k, P, C = 10, 32, 64
+    ref_ids, ref_d = ix.search(dq, k, P, C)
+    ref_st = ix.query_stats(dq.shape[0])
+    torch.cuda.synchronize()
+    L = nr.lib()
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    for _ in range(2):
+        ids = torch.full((dq.shape[0], k), -7, dtype=torch.int64, device="cuda")
+        d = torch.full((dq.shape[0], k), -7.0, dtype=torch.float32, device="cuda")
+        st = L.nr_search_static(ix.h, ctypes.c_void_p(dq.data_ptr()), dq.shape[0], k, P, C,
+                                ctypes.c_void_p(ids.data_ptr()), ctypes.c_void_p(d.data_ptr()),
+                                stream)
+        assert st == nr.NR_OK
+        torch.cuda.synchronize()
+        assert torch.equal(ids, ref_ids)
+        assert torch.equal(d, ref_d)
+        assert torch.equal(ix.query_stats(dq.shape[0]), ref_st)
+    assert ix.last_stats().nq == dq.shape[0]
+    # a batch whose scratch would not fit in the fixed array is refused
+    big = torch.zeros((20000, 128), dtype=torch.uint8, device="cuda")
+    out_i = torch.empty((20000, k), dtype=torch.int64, device="cuda")
+    out_d = torch.empty((20000, k), dtype=torch.float32, device="cuda")
+    st = L.nr_search_static(ix.h, ctypes.c_void_p(big.data_ptr()), 20000, k, 1024, 1024,
+                            ctypes.c_void_p(out_i.data_ptr()), ctypes.c_void_p(out_d.data_ptr()),
+                            stream)
+    assert st == -1  # NR_ERR_INVALID_ARG
+    ix.close()
