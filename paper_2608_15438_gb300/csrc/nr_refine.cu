@@ -64,65 +64,77 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
 }
 
-template <int DT, int TR, int STAGES>
+// CPR = 16-byte chunks per row when known at compile time (0: a.cpr)
+template <int DT, int TR, int STAGES, int CPR>
 __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int64_t RB = a.row_bytes;
-  unsigned char *stage_base = smem;                                        // STAGES x TR x RB
-  unsigned char *sq = smem + (size_t)STAGES * TR * RB;                     // RB (query)
-  uint32_t *srow = reinterpret_cast<uint32_t *>(sq + ((RB + 15) & ~15));   // STAGES x TR
-  uint64_t *hkey = reinterpret_cast<uint64_t *>(srow + STAGES * TR);       // 2 x kMaxK
-  int *htag = reinterpret_cast<int *>(hkey + 2 * kMaxK);                   // 2 x kMaxK
-  uint64_t *skey = reinterpret_cast<uint64_t *>(htag + 2 * kMaxK);         // TR survivors
-  int *sctl = reinterpret_cast<int *>(skey + TR);                          // control words
-  // sctl: 0 query, 1 survivors, 2 stop
+  const int cpr = CPR > 0 ? CPR : a.cpr;
+  const int swz = CPR > 0 ? ((CPR % 8 == 0) ? 7 : (CPR % 4 == 0) ? 3 : (CPR % 2 == 0) ? 1 : 0)
+                          : a.swz_mask;
+  const int64_t RB = (int64_t)cpr * 16;
+  unsigned char *stage_base = smem;                                       // STAGES x TR x RB
+  unsigned char *sq = smem + (size_t)STAGES * TR * RB;                    // RB (query)
+  uint32_t *srow = reinterpret_cast<uint32_t *>(sq + RB);                 // STAGES x TR
+  uint64_t *hkey = reinterpret_cast<uint64_t *>(srow + STAGES * TR);      // 2 x kMaxK
+  int *htag = reinterpret_cast<int *>(hkey + 2 * kMaxK);                  // 2 x kMaxK
+  uint64_t *skey = reinterpret_cast<uint64_t *>(htag + 2 * kMaxK);        // 2 x TR survivors
+  int *sctl = reinterpret_cast<int *>(skey + 2 * TR);                     // [0] query, [1..3] counters
   const uint32_t stage_s = (uint32_t)__cvta_generic_to_shared(stage_base);
   const int k = a.k;
   const int chunk = a.R < TR ? a.R : TR;
 
   for (;;) {
-    if (tid == 0) sctl[0] = (int)atomicAdd(a.counter, 1u);
+    if (tid == 0) {
+      sctl[0] = (int)atomicAdd(a.counter, 1u);
+      sctl[1] = sctl[2] = sctl[3] = 0;
+    }
     __syncthreads();
     const int64_t q = sctl[0];
     if (q >= a.nq) break;
-    // query row to shared memory
-    for (int c = tid; c < a.cpr; c += TR)
+    for (int c = tid; c < cpr; c += TR)
       reinterpret_cast<uint4 *>(sq)[c] = reinterpret_cast<const uint4 *>(a.q + q * RB)[c];
     const int64_t n = a.slen[q];
     const int nl = a.nL[q];
     const nr_seg *segs = a.seg + (size_t)q * a.Lmax;
     const int64_t ntiles = (n + TR - 1) / TR;
-    if (tid == 0) {
-      sctl[1] = 0;
-      sctl[2] = 0;
-    }
     __syncthreads();
+    uint4 qreg[DT == 0 && CPR > 0 && CPR <= 8 ? CPR : 1];
+    if (DT == 0 && CPR > 0 && CPR <= 8) {
+#pragma unroll
+      for (int c = 0; c < (CPR > 0 && CPR <= 8 ? CPR : 1); ++c) qreg[c] = reinterpret_cast<const uint4 *>(sq)[c];
+    }
 
-    // gather the rows of tile t into stage t % STAGES (each warp its own 32 rows)
+    // Gather the rows of tile t into stage t % STAGES. A warp copies and later
+    // reads only its own 32 rows, so stage reuse needs no block barrier.
+    int seg_i = 0;  // this thread's segment cursor (positions only grow)
     auto issue = [&](int64_t t) {
       if (t < ntiles) {
         const int st = (int)(t % STAGES);
         const int64_t p = t * TR + tid;
         uint32_t grow = 0;
         if (p < n) {
-          int lo = 0, hi = nl - 1;  // last segment starting at or before p
-          while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if ((int64_t)__ldg(&segs[mid].pos) <= p) lo = mid; else hi = mid - 1;
+          // last segment starting at or before p: exponential search from the cursor
+          int step = 1;
+          while (seg_i + step < nl && (int64_t)__ldg(&segs[seg_i + step].pos) <= p) {
+            seg_i += step;
+            step <<= 1;
           }
-          grow = __ldg(&segs[lo].row0) + (uint32_t)(p - (int64_t)__ldg(&segs[lo].pos));
+          for (step >>= 1; step > 0; step >>= 1)
+            if (seg_i + step < nl && (int64_t)__ldg(&segs[seg_i + step].pos) <= p) seg_i += step;
+          grow = __ldg(&segs[seg_i].row0) + (uint32_t)(p - (int64_t)__ldg(&segs[seg_i].pos));
           srow[st * TR + tid] = grow;
         }
         const int64_t wbase = t * TR + warp * 32;
         const uint32_t sbase = stage_s + (uint32_t)((size_t)st * TR * RB);
-        for (int f = lane; f < 32 * a.cpr; f += 32) {
-          const int rr = f / a.cpr;
-          const int c = f - rr * a.cpr;
+#pragma unroll 4
+        for (int f = lane; f < 32 * cpr; f += 32) {
+          const int rr = f / cpr;
+          const int c = f - rr * cpr;
           const uint32_t gr = __shfl_sync(kFull, grow, rr);
           if (wbase + rr < n) {
             const int r = warp * 32 + rr;
-            const uint32_t dst = sbase + (uint32_t)(r * RB) + (uint32_t)(((c ^ (r & a.swz_mask))) << 4);
+            const uint32_t dst = sbase + (uint32_t)(r * RB) + (uint32_t)((c ^ (r & swz)) << 4);
             cp_async16(dst, a.vec + (size_t)gr * RB + ((size_t)c << 4));
           }
         }
@@ -131,7 +143,7 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
     };
 
     for (int s = 0; s < STAGES - 1; ++s) issue(s);
-    int cur = 0, hn = 0, rounds = 0, low = 0;
+    int cur = 0, hn = 0, rounds = 0, low = 0, ci = 0;
     bool stop = false;
     int64_t done = 0;  // stream positions consumed in completed rounds
     for (int64_t t = 0; t < ntiles && !stop; ++t) {
@@ -144,23 +156,25 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
       if (p < n) {
         const unsigned char *row = stage_base + (size_t)st * TR * RB + (size_t)tid * RB;
         if (DT == 0) {
-          unsigned acc = 0;
+          unsigned a0 = 0, a1 = 0, a2 = 0, a3 = 0;  // integer sums: any order is exact
 #pragma unroll 8
-          for (int c = 0; c < a.cpr; ++c) {
-            const uint4 v = *reinterpret_cast<const uint4 *>(row + ((c ^ (tid & a.swz_mask)) << 4));
-            const uint4 w = reinterpret_cast<const uint4 *>(sq)[c];
+          for (int c = 0; c < cpr; ++c) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(row + ((c ^ (tid & swz)) << 4));
+            uint4 w;
+            if (CPR > 0 && CPR <= 8) w = qreg[c < (CPR > 0 && CPR <= 8 ? CPR : 1) ? c : 0];
+            else w = reinterpret_cast<const uint4 *>(sq)[c];
             unsigned d;
-            d = __vabsdiffu4(v.x, w.x); acc = __dp4a(d, d, acc);
-            d = __vabsdiffu4(v.y, w.y); acc = __dp4a(d, d, acc);
-            d = __vabsdiffu4(v.z, w.z); acc = __dp4a(d, d, acc);
-            d = __vabsdiffu4(v.w, w.w); acc = __dp4a(d, d, acc);
+            d = __vabsdiffu4(v.x, w.x); a0 = __dp4a(d, d, a0);
+            d = __vabsdiffu4(v.y, w.y); a1 = __dp4a(d, d, a1);
+            d = __vabsdiffu4(v.z, w.z); a2 = __dp4a(d, d, a2);
+            d = __vabsdiffu4(v.w, w.w); a3 = __dp4a(d, d, a3);
           }
-          dkey = acc;
+          dkey = (a0 + a1) + (a2 + a3);
         } else {
-          float acc = 0.0f;
+          float acc = 0.0f;  // sequential over j: the order fixes the rounding
 #pragma unroll 4
-          for (int c = 0; c < a.cpr; ++c) {
-            const float4 v = *reinterpret_cast<const float4 *>(row + ((c ^ (tid & a.swz_mask)) << 4));
+          for (int c = 0; c < cpr; ++c) {
+            const float4 v = *reinterpret_cast<const float4 *>(row + ((c ^ (tid & swz)) << 4));
             const float4 w = reinterpret_cast<const float4 *>(sq)[c];
             float d;
             d = __fsub_rn(v.x, w.x); acc = __fmaf_rn(d, d, acc);
@@ -171,19 +185,25 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
           dkey = __float_as_uint(acc);
         }
       }
-      // merge chunk by chunk; a round ends every R stream positions
-      for (int cs = 0; cs < TR && !stop; cs += chunk) {
+      // Merge chunk by chunk; a round ends every R stream positions. One block
+      // barrier per chunk (two when the top-k changes): survivor counters
+      // rotate over three slots and survivor buffers over two, and every warp
+      // evaluates the stop rule itself from the shared top-k.
+      for (int cs = 0; cs < TR && !stop; cs += chunk, ++ci) {
         const int64_t cstart = t * TR + cs;
         if (cstart >= n) break;
+        int *cnt = &sctl[1 + ci % 3];
+        uint64_t *sk_buf = skey + (ci & 1) * TR;
         const uint64_t thr = hn == k ? hkey[cur * kMaxK + k - 1] : kMaxKey;
         const uint32_t thr_hi = (uint32_t)(thr >> 32);
         if (tid >= cs && tid < cs + chunk && p < n && dkey <= thr_hi) {
           const uint32_t id = __ldg(&a.ids[srow[st * TR + tid]]);
           const uint64_t key = ((uint64_t)dkey << 32) | id;
-          if (key < thr) skey[atomicAdd(&sctl[1], 1)] = key;
+          if (key < thr) sk_buf[atomicAdd(cnt, 1)] = key;
         }
+        if (tid == 0) sctl[1 + (ci + 1) % 3] = 0;  // counter of the next chunk
         __syncthreads();
-        const int ns = sctl[1];
+        const int ns = *cnt;
         const int roundno = rounds + 1;
         if (ns > 0) {
           const int nxt = cur ^ 1;
@@ -191,14 +211,14 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
           // merged order: by key; on equal keys (possible only when an index
           // stores a row twice) H before S, and S by slot, so ranks are unique
           for (int i = tid; i < ns; i += TR) {
-            const uint64_t sk = skey[i];
+            const uint64_t sk = sk_buf[i];
             int lo = 0, hi = hn;  // # of H at or below sk
             while (lo < hi) {
               const int mid = (lo + hi) >> 1;
               if (H[mid] <= sk) lo = mid + 1; else hi = mid;
             }
             int r = lo;
-            for (int j = 0; j < ns; ++j) r += (skey[j] < sk || (skey[j] == sk && j < i)) ? 1 : 0;
+            for (int j = 0; j < ns; ++j) r += (sk_buf[j] < sk || (sk_buf[j] == sk && j < i)) ? 1 : 0;
             if (r < k) {
               hkey[nxt * kMaxK + r] = sk;
               htag[nxt * kMaxK + r] = roundno;
@@ -207,7 +227,7 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
           for (int j = tid; j < hn; j += TR) {
             const uint64_t hk = H[j];
             int r = j;
-            for (int i = 0; i < ns; ++i) r += skey[i] < hk ? 1 : 0;
+            for (int i = 0; i < ns; ++i) r += sk_buf[i] < hk ? 1 : 0;
             if (r < k) {
               hkey[nxt * kMaxK + r] = hk;
               htag[nxt * kMaxK + r] = htag[cur * kMaxK + j];
@@ -216,33 +236,25 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
           __syncthreads();
           cur = nxt;
           hn = hn + ns < k ? hn + ns : k;
-          if (tid == 0) sctl[1] = 0;
         }
         const int64_t cend = cstart + chunk < n ? cstart + chunk : n;
         if ((cend % a.R) == 0 || cend >= n) {  // round complete
           rounds = roundno;
           done = cend;
-          if (warp == 0) {
-            int newc = 0, frontc = 0;
-            for (int i = lane; i < hn; i += 32) {
-              const bool nw = htag[cur * kMaxK + i] == roundno;
-              newc += nw ? 1 : 0;
-              frontc += (nw && i < a.nfront) ? 1 : 0;
-            }
-            for (int o = 16; o > 0; o >>= 1) {
-              newc += __shfl_xor_sync(kFull, newc, o);
-              frontc += __shfl_xor_sync(kFull, frontc, o);
-            }
-            const bool lowq = newc < a.u_min && frontc < a.f_min;
-            const int nlow = lowq ? low + 1 : 0;
-            if (lane == 0)
-              sctl[2] = (a.t_low > 0 && hn == k && roundno >= a.r_min && nlow >= a.t_low) ? 1 : 0;
-            low = nlow;
+          int newc = 0, frontc = 0;
+          for (int i = lane; i < hn; i += 32) {
+            const bool nw = htag[cur * kMaxK + i] == roundno;
+            newc += nw ? 1 : 0;
+            frontc += (nw && i < a.nfront) ? 1 : 0;
           }
-          __syncthreads();  // only warp 0 tracks `low`; everyone reads the decision
-          stop = sctl[2] != 0;
+          for (int o = 16; o > 0; o >>= 1) {
+            newc += __shfl_xor_sync(kFull, newc, o);
+            frontc += __shfl_xor_sync(kFull, frontc, o);
+          }
+          const bool lowq = newc < a.u_min && frontc < a.f_min;
+          low = lowq ? low + 1 : 0;
+          stop = a.t_low > 0 && hn == k && roundno >= a.r_min && low >= a.t_low;
         }
-        __syncthreads();
       }
     }
     cp_async_wait<0>();
@@ -269,11 +281,11 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
   }
 }
 
-template <int DT, int TR, int STAGES>
+template <int DT, int TR, int STAGES, int CPR>
 cudaError_t launch(nr_index *ix, const RefineArgs &a, cudaStream_t s) {
-  const size_t smem = (size_t)STAGES * TR * a.row_bytes + ((a.row_bytes + 15) & ~15) +
-                      (size_t)STAGES * TR * 4 + 2 * kMaxK * 8 + 2 * kMaxK * 4 + (size_t)TR * 8 + 16;
-  auto kern = refine_kernel<DT, TR, STAGES>;
+  const size_t smem = (size_t)STAGES * TR * a.row_bytes + (size_t)a.row_bytes +
+                      (size_t)STAGES * TR * 4 + 2 * kMaxK * 8 + 2 * kMaxK * 4 + (size_t)2 * TR * 8 + 32;
+  auto kern = refine_kernel<DT, TR, STAGES, CPR>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   int per_sm = 0;
@@ -326,11 +338,13 @@ cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, i
   cudaError_t e = cudaMemsetAsync(d_counter, 0, sizeof(unsigned int), s);
   if (e != cudaSuccess) return e;
   if (ix->dtype == 0) {
-    if (ix->row_bytes <= 256) return launch<0, 256, 3>(ix, a, s);
-    if (ix->row_bytes <= 512) return launch<0, 128, 3>(ix, a, s);
-    return launch<0, 64, 3>(ix, a, s);
+    if (a.cpr == 8) return launch<0, 256, 3, 8>(ix, a, s);  // uint8, D = 128
+    if (ix->row_bytes <= 256) return launch<0, 256, 3, 0>(ix, a, s);
+    if (ix->row_bytes <= 512) return launch<0, 128, 3, 0>(ix, a, s);
+    return launch<0, 64, 3, 0>(ix, a, s);
   }
-  if (ix->row_bytes <= 384) return launch<1, 256, 2>(ix, a, s);
-  if (ix->row_bytes <= 768) return launch<1, 128, 2>(ix, a, s);
-  return launch<1, 64, 2>(ix, a, s);
+  if (a.cpr == 24) return launch<1, 256, 2, 24>(ix, a, s);  // fp32, D = 96
+  if (ix->row_bytes <= 384) return launch<1, 256, 2, 0>(ix, a, s);
+  if (ix->row_bytes <= 768) return launch<1, 128, 2, 0>(ix, a, s);
+  return launch<1, 64, 2, 0>(ix, a, s);
 }
