@@ -1,5 +1,6 @@
 // C ABI of the query path: index loading, argument checks, workspace and the
 // launch sequence encode -> route -> select -> refine (see neuroute.h).
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -167,7 +168,7 @@ void nr_index_free(nr_index *ix) {
     cudaEventDestroy(t.a);
     cudaEventDestroy(t.b);
   }
-  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->bkt_off,
+  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
                   ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->single, e->io};
   for (void *p : ptrs)
     if (p) cudaFree(p);
@@ -283,6 +284,16 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   if ((st = up((void **)&ix->b2, b2.data(), sz[3])) != NR_OK) return bad(st);
   if ((st = up((void **)&ix->tau, tau.data(), sz[4])) != NR_OK) return bad(st);
   if ((st = up((void **)&ix->W1T, W1T.data(), sz[0])) != NR_OK) return bad(st);
+  {
+    // fp16 operands of the tensor-core encoder; layer 2 padded to 16 or 32 rows
+    const int n2 = ix->b <= 16 ? 16 : 32;
+    std::vector<__half> w1h((size_t)ix->H * ix->D), w2h((size_t)n2 * ix->H, __float2half_rn(0.0f));
+    for (size_t i = 0; i < w1h.size(); ++i) w1h[i] = __float2half_rn(W1[i]);
+    for (int o = 0; o < ix->b; ++o)
+      for (int u = 0; u < ix->H; ++u) w2h[(size_t)o * ix->H + u] = __float2half_rn(W2[(size_t)o * ix->H + u]);
+    if ((st = up(&ix->W1h, w1h.data(), w1h.size() * 2)) != NR_OK) return bad(st);
+    if ((st = up(&ix->W2h, w2h.data(), w2h.size() * 2)) != NR_OK) return bad(st);
+  }
   if ((st = up((void **)&ix->bkt_off, bkt.data(), sz[5])) != NR_OK) return bad(st);
   if ((st = up((void **)&ext_of(ix)->single, single.data(), single.size())) != NR_OK) return bad(st);
   if ((st = up((void **)&ix->d_err, nullptr, 16)) != NR_OK) return bad(st);

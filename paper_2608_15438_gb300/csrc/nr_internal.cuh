@@ -12,7 +12,8 @@ enum : int {
   NR_DEV_BAD_BUCKET = 1,   // bkt_off range reversed or past n_clusters
   NR_DEV_BAD_CLUSTER = 2,  // cl_off range reversed or past N
   NR_DEV_TOO_MANY = 3,     // a bucket holds more than K_max clusters
-  NR_DEV_BAD_CODE = 4      // a probe code >= 2^b
+  NR_DEV_BAD_CODE = 4,     // a probe code >= 2^b
+  NR_DEV_TIMEOUT = 5       // a bounded wait on an MMA completion barrier expired
 };
 
 struct nr_index {
@@ -27,6 +28,8 @@ struct nr_index {
   float *W1 = nullptr, *b1 = nullptr, *W2 = nullptr, *b2 = nullptr, *tau = nullptr;
   float *cent = nullptr;
   float *W1T = nullptr;  // [D][H]
+  void *W1h = nullptr;   // fp16 [H][D] (tensor-core encoder)
+  void *W2h = nullptr;   // fp16 [16 or 32][H], rows >= b zero
   uint32_t *bkt_off = nullptr, *cl_off = nullptr, *ids = nullptr;
   void *vec = nullptr;
   int *d_err = nullptr;
@@ -51,6 +54,7 @@ struct nr_seg {
 };
 
 // kernel launchers (each returns cudaGetLastError() after the launch)
+bool nr_encode_uses_tensor_cores(const nr_index *ix);
 cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
                              cudaStream_t s);
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
