@@ -1,8 +1,7 @@
 // K2 route: binarisation (Eq. 10), deviation scores (Sec. 3.2.3) and the
 // probe list of Algorithm 1 as an exact best-first enumeration of flip sets.
 //
-// One warp per query. Lane j holds bit j. Ranks order the bits by
-// (delta_j, j); a flip set F is a set of ranks with key
+// Ranks order the bits by (delta_j, j); a flip set F is a set of ranks with key
 //   (cost(F), |F|, rank mask),  cost = fp32 sum of delta over F, ascending rank.
 // Flip sets form a tree rooted at {0}: a set whose largest rank is m has the
 // children "shift" (m -> m+1) and "expand" (add m+1). Every child's key is
@@ -11,10 +10,6 @@
 // first P sets in key order, the empty set (the base bucket) first. Costs are
 // carried as (cost, cost without the largest rank), so each child's cost is
 // one addition in the same left-to-right order a sequential sum would use.
-//
-// The frontier lives in shared memory; slot s belongs to lane s % 32, which
-// keeps the minimum of its own slots in registers. A pop is two warp
-// min-reductions, a ballot and one rescan by the owning lane.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -24,140 +19,201 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr uint64_t kEmpty = ~0ull;
+constexpr int kGroup = 8;             // lanes per query
+constexpr int kQPW = 32 / kGroup;     // queries per warp
 
 __device__ __forceinline__ uint64_t pack_key(float cost, uint32_t size, uint32_t mask) {
   return ((uint64_t)__float_as_uint(cost) << 32) | ((uint64_t)size << 24) | (uint64_t)mask;
 }
 
-__global__ void route_kernel(const float *__restrict__ logits, const float *__restrict__ tau, int b,
-                             int bsel, int rmax, float smax, int64_t nq, int P, int cap,
-                             uint32_t *__restrict__ codes, int32_t *__restrict__ nprobe) {
+__device__ __forceinline__ uint64_t shfl_xor64(uint64_t v, int o) {
+  const uint32_t lo = __shfl_xor_sync(kFull, (uint32_t)v, o, kGroup);
+  const uint32_t hi = __shfl_xor_sync(kFull, (uint32_t)(v >> 32), o, kGroup);
+  return ((uint64_t)hi << 32) | lo;
+}
+
+// One 8-lane group per query, four queries per warp. Lane gl of a group holds
+// bits gl, gl + 8, gl + 16. The frontier is an 8-ary min-heap of
+// (key, prefix cost) in shared memory: a pop that also inserts the shift child
+// is one sift-down (the 8 lanes compare the 8 children of a node at once); the
+// expand child is a sift-up by the group leader. The frontier never holds more
+// than P + 1 entries.
+__global__ void route_heap_kernel(const float *__restrict__ logits, const float *__restrict__ tau,
+                                  int b, int bsel, int rmax, float smax, int64_t nq, int P, int cap,
+                                  uint32_t *__restrict__ codes, int32_t *__restrict__ nprobe) {
   extern __shared__ __align__(16) unsigned char smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
-  const int64_t q = (int64_t)blockIdx.x * wpb + warp;
-  if (q >= nq) return;  // uniform per warp
-  uint64_t *skey = reinterpret_cast<uint64_t *>(smem) + (size_t)warp * cap;
-  float *scostp = reinterpret_cast<float *>(smem + (size_t)wpb * cap * 8) + (size_t)warp * cap;
-  float *ssd = reinterpret_cast<float *>(smem + (size_t)wpb * cap * 12) + warp * 32;
-  int *spi = reinterpret_cast<int *>(smem + (size_t)wpb * cap * 12 + (size_t)wpb * 128) + warp * 32;
+  const int g = lane / kGroup, gl = lane % kGroup;
+  const int slot = warp * kQPW + g;                 // group slot within the block
+  const int nslot = wpb * kQPW;
+  const int64_t q = ((int64_t)blockIdx.x * wpb + warp) * kQPW + g;
+  const bool live = q < nq;
+  uint64_t *hkey = reinterpret_cast<uint64_t *>(smem) + (size_t)slot * cap;
+  float *hcp = reinterpret_cast<float *>(smem + (size_t)nslot * cap * 8) + (size_t)slot * cap;
+  float *ssd = reinterpret_cast<float *>(smem + (size_t)nslot * cap * 12) + slot * 32;
+  int *spi = reinterpret_cast<int *>(smem + (size_t)nslot * cap * 12 + (size_t)nslot * 128) + slot * 32;
 
-  // Eq. 10: bit j set iff l_j >= tau_j; deviation delta_j = |l_j - tau_j|
-  float dj = __int_as_float(0x7f800000);
-  bool bit = false;
-  if (lane < b) {
-    const float l = logits[q * b + lane];
-    const float tj = tau[lane];
-    bit = l >= tj;
-    dj = fabsf(__fsub_rn(l, tj));
+  // Eq. 10 and the deviations of this lane's three bits
+  float dj[3];
+  uint32_t mybits = 0;
+#pragma unroll
+  for (int t = 0; t < 3; ++t) {
+    const int j = gl + kGroup * t;
+    dj[t] = __int_as_float(0x7f800000);
+    if (live && j < b) {
+      const float l = logits[q * b + j];
+      const float tj = tau[j];
+      if (l >= tj) mybits |= 1u << j;
+      dj[t] = fabsf(__fsub_rn(l, tj));
+    }
   }
-  const uint32_t u0 = __ballot_sync(kFull, bit);
-  // rank of bit `lane` by (delta, bit index)
-  int rank = 0;
+  uint32_t u0 = mybits;
+#pragma unroll
+  for (int o = 1; o < kGroup; o <<= 1) u0 |= __shfl_xor_sync(kFull, u0, o, kGroup);
+  // ranks by (delta, bit index)
+  int rank[3] = {0, 0, 0};
   for (int i = 0; i < b; ++i) {
-    const float di = __shfl_sync(kFull, dj, i);
-    if (di < dj || (di == dj && i < lane)) ++rank;
-  }
-  if (lane < b) {
-    ssd[rank] = dj;
-    spi[rank] = lane;
-  }
-  __syncwarp();
-  const float sd = lane < b ? ssd[lane] : 0.0f;  // delta of rank `lane`
-  const int pi = lane < b ? spi[lane] : 0;        // bit index of rank `lane`
-
-  uint32_t *out = codes + (size_t)q * P;
-  if (lane == 0) out[0] = u0;
-  int n = 1;
-  int nslots = 0;
-  uint32_t my_hi = 0xffffffffu, my_lo = 0xffffffffu;
-  int my_slot = -1;
-
-  const float sd0 = __shfl_sync(kFull, sd, 0);
-  if (P > 1 && bsel >= 1 && sd0 <= smax) {
-    if (lane == 0) {
-      const uint64_t key = pack_key(sd0, 1u, 1u);
-      skey[0] = key;
-      scostp[0] = 0.0f;
-      my_hi = (uint32_t)(key >> 32);
-      my_lo = (uint32_t)key;
-      my_slot = 0;
+    const float di = __shfl_sync(kFull, dj[i / kGroup], i % kGroup, kGroup);
+#pragma unroll
+    for (int t = 0; t < 3; ++t) {
+      const int j = gl + kGroup * t;
+      if (di < dj[t] || (di == dj[t] && i < j)) ++rank[t];
     }
-    nslots = 1;
+  }
+#pragma unroll
+  for (int t = 0; t < 3; ++t) {
+    const int j = gl + kGroup * t;
+    if (live && j < b) {
+      ssd[rank[t]] = dj[t];
+      spi[rank[t]] = j;
+    }
   }
   __syncwarp();
 
-  while (n < P) {
-    const uint32_t hmin = __reduce_min_sync(kFull, my_hi);
-    const uint32_t lmin = __reduce_min_sync(kFull, my_hi == hmin ? my_lo : 0xffffffffu);
-    if (hmin == 0xffffffffu && lmin == 0xffffffffu) break;  // frontier empty
-    const unsigned own = __ballot_sync(kFull, my_slot >= 0 && my_hi == hmin && my_lo == lmin);
-    const int owner = __ffs(own) - 1;
-    const int slot = __shfl_sync(kFull, my_slot, owner);
-    const float costp = scostp[slot];
-    const uint32_t rmask = lmin & 0xffffffu;
-    const uint32_t size = lmin >> 24;
-    const float cost = __uint_as_float(hmin);
-    // ApplyFlips: code = u0 XOR (bits of the ranks in F)
-    const uint32_t flips =
-        __reduce_or_sync(kFull, (lane < b && ((rmask >> lane) & 1u)) ? (1u << pi) : 0u);
-    if (lane == 0) out[n] = u0 ^ flips;
-    ++n;
-    __syncwarp();
-    if (lane == owner) {
-      skey[slot] = kEmpty;
-      uint64_t best = kEmpty;
-      int bs = -1;
-      for (int s = lane; s < nslots; s += 32) {
-        const uint64_t kk = skey[s];
-        if (kk < best) {
-          best = kk;
-          bs = s;
-        }
-      }
-      my_hi = (uint32_t)(best >> 32);
-      my_lo = (uint32_t)best;
-      my_slot = bs;
+  uint32_t *out = codes + (size_t)(live ? q : 0) * P;
+  if (live && gl == 0) out[0] = u0;
+  int n = 1, hs = 0;
+  if (live && P > 1 && bsel >= 1 && ssd[0] <= smax) {
+    if (gl == 0) {
+      hkey[0] = pack_key(ssd[0], 1u, 1u);
+      hcp[0] = 0.0f;
     }
-    const int m = 31 - __clz((int)rmask);  // largest rank in F
-    if (m + 1 < bsel) {
-      const float sdn = __shfl_sync(kFull, sd, m + 1);
-      // shift: replace rank m by m + 1
-      const float c1 = __fadd_rn(costp, sdn);
-      if (c1 <= smax) {
-        const int s = nslots++;
-        if (lane == (s & 31)) {
-          const uint64_t key = pack_key(c1, size, rmask + (1u << m));
-          skey[s] = key;
-          scostp[s] = costp;
-          if (key < (((uint64_t)my_hi << 32) | my_lo)) {
-            my_hi = (uint32_t)(key >> 32);
-            my_lo = (uint32_t)key;
-            my_slot = s;
-          }
-        }
-      }
-      // expand: add rank m + 1
-      if (rmax <= 0 || (int)size < rmax) {
-        const float c2 = __fadd_rn(cost, sdn);
-        if (c2 <= smax) {
-          const int s = nslots++;
-          if (lane == (s & 31)) {
-            const uint64_t key = pack_key(c2, size + 1, rmask | (1u << (m + 1)));
-            skey[s] = key;
-            scostp[s] = cost;
-            if (key < (((uint64_t)my_hi << 32) | my_lo)) {
-              my_hi = (uint32_t)(key >> 32);
-              my_lo = (uint32_t)key;
-              my_slot = s;
-            }
-          }
-        }
-      }
-    }
-    __syncwarp();
+    hs = 1;
   }
-  for (int i = n + lane; i < P; i += 32) out[i] = 0xffffffffu;
-  if (lane == 0) nprobe[q] = n;
+  __syncwarp();
+  bool active = live && n < P && hs > 0;
+  while (__any_sync(kFull, active)) {
+    uint64_t top = kEmpty, x = kEmpty, c2key = kEmpty;
+    float topcp = 0.0f, xcp = 0.0f, c2cp = 0.0f;
+    bool push2 = false;
+    if (active) {
+      top = hkey[0];
+      topcp = hcp[0];
+      const uint32_t rmask = (uint32_t)top & 0xffffffu;
+      const uint32_t size = ((uint32_t)top >> 24) & 0xffu;
+      const float cost = __uint_as_float((uint32_t)(top >> 32));
+      if (gl == 0) {  // ApplyFlips
+        uint32_t f = 0, mm = rmask;
+        while (mm) {
+          const int r = __ffs(mm) - 1;
+          f |= 1u << spi[r];
+          mm &= mm - 1;
+        }
+        out[n] = u0 ^ f;
+      }
+      ++n;
+      const int m = 31 - __clz((int)rmask);
+      bool v1 = false, v2 = false;
+      uint64_t k1 = kEmpty, k2 = kEmpty;
+      float cp1 = 0.0f, cp2 = 0.0f;
+      if (m + 1 < bsel) {
+        const float sdn = ssd[m + 1];
+        const float c1 = __fadd_rn(topcp, sdn);  // shift: rank m -> m + 1
+        if (c1 <= smax) {
+          v1 = true;
+          k1 = pack_key(c1, size, rmask + (1u << m));
+          cp1 = topcp;
+        }
+        if (rmax <= 0 || (int)size < rmax) {  // expand: add rank m + 1
+          const float c2 = __fadd_rn(cost, sdn);
+          if (c2 <= smax) {
+            v2 = true;
+            k2 = pack_key(c2, size + 1, rmask | (1u << (m + 1)));
+            cp2 = cost;
+          }
+        }
+      }
+      // the root is replaced by a child, or by the last entry
+      if (v1) {
+        x = k1; xcp = cp1;
+        if (v2) { push2 = true; c2key = k2; c2cp = cp2; }
+      } else if (v2) {
+        x = k2; xcp = cp2;
+      } else {
+        hs -= 1;
+        if (hs > 0) { x = hkey[hs]; xcp = hcp[hs]; }
+      }
+    }
+    __syncwarp();
+    // sift-down of x from the root (groups with nothing to place idle along)
+    int i = 0;
+    bool sifting = active && x != kEmpty;
+    while (__any_sync(kFull, sifting)) {
+      uint64_t ck = kEmpty;
+      int ci = -1;
+      if (sifting) {
+        const int c = kGroup * i + 1 + gl;
+        if (c < hs) { ck = hkey[c]; ci = c; }
+      }
+      // group minimum over the 8 children (keys are unique)
+      uint64_t mk = ck;
+#pragma unroll
+      for (int o = 1; o < kGroup; o <<= 1) {
+        const uint64_t ok = shfl_xor64(mk, o);
+        mk = ok < mk ? ok : mk;
+      }
+      const unsigned who = __ballot_sync(kFull, sifting && ck == mk && ci >= 0);
+      const int src = __ffs((who >> (g * kGroup)) & 0xffu) - 1;  // lane in group holding the min
+      const int mci = __shfl_sync(kFull, ci, src < 0 ? 0 : src, kGroup);
+      if (sifting) {
+        if (src >= 0 && mk < x) {
+          if (gl == 0) {
+            hkey[i] = mk;
+            hcp[i] = hcp[mci];
+          }
+          i = mci;
+        } else {
+          if (gl == 0) {
+            hkey[i] = x;
+            hcp[i] = xcp;
+          }
+          sifting = false;
+        }
+      }
+      __syncwarp();
+    }
+    // sift-up of the expand child
+    if (push2 && gl == 0) {
+      int j = hs;
+      while (j > 0) {
+        const int pj = (j - 1) / kGroup;
+        const uint64_t pk = hkey[pj];
+        if (pk < c2key) break;
+        hkey[j] = pk;
+        hcp[j] = hcp[pj];
+        j = pj;
+      }
+      hkey[j] = c2key;
+      hcp[j] = c2cp;
+    }
+    if (push2) hs += 1;
+    __syncwarp();
+    active = active && n < P && hs > 0;
+  }
+  if (live) {
+    for (int t = n + gl; t < P; t += kGroup) out[t] = 0xffffffffu;
+    if (gl == 0) nprobe[q] = n;
+  }
 }
 
 }  // namespace
@@ -165,20 +221,21 @@ __global__ void route_kernel(const float *__restrict__ logits, const float *__re
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
-  const int cap = 2 * P;
-  const size_t per_warp = (size_t)cap * 12 + 256;
-  int wpb = (int)((96u * 1024u) / per_warp);
-  if (wpb > 8) wpb = 8;
+  const int cap = P + 2;
+  const size_t per_group = (size_t)cap * 12 + 256;
+  int wpb = (int)((96u * 1024u) / (per_group * kQPW));
+  if (wpb > 4) wpb = 4;
   if (wpb < 1) wpb = 1;
-  const size_t smem = per_warp * (size_t)wpb;
-  cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const size_t smem = per_group * (size_t)(wpb * kQPW);
+  cudaError_t e = cudaFuncSetAttribute(route_heap_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   const nr_params &p = ix->params;
   const int bsel = (p.l_sel > 0 && p.l_sel < ix->b) ? p.l_sel : ix->b;
-  const int64_t grid = (nq + wpb - 1) / wpb;
-  route_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(d_logits, ix->tau, ix->b, bsel, p.r_max,
-                                                       p.s_max, nq, P, cap, d_codes, d_nprobe);
+  const int64_t qpb = (int64_t)wpb * kQPW;
+  const int64_t grid = (nq + qpb - 1) / qpb;
+  route_heap_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(d_logits, ix->tau, ix->b, bsel, p.r_max,
+                                                            p.s_max, nq, P, cap, d_codes, d_nprobe);
   ix->launches += 1;
   return cudaGetLastError();
 }
