@@ -29,11 +29,13 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+METRIC = "QPS at Recall@10~0.90 (batched query path); refine-scan HBM GB/s"
+
 # operating points (P, C, t_low) with Recall@10 in [0.88, 0.92], from `--sweep`
 OPERATING_POINTS = {
     "tiny": (128, 256, 4),
     "u8-10m": (256, 256, 64),
-    "f32-10m": (256, 512, 4),
+    "f32-10m": (512, 256, 16),
 }
 
 
@@ -247,7 +249,7 @@ def run_reference(args, w, rank, world):
         times.append(time.perf_counter() - t)
     tot = sum(times)
     v = ns * args.steps / tot
-    line = {"impl": "reference", "metric": "QPS at Recall@10~0.90 (batched query path)", "value": v,
+    line = {"impl": "reference", "metric": METRIC, "value": v,
             "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
@@ -398,7 +400,7 @@ def main():
     peaks, peak_src = measured_peaks()
     traffic = traffic_from_profile(w.name, P, C)
     out = {
-        "metric": "QPS at Recall@10~0.90 (batched query path); refine-scan HBM GB/s",
+        "metric": METRIC,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
         "warmup": max(3, args.warmup), "ms_per_step": tot_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

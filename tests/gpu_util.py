@@ -35,3 +35,24 @@ def recall(found, truth, k=10):
         f = set(int(v) for v in f[:k] if v >= 0)
         r.append(len(f & g) / min(k, len(g)) if g else 1.0)
     return float(np.mean(r))
+
+
+def cached_index(workload_name, tmp_root="/tmp"):
+    """Full-size index of a workload, built once per machine and reused by
+    content digest (workload definition + generator and builder sources)."""
+    import hashlib
+
+    from paper_2608_15438_gb300.builder import build_index, config
+
+    w = synth.WORKLOADS[workload_name]
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    h = hashlib.sha256(repr(w).encode())
+    for f in ("synth/synth.c", "paper_2608_15438_gb300/builder/nrbuild.cpp"):
+        h.update(open(os.path.join(root, f), "rb").read())
+    path = os.path.join(tmp_root, f"neuroute_{w.name}_{h.hexdigest()[:16]}.nrix")
+    if not os.path.exists(path):
+        base = synth.base(w)
+        build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t), base,
+                    synth.encoder_weights(w), path + f".tmp{os.getpid()}")
+        os.replace(path + f".tmp{os.getpid()}", path)
+    return path

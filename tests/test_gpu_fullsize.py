@@ -1,0 +1,61 @@
+"""Parity at the benchmark's full sizes and launch configuration: 1e7-vector
+workloads, the whole 10,000-query batch in one nr_search_logits call with the
+benchmark's (P, C, t_low), checked against the oracle on a sample of queries
+spread over the batch (the oracle computes each one from scratch).
+
+Fed the oracle's logits, ids, distances and per-query statistics must match
+exactly; end to end (GPU encoder), Recall@10 on the sample must agree with the
+oracle's within 0.002 against brute-force ground truth."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from gpu_util import cached_index, need_cuda, recall
+
+pytestmark = pytest.mark.gpu
+
+SAMPLE = 200
+
+
+@pytest.mark.parametrize("name", ["u8-10m", "f32-10m"])
+def test_full_batch_sampled_parity(name):
+    torch = need_cuda()
+    import bench
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    w = synth.WORKLOADS[name]
+    P, C, t_low = bench.OPERATING_POINTS[name]
+    path = cached_index(name)
+    ix = nr.Index(path, 0)
+    orc = oracle.Index(path)
+    qs = synth.queries(w)
+    lg = orc.encode(qs)
+    dq = torch.from_numpy(qs).cuda()
+    ix.set_params(t_low=t_low)
+    ids, d = ix.search_logits(dq, torch.from_numpy(lg).cuda(), 10, P, C)
+    st = ix.query_stats(w.nq)
+    torch.cuda.synchronize()
+    ids, d, st = ids.cpu().numpy(), d.cpu().numpy(), st.cpu().numpy()
+    sample = np.linspace(0, w.nq - 1, SAMPLE).astype(np.int64)
+    p = oracle.params(t_low=t_low)
+    ids_o, d_o, st_o = orc.search(qs[sample], 10, P, C, p, logits=lg[sample])
+    assert np.array_equal(ids[sample], ids_o)
+    if w.dtype == "u8":
+        assert np.array_equal(d[sample], d_o)
+    else:
+        assert np.all(np.abs(d[sample] - d_o) <= 1e-5 * np.abs(d_o))
+    assert np.array_equal(st[sample], st_o)
+    # end to end through the GPU encoder, recall against exact k-NN on the sample
+    ids_e, _ = ix.search(dq, 10, P, C)
+    torch.cuda.synchronize()
+    ids_oe, _, _ = orc.search(qs[sample], 10, P, C, p)
+    base = torch.from_numpy(synth.base(w)).cuda().float()
+    qf = dq[torch.from_numpy(sample).cuda()].float()
+    dist = (qf * qf).sum(1, keepdim=True) + (base * base).sum(1)[None] - 2.0 * qf @ base.T
+    truth = torch.topk(dist, 10, dim=1, largest=False).indices.cpu().numpy()
+    del base, dist
+    r_gpu = recall(ids_e.cpu().numpy()[sample], truth)
+    r_orc = recall(ids_oe, truth)
+    assert abs(r_gpu - r_orc) <= 0.002 + 1e-12, (r_gpu, r_orc)
+    ix.close()
