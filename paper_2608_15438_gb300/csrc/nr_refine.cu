@@ -12,8 +12,9 @@
 // thread). Each warp gathers its own 32 rows of a tile with 16-byte cp.async
 // copies issued across lanes so that a warp-wide copy covers whole 128-byte
 // lines, into a shared-memory stage whose 16-byte chunks are XOR-swizzled by
-// row so that one-row-per-thread reads are bank-conflict free. STAGES tiles
-// are in flight per CTA.
+// row so that one-row-per-thread reads are bank-conflict free. Tiles are small
+// (128 uint8 rows, 32 fp32 rows) and two stages deep, so that many queries
+// stream concurrently on every SM.
 //
 // Distances: uint8 rows use per-byte |x - q| (__vabsdiffu4) squared and summed
 // with __dp4a in int32 (exact); fp32 rows use the sequential fmaf chain over
@@ -33,7 +34,6 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr uint64_t kMaxKey = ~0ull;
-constexpr int kMaxK = 256;
 
 struct RefineArgs {
   const uint8_t *q;  // [nq x row_bytes]
@@ -65,8 +65,8 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 // CPR = 16-byte chunks per row when known at compile time (0: a.cpr)
-template <int DT, int TR, int STAGES, int CPR>
-__global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
+template <int DT, int TR, int STAGES, int CPR, int MINB>
+__global__ void __launch_bounds__(TR, MINB) refine_kernel(RefineArgs a) {
   extern __shared__ __align__(128) unsigned char smem[];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int cpr = CPR > 0 ? CPR : a.cpr;
@@ -76,10 +76,11 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
   unsigned char *stage_base = smem;                                       // STAGES x TR x RB
   unsigned char *sq = smem + (size_t)STAGES * TR * RB;                    // RB (query)
   uint32_t *srow = reinterpret_cast<uint32_t *>(sq + RB);                 // STAGES x TR
-  uint64_t *hkey = reinterpret_cast<uint64_t *>(srow + STAGES * TR);      // 2 x kMaxK
-  int *htag = reinterpret_cast<int *>(hkey + 2 * kMaxK);                  // 2 x kMaxK
-  uint64_t *skey = reinterpret_cast<uint64_t *>(htag + 2 * kMaxK);        // 2 x TR survivors
-  int *sctl = reinterpret_cast<int *>(skey + 2 * TR);                     // [0] query, [1..3] counters
+  const int kMaxK = a.k;                                                  // top-k buffers sized by k
+  uint64_t *hkey = reinterpret_cast<uint64_t *>(srow + STAGES * TR);      // 2 x k
+  uint64_t *skey = hkey + 2 * kMaxK;                                      // 2 x TR survivors
+  int *htag = reinterpret_cast<int *>(skey + 2 * TR);                     // 2 x k
+  int *sctl = htag + 2 * kMaxK;                                           // [0] query, [1..3] counters
   const uint32_t stage_s = (uint32_t)__cvta_generic_to_shared(stage_base);
   const int k = a.k;
   const int chunk = a.R < TR ? a.R : TR;
@@ -94,10 +95,10 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
     if (q >= a.nq) break;
     for (int c = tid; c < cpr; c += TR)
       reinterpret_cast<uint4 *>(sq)[c] = reinterpret_cast<const uint4 *>(a.q + q * RB)[c];
-    const int64_t n = a.slen[q];
+    const uint32_t n = a.slen[q];  // stream positions fit 32 bits (N < 2^32)
     const int nl = a.nL[q];
     const nr_seg *segs = a.seg + (size_t)q * a.Lmax;
-    const int64_t ntiles = (n + TR - 1) / TR;
+    const uint32_t ntiles = (uint32_t)(((uint64_t)n + TR - 1) / TR);
     __syncthreads();
     uint4 qreg[DT == 0 && CPR > 0 && CPR <= 8 ? CPR : 1];
     if (DT == 0 && CPR > 0 && CPR <= 8) {
@@ -108,24 +109,23 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
     // Gather the rows of tile t into stage t % STAGES. A warp copies and later
     // reads only its own 32 rows, so stage reuse needs no block barrier.
     int seg_i = 0;  // this thread's segment cursor (positions only grow)
-    auto issue = [&](int64_t t) {
+    auto issue = [&](uint32_t t, int st) {
       if (t < ntiles) {
-        const int st = (int)(t % STAGES);
-        const int64_t p = t * TR + tid;
+        const uint32_t p = t * TR + tid;
         uint32_t grow = 0;
         if (p < n) {
           // last segment starting at or before p: exponential search from the cursor
           int step = 1;
-          while (seg_i + step < nl && (int64_t)__ldg(&segs[seg_i + step].pos) <= p) {
+          while (seg_i + step < nl && __ldg(&segs[seg_i + step].pos) <= p) {
             seg_i += step;
             step <<= 1;
           }
           for (step >>= 1; step > 0; step >>= 1)
-            if (seg_i + step < nl && (int64_t)__ldg(&segs[seg_i + step].pos) <= p) seg_i += step;
-          grow = __ldg(&segs[seg_i].row0) + (uint32_t)(p - (int64_t)__ldg(&segs[seg_i].pos));
+            if (seg_i + step < nl && __ldg(&segs[seg_i + step].pos) <= p) seg_i += step;
+          grow = __ldg(&segs[seg_i].row0) + (p - __ldg(&segs[seg_i].pos));
           srow[st * TR + tid] = grow;
         }
-        const int64_t wbase = t * TR + warp * 32;
+        const uint32_t wbase = t * TR + warp * 32;
         const uint32_t sbase = stage_s + (uint32_t)((size_t)st * TR * RB);
 #pragma unroll 4
         for (int f = lane; f < 32 * cpr; f += 32) {
@@ -142,16 +142,17 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
       cp_async_commit();
     };
 
-    for (int s = 0; s < STAGES - 1; ++s) issue(s);
+    for (int s = 0; s < STAGES - 1; ++s) issue((uint32_t)s, s);
     int cur = 0, hn = 0, rounds = 0, low = 0, ci = 0;
     bool stop = false;
-    int64_t done = 0;  // stream positions consumed in completed rounds
-    for (int64_t t = 0; t < ntiles && !stop; ++t) {
-      issue(t + STAGES - 1);
+    uint32_t done = 0;  // stream positions consumed in completed rounds
+    const uint32_t rmask_round = (uint32_t)a.R - 1u;  // R is a power of two
+    int st = 0;                                        // stage of tile t
+    for (uint32_t t = 0; t < ntiles && !stop; ++t) {
+      issue(t + STAGES - 1, st == 0 ? STAGES - 1 : st - 1);
       cp_async_wait<STAGES - 1>();
       __syncwarp();
-      const int st = (int)(t % STAGES);
-      const int64_t p = t * TR + tid;
+      const uint32_t p = t * TR + tid;
       uint32_t dkey = 0xffffffffu;
       if (p < n) {
         const unsigned char *row = stage_base + (size_t)st * TR * RB + (size_t)tid * RB;
@@ -190,7 +191,7 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
       // rotate over three slots and survivor buffers over two, and every warp
       // evaluates the stop rule itself from the shared top-k.
       for (int cs = 0; cs < TR && !stop; cs += chunk, ++ci) {
-        const int64_t cstart = t * TR + cs;
+        const uint32_t cstart = t * TR + cs;
         if (cstart >= n) break;
         int *cnt = &sctl[1 + ci % 3];
         uint64_t *sk_buf = skey + (ci & 1) * TR;
@@ -237,8 +238,8 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
           cur = nxt;
           hn = hn + ns < k ? hn + ns : k;
         }
-        const int64_t cend = cstart + chunk < n ? cstart + chunk : n;
-        if ((cend % a.R) == 0 || cend >= n) {  // round complete
+        const uint32_t cend = n - cstart > (uint32_t)chunk ? cstart + chunk : n;
+        if ((cend & rmask_round) == 0 || cend >= n) {  // round complete
           rounds = roundno;
           done = cend;
           int newc = 0, frontc = 0;
@@ -256,6 +257,7 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
           stop = a.t_low > 0 && hn == k && roundno >= a.r_min && low >= a.t_low;
         }
       }
+      st = st + 1 == STAGES ? 0 : st + 1;
     }
     cp_async_wait<0>();
     __syncthreads();
@@ -274,18 +276,18 @@ __global__ void __launch_bounds__(TR) refine_kernel(RefineArgs a) {
       a.out_d[q * k + i] = d;
     }
     if (tid == 0 && a.stats) {
-      a.stats[q * 4 + 0] = done;
+      a.stats[q * 4 + 0] = (int64_t)done;
       a.stats[q * 4 + 1] = rounds;
     }
     __syncthreads();
   }
 }
 
-template <int DT, int TR, int STAGES, int CPR>
+template <int DT, int TR, int STAGES, int CPR, int MINB = 1>
 cudaError_t launch(nr_index *ix, const RefineArgs &a, cudaStream_t s) {
   const size_t smem = (size_t)STAGES * TR * a.row_bytes + (size_t)a.row_bytes +
-                      (size_t)STAGES * TR * 4 + 2 * kMaxK * 8 + 2 * kMaxK * 4 + (size_t)2 * TR * 8 + 32;
-  auto kern = refine_kernel<DT, TR, STAGES, CPR>;
+                      (size_t)STAGES * TR * 4 + (size_t)2 * a.k * 12 + (size_t)2 * TR * 8 + 32;
+  auto kern = refine_kernel<DT, TR, STAGES, CPR, MINB>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   int per_sm = 0;
@@ -337,14 +339,15 @@ cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, i
   a.counter = d_counter;
   cudaError_t e = cudaMemsetAsync(d_counter, 0, sizeof(unsigned int), s);
   if (e != cudaSuccess) return e;
+  // Launch shapes measured on GB300 (u8-10m / f32-10m operating points): the
+  // scan is limited by how many queries stream concurrently per SM, so tiles
+  // are small, two stages deep, and registers are capped for many CTAs per SM.
   if (ix->dtype == 0) {
-    if (a.cpr == 8) return launch<0, 256, 3, 8>(ix, a, s);  // uint8, D = 128
-    if (ix->row_bytes <= 256) return launch<0, 256, 3, 0>(ix, a, s);
-    if (ix->row_bytes <= 512) return launch<0, 128, 3, 0>(ix, a, s);
-    return launch<0, 64, 3, 0>(ix, a, s);
+    if (a.cpr == 8) return launch<0, 128, 2, 8, 6>(ix, a, s);  // uint8, D = 128
+    if (ix->row_bytes <= 512) return launch<0, 128, 2, 0, 4>(ix, a, s);
+    return launch<0, 64, 2, 0, 4>(ix, a, s);
   }
-  if (a.cpr == 24) return launch<1, 256, 2, 24>(ix, a, s);  // fp32, D = 96
-  if (ix->row_bytes <= 384) return launch<1, 256, 2, 0>(ix, a, s);
-  if (ix->row_bytes <= 768) return launch<1, 128, 2, 0>(ix, a, s);
-  return launch<1, 64, 2, 0>(ix, a, s);
+  if (a.cpr == 24) return launch<1, 32, 2, 24, 12>(ix, a, s);  // fp32, D = 96
+  if (ix->row_bytes <= 512) return launch<1, 64, 2, 0, 4>(ix, a, s);
+  return launch<1, 32, 2, 0, 4>(ix, a, s);
 }
