@@ -216,11 +216,176 @@ __global__ void route_heap_kernel(const float *__restrict__ logits, const float 
   }
 }
 
+
+// Warp-per-query variant: the frontier is a 32-ary min-heap in shared memory,
+// so a sift-down level is one load per lane and two warp min-reductions
+// (redux.sync) over the 32 children of a node; a 512-entry frontier is two
+// levels deep. Lane j holds bit j.
+__global__ void route_warp_kernel(const float *__restrict__ logits, const float *__restrict__ tau,
+                                  int b, int bsel, int rmax, float smax, int64_t nq, int P, int cap,
+                                  uint32_t *__restrict__ codes, int32_t *__restrict__ nprobe) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
+  const int64_t q = (int64_t)blockIdx.x * wpb + warp;
+  if (q >= nq) return;  // uniform per warp
+  uint64_t *hkey = reinterpret_cast<uint64_t *>(smem) + (size_t)warp * cap;
+  float *hcp = reinterpret_cast<float *>(smem + (size_t)wpb * cap * 8) + (size_t)warp * cap;
+  float *ssd = reinterpret_cast<float *>(smem + (size_t)wpb * cap * 12) + warp * 32;
+
+  float dj = __int_as_float(0x7f800000);
+  bool bit = false;
+  if (lane < b) {
+    const float l = logits[q * b + lane];
+    const float tj = tau[lane];
+    bit = l >= tj;
+    dj = fabsf(__fsub_rn(l, tj));
+  }
+  const uint32_t u0 = __ballot_sync(kFull, bit);
+  int rank = 0;
+  for (int i = 0; i < b; ++i) {
+    const float di = __shfl_sync(kFull, dj, i);
+    if (di < dj || (di == dj && i < lane)) ++rank;
+  }
+  // bit mask of the bit holding each rank: lane r gets 1 << pi[r]
+  uint32_t rbit = 0;
+  for (int j = 0; j < b; ++j) {
+    const int rj = __shfl_sync(kFull, rank, j);
+    if (rj == lane) rbit = 1u << j;
+  }
+  if (lane < b) ssd[rank] = dj;
+  __syncwarp();
+
+  uint32_t *out = codes + (size_t)q * P;
+  if (lane == 0) out[0] = u0;
+  int n = 1, hs = 0;
+  if (P > 1 && bsel >= 1 && ssd[0] <= smax) {
+    if (lane == 0) {
+      hkey[0] = pack_key(ssd[0], 1u, 1u);
+      hcp[0] = 0.0f;
+    }
+    hs = 1;
+  }
+  __syncwarp();
+  while (n < P && hs > 0) {
+    const uint64_t top = hkey[0];
+    const float topcp = hcp[0];
+    const uint32_t rmask = (uint32_t)top & 0xffffffu;
+    const uint32_t size = ((uint32_t)top >> 24) & 0xffu;
+    const float cost = __uint_as_float((uint32_t)(top >> 32));
+    const uint32_t flips = __reduce_or_sync(kFull, ((rmask >> lane) & 1u) ? rbit : 0u);
+    if (lane == 0) out[n] = u0 ^ flips;
+    ++n;
+    const int m = 31 - __clz((int)rmask);
+    bool v1 = false, v2 = false;
+    uint64_t k1 = kEmpty, k2 = kEmpty;
+    float cp1 = 0.0f, cp2 = 0.0f;
+    if (m + 1 < bsel) {
+      const float sdn = ssd[m + 1];
+      const float c1 = __fadd_rn(topcp, sdn);  // shift: rank m -> m + 1
+      if (c1 <= smax) {
+        v1 = true;
+        k1 = pack_key(c1, size, rmask + (1u << m));
+        cp1 = topcp;
+      }
+      if (rmax <= 0 || (int)size < rmax) {  // expand: add rank m + 1
+        const float c2 = __fadd_rn(cost, sdn);
+        if (c2 <= smax) {
+          v2 = true;
+          k2 = pack_key(c2, size + 1, rmask | (1u << (m + 1)));
+          cp2 = cost;
+        }
+      }
+    }
+    uint64_t x = kEmpty;
+    float xcp = 0.0f;
+    if (v1) {
+      x = k1;
+      xcp = cp1;
+    } else if (v2) {
+      x = k2;
+      xcp = cp2;
+    } else {
+      hs -= 1;
+      if (hs > 0) {
+        x = hkey[hs];
+        xcp = hcp[hs];
+      }
+    }
+    // sift-down of x from the root
+    if (x != kEmpty) {
+      int i = 0;
+      for (;;) {
+        const int c = 32 * i + 1 + lane;
+        const uint64_t ck = c < hs ? hkey[c] : kEmpty;
+        const uint32_t chi = (uint32_t)(ck >> 32), clo = (uint32_t)ck;
+        const uint32_t mhi = __reduce_min_sync(kFull, chi);
+        const uint32_t mlo = __reduce_min_sync(kFull, chi == mhi ? clo : 0xffffffffu);
+        const uint64_t mk = ((uint64_t)mhi << 32) | mlo;
+        if (mk < x) {
+          const int src = __ffs(__ballot_sync(kFull, ck == mk)) - 1;
+          const int mc = 32 * i + 1 + src;
+          if (lane == src) {
+            hkey[i] = mk;
+            hcp[i] = hcp[mc];
+          }
+          i = mc;
+          __syncwarp();
+        } else {
+          if (lane == 0) {
+            hkey[i] = x;
+            hcp[i] = xcp;
+          }
+          break;
+        }
+      }
+    }
+    __syncwarp();
+    if (v1 && v2) {  // sift-up of the expand child
+      if (lane == 0) {
+        int j = hs;
+        while (j > 0) {
+          const int pj = (j - 1) >> 5;
+          const uint64_t pk = hkey[pj];
+          if (pk < k2) break;
+          hkey[j] = pk;
+          hcp[j] = hcp[pj];
+          j = pj;
+        }
+        hkey[j] = k2;
+        hcp[j] = cp2;
+      }
+      hs += 1;
+    }
+    __syncwarp();
+  }
+  for (int t = n + lane; t < P; t += 32) out[t] = 0xffffffffu;
+  if (lane == 0) nprobe[q] = n;
+}
+
 }  // namespace
 
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
+  {
+    const int cap = P + 2;
+    const size_t per_warp = (size_t)cap * 12 + 128;
+    int wpb = (int)((48u * 1024u) / per_warp);
+    if (wpb > 4) wpb = 4;
+    if (wpb < 1) wpb = 1;
+    const size_t smem = per_warp * (size_t)wpb;
+    cudaError_t e = cudaFuncSetAttribute(route_warp_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const nr_params &p = ix->params;
+    const int bsel = (p.l_sel > 0 && p.l_sel < ix->b) ? p.l_sel : ix->b;
+    const int64_t grid = (nq + wpb - 1) / wpb;
+    route_warp_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(d_logits, ix->tau, ix->b, bsel,
+                                                              p.r_max, p.s_max, nq, P, cap, d_codes,
+                                                              d_nprobe);
+    ix->launches += 1;
+    return cudaGetLastError();
+  }
   const int cap = P + 2;
   const size_t per_group = (size_t)cap * 12 + 256;
   int wpb = (int)((96u * 1024u) / (per_group * kQPW));

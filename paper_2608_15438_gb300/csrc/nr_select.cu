@@ -21,7 +21,7 @@
 
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 128;
 constexpr uint64_t kMaxKey = ~0ull;
 
 __device__ __forceinline__ void set_err(int *err, int code) { atomicCAS(err, 0, code); }
@@ -60,7 +60,11 @@ __device__ int block_exclusive_scan(int *a, int n, int *warp_sums) {
   return total;
 }
 
-__device__ void bitonic_sort(uint64_t *k, int n) {  // n a power of two
+// Bitonic sort of k[0..n), n a power of two. Thread i owns the pairs
+// (lo, lo + stride) with lo = 2i - (i mod stride); for strides up to 32 the
+// pairs of one warp stay inside its own 64-element blocks, so consecutive
+// such stages need only a warp barrier.
+__device__ void bitonic_sort(uint64_t *k, int n) {
   for (int size = 2; size <= n; size <<= 1) {
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
       for (int i = threadIdx.x; i < n / 2; i += kThreads) {
@@ -73,9 +77,13 @@ __device__ void bitonic_sort(uint64_t *k, int n) {  // n a power of two
           k[hi] = a;
         }
       }
-      __syncthreads();
+      // a block barrier whenever this stage or the next one crosses warps
+      const int next = stride > 1 ? stride >> 1 : size;
+      if (stride > 32 || next > 32) __syncthreads();
+      else __syncwarp();
     }
   }
+  __syncthreads();
 }
 
 struct SelectArgs {
@@ -138,14 +146,15 @@ __global__ void __launch_bounds__(kThreads) select_kernel(SelectArgs a) {
   }
   __syncthreads();
   const int M = block_exclusive_scan(cnt, np, warp_sums);
+  // each probe writes its clusters' indices into the key slots
+  for (int i = tid; i < np; i += kThreads) {
+    const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
+    for (int j = 0; j < n; ++j) keys[o + j] = (uint64_t)(uint32_t)(c0s[i] + j);
+  }
+  __syncthreads();
   // centroid distances; keys of all candidates (exclusion decided after d_min)
   for (int s = tid; s < M; s += kThreads) {
-    int lo = 0, hi = np - 1;  // largest i with cnt[i] <= s
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (cnt[mid] <= s) lo = mid; else hi = mid - 1;
-    }
-    const uint32_t c = (uint32_t)(c0s[lo] + (s - cnt[lo]));
+    const uint32_t c = (uint32_t)keys[s];
     const float *mu = a.cent + (size_t)c * a.b;
     float acc = 0.0f;
     for (int j = 0; j < a.b; ++j) {
