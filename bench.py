@@ -31,12 +31,23 @@ sys.path.insert(0, ROOT)
 
 METRIC = "QPS at Recall@10~0.90 (batched query path); refine-scan HBM GB/s"
 
-# operating points (P, C, t_low) with Recall@10 in [0.88, 0.92], from `--sweep`
+# operating points (P, C, t_low, gate m1) with Recall@10 in [0.88, 0.92], from
+# `--sweep` / `--sweep-gate`; gate m1 = None: gate off, else M(x) = m1 x
 OPERATING_POINTS = {
-    "tiny": (128, 256, 4),
-    "u8-10m": (256, 256, 64),
-    "f32-10m": (512, 256, 16),
+    "tiny": (128, 256, 4, None),
+    "u8-10m": (256, 256, 0, 4.0),
+    "f32-10m": (512, 256, 16, None),
+    "u8-100m": (1024, 256, 32, None),
 }
+
+
+def op_params(w):
+    """nr_params keyword arguments of the workload's operating point."""
+    _, _, t_low, m1 = OPERATING_POINTS.get(w.name, (64, 128, 4, None))
+    kw = {"t_low": t_low}
+    if m1 is not None:
+        kw.update(gate_m0=0.0, gate_m1=m1)
+    return kw
 
 
 def parse():
@@ -52,6 +63,8 @@ def parse():
     ap.add_argument("--nq", type=int, default=None)
     ap.add_argument("--impl", default="neuroute", choices=["neuroute", "reference"])
     ap.add_argument("--sweep", action="store_true")
+    ap.add_argument("--sweep-gate", action="store_true",
+                    help="sweep the centroid gate M(x) = m1 x around the (P, C) grid")
     ap.add_argument("--index", default=None, help="reuse an index file")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-gt", action="store_true", help="skip ground truth (profiling runs)")
@@ -182,14 +195,21 @@ def recall_at(found, truth, k=10):
     return float(np.mean(r))
 
 
+def refine_sources_digest():
+    """sha256 over the sources that define the refine kernel."""
+    h = hashlib.sha256()
+    for f in ("nr_refine.cu", "nr_query.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2608_15438_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()
+
+
 def traffic_from_profile(workload, P, C):
     """Per-launch DRAM bytes of the refine kernel from a committed ncu summary,
     valid only while the kernel source is unchanged since the capture."""
     path = os.path.join(ROOT, "profiles", "refine_traffic.json")
     try:
         rec = json.load(open(path))
-        src = open(os.path.join(ROOT, "paper_2608_15438_gb300", "csrc", "nr_refine.cu"), "rb").read()
-        if rec.get("nr_refine_sha256") != hashlib.sha256(src).hexdigest():
+        if rec.get("sources_sha256") != refine_sources_digest():
             return None
         e = rec.get("captures", {}).get(f"{workload}/P{P}/C{C}")
         return None if e is None else e.get("bytes_per_launch")
@@ -201,7 +221,9 @@ def cpu_baseline(w, path, queries, k, P, C, t_low, seconds, truth=None):
     import oracle
 
     orc = oracle.Index(path)
-    p = oracle.params(t_low=t_low)
+    kw = op_params(w)
+    kw["t_low"] = t_low
+    p = oracle.params(**kw)
     cores = os.cpu_count() or 1
     n = 16
     t = time.perf_counter()
@@ -232,7 +254,9 @@ def run_reference(args, w, rank, world):
     import oracle
 
     orc = oracle.Index(path)
-    p = oracle.params(t_low=t_low)
+    kw = op_params(w)
+    kw["t_low"] = t_low
+    p = oracle.params(**kw)
     cores = os.cpu_count() or 1
     n = 16
     t = time.perf_counter()
@@ -262,7 +286,7 @@ def run_reference(args, w, rank, world):
 
 
 def op_point(args, w):
-    P, C, t_low = OPERATING_POINTS.get(w.name, (64, 128, 4))
+    P, C, t_low, _ = OPERATING_POINTS.get(w.name, (64, 128, 4, None))
     return (args.P or P, args.C or C, t_low if args.t_low is None else args.t_low)
 
 
@@ -318,10 +342,33 @@ def main():
         del base_t
         torch.cuda.empty_cache()
 
+    if args.sweep_gate:
+        for Pp in (128, 256, 512):
+            for Cc in (128, 256, 1024):
+                for tl in (0, 32, 64):
+                    for m1 in (None, 0.5, 1.0, 2.0, 4.0):
+                        kw = {"t_low": tl}
+                        if m1 is not None:
+                            kw.update(gate_m0=0.0, gate_m1=m1)
+                        ix.set_params(**kw)
+                        ix.search(dq, k, Pp, Cc, out=(ids, dd))
+                        torch.cuda.synchronize()
+                        t = time.perf_counter()
+                        ix.search(dq, k, Pp, Cc, out=(ids, dd))
+                        torch.cuda.synchronize()
+                        el = time.perf_counter() - t
+                        st = ix.last_stats()
+                        print(json.dumps({"P": Pp, "C": Cc, "t_low": tl, "gate_m1": m1,
+                                          "recall": recall_at(ids.cpu().numpy(), truth, k),
+                                          "qps": nq / el, "cand_per_q": st.candidates / nq}), flush=True)
+        return 0
+
     if args.sweep:
         rows = []
-        for Pp in (64, 128, 256, 512, 1024):
-            for Cc in (256, 512, 1024, 2048):
+        grid_p = (64, 128, 256, 512, 1024) if w.bits <= 20 else (256, 512, 1024)
+        grid_c = (256, 512, 1024, 2048) if w.bits <= 20 else (256, 1024)
+        for Pp in grid_p:
+            for Cc in grid_c:
                 if Pp * ix.k_max > 16384:
                     continue
                 for tl in (0, 8, 16, 32, 64):
@@ -338,7 +385,9 @@ def main():
                     print(json.dumps(rows[-1]), flush=True)
         return 0
 
-    ix.set_params(t_low=t_low)
+    kw = op_params(w)
+    kw["t_low"] = t_low
+    ix.set_params(**kw)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     for _ in range(max(3, args.warmup)):
         ix.search(dq, k, P, C, out=(ids, dd), stream=stream)
@@ -407,6 +456,7 @@ def main():
         "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
         "config": {"workload": w.name, "N": w.n, "D": w.dim, "nq": nq, "k": k, "bits": w.bits,
                    "hidden": w.hidden, "K_max": w.k_max, "P": P, "C": C, "t_low": t_low,
+                   "gate_m1": kw.get("gate_m1"),
                    "round": 256, "recall_at_10": rec, "cand_per_query": cand / nq,
                    "l2": "flushed between timed steps (256 MB write)",
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},

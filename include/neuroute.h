@@ -171,9 +171,10 @@ nr_status nr_search_host(nr_index *ix, const void *h_queries, int64_t nq, int k,
  * inference server, and latency-critical loops in which cudaMalloc / cudaFree
  * (which can synchronise the device) are not acceptable. The paper has no
  * counterpart; results are identical to nr_search.
- * Limit: a call needs about nq * (4b + 4P + 12(P + C) + 48) bytes (each of its
- * nine buffers rounded up to 256 bytes); larger requests return
- * NR_ERR_INVALID_ARG without enqueuing work, so split the batch.
+ * Limit: a call needs about nq * (4b + 4P + 12(P + C) + 48) bytes, plus
+ * nq * 12 * P * K_max bytes when P * K_max exceeds 2048 (each buffer rounded up
+ * to 256 bytes); larger requests return NR_ERR_INVALID_ARG without enqueuing
+ * work, so split the batch.
  * The first call on a device looks up the array's device address with that
  * device made current; make that first call before any stream capture.
  * All calls share the one array and it keeps the last call's contents: two

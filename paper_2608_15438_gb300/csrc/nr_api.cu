@@ -54,7 +54,7 @@ size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 // Per-chunk workspace layout of a search over qc queries.
 struct Layout {
-  size_t logits, codes, nprobe, L, nL, seg, slen, total;
+  size_t logits, codes, nprobe, L, nL, seg, slen, slab, total;
 };
 Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   Layout l;
@@ -67,6 +67,7 @@ Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   l.nL = o;     o = align256(o + (size_t)qc * 4);
   l.seg = o;    o = align256(o + (size_t)qc * Lmax * sizeof(nr_seg));
   l.slen = o;   o = align256(o + (size_t)qc * 4);
+  l.slab = o;   o = align256(o + (size_t)qc * nr_select_slab_bytes(P, ix->K_max));
   l.total = o;
   return l;
 }
@@ -400,7 +401,7 @@ nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int
   if (e == cudaSuccess)
     e = nr_launch_select(ix, d_logits, (uint32_t *)(w + l.codes), (int32_t *)(w + l.nprobe), nq,
                          P, C, d_clusters, d_ncl, (nr_seg *)(w + l.seg), (uint32_t *)(w + l.slen),
-                         nullptr, s);
+                         nullptr, nr_select_slab_bytes(P, ix->K_max) ? w + l.slab : nullptr, s);
   return cuda_status(e);
 }
 
@@ -463,7 +464,8 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
     ev = tstart(2);
     e = nr_launch_select(ix, lg, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), n, P, C,
                          (int32_t *)(cw + l.L), (int32_t *)(cw + l.nL), (nr_seg *)(cw + l.seg),
-                         (uint32_t *)(cw + l.slen), stats + q0 * 4, s);
+                         (uint32_t *)(cw + l.slen), stats + q0 * 4,
+                         nr_select_slab_bytes(P, ix->K_max) ? cw + l.slab : nullptr, s);
     tend(ev);
     if (e != cudaSuccess) break;
     ev = tstart(3);

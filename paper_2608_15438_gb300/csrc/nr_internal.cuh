@@ -60,10 +60,12 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s);
 size_t nr_select_smem_bytes(int P, int C, int K_max);
+// global scratch per query that select needs for probe budget P (0: none)
+size_t nr_select_slab_bytes(int P, int K_max);
 cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t *d_codes,
                              const int32_t *d_nprobe, int64_t nq, int P, int C, int32_t *d_L,
                              int32_t *d_nL, nr_seg *d_seg, uint32_t *d_slen, int64_t *d_stats,
-                             cudaStream_t s);
+                             void *d_slab, cudaStream_t s);
 cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, int Lmax,
                              const nr_seg *d_seg, const int32_t *d_nL, const uint32_t *d_slen,
                              int64_t *d_ids, float *d_dists, int64_t *d_stats,

@@ -260,32 +260,46 @@ struct SelectParams {
   int *err;
 };
 
-// Scratch (shared memory) of select_block for probe budget P.
+// Sort capacity for probe budget P: all clusters of P buckets. Shared memory
+// holds at most kSelectSmemKeys keys; a query with more candidate clusters
+// sorts in its slab of global memory (select_slab_bytes, 0 when unneeded).
+constexpr int kSelectSmemKeys = 2048;
 __host__ __device__ inline int select_sort_cap(int P, int K_max) {
   int s = 1;
   while (s < P * K_max) s <<= 1;
   return s;
 }
+__host__ __device__ inline int select_smem_cap(int P, int K_max) {
+  const int s = select_sort_cap(P, K_max);
+  return s < kSelectSmemKeys ? s : kSelectSmemKeys;
+}
 __host__ __device__ inline size_t select_scratch_bytes(int P, int K_max) {
-  const int S = select_sort_cap(P, K_max);
+  const int S = select_smem_cap(P, K_max);
   const int ib = S > 2 * P + 1 ? S : 2 * P + 1;
   return (size_t)S * 8 + (size_t)ib * 4;
+}
+__host__ __device__ inline size_t select_slab_bytes(int P, int K_max) {
+  const int full = select_sort_cap(P, K_max);
+  return full > select_smem_cap(P, K_max) ? (size_t)full * 12 : 0;
 }
 
 // One query: codes[0..np) -> the kept clusters C^dir U C^cent in (d, cluster)
 // order and their refinement segments. Writes seg[i] = (first row, stream
 // position) for i < nl, and L[i] (cluster index, -1 padded to Lmax) when L is
 // not null. slog: the query's b logits in shared memory; scratch:
-// select_scratch_bytes(P, K_max) bytes of shared memory; warp_sums: 32 ints;
-// sred: 1 unsigned. Returns nl; *total = stream length. Whole block calls.
+// select_scratch_bytes(P, K_max) bytes of shared memory; slab: this query's
+// select_slab_bytes(P, K_max) bytes of global memory (null when that is 0);
+// warp_sums: 32 ints; sred: 1 unsigned. Returns nl; *total = stream length.
+// Whole block calls.
 __device__ __forceinline__ int select_block(const SelectParams &sp, const float *slog,
                                             const uint32_t *codes, int np, unsigned char *scratch,
-                                            int *warp_sums, unsigned *sred, nr_seg *seg,
-                                            int32_t *L, int Lmax, uint32_t *total) {
+                                            unsigned char *slab, int *warp_sums, unsigned *sred,
+                                            nr_seg *seg, int32_t *L, int Lmax, uint32_t *total) {
   const int tid = threadIdx.x, nt = blockDim.x;
-  const int S_pow = select_sort_cap(sp.P, sp.K_max);
+  const int S_smem = select_smem_cap(sp.P, sp.K_max);
+  const int S_full = select_sort_cap(sp.P, sp.K_max);
   uint64_t *keys = reinterpret_cast<uint64_t *>(scratch);
-  int *ibuf = reinterpret_cast<int *>(scratch + (size_t)S_pow * 8);
+  int *ibuf = reinterpret_cast<int *>(scratch + (size_t)S_smem * 8);
   if (tid == 0) *sred = 0xffffffffu;
   int *cnt = ibuf;        // [P] clusters per probe -> exclusive offsets
   int *c0s = ibuf + sp.P;  // [P] first cluster per probe
@@ -313,6 +327,18 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   }
   __syncthreads();
   const int M = block_exclusive_scan(cnt, np, warp_sums);
+  int Sn = 1;
+  while (Sn < M) Sn <<= 1;
+  // many candidate clusters: keys and per-key integers move to the global slab
+  int *ints = ibuf;
+  if (M > S_smem && slab != nullptr && Sn <= S_full) {
+    keys = reinterpret_cast<uint64_t *>(slab);
+    ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
+  } else if (M > S_smem) {
+    if (tid == 0) set_err(sp.err, NR_DEV_TOO_MANY);
+    *total = 0;
+    return 0;
+  }
   for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
     const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
     for (int j = 0; j < n; ++j) keys[o + j] = (uint64_t)(uint32_t)(c0s[i] + j);
@@ -330,8 +356,6 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     keys[s] = ((uint64_t)__float_as_uint(acc) << 32) | c;
     if (!__ldg(&sp.single[c])) atomicMin(sred, __float_as_uint(acc));  // d >= 0: bits order as values
   }
-  int Sn = 1;
-  while (Sn < M) Sn <<= 1;
   for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
   __syncthreads();
   const uint32_t dmin_bits = *sred;
@@ -348,7 +372,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   __syncthreads();
   bitonic_sort(keys, Sn);
   // keep C^dir and the first C survivors in key order
-  int *keep = ibuf;  // [Sn]
+  int *keep = ints;  // [Sn]
   for (int s = tid; s < Sn; s += nt) {
     const uint64_t kk = keys[s];
     keep[s] = (s < M && kk != kEmpty && !__ldg(&sp.single[(uint32_t)kk])) ? 1 : 0;
@@ -372,7 +396,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     }
   }
   __syncthreads();
-  int *len = ibuf;  // [nl]
+  int *len = ints;  // [nl]
   for (int i = tid; i < nl; i += nt) {
     const uint32_t c = seg[i].row0;
     if (L) L[i] = (int32_t)c;

@@ -25,7 +25,8 @@ constexpr int kThreads = 128;
 __global__ void __launch_bounds__(kThreads)
     select_kernel(nrq::SelectParams sp, const float *__restrict__ logits,
                   const uint32_t *__restrict__ codes, const int32_t *__restrict__ nprobe,
-                  int32_t *L, int32_t *nL, nr_seg *seg, uint32_t *slen, int64_t *stats) {
+                  int32_t *L, int32_t *nL, nr_seg *seg, uint32_t *slen, int64_t *stats,
+                  unsigned char *slab, size_t slab_bytes) {
   extern __shared__ __align__(16) unsigned char smem[];
   const int q = blockIdx.x, tid = threadIdx.x;
   const int Lmax = sp.P + sp.C;
@@ -37,7 +38,8 @@ __global__ void __launch_bounds__(kThreads)
   if (tid < sp.b) slog[tid] = logits[(size_t)q * sp.b + tid];
   __syncthreads();
   uint32_t total = 0;
-  const int nl = nrq::select_block(sp, slog, codes + (size_t)q * sp.P, np, scratch, warp_sums, sred,
+  unsigned char *qslab = slab ? slab + (size_t)q * slab_bytes : nullptr;
+  const int nl = nrq::select_block(sp, slog, codes + (size_t)q * sp.P, np, scratch, qslab, warp_sums, sred,
                                    seg + (size_t)q * Lmax, L ? L + (size_t)q * Lmax : nullptr,
                                    Lmax, &total);
   if (tid == 0) {
@@ -75,6 +77,8 @@ nrq::SelectParams nr_select_params(nr_index *ix, int P, int C) {
   return sp;
 }
 
+size_t nr_select_slab_bytes(int P, int K_max) { return nrq::select_slab_bytes(P, K_max); }
+
 size_t nr_select_smem_bytes(int P, int C, int K_max) {
   (void)C;
   return nrq::select_scratch_bytes(P, K_max) + 32 * 4 + 32 * 4 + 16;
@@ -83,14 +87,16 @@ size_t nr_select_smem_bytes(int P, int C, int K_max) {
 cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t *d_codes,
                              const int32_t *d_nprobe, int64_t nq, int P, int C, int32_t *d_L,
                              int32_t *d_nL, nr_seg *d_seg, uint32_t *d_slen, int64_t *d_stats,
-                             cudaStream_t s) {
+                             void *d_slab, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
   const size_t smem = nr_select_smem_bytes(P, C, ix->K_max);
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   select_kernel<<<(unsigned)nq, kThreads, smem, s>>>(nr_select_params(ix, P, C), d_logits, d_codes,
-                                                      d_nprobe, d_L, d_nL, d_seg, d_slen, d_stats);
+                                                      d_nprobe, d_L, d_nL, d_seg, d_slen, d_stats,
+                                                      static_cast<unsigned char *>(d_slab),
+                                                      nrq::select_slab_bytes(P, ix->K_max));
   ix->launches += 1;
   return cudaGetLastError();
 }

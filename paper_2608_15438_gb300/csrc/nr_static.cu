@@ -88,6 +88,8 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   const size_t o_seg = o;    o = up256(o + q * Lmax * sizeof(nr_seg));
   const size_t o_slen = o;   o = up256(o + q * 4);
   const size_t o_stats = o;  o = up256(o + q * 4 * 8);
+  const size_t slab_q = nr_select_slab_bytes(P, ix->K_max);
+  const size_t o_slab = o;   o = up256(o + q * slab_q);
   const size_t o_count = o;  o = up256(o + 16);
   if (o > NR_STATIC_SCRATCH_BYTES) return NR_ERR_INVALID_ARG;  // request too large for the array
   CurrentDevice cd(ix->device);
@@ -107,7 +109,7 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   if (e == cudaSuccess)
     e = nr_launch_select(ix, logits, (uint32_t *)(w + o_codes), (int32_t *)(w + o_nprobe), nq, P, C,
                          (int32_t *)(w + o_L), (int32_t *)(w + o_nL), (nr_seg *)(w + o_seg),
-                         (uint32_t *)(w + o_slen), stats, s);
+                         (uint32_t *)(w + o_slen), stats, slab_q ? w + o_slab : nullptr, s);
   if (e == cudaSuccess)
     e = nr_launch_refine(ix, d_queries, nq, k, (int)Lmax, (nr_seg *)(w + o_seg),
                          (int32_t *)(w + o_nL), (uint32_t *)(w + o_slen), d_out_ids, d_out_dists,

@@ -25,20 +25,21 @@ def test_full_batch_sampled_parity(name):
     from paper_2608_15438_gb300 import neuroute as nr
 
     w = synth.WORKLOADS[name]
-    P, C, t_low = bench.OPERATING_POINTS[name]
+    P, C, _, _ = bench.OPERATING_POINTS[name]
+    kw = bench.op_params(w)
     path = cached_index(name)
     ix = nr.Index(path, 0)
     orc = oracle.Index(path)
     qs = synth.queries(w)
     lg = orc.encode(qs)
     dq = torch.from_numpy(qs).cuda()
-    ix.set_params(t_low=t_low)
+    ix.set_params(**kw)
     ids, d = ix.search_logits(dq, torch.from_numpy(lg).cuda(), 10, P, C)
     st = ix.query_stats(w.nq)
     torch.cuda.synchronize()
     ids, d, st = ids.cpu().numpy(), d.cpu().numpy(), st.cpu().numpy()
     sample = np.linspace(0, w.nq - 1, SAMPLE).astype(np.int64)
-    p = oracle.params(t_low=t_low)
+    p = oracle.params(**kw)
     ids_o, d_o, st_o = orc.search(qs[sample], 10, P, C, p, logits=lg[sample])
     assert np.array_equal(ids[sample], ids_o)
     if w.dtype == "u8":

@@ -270,3 +270,38 @@ def test_out_of_range_directory_is_flagged_not_faulted(torch, tmp_path):
     torch.cuda.synchronize()
     assert torch.equal(ids, ids2)
     assert ids.cpu().tolist()[0] == [0, 1, 1, 2, 3]
+
+
+@pytest.fixture(scope="module")
+def many_clusters(torch, tmp_path_factory):
+    """b = 8 and up to 16 clusters per bucket: probing all 256 buckets gives
+    about 4096 candidate clusters, more than select keeps in shared memory."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, base, info = build_small(tmp_path_factory.mktemp("mc"), "tiny", n=20000, bits=8,
+                                   k_max=16, t=4, name="mc")
+    w = synth.WORKLOADS["tiny"]
+    qs = synth.queries(w, 300)
+    orc = oracle.Index(path)
+    lg = orc.encode(qs)
+    return {"ix": nr.Index(path, 0), "orc": orc, "q": qs, "lg": lg, "info": info,
+            "dq": torch.from_numpy(qs).cuda(), "dl": torch.from_numpy(lg).cuda()}
+
+
+@pytest.mark.parametrize("C", [64, 4096])
+def test_select_overflow_to_global_slab(many_clusters, torch, C):
+    mc = many_clusters
+    assert mc["info"]["n_clusters"] > 2048
+    ix, orc = mc["ix"], mc["orc"]
+    cl, ncl = ix.debug_clusters(mc["dl"], 256, C)
+    cl, ncl = cl.cpu().numpy(), ncl.cpu().numpy()
+    tau = orc.tau()
+    p = oracle.params()
+    for i in range(0, len(mc["q"]), 7):
+        codes, _, _ = oracle.probe_list(mc["lg"][i], tau, 256, p)
+        L, _, _ = orc.cluster_list(mc["lg"][i], codes, C, p)
+        assert ncl[i] == len(L)
+        assert np.array_equal(cl[i, : len(L)], L)
+    ids, d = ix.search_logits(mc["dq"], mc["dl"], 10, 256, C)
+    ids_o, d_o, _ = orc.search(mc["q"], 10, 256, C, p, logits=mc["lg"])
+    assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
