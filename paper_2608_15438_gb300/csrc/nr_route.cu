@@ -44,9 +44,21 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
   if (nq <= 0) return cudaSuccess;
   const int cap = P + 2;
   const size_t per_warp = nr_route_heap_bytes(P);
-  int wpb = (int)((48u * 1024u) / per_warp);
-  if (wpb > 4) wpb = 4;
-  if (wpb < 1) wpb = 1;
+  // warps per block: the choice that packs the most warps into an SM's
+  // shared memory (the heap is the limit at large probe budgets)
+  const size_t sm_bytes = (size_t)227 * 1024;
+  int wpb = 1, best = 0;
+  for (int w = 4; w >= 1; w >>= 1) {
+    const size_t blk = per_warp * (size_t)w;
+    if (blk > sm_bytes) continue;
+    int blocks = (int)(sm_bytes / (blk + 1024));
+    if (blocks > 32) blocks = 32;
+    const int warps = blocks * w > 64 ? 64 : blocks * w;
+    if (warps > best) {
+      best = warps;
+      wpb = w;
+    }
+  }
   const size_t smem = per_warp * (size_t)wpb;
   cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
