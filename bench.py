@@ -68,6 +68,8 @@ def parse():
     ap.add_argument("--index", default=None, help="reuse an index file")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-gt", action="store_true", help="skip ground truth (profiling runs)")
+    ap.add_argument("--encode", type=int, default=0,
+                    help="time only the tensor-core encoder over this many base vectors")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     return ap.parse_args()
 
@@ -285,6 +287,48 @@ def run_reference(args, w, rank, world):
     return 0
 
 
+def encode_bench(args, w, torch, nr, dev):
+    """Throughput of the encoder (K1, tensor cores) over a batch of base
+    vectors, the operation an index build runs over the whole base."""
+    path = args.index or index_path(w)
+    build_or_load_index(w, path, 0, 1)
+    ix = nr.Index(path, dev.index or 0)
+    import synth
+
+    x = torch.from_numpy(synth.base(w, args.encode)).to(dev)
+    out = torch.empty((args.encode, w.bits), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    L = nr.lib()
+    import ctypes
+
+    def run():
+        st = L.nr_encode(ix.h, ctypes.c_void_p(x.data_ptr()), args.encode, ctypes.c_void_p(out.data_ptr()),
+                         ctypes.c_void_p(stream.cuda_stream))
+        if st != 0:
+            raise RuntimeError(f"nr_encode failed {st}")
+
+    for _ in range(max(3, args.warmup)):
+        run()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record(stream)
+    for _ in range(args.steps):
+        run()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    flops = 2.0 * args.encode * (w.dim * w.hidden + w.hidden * w.bits)
+    peaks, src = measured_peaks()
+    tf = flops / (ms / 1e3) / 1e12
+    print(json.dumps({"metric": "encoder TFLOP/s (fp16 tensor cores, fp32 accumulate)", "value": tf,
+                      "unit": "TFLOP/s", "rows": args.encode, "ms_per_launch": ms,
+                      "roofline": {"bound": "tensor", "achieved": tf, "peak": peaks.get("bf16_tflops"),
+                                   "unit": "TFLOP/s", "frac": tf / peaks.get("bf16_tflops"),
+                                   "peak_source": src + " bf16 dense (fp16 dense runs at the same nominal rate)"},
+                      "config": {"workload": w.name, "D": w.dim, "H": w.hidden, "b": w.bits}}), flush=True)
+    return 0
+
+
 def op_point(args, w):
     P, C, t_low, _ = OPERATING_POINTS.get(w.name, (64, 128, 4, None))
     return (args.P or P, args.C or C, t_low if args.t_low is None else args.t_low)
@@ -317,6 +361,8 @@ def main():
 
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
+    if args.encode:
+        return encode_bench(args, w, torch, nr, dev)
     P, C, t_low = op_point(args, w)
     k = args.k
     path = args.index or index_path(w)

@@ -156,8 +156,10 @@ __global__ void __launch_bounds__(128, 1)
     fence_mbar_init();
   }
   // X tile to fp16 (rows past nq are zero)
+  // thread i fills row 8 (i / 8 / kx) + i % 8, chunk (i / 8) % kx: eight
+  // consecutive threads write one 128-byte core matrix (no bank conflicts)
   for (int i = tid; i < kRows * kx; i += 128) {
-    const int r = i / kx, c = i - r * kx;
+    const int c = (i >> 3) % kx, r = ((i >> 3) / kx) * 8 + (i & 7);
     const int64_t row = row0 + r;
     __align__(16) __half hv[8];
     if (row < nq) {
@@ -195,12 +197,12 @@ __global__ void __launch_bounds__(128, 1)
   for (int hc = 0; hc < H / kHC && ok; ++hc) {
     // operands of this chunk: W1 rows [hc*128, +128), W2 columns [hc*128, +128)
     for (int i = tid; i < kHC * kx; i += 128) {
-      const int n = i / kx, c = i - n * kx;
+      const int c = (i >> 3) % kx, n = ((i >> 3) / kx) * 8 + (i & 7);
       *reinterpret_cast<uint4 *>(sW1 + kmajor_off(n, c, kx)) =
           *reinterpret_cast<const uint4 *>(W1h + (size_t)(hc * kHC + n) * D + c * 8);
     }
     for (int i = tid; i < n2 * 16; i += 128) {
-      const int n = i >> 4, c = i & 15;
+      const int c = (i >> 3) & 15, n = (i >> 7) * 8 + (i & 7);
       *reinterpret_cast<uint4 *>(sW2 + kmajor_off(n, c, 16)) =
           *reinterpret_cast<const uint4 *>(W2h + (size_t)n * H + hc * kHC + c * 8);
     }

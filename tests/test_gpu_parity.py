@@ -305,3 +305,20 @@ def test_select_overflow_to_global_slab(many_clusters, torch, C):
     ids, d = ix.search_logits(mc["dq"], mc["dl"], 10, 256, C)
     ids_o, d_o, _ = orc.search(mc["q"], 10, 256, C, p, logits=mc["lg"])
     assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
+
+
+@pytest.mark.parametrize("workload", ["tiny", "u8-10m", "f32-10m"])
+def test_encoder_large_batch(torch, tmp_path, workload):
+    """Large batches (many 128-row tiles) through the tensor-core encoder, for
+    the three encoder shapes (H = 256, 512, 384)."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, _, _ = build_small(tmp_path, workload, n=20000, name="enc")
+    w = synth.WORKLOADS[workload]
+    x = synth.base(w, 60000)
+    ix, orc = nr.Index(path, 0), oracle.Index(path)
+    lg = ix.encode(torch.from_numpy(x).cuda()).cpu().numpy().astype(np.float64)
+    ref = orc.encode(x).astype(np.float64)
+    err = np.abs(lg - ref).max(1)
+    assert np.all(err <= 1e-2 * np.abs(ref).max(1))
+    assert np.median(err / np.abs(ref).max(1)) < 2e-3
