@@ -45,9 +45,11 @@ __device__ __forceinline__ void cp_async_wait() {
 // carried as (cost, cost without the largest rank), so each child's cost is
 // one addition in the same left-to-right order a sequential sum would use.
 //
-// The frontier is a 32-ary min-heap in shared memory (hkey/hcp, capacity
-// P + 2): a sift-down level is one load per lane and two warp min-reductions;
-// the frontier never holds more than P + 1 entries. Lane j holds bit j.
+// The frontier is a 32-ary min-heap of keys in shared memory (capacity P + 2,
+// 8 bytes an entry): a sift-down level is one load per lane and two warp
+// min-reductions; the frontier never holds more than P + 1 entries. The cost
+// without the largest rank, needed for the shift child, is recomputed from
+// the popped rank mask in the same left-to-right fp32 order. Lane j holds bit j.
 struct RouteParams {
   const float *tau;
   int b, bsel, rmax;
@@ -55,12 +57,18 @@ struct RouteParams {
   int P;
 };
 
+// Bytes of shared memory route_warp needs for probe budget P.
+__host__ __device__ inline size_t route_heap_bytes(int P) { return (size_t)(P + 2) * 8 + 128; }
+
 // Writes codes[0..n) (any address space) and returns n, uniform in the warp.
-// Must be called by a whole warp. ssd: 32 floats of shared memory.
+// Must be called by a whole warp. heap: route_heap_bytes(P) bytes of shared
+// memory (8-byte aligned).
 __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__restrict__ logit,
-                                          uint64_t *hkey, float *hcp, float *ssd, uint32_t *codes) {
+                                          unsigned char *heap, uint32_t *codes) {
   const int lane = threadIdx.x & 31;
   const int b = rp.b;
+  uint64_t *hkey = reinterpret_cast<uint64_t *>(heap);
+  float *ssd = reinterpret_cast<float *>(heap + (size_t)(rp.P + 2) * 8);
   float dj = __int_as_float(0x7f800000);
   bool bit = false;
   if (lane < b) {
@@ -85,16 +93,12 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
   if (lane == 0) codes[0] = u0;
   int n = 1, hs = 0;
   if (rp.P > 1 && rp.bsel >= 1 && ssd[0] <= rp.smax) {
-    if (lane == 0) {
-      hkey[0] = pack_key(ssd[0], 1u, 1u);
-      hcp[0] = 0.0f;
-    }
+    if (lane == 0) hkey[0] = pack_key(ssd[0], 1u, 1u);
     hs = 1;
   }
   __syncwarp();
   while (n < rp.P && hs > 0) {
     const uint64_t top = hkey[0];
-    const float topcp = hcp[0];
     const uint32_t rmask = (uint32_t)top & 0xffffffu;
     const uint32_t size = ((uint32_t)top >> 24) & 0xffu;
     const float cost = __uint_as_float((uint32_t)(top >> 32));
@@ -105,38 +109,32 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
     const int m = 31 - __clz((int)rmask);
     bool v1 = false, v2 = false;
     uint64_t k1 = kEmpty, k2 = kEmpty;
-    float cp1 = 0.0f, cp2 = 0.0f;
     if (m + 1 < rp.bsel) {
       const float sdn = ssd[m + 1];
-      const float c1 = __fadd_rn(topcp, sdn);  // shift: rank m -> m + 1
+      // cost without rank m: fp32 sum from 0 over the other ranks, ascending
+      float costp = 0.0f;
+      for (uint32_t mm = rmask & ~(1u << m); mm; mm &= mm - 1) costp = __fadd_rn(costp, ssd[__ffs(mm) - 1]);
+      const float c1 = __fadd_rn(costp, sdn);  // shift: rank m -> m + 1
       if (c1 <= rp.smax) {
         v1 = true;
         k1 = pack_key(c1, size, rmask + (1u << m));
-        cp1 = topcp;
       }
       if (rp.rmax <= 0 || (int)size < rp.rmax) {  // expand: add rank m + 1
         const float c2 = __fadd_rn(cost, sdn);
         if (c2 <= rp.smax) {
           v2 = true;
           k2 = pack_key(c2, size + 1, rmask | (1u << (m + 1)));
-          cp2 = cost;
         }
       }
     }
     uint64_t x = kEmpty;
-    float xcp = 0.0f;
     if (v1) {
       x = k1;
-      xcp = cp1;
     } else if (v2) {
       x = k2;
-      xcp = cp2;
     } else {
       hs -= 1;
-      if (hs > 0) {
-        x = hkey[hs];
-        xcp = hcp[hs];
-      }
+      if (hs > 0) x = hkey[hs];
     }
     if (x != kEmpty) {  // sift-down of x from the root
       int i = 0;
@@ -149,18 +147,11 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
         const uint64_t mk = ((uint64_t)mhi << 32) | mlo;
         if (mk < x) {
           const int src = __ffs(__ballot_sync(kFull, ck == mk)) - 1;
-          const int mc = 32 * i + 1 + src;
-          if (lane == src) {
-            hkey[i] = mk;
-            hcp[i] = hcp[mc];
-          }
-          i = mc;
+          if (lane == src) hkey[i] = mk;
+          i = 32 * i + 1 + src;
           __syncwarp();
         } else {
-          if (lane == 0) {
-            hkey[i] = x;
-            hcp[i] = xcp;
-          }
+          if (lane == 0) hkey[i] = x;
           break;
         }
       }
@@ -174,11 +165,9 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
           const uint64_t pk = hkey[pj];
           if (pk < k2) break;
           hkey[j] = pk;
-          hcp[j] = hcp[pj];
           j = pj;
         }
         hkey[j] = k2;
-        hcp[j] = cp2;
       }
       hs += 1;
     }

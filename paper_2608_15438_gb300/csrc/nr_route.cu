@@ -9,16 +9,14 @@
 namespace {
 
 __global__ void route_kernel(nrq::RouteParams rp, const float *__restrict__ logits, int64_t nq,
-                             int cap, uint32_t *__restrict__ codes, int32_t *__restrict__ nprobe) {
+                             uint32_t *__restrict__ codes, int32_t *__restrict__ nprobe) {
   extern __shared__ __align__(16) unsigned char smem[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int64_t q = (int64_t)blockIdx.x * wpb + warp;
   if (q >= nq) return;  // uniform per warp
-  uint64_t *hkey = reinterpret_cast<uint64_t *>(smem) + (size_t)warp * cap;
-  float *hcp = reinterpret_cast<float *>(smem + (size_t)wpb * cap * 8) + (size_t)warp * cap;
-  float *ssd = reinterpret_cast<float *>(smem + (size_t)wpb * cap * 12) + warp * 32;
+  unsigned char *heap = smem + (size_t)warp * nrq::route_heap_bytes(rp.P);
   uint32_t *out = codes + (size_t)q * rp.P;
-  const int n = nrq::route_warp(rp, logits + q * rp.b, hkey, hcp, ssd, out);
+  const int n = nrq::route_warp(rp, logits + q * rp.b, heap, out);
   for (int t = n + lane; t < rp.P; t += 32) out[t] = 0xffffffffu;
   if (lane == 0) nprobe[q] = n;
 }
@@ -37,12 +35,11 @@ nrq::RouteParams nr_route_params(const nr_index *ix, int P) {
   return rp;
 }
 
-size_t nr_route_heap_bytes(int P) { return (size_t)(P + 2) * 12 + 128; }
+size_t nr_route_heap_bytes(int P) { return nrq::route_heap_bytes(P); }
 
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
-  const int cap = P + 2;
   const size_t per_warp = nr_route_heap_bytes(P);
   // warps per block: the choice that packs the most warps into an SM's
   // shared memory (the heap is the limit at large probe budgets)
@@ -64,7 +61,7 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
                                        (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t grid = (nq + wpb - 1) / wpb;
-  route_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(nr_route_params(ix, P), d_logits, nq, cap,
+  route_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(nr_route_params(ix, P), d_logits, nq,
                                                        d_codes, d_nprobe);
   ix->launches += 1;
   return cudaGetLastError();
