@@ -54,7 +54,7 @@ size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 // Per-chunk workspace layout of a search over qc queries.
 struct Layout {
-  size_t logits, codes, nprobe, L, nL, seg, slen, slab, total;
+  size_t logits, codes, nprobe, L, nL, seg, slen, slab, perm, total;
 };
 Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   Layout l;
@@ -68,6 +68,7 @@ Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   l.seg = o;    o = align256(o + (size_t)qc * Lmax * sizeof(nr_seg));
   l.slen = o;   o = align256(o + (size_t)qc * 4);
   l.slab = o;   o = align256(o + (size_t)qc * nr_select_slab_bytes(P, ix->K_max));
+  l.perm = o;   o = align256(o + (size_t)qc * 4);
   l.total = o;
   return l;
 }
@@ -471,7 +472,7 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
     ev = tstart(3);
     e = nr_launch_refine(ix, qp, n, k, P + C, (nr_seg *)(cw + l.seg), (int32_t *)(cw + l.nL),
                          (uint32_t *)(cw + l.slen), d_ids + q0 * k, d_d + q0 * k, stats + q0 * 4,
-                         counter, s);
+                         counter, (int32_t *)(cw + l.perm), s);
     tend(ev);
   }
   ix->timed_last = ix->timing;

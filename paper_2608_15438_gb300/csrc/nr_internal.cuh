@@ -69,4 +69,4 @@ cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t
 cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, int Lmax,
                              const nr_seg *d_seg, const int32_t *d_nL, const uint32_t *d_slen,
                              int64_t *d_ids, float *d_dists, int64_t *d_stats,
-                             unsigned int *d_counter, cudaStream_t s);
+                             unsigned int *d_counter, int32_t *d_perm, cudaStream_t s);

@@ -14,6 +14,44 @@
 
 namespace {
 
+// Longest streams first: one CTA buckets the queries by stream length
+// (1024 buckets scaled to the longest stream) and writes them in decreasing
+// bucket order, so the persistent refinement CTAs finish together instead of
+// waiting on a long query picked up last. Order inside a bucket is arbitrary;
+// it does not affect any result.
+constexpr int kOrderBins = 1024;
+
+__global__ void __launch_bounds__(1024) order_kernel(const uint32_t *__restrict__ slen, int64_t nq,
+                                                     int32_t *__restrict__ perm) {
+  __shared__ unsigned int hist[kOrderBins];
+  __shared__ unsigned int smax;
+  const int tid = threadIdx.x;
+  if (tid == 0) smax = 1;
+  for (int i = tid; i < kOrderBins; i += blockDim.x) hist[i] = 0;
+  __syncthreads();
+  unsigned int m = 1;
+  for (int64_t q = tid; q < nq; q += blockDim.x) m = max(m, slen[q]);
+  atomicMax(&smax, m);
+  __syncthreads();
+  const uint64_t top = (uint64_t)smax + 1;
+  for (int64_t q = tid; q < nq; q += blockDim.x)
+    atomicAdd(&hist[kOrderBins - 1 - (int)((uint64_t)slen[q] * kOrderBins / top)], 1u);
+  __syncthreads();
+  if (tid == 0) {  // exclusive scan (1024 entries)
+    unsigned int run = 0;
+    for (int i = 0; i < kOrderBins; ++i) {
+      const unsigned int v = hist[i];
+      hist[i] = run;
+      run += v;
+    }
+  }
+  __syncthreads();
+  for (int64_t q = tid; q < nq; q += blockDim.x) {
+    const int bin = kOrderBins - 1 - (int)((uint64_t)slen[q] * kOrderBins / top);
+    perm[atomicAdd(&hist[bin], 1u)] = (int32_t)q;
+  }
+}
+
 struct RefineArgs {
   nrq::RefineParams rf;
   const uint8_t *q;  // [nq x row_bytes]
@@ -27,6 +65,7 @@ struct RefineArgs {
   float *out_d;
   int64_t *stats;
   unsigned int *counter;
+  const int32_t *perm;  // processing order (null: index order)
 };
 
 template <int DT, int TR, int STAGES, int CPR, int MINB>
@@ -37,10 +76,13 @@ __global__ void __launch_bounds__(TR, MINB) refine_kernel(RefineArgs a) {
   const nrq::RefineSmem m = nrq::refine_carve<TR, STAGES>(smem, a.row_bytes, k);
   int *qslot = m.sctl + 4;
   for (;;) {
-    if (tid == 0) *qslot = (int)atomicAdd(a.counter, 1u);
+    if (tid == 0) {
+      const unsigned int slot = atomicAdd(a.counter, 1u);
+      *qslot = slot < a.nq ? (a.perm ? a.perm[slot] : (int)slot) : -1;
+    }
     __syncthreads();
     const int64_t q = *qslot;
-    if (q >= a.nq) break;
+    if (q < 0) break;
     for (int c = tid; c * 16 < a.row_bytes; c += TR)
       reinterpret_cast<uint4 *>(m.sq)[c] = reinterpret_cast<const uint4 *>(a.q + q * a.row_bytes)[c];
     nrq::refine_block<DT, TR, STAGES, CPR>(a.rf, m, a.slen[q], a.nL[q], a.seg + (size_t)q * a.Lmax,
@@ -104,8 +146,14 @@ nrq::RefineParams refine_params(const nr_index *ix, int k) {
 cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, int Lmax,
                              const nr_seg *d_seg, const int32_t *d_nL, const uint32_t *d_slen,
                              int64_t *d_ids, float *d_dists, int64_t *d_stats,
-                             unsigned int *d_counter, cudaStream_t s) {
+                             unsigned int *d_counter, int32_t *d_perm, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
+  if (d_perm) {
+    order_kernel<<<1, 1024, 0, s>>>(d_slen, nq, d_perm);
+    ix->launches += 1;
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
   RefineArgs a;
   a.rf = refine_params(ix, k);
   a.q = static_cast<const uint8_t *>(d_q);
@@ -119,6 +167,7 @@ cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, i
   a.out_d = d_dists;
   a.stats = d_stats;
   a.counter = d_counter;
+  a.perm = d_perm;
   cudaError_t e = cudaMemsetAsync(d_counter, 0, sizeof(unsigned int), s);
   if (e != cudaSuccess) return e;
   if (ix->dtype == 0) {

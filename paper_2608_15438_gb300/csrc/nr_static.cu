@@ -113,7 +113,7 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   if (e == cudaSuccess)
     e = nr_launch_refine(ix, d_queries, nq, k, (int)Lmax, (nr_seg *)(w + o_seg),
                          (int32_t *)(w + o_nL), (uint32_t *)(w + o_slen), d_out_ids, d_out_dists,
-                         stats, (unsigned int *)(w + o_count), s);
+                         stats, (unsigned int *)(w + o_count), nullptr, s);
   // statistics of this call are read from the array by nr_last_stats / nr_query_stats
   ix->d_stats = stats;
   ix->last_nq = nq;
