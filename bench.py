@@ -413,6 +413,8 @@ def main():
         rows = []
         grid_p = (64, 128, 256, 512, 1024) if w.bits <= 20 else (256, 512, 1024)
         grid_c = (256, 512, 1024, 2048) if w.bits <= 20 else (256, 1024)
+        if w.k_max == 1:  # no bucket-local clustering: C never binds
+            grid_p, grid_c = (64, 128, 256, 512, 1024, 2048), (256,)
         for Pp in grid_p:
             for Cc in grid_c:
                 if Pp * ix.k_max > 16384:

@@ -97,6 +97,10 @@ WORKLOADS = {
     # 1e7 fp32 x 96, L2-normalised, b = 20
     "f32-10m": Workload("f32-10m", 10_000_000, 96, "f32", 1024, 0.3, 10_000, 384, 20, 8, 64,
                         probe=(8, 32), clusters=(64,)),
+    # the 1e7 uint8 workload indexed without bucket-local clustering (one
+    # cluster per bucket): the analogue of the paper's bucket-clustering ablation
+    "u8-10m-nocl": Workload("u8-10m-nocl", 10_000_000, 128, "u8", 256, 18.0, 10_000, 512, 20, 1, 64,
+                            probe=(64, 256), clusters=(256,)),
     # 1e8 uint8 x 128, b = 24
     "u8-100m": Workload("u8-100m", 100_000_000, 128, "u8", 4096, 18.0, 10_000, 512, 24, 16, 64),
     # 1e9 uint8 x 128, b = 24
