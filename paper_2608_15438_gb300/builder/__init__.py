@@ -33,6 +33,9 @@ def lib():
         L.nrb_build.argtypes = [ctypes.POINTER(Config), vp, ctypes.c_int64, vp, vp, vp, vp,
                                 ctypes.c_char_p, ctypes.c_int, vp]
         L.nrb_build.restype = ctypes.c_int
+        L.nrb_build_logits.argtypes = [ctypes.POINTER(Config), vp, ctypes.c_int64, vp, vp, vp, vp,
+                                       vp, ctypes.c_char_p, ctypes.c_int, vp]
+        L.nrb_build_logits.restype = ctypes.c_int
         L.nrb_encode.argtypes = [ctypes.POINTER(Config), vp, ctypes.c_int64, vp, vp, vp, vp, vp,
                                  ctypes.c_int]
         L.nrb_encode.restype = ctypes.c_int
@@ -63,5 +66,41 @@ def build_index(cfg: Config, base: np.ndarray, weights, path: str, nthreads: int
                          nthreads or os.cpu_count() or 1, info.ctypes.data)
     if rc != 0:
         raise RuntimeError(f"nrb_build failed ({rc})")
+    return _info(info)
+
+
+def _info(info):
     return {"n_clusters": int(info[0]), "n_buckets": int(info[1]), "max_bucket": int(info[2]),
             "max_cluster": int(info[3]), "single_cluster_buckets": int(info[4])}
+
+
+def build_index_from_logits(cfg: Config, base: np.ndarray, logits: np.ndarray, weights, path: str,
+                            nthreads: int | None = None):
+    """Build the index over base [N x D] from given base logits [N x b] (the
+    encoder step skipped) and write it to path. weights are stored in the file."""
+    base = np.ascontiguousarray(base)
+    logits = np.ascontiguousarray(logits, np.float32)
+    if logits.shape != (base.shape[0], cfg.b):
+        raise ValueError("logits must be [N x b]")
+    W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights)
+    info = np.zeros(5, np.int64)
+    rc = lib().nrb_build_logits(ctypes.byref(cfg), base.ctypes.data, base.shape[0],
+                                logits.ctypes.data, W1.ctypes.data, b1.ctypes.data, W2.ctypes.data,
+                                b2.ctypes.data, path.encode(), nthreads or os.cpu_count() or 1,
+                                info.ctypes.data)
+    if rc != 0:
+        raise RuntimeError(f"nrb_build_logits failed ({rc})")
+    return _info(info)
+
+
+def encode(cfg: Config, base: np.ndarray, weights, nthreads: int | None = None) -> np.ndarray:
+    """The builder's fp32 encoder over base [N x D]: logits [N x b]."""
+    base = np.ascontiguousarray(base)
+    W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights)
+    out = np.empty((base.shape[0], cfg.b), np.float32)
+    rc = lib().nrb_encode(ctypes.byref(cfg), base.ctypes.data, base.shape[0], W1.ctypes.data,
+                          b1.ctypes.data, W2.ctypes.data, b2.ctypes.data, out.ctypes.data,
+                          nthreads or os.cpu_count() or 1)
+    if rc != 0:
+        raise RuntimeError(f"nrb_encode failed ({rc})")
+    return out

@@ -2,7 +2,8 @@
 //
 // Paper Sec. 3.3 (Index Construction) and Sec. 3.2.3 (Binarization):
 //   1. encode every base vector with the encoder, l_i = E(x_i);
-//   2. per-bit threshold tau_j = median of column j (lower median, exact);
+//   2. per-bit threshold tau_j = median of column j (lower median, exact, in
+//      the total order of the fp32 bit patterns);
 //   3. code u_i with bit j = [l_ij >= tau_j]; bucket = code;
 //   4. per non-empty bucket B, K_B = min(K_max, ceil(|B| / t)) clusters found by
 //      k-means++ seeding on a sample and a few Lloyd passes on the whole bucket,
@@ -12,7 +13,8 @@
 // The file it writes is the input of the query path (format in neuroute.h).
 //
 // Host-only C++, threads over rows and buckets. It is deterministic for a
-// given seed and thread count does not change the result.
+// given seed and thread count does not change the result. Given the same
+// logits (nrb_build_logits), the library's GPU builder writes the same bytes.
 #include <algorithm>
 #include <atomic>
 #include <cmath>
@@ -62,7 +64,6 @@ uint64_t splitmix64(uint64_t &s) {
   z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
   return z ^ (z >> 31);
 }
-double unif(uint64_t &s) { return (double)(splitmix64(s) >> 11) * (1.0 / 9007199254740992.0); }
 
 // Encoder forward over rows [r0, r0 + n): blocks of 16 rows so the inner loop
 // runs over independent accumulators.
@@ -101,98 +102,162 @@ void encode_block(const nrb_config &c, const void *x, int64_t r0, int n, const f
   }
 }
 
-double sqdist(const float *a, const double *m, int b) {
-  double s = 0.0;
+// ---------------------------------------------------------------------------
+// Arithmetic of the build, fixed so that a parallel implementation reproduces
+// it bit for bit (the library's GPU builder follows the same definition):
+//  * distances in logit space are fp32 with every product and sum rounded
+//    (t = a_j - c_j, s = s + t*t over j ascending from s = 0, no fused
+//    multiply-add);
+//  * a centroid is the mean of its members' logits, summed exactly as
+//    integers in fixed point (x * 2^G rounded to nearest, G = 30 - e with
+//    max |logit| = f 2^e, f in [0.5, 1)), then ((double)sum * 2^-G) / count
+//    rounded to fp32 -- the order of the additions cannot change it;
+//  * the k-means++ sample is every (n/m)-th member of the bucket (positions
+//    floor(i n / m), members in id order), and the D^2-weighted draw uses
+//    integer weights trunc(dmin_i * 2^F), F = 50 - e(max dmin), so the prefix
+//    sums are exact.
+// ---------------------------------------------------------------------------
+
+// e with v = f * 2^e, f in [0.5, 1), for a positive finite double
+int exponent_of(double v) {
+  uint64_t bits;
+  memcpy(&bits, &v, 8);
+  return (int)((bits >> 52) & 0x7FF) - 1022;
+}
+double pow2(int e) {
+  const uint64_t bits = (uint64_t)(e + 1023) << 52;
+  double v;
+  memcpy(&v, &bits, 8);
+  return v;
+}
+uint64_t mulhi64(uint64_t a, uint64_t b) {
+  return (uint64_t)(((unsigned __int128)a * (unsigned __int128)b) >> 64);
+}
+
+// order-preserving map of fp32 bit patterns to uint32 (total order, -0 < +0)
+uint32_t float_key(float x) {
+  uint32_t u;
+  memcpy(&u, &x, 4);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+float key_float(uint32_t k) {
+  const uint32_t u = (k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k;
+  float x;
+  memcpy(&x, &u, 4);
+  return x;
+}
+
+float sqdist_f(const float *a, const float *c, int b) {
+  float s = 0.0f;
   for (int j = 0; j < b; ++j) {
-    double t = (double)a[j] - m[j];
-    s += t * t;
+    const float t = a[j] - c[j];
+    const float p = t * t;
+    s = s + p;
   }
   return s;
 }
 
-// k-means in logit space for one bucket. rows: member row numbers (ascending
-// id). Returns the number of (non-empty) clusters; labels[i] in [0, K).
-int cluster_bucket(const nrb_config &c, const float *logits, const int64_t *rows, int64_t n,
-                   uint32_t code, std::vector<int> &labels, std::vector<float> &cent_out) {
+struct Fixed {
+  double scale, inv_scale;
+};
+
+// Fixed-point means of the labelled members; clusters without members keep
+// their centroid. cnt[k] = members of cluster k.
+void update_means(const float *logits, const uint32_t *rows, int64_t n, const uint8_t *lab, int K,
+                  int b, const Fixed &fx, float *cent, std::vector<int64_t> &cnt) {
+  std::vector<int64_t> sum((size_t)K * b, 0);
+  cnt.assign((size_t)K, 0);
+  for (int64_t i = 0; i < n; ++i) {
+    const float *l = &logits[(size_t)rows[i] * b];
+    const int k = lab[i];
+    cnt[k] += 1;
+    for (int j = 0; j < b; ++j) sum[(size_t)k * b + j] += llrint((double)l[j] * fx.scale);
+  }
+  for (int k = 0; k < K; ++k)
+    if (cnt[k] > 0)
+      for (int j = 0; j < b; ++j)
+        cent[(size_t)k * b + j] =
+            (float)(((double)sum[(size_t)k * b + j] * fx.inv_scale) / (double)cnt[k]);
+}
+
+// k-means in logit space for one bucket. rows: member ids, ascending.
+// On return labels[i] in [0, kk) and cent_out / cnt_out hold the kk non-empty
+// clusters in label order.
+int cluster_bucket(const nrb_config &c, const float *logits, const uint32_t *rows, int64_t n,
+                   uint32_t code, const Fixed &fx, std::vector<uint8_t> &labels,
+                   std::vector<float> &cent_out, std::vector<int64_t> &cnt_out) {
   const int b = c.b;
   labels.assign((size_t)n, 0);
   int64_t K = (n + c.t - 1) / c.t;
   if (K > c.K_max) K = c.K_max;
-  if (K < 1) K = 1;
   if (K > n) K = n;
-  std::vector<double> cent((size_t)K * b, 0.0);
-  if (K == 1) {
-    for (int64_t i = 0; i < n; ++i)
-      for (int j = 0; j < b; ++j) cent[j] += logits[(size_t)rows[i] * b + j];
-    cent_out.resize((size_t)b);
-    for (int j = 0; j < b; ++j) cent_out[j] = (float)(cent[j] / (double)n);
-    return 1;
-  }
-  uint64_t s = c.seed * 0x100000001B3ull ^ ((uint64_t)code * 0x9E3779B97F4A7C15ull);
-  // sample without replacement (partial Fisher-Yates on member positions)
-  int64_t m = std::min<int64_t>(n, (int64_t)c.sample_per_cluster * K);
-  std::vector<int64_t> pos((size_t)n);
-  for (int64_t i = 0; i < n; ++i) pos[i] = i;
-  for (int64_t i = 0; i < m; ++i) {
-    int64_t j = i + (int64_t)(unif(s) * (double)(n - i));
-    if (j >= n) j = n - 1;
-    std::swap(pos[i], pos[j]);
-  }
-  // k-means++ seeding on the sample
-  std::vector<double> dmin((size_t)m, 1e300);
-  int64_t first = (int64_t)(unif(s) * (double)m);
-  if (first >= m) first = m - 1;
-  for (int j = 0; j < b; ++j) cent[j] = logits[(size_t)rows[pos[first]] * b + j];
-  for (int64_t k = 1; k < K; ++k) {
-    double tot = 0.0;
-    for (int64_t i = 0; i < m; ++i) {
-      double d = sqdist(&logits[(size_t)rows[pos[i]] * b], &cent[(size_t)(k - 1) * b], b);
-      if (d < dmin[i]) dmin[i] = d;
-      tot += dmin[i];
-    }
-    int64_t pick = m - 1;
-    if (tot > 0.0) {
-      double r = unif(s) * tot, acc = 0.0;
+  if (K < 1) K = 1;
+  std::vector<float> cent((size_t)K * b, 0.0f);
+  std::vector<int64_t> cnt;
+  if (K > 1) {
+    uint64_t s = c.seed * 0x100000001B3ull ^ ((uint64_t)code * 0x9E3779B97F4A7C15ull);
+    const int64_t m = std::min<int64_t>(n, (int64_t)c.sample_per_cluster * K);
+    auto sample = [&](int64_t i) {
+      return &logits[(size_t)rows[(uint64_t)i * (uint64_t)n / (uint64_t)m] * b];
+    };
+    auto uniform_pick = [&](uint64_t draw) {
+      int64_t p = (int64_t)((double)(draw >> 11) * (1.0 / 9007199254740992.0) * (double)m);
+      return p < m ? p : m - 1;
+    };
+    memcpy(&cent[0], sample(uniform_pick(splitmix64(s))), sizeof(float) * b);
+    std::vector<float> dmin((size_t)m, INFINITY);
+    std::vector<uint64_t> w((size_t)m);
+    for (int64_t k = 1; k < K; ++k) {
+      float mx = 0.0f;
       for (int64_t i = 0; i < m; ++i) {
-        acc += dmin[i];
-        if (acc > r) {
-          pick = i;
-          break;
+        const float d = sqdist_f(sample(i), &cent[(size_t)(k - 1) * b], b);
+        if (d < dmin[i]) dmin[i] = d;
+        if (dmin[i] > mx) mx = dmin[i];
+      }
+      const uint64_t draw = splitmix64(s);
+      int64_t pick = -1;
+      if (mx > 0.0f) {
+        const double mult = pow2(50 - exponent_of((double)mx));
+        uint64_t tot = 0;
+        for (int64_t i = 0; i < m; ++i) {
+          w[i] = (uint64_t)((double)dmin[i] * mult);
+          tot += w[i];
+        }
+        if (tot > 0) {
+          const uint64_t r = mulhi64(draw, tot);
+          uint64_t acc = 0;
+          for (int64_t i = 0; i < m; ++i) {
+            acc += w[i];
+            if (acc > r) {
+              pick = i;
+              break;
+            }
+          }
         }
       }
-    } else {
-      pick = (int64_t)(unif(s) * (double)m);
-      if (pick >= m) pick = m - 1;
+      if (pick < 0) pick = uniform_pick(draw);
+      memcpy(&cent[(size_t)k * b], sample(pick), sizeof(float) * b);
     }
-    for (int j = 0; j < b; ++j) cent[(size_t)k * b + j] = logits[(size_t)rows[pos[pick]] * b + j];
-  }
-  // Lloyd passes on the whole bucket: assign (ties to the lower index), update
-  std::vector<double> sum((size_t)K * b);
-  std::vector<int64_t> cnt((size_t)K);
-  const int iters = c.lloyd_iters > 0 ? c.lloyd_iters : 1;
-  for (int it = 0; it < iters; ++it) {
-    for (int64_t i = 0; i < n; ++i) {
-      const float *l = &logits[(size_t)rows[i] * b];
-      int best = 0;
-      double bd = sqdist(l, &cent[0], b);
-      for (int k = 1; k < K; ++k) {
-        double d = sqdist(l, &cent[(size_t)k * b], b);
-        if (d < bd) {
-          bd = d;
-          best = k;
+    // Lloyd passes on the whole bucket: assign (ties to the lower index), update
+    const int iters = c.lloyd_iters > 0 ? c.lloyd_iters : 1;
+    for (int it = 0; it < iters; ++it) {
+      for (int64_t i = 0; i < n; ++i) {
+        const float *l = &logits[(size_t)rows[i] * b];
+        int best = 0;
+        float bd = sqdist_f(l, &cent[0], b);
+        for (int k = 1; k < K; ++k) {
+          const float d = sqdist_f(l, &cent[(size_t)k * b], b);
+          if (d < bd) {
+            bd = d;
+            best = k;
+          }
         }
+        labels[i] = (uint8_t)best;
       }
-      labels[i] = best;
+      update_means(logits, rows, n, labels.data(), (int)K, b, fx, cent.data(), cnt);
     }
-    std::fill(sum.begin(), sum.end(), 0.0);
-    std::fill(cnt.begin(), cnt.end(), 0);
-    for (int64_t i = 0; i < n; ++i) {
-      cnt[labels[i]] += 1;
-      for (int j = 0; j < b; ++j) sum[(size_t)labels[i] * b + j] += logits[(size_t)rows[i] * b + j];
-    }
-    for (int k = 0; k < K; ++k)
-      if (cnt[k] > 0)
-        for (int j = 0; j < b; ++j) cent[(size_t)k * b + j] = sum[(size_t)k * b + j] / (double)cnt[k];
+  } else {
+    update_means(logits, rows, n, labels.data(), 1, b, fx, cent.data(), cnt);
   }
   // drop empty clusters, renumber in label order
   std::vector<int> remap((size_t)K, -1);
@@ -200,10 +265,13 @@ int cluster_bucket(const nrb_config &c, const float *logits, const int64_t *rows
   for (int k = 0; k < K; ++k)
     if (cnt[k] > 0) remap[k] = kk++;
   cent_out.resize((size_t)kk * b);
+  cnt_out.resize((size_t)kk);
   for (int k = 0; k < K; ++k)
-    if (remap[k] >= 0)
-      for (int j = 0; j < b; ++j) cent_out[(size_t)remap[k] * b + j] = (float)cent[(size_t)k * b + j];
-  for (int64_t i = 0; i < n; ++i) labels[i] = remap[labels[i]];
+    if (remap[k] >= 0) {
+      memcpy(&cent_out[(size_t)remap[k] * b], &cent[(size_t)k * b], sizeof(float) * b);
+      cnt_out[remap[k]] = cnt[k];
+    }
+  for (int64_t i = 0; i < n; ++i) labels[i] = (uint8_t)remap[labels[i]];
   return kk;
 }
 
@@ -228,26 +296,45 @@ int nrb_encode(const nrb_config *c, const void *x, int64_t n, const float *W1, c
   return 0;
 }
 
-// Build the index over base x [N x D] and write it to path.
-// Returns 0, -1 bad argument, -2 I/O error.
-int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, const float *b1,
-              const float *W2, const float *b2, const char *path, int nthreads, int64_t *info_out) {
-  if (!c || !x || !path || N < 1 || N >= (int64_t)0xFFFFFFFFll || c->b < 1 || c->b > 24 ||
-      c->D < 1 || c->H < 1 || c->K_max < 1 || c->t < 1 || (c->dtype != 0 && c->dtype != 1))
+// Build the index over base x [N x D] from the base's logits [N x b] and
+// write it to path. Returns 0, -1 bad argument (including non-finite
+// logits), -2 I/O error.
+int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float *logits_in,
+                     const float *W1, const float *b1, const float *W2, const float *b2,
+                     const char *path, int nthreads, int64_t *info_out) {
+  if (!c || !x || !logits_in || !path || N < 1 || N >= (int64_t)0xFFFFFFFFll || c->b < 1 ||
+      c->b > 24 || c->D < 1 || c->H < 1 || c->K_max < 1 || c->K_max > 64 || c->t < 1 ||
+      c->sample_per_cluster < 1 || (c->dtype != 0 && c->dtype != 1))
     return -1;
   const int b = c->b, D = c->D;
   const size_t esz = c->dtype == 0 ? 1 : 4;
-  // 1. logits of the whole base
-  std::vector<float> logits((size_t)N * b);
-  nrb_encode(c, x, N, W1, b1, W2, b2, logits.data(), nthreads);
-  // 2. per-bit lower median
+  const float *logits = logits_in;
+  // fixed-point scale of the centroid sums from the largest |logit|
+  uint32_t amax = 0;
+  for (int64_t i = 0; i < N * b; ++i) {
+    uint32_t u;
+    memcpy(&u, &logits[i], 4);
+    u &= 0x7FFFFFFFu;
+    if (u > amax) amax = u;
+  }
+  if (amax >= 0x7F800000u) return -1;
+  Fixed fx;
+  {
+    float am;
+    memcpy(&am, &amax, 4);
+    const int G = 30 - (am > 0.0f ? exponent_of((double)am) : 0);
+    fx.scale = pow2(G);
+    fx.inv_scale = pow2(-G);
+  }
+  // 2. per-bit lower median (rank floor((N-1)/2) in the total order of the
+  // fp32 bit patterns)
   std::vector<float> tau((size_t)b);
   parallel_for(b, nthreads, [&](int64_t j) {
-    std::vector<float> col((size_t)N);
-    for (int64_t i = 0; i < N; ++i) col[i] = logits[(size_t)i * b + j];
+    std::vector<uint32_t> col((size_t)N);
+    for (int64_t i = 0; i < N; ++i) col[i] = float_key(logits[(size_t)i * b + j]);
     size_t mid = (size_t)((N - 1) / 2);
     std::nth_element(col.begin(), col.begin() + mid, col.end());
-    tau[j] = col[mid];
+    tau[j] = key_float(col[mid]);
   });
   // 3. codes and a stable counting sort of ids by code
   const size_t nb = (size_t)1 << b;
@@ -264,10 +351,10 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
   std::vector<int64_t> bstart(nb + 1, 0);
   for (int64_t i = 0; i < N; ++i) bstart[code[i] + 1] += 1;
   for (size_t u = 0; u < nb; ++u) bstart[u + 1] += bstart[u];
-  std::vector<int64_t> order((size_t)N);
+  std::vector<uint32_t> order((size_t)N);
   {
     std::vector<int64_t> fill(bstart.begin(), bstart.end() - 1);
-    for (int64_t i = 0; i < N; ++i) order[fill[code[i]]++] = i;
+    for (int64_t i = 0; i < N; ++i) order[fill[code[i]]++] = (uint32_t)i;
   }
   std::vector<uint32_t>().swap(code);
   // 4. bucket-local clustering
@@ -275,8 +362,8 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
   for (size_t u = 0; u < nb; ++u)
     if (bstart[u + 1] > bstart[u]) nonempty.push_back((uint32_t)u);
   std::vector<std::vector<float>> bcent(nonempty.size());
+  std::vector<std::vector<int64_t>> bcnt(nonempty.size());
   std::vector<int> ncl(nonempty.size());
-  std::vector<int> label((size_t)N);  // by position in `order`
   // largest buckets first for load balance
   std::vector<int64_t> sched(nonempty.size());
   for (size_t i = 0; i < sched.size(); ++i) sched[i] = (int64_t)i;
@@ -289,23 +376,14 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
     int64_t i = sched[si];
     uint32_t u = nonempty[i];
     int64_t lo = bstart[u], n = bstart[u + 1] - lo;
-    std::vector<int> lab;
-    ncl[i] = cluster_bucket(*c, logits.data(), &order[lo], n, u, lab, bcent[i]);
+    std::vector<uint8_t> lab;
+    ncl[i] = cluster_bucket(*c, logits, &order[lo], n, u, fx, lab, bcent[i], bcnt[i]);
     // rows in (label, id) order inside the bucket: stable counting sort
-    std::vector<int64_t> cnt((size_t)ncl[i] + 1, 0);
-    for (int64_t r = 0; r < n; ++r) cnt[lab[r] + 1] += 1;
-    for (int k = 0; k < ncl[i]; ++k) cnt[k + 1] += cnt[k];
-    std::vector<int64_t> tmp((size_t)n);
-    std::vector<int> tl((size_t)n);
-    for (int64_t r = 0; r < n; ++r) {
-      int64_t p = cnt[lab[r]]++;
-      tmp[p] = order[lo + r];
-      tl[p] = lab[r];
-    }
-    for (int64_t r = 0; r < n; ++r) {
-      order[lo + r] = tmp[r];
-      label[lo + r] = tl[r];
-    }
+    std::vector<int64_t> pos((size_t)ncl[i] + 1, 0);
+    for (int k = 0; k < ncl[i]; ++k) pos[k + 1] = pos[k] + bcnt[i][k];
+    std::vector<uint32_t> tmp((size_t)n);
+    for (int64_t r = 0; r < n; ++r) tmp[pos[lab[r]]++] = order[lo + r];
+    memcpy(&order[lo], tmp.data(), sizeof(uint32_t) * (size_t)n);
   });
   // 5. two CSR levels
   int64_t n_cl = 0;
@@ -318,12 +396,11 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
     for (size_t u = 0; u < nb; ++u) {
       bkt_off[u] = (uint32_t)cidx;
       if (e < nonempty.size() && nonempty[e] == u) {
-        int64_t lo = bstart[u], n = bstart[u + 1] - lo;
-        int64_t r = 0;
+        int64_t r = bstart[u];
         for (int k = 0; k < ncl[e]; ++k) {
-          cl_off[cidx + k] = (uint32_t)(lo + r);
-          while (r < n && label[lo + r] == k) ++r;
-          for (int j = 0; j < b; ++j) cent[(size_t)(cidx + k) * b + j] = bcent[e][(size_t)k * b + j];
+          cl_off[cidx + k] = (uint32_t)r;
+          r += bcnt[e][k];
+          memcpy(&cent[(size_t)(cidx + k) * b], &bcent[e][(size_t)k * b], sizeof(float) * b);
         }
         cidx += ncl[e];
         ++e;
@@ -332,8 +409,7 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
     bkt_off[nb] = (uint32_t)cidx;
     cl_off[n_cl] = (uint32_t)N;
   }
-  std::vector<uint32_t> ids((size_t)N);
-  for (int64_t r = 0; r < N; ++r) ids[r] = (uint32_t)order[r];
+  const std::vector<uint32_t> &ids = order;
   // 6. write
   FILE *f = fopen(path, "wb");
   if (!f) return -2;
@@ -406,6 +482,21 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
     info_out[4] = nsingle;
   }
   return 0;
+}
+
+// Build the index over base x [N x D] with the builder's fp32 encoder and
+// write it to path (nrb_build_logits on the encoded base).
+int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, const float *b1,
+              const float *W2, const float *b2, const char *path, int nthreads, int64_t *info_out) {
+  if (!c || !x || N < 1 || N >= (int64_t)0xFFFFFFFFll || c->b < 1 || c->b > 24) return -1;
+  std::vector<float> logits;
+  try {
+    logits.resize((size_t)N * c->b);
+  } catch (...) {
+    return -1;
+  }
+  nrb_encode(c, x, N, W1, b1, W2, b2, logits.data(), nthreads);
+  return nrb_build_logits(c, x, N, logits.data(), W1, b1, W2, b2, path, nthreads, info_out);
 }
 
 }  // extern "C"
