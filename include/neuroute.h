@@ -114,6 +114,12 @@ void nr_index_free(nr_index *ix);
 /* info[0..7] = N, D, H, b, n_clusters, dtype (0 uint8, 1 fp32), K_max, t */
 nr_status nr_index_info(const nr_index *ix, int64_t *info);
 
+/* Write the index to `path` in the file format above (the bytes nr_index_load
+ * reads back). Waits for the device to finish its work first, then copies the
+ * sections out through a pinned buffer. Errors: NR_ERR_IO (open or write),
+ * NR_ERR_OOM, NR_ERR_CUDA. A failed call may leave a partial file. */
+nr_status nr_index_save(nr_index *ix, const char *path);
+
 /* Validate and set the query-time knobs (p = NULL restores the defaults).
  * NR_ERR_INVALID_ARG if a field is out of range. */
 nr_status nr_set_params(nr_index *ix, const nr_params *p);

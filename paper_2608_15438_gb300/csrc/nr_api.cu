@@ -131,6 +131,64 @@ static nr_index_ext *ext_of(nr_index *ix) { return &reinterpret_cast<nr_index_fu
 
 const uint8_t *nr_single_table(nr_index *ix) { return ext_of(ix)->single; }
 
+nr_index *nr_index_alloc() {
+  auto *full = new (std::nothrow) nr_index_full();
+  if (!full) return nullptr;
+  nr_params_default(&full->ix.params);
+  return &full->ix;
+}
+
+void nr_index_set_single(nr_index *ix, uint8_t *d_single) { ext_of(ix)->single = d_single; }
+
+nr_status nr_index_init_device(nr_index *ix) {
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, ix->device) != cudaSuccess) {
+    cudaGetLastError();
+    return NR_ERR_CUDA;
+  }
+  ix->num_sms = prop.multiProcessorCount;
+  if (cudaMalloc((void **)&ix->d_err, 16) != cudaSuccess) {
+    cudaGetLastError();
+    ix->d_err = nullptr;
+    return NR_ERR_OOM;
+  }
+  if (cudaMemset(ix->d_err, 0, 16) != cudaSuccess) return NR_ERR_CUDA;
+  return NR_OK;
+}
+
+nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1, const float *W2,
+                                  const float *b2) {
+  const int D = ix->D, H = ix->H, b = ix->b;
+  auto up = [&](void **dptr, const void *src, size_t bytes) -> nr_status {
+    if (cudaMalloc(dptr, bytes > 0 ? bytes : 16) != cudaSuccess) {
+      cudaGetLastError();
+      *dptr = nullptr;
+      return NR_ERR_OOM;
+    }
+    if (src && bytes && cudaMemcpy(*dptr, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess)
+      return NR_ERR_CUDA;
+    return NR_OK;
+  };
+  std::vector<float> W1T((size_t)D * H);
+  for (int u = 0; u < H; ++u)
+    for (int j = 0; j < D; ++j) W1T[(size_t)j * H + u] = W1[(size_t)u * D + j];
+  // fp16 operands of the tensor-core encoder; layer 2 padded to 16 or 32 rows
+  const int n2 = b <= 16 ? 16 : 32;
+  std::vector<__half> w1h((size_t)H * D), w2h((size_t)n2 * H, __float2half_rn(0.0f));
+  for (size_t i = 0; i < w1h.size(); ++i) w1h[i] = __float2half_rn(W1[i]);
+  for (int o = 0; o < b; ++o)
+    for (int u = 0; u < H; ++u) w2h[(size_t)o * H + u] = __float2half_rn(W2[(size_t)o * H + u]);
+  nr_status st;
+  if ((st = up((void **)&ix->W1, W1, (size_t)H * D * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->b1, b1, (size_t)H * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->W2, W2, (size_t)b * H * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->b2, b2, (size_t)b * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->W1T, W1T.data(), W1T.size() * 4)) != NR_OK) return st;
+  if ((st = up(&ix->W1h, w1h.data(), w1h.size() * 2)) != NR_OK) return st;
+  if ((st = up(&ix->W2h, w2h.data(), w2h.size() * 2)) != NR_OK) return st;
+  return NR_OK;
+}
+
 extern "C" {
 
 const char *nr_status_string(nr_status s) {
@@ -202,12 +260,11 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
     fclose(f);
     return NR_ERR_FORMAT;
   }
-  auto *full = new (std::nothrow) nr_index_full();
-  if (!full) {
+  nr_index *ix = nr_index_alloc();
+  if (!ix) {
     fclose(f);
     return NR_ERR_OOM;
   }
-  nr_index *ix = &full->ix;
   ix->device = device;
   ix->dtype = (int)rd32(h, 12);
   ix->N = (int64_t)rd64(h, 16);
@@ -218,7 +275,6 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   ix->t = (int)rd32(h, 40);
   ix->n_cl = (int64_t)rd64(h, 48);
   memcpy(&ix->in_scale, h + 56, 4);
-  nr_params_default(&ix->params);
   uint64_t off[10];
   for (int i = 0; i < 10; ++i) off[i] = rd64(h, 64 + 8 * i);
   const size_t esz = ix->dtype == 0 ? 1 : 4;
@@ -263,12 +319,10 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   }
   if (ix->K_max < 1) ix->K_max = kmax_dir;
   DeviceGuard g(device);
-  cudaDeviceProp prop;
-  if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) return bad(NR_ERR_CUDA);
-  ix->num_sms = prop.multiProcessorCount;
-  std::vector<float> W1T((size_t)ix->D * ix->H);
-  for (int u = 0; u < ix->H; ++u)
-    for (int j = 0; j < ix->D; ++j) W1T[(size_t)j * ix->H + u] = W1[(size_t)u * ix->D + j];
+  nr_status st = nr_index_init_device(ix);
+  if (st != NR_OK) return bad(st);
+  if ((st = nr_index_upload_encoder(ix, W1.data(), b1.data(), W2.data(), b2.data())) != NR_OK)
+    return bad(st);
   auto up = [&](void **dptr, const void *src, size_t bytes) -> nr_status {
     if (cudaMalloc(dptr, bytes > 0 ? bytes : 16) != cudaSuccess) {
       cudaGetLastError();
@@ -279,27 +333,9 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
       return NR_ERR_CUDA;
     return NR_OK;
   };
-  nr_status st;
-  if ((st = up((void **)&ix->W1, W1.data(), sz[0])) != NR_OK) return bad(st);
-  if ((st = up((void **)&ix->b1, b1.data(), sz[1])) != NR_OK) return bad(st);
-  if ((st = up((void **)&ix->W2, W2.data(), sz[2])) != NR_OK) return bad(st);
-  if ((st = up((void **)&ix->b2, b2.data(), sz[3])) != NR_OK) return bad(st);
   if ((st = up((void **)&ix->tau, tau.data(), sz[4])) != NR_OK) return bad(st);
-  if ((st = up((void **)&ix->W1T, W1T.data(), sz[0])) != NR_OK) return bad(st);
-  {
-    // fp16 operands of the tensor-core encoder; layer 2 padded to 16 or 32 rows
-    const int n2 = ix->b <= 16 ? 16 : 32;
-    std::vector<__half> w1h((size_t)ix->H * ix->D), w2h((size_t)n2 * ix->H, __float2half_rn(0.0f));
-    for (size_t i = 0; i < w1h.size(); ++i) w1h[i] = __float2half_rn(W1[i]);
-    for (int o = 0; o < ix->b; ++o)
-      for (int u = 0; u < ix->H; ++u) w2h[(size_t)o * ix->H + u] = __float2half_rn(W2[(size_t)o * ix->H + u]);
-    if ((st = up(&ix->W1h, w1h.data(), w1h.size() * 2)) != NR_OK) return bad(st);
-    if ((st = up(&ix->W2h, w2h.data(), w2h.size() * 2)) != NR_OK) return bad(st);
-  }
   if ((st = up((void **)&ix->bkt_off, bkt.data(), sz[5])) != NR_OK) return bad(st);
   if ((st = up((void **)&ext_of(ix)->single, single.data(), single.size())) != NR_OK) return bad(st);
-  if ((st = up((void **)&ix->d_err, nullptr, 16)) != NR_OK) return bad(st);
-  if (cudaMemset(ix->d_err, 0, 16) != cudaSuccess) return bad(NR_ERR_CUDA);
   // large sections streamed through a pinned staging buffer
   const size_t stage_bytes = (size_t)64 << 20;
   void *stage = nullptr;
@@ -332,6 +368,79 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   fclose(f);
   *out = ix;
   return NR_OK;
+}
+
+nr_status nr_index_save(nr_index *ix, const char *path) {
+  if (!ix || !path) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    cudaGetLastError();
+    return NR_ERR_CUDA;
+  }
+  const uint64_t nb = ((uint64_t)1 << ix->b) + 1;
+  const uint64_t sz[10] = {(uint64_t)ix->H * ix->D * 4, (uint64_t)ix->H * 4,
+                           (uint64_t)ix->b * ix->H * 4, (uint64_t)ix->b * 4,
+                           (uint64_t)ix->b * 4,         nb * 4,
+                           (uint64_t)(ix->n_cl + 1) * 4, (uint64_t)ix->n_cl * ix->b * 4,
+                           (uint64_t)ix->N * 4,         (uint64_t)ix->N * ix->row_bytes};
+  const void *src[10] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->bkt_off,
+                         ix->cl_off, ix->cent, ix->ids, ix->vec};
+  uint64_t off[10], cur = 256;
+  for (int i = 0; i < 10; ++i) {
+    off[i] = cur;
+    cur = (cur + sz[i] + 255) & ~(uint64_t)255;
+  }
+  unsigned char h[256];
+  memset(h, 0, sizeof(h));
+  memcpy(h, "NRIXv001", 8);
+  auto w32 = [&](int o, uint32_t v) { memcpy(h + o, &v, 4); };
+  auto w64 = [&](int o, uint64_t v) { memcpy(h + o, &v, 8); };
+  w32(8, 1);
+  w32(12, (uint32_t)ix->dtype);
+  w64(16, (uint64_t)ix->N);
+  w32(24, (uint32_t)ix->D);
+  w32(28, (uint32_t)ix->H);
+  w32(32, (uint32_t)ix->b);
+  w32(36, (uint32_t)ix->K_max);
+  w32(40, (uint32_t)ix->t);
+  w64(48, (uint64_t)ix->n_cl);
+  memcpy(h + 56, &ix->in_scale, 4);
+  for (int i = 0; i < 10; ++i) w64(64 + 8 * i, off[i]);
+  w64(144, cur);
+  FILE *f = fopen(path, "wb");
+  if (!f) return NR_ERR_IO;
+  const size_t stage_bytes = (size_t)64 << 20;
+  void *stage = nullptr;
+  if (cudaMallocHost(&stage, stage_bytes) != cudaSuccess) {
+    cudaGetLastError();
+    fclose(f);
+    return NR_ERR_OOM;
+  }
+  nr_status st = NR_OK;
+  static const unsigned char zeros[256] = {0};
+  uint64_t at = 0;
+  auto put = [&](const void *p, size_t n) {
+    if (st == NR_OK && n && fwrite(p, 1, n, f) != n) st = NR_ERR_IO;
+    at += n;
+  };
+  put(h, 256);
+  for (int i = 0; i < 10 && st == NR_OK; ++i) {
+    put(zeros, (size_t)(off[i] - at));
+    for (uint64_t done = 0; done < sz[i] && st == NR_OK;) {
+      const size_t n = (size_t)((sz[i] - done) < stage_bytes ? (sz[i] - done) : stage_bytes);
+      if (cudaMemcpy(stage, (const char *)src[i] + done, n, cudaMemcpyDeviceToHost) != cudaSuccess) {
+        cudaGetLastError();
+        st = NR_ERR_CUDA;
+        break;
+      }
+      put(stage, n);
+      done += n;
+    }
+  }
+  put(zeros, (size_t)(cur - at));
+  cudaFreeHost(stage);
+  if (fclose(f) != 0 && st == NR_OK) st = NR_ERR_IO;
+  return st;
 }
 
 nr_status nr_index_info(const nr_index *ix, int64_t *info) {

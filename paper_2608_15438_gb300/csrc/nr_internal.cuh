@@ -53,6 +53,16 @@ struct nr_seg {
   uint32_t pos;
 };
 
+// Index object helpers shared by the file loader and the GPU builder
+// (nr_api.cu). The device must be current.
+nr_index *nr_index_alloc();  // zeroed object with default params and host extras
+nr_status nr_index_init_device(nr_index *ix);  // num_sms and the device check flag
+// uploads fp32 W1 [H x D], b1 [H], W2 [b x H], b2 [b] (host) and the encoder's
+// derived forms; needs D, H and b set
+nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1, const float *W2,
+                                  const float *b2);
+void nr_index_set_single(nr_index *ix, uint8_t *d_single);  // takes ownership
+
 // kernel launchers (each returns cudaGetLastError() after the launch)
 bool nr_encode_uses_tensor_cores(const nr_index *ix);
 cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,

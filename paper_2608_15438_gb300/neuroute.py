@@ -22,7 +22,9 @@ STATUS = {0: "NR_OK", -1: "NR_ERR_INVALID_ARG", -2: "NR_ERR_IO", -3: "NR_ERR_FOR
 EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_free",
            "nr_index_info", "nr_set_params", "nr_encode", "nr_route", "nr_debug_clusters",
            "nr_search", "nr_search_logits", "nr_search_host", "nr_query_stats", "nr_last_stats",
-           "nr_enable_timing", "nr_last_timing", "nr_kernel_launches", "nr_search_static"]
+           "nr_enable_timing", "nr_last_timing", "nr_kernel_launches", "nr_search_static",
+           "nr_index_save", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
+           "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free"]
 
 
 class NRError(RuntimeError):
@@ -71,8 +73,18 @@ def lib():
         L.nr_last_timing.argtypes = [vp, vp]
         L.nr_kernel_launches.argtypes = [vp]
         L.nr_kernel_launches.restype = i64
+        L.nr_index_save.argtypes = [vp, ctypes.c_char_p]
+        L.nr_build_begin.argtypes = [vp, i64, vp, vp, vp, vp, i32, ctypes.POINTER(vp)]
+        L.nr_build_encode.argtypes = [vp, vp, i64, i64, vp]
+        L.nr_build_set_logits.argtypes = [vp, vp, i64, i64, vp]
+        L.nr_build_finish.argtypes = [vp, vp]
+        L.nr_build_place.argtypes = [vp, vp, i64, i64, vp]
+        L.nr_build_end.argtypes = [vp, ctypes.POINTER(vp)]
+        L.nr_build_free.argtypes = [vp]
+        L.nr_build_free.restype = None
         for name in EXPORTS:
-            if name not in ("nr_status_string", "nr_index_free", "nr_kernel_launches"):
+            if name not in ("nr_status_string", "nr_index_free", "nr_kernel_launches",
+                            "nr_build_free"):
                 getattr(L, name).restype = i32
         _LIB = L
     return _LIB
@@ -107,9 +119,12 @@ def _stream(stream):
 class Index:
     """A loaded index on one GPU."""
 
-    def __init__(self, path: str, device: int = 0):
-        h = ctypes.c_void_p()
-        _check("nr_index_load", lib().nr_index_load(path.encode(), device, ctypes.byref(h)))
+    def __init__(self, path: str | None, device: int = 0, _handle=None):
+        if _handle is None:
+            h = ctypes.c_void_p()
+            _check("nr_index_load", lib().nr_index_load(path.encode(), device, ctypes.byref(h)))
+        else:
+            h = _handle
         self.h = h
         self.device = device
         info = np.zeros(8, np.int64)
@@ -131,6 +146,10 @@ class Index:
     @property
     def row_bytes(self):
         return self.D * (1 if self.dtype_code == 0 else 4)
+
+    def save(self, path: str):
+        """Write the index file (nr_index_save)."""
+        _check("nr_index_save", lib().nr_index_save(self.h, path.encode()))
 
     def set_params(self, p: Params | None = None, **kw):
         if p is None:
@@ -234,3 +253,58 @@ class Index:
 
     def kernel_launches(self) -> int:
         return int(lib().nr_kernel_launches(self.h))
+
+
+class Builder:
+    """A GPU index build (neuroute_build.h): pass 1 gives every row's logits
+    (encode or set_logits), finish() builds thresholds, codes, clusters and
+    the CSR levels, pass 2 places the rows, end() returns the Index.
+
+    cfg is a ctypes structure with the fields of nr_build_config (the host
+    builder's Config has the same layout); weights = (W1, b1, W2, b2) fp32."""
+
+    def __init__(self, cfg, N: int, weights, device: int = 0):
+        W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights)
+        h = ctypes.c_void_p()
+        _check("nr_build_begin", lib().nr_build_begin(
+            ctypes.byref(cfg), N, W1.ctypes.data, b1.ctypes.data, W2.ctypes.data, b2.ctypes.data,
+            device, ctypes.byref(h)))
+        self.h, self.N, self.device, self.b = h, N, device, cfg.b
+
+    def encode(self, rows, row0: int, stream=None):
+        """Logits of rows [row0, row0 + len(rows)) from a CUDA tensor [n x D]."""
+        _check("nr_build_encode", lib().nr_build_encode(self.h, _ptr(rows), row0, rows.shape[0],
+                                                         _stream(stream)))
+
+    def set_logits(self, logits, row0: int, stream=None):
+        """Given logits [n x b] fp32 (CUDA tensor) of rows [row0, row0 + n)."""
+        _check("nr_build_set_logits", lib().nr_build_set_logits(self.h, _ptr(logits), row0,
+                                                                 logits.shape[0], _stream(stream)))
+
+    def finish(self):
+        info = np.zeros(5, np.int64)
+        _check("nr_build_finish", lib().nr_build_finish(self.h, info.ctypes.data))
+        return {"n_clusters": int(info[0]), "n_buckets": int(info[1]), "max_bucket": int(info[2]),
+                "max_cluster": int(info[3]), "single_cluster_buckets": int(info[4])}
+
+    def place(self, rows, row0: int, stream=None):
+        """Store rows [row0, row0 + len(rows)) from a CUDA tensor [n x D]."""
+        _check("nr_build_place", lib().nr_build_place(self.h, _ptr(rows), row0, rows.shape[0],
+                                                      _stream(stream)))
+
+    def end(self) -> Index:
+        out = ctypes.c_void_p()
+        h, self.h = self.h, None
+        _check("nr_build_end", lib().nr_build_end(h, ctypes.byref(out)))
+        return Index(None, self.device, _handle=out)
+
+    def close(self):
+        if self.h:
+            lib().nr_build_free(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -44,8 +44,28 @@ def lib():
                                        ctypes.c_int64, ctypes.c_void_p]
         L.synth_normal.argtypes = [ctypes.c_uint64, ctypes.c_uint32, ctypes.c_int64,
                                    ctypes.c_double, ctypes.c_void_p]
+        L.synth_centres.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int,
+                                    ctypes.c_void_p]
         _LIB = L
     return _LIB
+
+
+_CUDA_LIB = None
+
+
+def cuda_lib():
+    """The GPU row generator (synth_cuda.cu)."""
+    global _CUDA_LIB
+    if _CUDA_LIB is None:
+        path = os.path.join(_HERE, "libsynth_cuda.so")
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} missing: run __graft_entry__.build() first")
+        L = ctypes.CDLL(path)
+        L.synth_mixture_cuda.argtypes = [ctypes.c_int, ctypes.c_uint64, ctypes.c_int, ctypes.c_int,
+                                         ctypes.c_double, ctypes.c_int64, ctypes.c_int64,
+                                         ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+        _CUDA_LIB = L
+    return _CUDA_LIB
 
 
 def philox4x32_10(ctr, key):
@@ -132,6 +152,44 @@ def components(w: Workload, seed_rows: int, row0: int, n: int) -> np.ndarray:
     out = np.empty(n, dtype=np.int32)
     lib().synth_components(seed_rows, w.mixture, row0, n, out.ctypes.data)
     return out
+
+
+def centres(w: Workload, seed_centres: int = SEED_DATA) -> np.ndarray:
+    """The mixture centres [M x D] (float64) that the rows are drawn around."""
+    out = np.empty((w.mixture, w.dim), np.float64)
+    if lib().synth_centres(w.dtype_code, seed_centres, w.mixture, w.dim, out.ctypes.data) != 0:
+        raise RuntimeError("synth_centres failed")
+    return out
+
+
+class DeviceRows:
+    """Rows of a workload's mixture generated on a GPU (the definition of
+    ``mixture``, computed by synth_cuda.cu), for bases too large for the host."""
+
+    def __init__(self, w: Workload, seed_rows: int = SEED_DATA, seed_centres: int = SEED_DATA,
+                 device: int = 0):
+        import torch
+
+        self.w, self.seed_rows, self.device = w, seed_rows, device
+        self.cent = torch.from_numpy(centres(w, seed_centres)).to(f"cuda:{device}")
+
+    def rows(self, row0: int, n: int, out=None, stream=None):
+        """Rows [row0, row0 + n) as a CUDA tensor [n x D] (uint8 or float32)."""
+        import torch
+
+        w = self.w
+        dt = torch.uint8 if w.dtype == "u8" else torch.float32
+        if out is None:
+            out = torch.empty((n, w.dim), dtype=dt, device=f"cuda:{self.device}")
+        assert out.dtype == dt and out.is_contiguous() and out.shape[0] >= n
+        s = stream if stream is not None else torch.cuda.current_stream(self.device)
+        rc = cuda_lib().synth_mixture_cuda(w.dtype_code, self.seed_rows, w.mixture, w.dim, w.sigma,
+                                           row0, n, ctypes.c_void_p(self.cent.data_ptr()),
+                                           ctypes.c_void_p(out.data_ptr()),
+                                           ctypes.c_void_p(s.cuda_stream))
+        if rc != 0:
+            raise RuntimeError("synth_mixture_cuda failed")
+        return out[:n]
 
 
 def normal(seed: int, stream: int, n: int, scale: float) -> np.ndarray:

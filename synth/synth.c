@@ -228,3 +228,13 @@ int synth_normal(uint64_t seed, uint32_t stream, int64_t n, double scale, float 
   }
   return 0;
 }
+
+/* Mixture centres [M x D] as doubles (kind 0 = u8, 1 = f32), the values every
+ * row generator adds its noise to. */
+int synth_centres(int kind, uint64_t seed_centres, int M, int D, double *out) {
+  if ((kind != 0 && kind != 1) || M < 1 || D < 1 || !out) return -1;
+  for (int64_t m = 0; m < M; ++m)
+    for (int j = 0; j < D; ++j)
+      out[(size_t)m * D + j] = kind == 0 ? centre_u8(seed_centres, m, j) : centre_f32(seed_centres, m, j);
+  return 0;
+}

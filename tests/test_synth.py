@@ -64,3 +64,17 @@ def test_encoder_weights_scale():
     assert abs(W1.std() * np.sqrt(w.dim) - 1.0) < 0.02
     assert abs(W2.std() * np.sqrt(w.hidden) - 1.0) < 0.05
     assert not b1.any() and not b2.any()
+
+
+def test_centres_are_the_rows_centres():
+    """The exported centres are the ones the rows scatter around: the mean of
+    a component's rows approaches its centre (u8: uniform in [20, 235])."""
+    w = synth.WORKLOADS["tiny"]
+    c = synth.centres(w)
+    assert c.shape == (w.mixture, w.dim) and c.min() >= 20.0 and c.max() <= 235.0
+    rows = synth.mixture(w, synth.SEED_DATA, 0, 20_000).astype(np.float64)
+    comp = synth.components(w, synth.SEED_DATA, 0, 20_000)
+    for m in range(3):
+        sel = rows[comp == m]
+        assert len(sel) > 30
+        assert np.abs(sel.mean(0) - c[m]).max() < 5 * w.sigma / np.sqrt(len(sel)) + 1.0
