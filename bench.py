@@ -3,7 +3,7 @@
 One step = one nr_search call over the workload's whole query batch (encode,
 route, select, refine) with the index and the queries resident in HBM.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload u8-10m]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload u8-1b]
                   [--P 64 --C 128 --t-low 4] [--impl neuroute|reference] [--sweep]
 
 Prints one JSON line (rank 0). Metric: queries per second at the workload's
@@ -38,6 +38,7 @@ OPERATING_POINTS = {
     "u8-10m": (256, 256, 0, 4.0),
     "f32-10m": (512, 256, 16, None),
     "u8-100m": (1024, 256, 32, None),
+    "u8-1b": (1024, 1024, 64, 4.0),
 }
 
 
@@ -55,7 +56,7 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", default="u8-10m")
+    ap.add_argument("--workload", default="u8-1b")
     ap.add_argument("--P", type=int, default=None)
     ap.add_argument("--C", type=int, default=None)
     ap.add_argument("--t-low", type=int, default=None)
@@ -65,7 +66,11 @@ def parse():
     ap.add_argument("--sweep", action="store_true")
     ap.add_argument("--sweep-gate", action="store_true",
                     help="sweep the centroid gate M(x) = m1 x around the (P, C) grid")
-    ap.add_argument("--index", default=None, help="reuse an index file")
+    ap.add_argument("--grid", default=None,
+                    help="sweep grid 'P=..;C=..;t_low=..;m1=..' (comma lists, m1 'none' = gate off)")
+    ap.add_argument("--index", default=None, help="reuse an index file (host builder)")
+    ap.add_argument("--builder", default="gpu", choices=["gpu", "host"],
+                    help="build the index on the GPU from generated rows (default) or on the host")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-gt", action="store_true", help="skip ground truth (profiling runs)")
     ap.add_argument("--encode", type=int, default=0,
@@ -172,6 +177,94 @@ def build_or_load_index(w, path, rank, world):
     return path
 
 
+def gpu_index(w, torch, nr, dev):
+    """The workload's index built on the GPU (neuroute_build.h) from rows that
+    the GPU generator draws twice: once to encode, once to store."""
+    import synth
+    from paper_2608_15438_gb300.builder import config
+
+    d = dev.index or 0
+    gen = synth.DeviceRows(w, synth.SEED_DATA, device=d)
+    bd = nr.Builder(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t), w.n,
+                    synth.encoder_weights(w), d)
+    chunk = min(w.n, (4 << 30) // w.row_bytes)
+    buf = torch.empty((chunk, w.dim), dtype=torch.uint8 if w.dtype == "u8" else torch.float32,
+                      device=dev)
+    for r0 in range(0, w.n, chunk):
+        m = min(chunk, w.n - r0)
+        bd.encode(gen.rows(r0, m, out=buf), r0)
+    torch.cuda.synchronize()
+    info = bd.finish()
+    for r0 in range(0, w.n, chunk):
+        m = min(chunk, w.n - r0)
+        bd.place(gen.rows(r0, m, out=buf), r0)
+    ix = bd.end()
+    del buf
+    torch.cuda.empty_cache()
+    return ix, info
+
+
+def ground_truth_rows(torch, w, dq, k, dev, chunk=1 << 22, qblock=2500, group=1024):
+    """Exact k-NN of the queries over the whole base, rows regenerated on the
+    GPU chunk by chunk. Distances are |x|^2 - 2 q.x (the query norm does not
+    change the order); for uint8 rows every product and partial sum is an
+    integer below 2^24, so the TF32 tensor-core matmul is exact. Per chunk the
+    k nearest rows lie in the k groups of `group` rows with the smallest
+    minimum distance, so the top-k runs only over those groups."""
+    import synth
+
+    gen = synth.DeviceRows(w, synth.SEED_DATA, device=dev.index or 0)
+    Q = dq.float()
+    nq = Q.shape[0]
+    best_d = torch.full((nq, k), float("inf"), device=dev)
+    best_i = torch.full((nq, k), -1, dtype=torch.int64, device=dev)
+    tf32 = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = w.dtype == "u8"
+    try:
+        for r0 in range(0, w.n, chunk):
+            m = min(chunk, w.n - r0)
+            X = gen.rows(r0, m).float()
+            bn = (X * X).sum(1)
+            for q0 in range(0, nq, qblock):
+                q1 = min(nq, q0 + qblock)
+                dmat = bn[None, :] - 2.0 * (Q[q0:q1] @ X.T)
+                if m % group == 0 and m // group > k:
+                    g = dmat.view(q1 - q0, m // group, group)
+                    top_g = torch.topk(g.amin(2), k, dim=1, largest=False).indices
+                    cand = torch.gather(g, 1, top_g[:, :, None].expand(-1, -1, group))
+                    v, i = torch.topk(cand.reshape(q1 - q0, -1), k, dim=1, largest=False)
+                    i = torch.gather(top_g, 1, i // group) * group + i % group
+                else:
+                    v, i = torch.topk(dmat, min(k, m), dim=1, largest=False)
+                cv = torch.cat([best_d[q0:q1], v], 1)
+                ci = torch.cat([best_i[q0:q1], i + r0], 1)
+                vv, ii = torch.topk(cv, k, dim=1, largest=False)
+                best_d[q0:q1] = vv
+                best_i[q0:q1] = torch.gather(ci, 1, ii)
+                del dmat
+            del X
+        torch.cuda.synchronize()
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = tf32
+    return best_i.cpu().numpy()
+
+
+def oracle_subindex(w, ix, qs, P, kw, path):
+    """Sub-index of the buckets that the oracle probes for queries qs: the
+    oracle's own logits (double-precision encoder) and probe lists pick the
+    codes, the library copies those buckets out (nr_index_extract). The oracle
+    then answers these queries on the file exactly as on the whole index."""
+    import oracle
+    import synth
+
+    lg = oracle.encode_weights(synth.encoder_weights(w), w.in_scale, qs)
+    tau = ix.thresholds()
+    p = oracle.params(**kw)
+    codes = np.concatenate([oracle.probe_list(lg[i], tau, P, p)[0] for i in range(len(qs))])
+    rows, _ = ix.extract(codes, path)
+    return lg, rows
+
+
 def ground_truth(torch, base_t, q_t, k, dtype):
     """Exact k-NN by brute force on the GPU (torch fp32 matmul; exact for uint8
     data, whose dot products and norms are integers below 2^24)."""
@@ -242,6 +335,54 @@ def cpu_baseline(w, path, queries, k, P, C, t_low, seconds, truth=None):
     return res, ids
 
 
+def calibrate_subindex(w, ix, queries, k, P, C, kw, seconds, path, row_budget):
+    """Number of queries whose oracle run takes about `seconds` on the host
+    cores, bounded by the query count and by a sub-index of at most
+    row_budget rows (estimated from the first 16 queries)."""
+    import oracle
+
+    n = min(16, len(queries))
+    lg, rows = oracle_subindex(w, ix, queries[:n], P, kw, path)
+    orc = oracle.Index(path)
+    t = time.perf_counter()
+    orc.search(queries[:n], k, P, C, oracle.params(**kw), logits=lg, nthreads=os.cpu_count() or 1)
+    dt = max(time.perf_counter() - t, 1e-6)
+    orc.close()
+    per_q = max(1.0, rows / n)
+    return int(min(len(queries), max(n, row_budget / per_q), max(n, n * seconds / dt)))
+
+
+def cpu_baseline_subindex(w, ix, queries, k, P, C, t_low, seconds, row_budget=100_000_000):
+    """The oracle timed on the host cores for a bounded query sample, on the
+    sub-index of the buckets those queries probe (the index may be too large
+    for host memory)."""
+    import oracle
+
+    kw = op_params(w)
+    kw["t_low"] = t_low
+    p = oracle.params(**kw)
+    cores = os.cpu_count() or 1
+    with tempfile.TemporaryDirectory() as td:
+        sub = os.path.join(td, "sub.nrix")
+        n2 = calibrate_subindex(w, ix, queries, k, P, C, kw, seconds, sub, row_budget)
+        _, rows = oracle_subindex(w, ix, queries[:n2], P, kw, sub)
+        orc = oracle.Index(sub)
+        t = time.perf_counter()
+        orc.search(queries[:n2], k, P, C, p, nthreads=cores)
+        dt1 = max(time.perf_counter() - t, 1e-6)
+        # repeat the sample (when the sub-index bound limits it) to about `seconds`
+        reps = int(max(1, min(50, seconds / dt1)))
+        t = time.perf_counter()
+        for _ in range(reps):
+            orc.search(queries[:n2], k, P, C, p, nthreads=cores)
+        dt2 = time.perf_counter() - t
+        orc.close()
+    return {"value": n2 * reps / dt2, "unit": "queries/s", "cores": cores, "kind": "oracle",
+            "sample": f"first {n2} of {len(queries)} queries of {w.name} (oracle encoder included), "
+                      f"{reps} passes, P={P} C={C} t_low={t_low}, {cores} threads, {dt2:.1f} s, on "
+                      f"the {rows}-row sub-index of the buckets they probe"}
+
+
 def run_reference(args, w, rank, world):
     """The oracle timed on the host cores (the CPU reference arm)."""
     if rank != 0:
@@ -249,13 +390,42 @@ def run_reference(args, w, rank, world):
     import synth
 
     P, C, t_low = op_point(args, w)
-    path = args.index or index_path(w)
-    build_or_load_index(w, path, 0, 1)
     nq = args.nq or w.nq
     qs = synth.queries(w, nq)
     import oracle
 
+    tmpdir = None
+    if args.builder == "gpu" and not args.index:
+        # the index is built on the GPU (setup, outside the timed region); the
+        # oracle answers a bounded query sample from the sub-index of the
+        # buckets those queries probe
+        import torch
+
+        import __graft_entry__
+
+        __graft_entry__.build()
+        from paper_2608_15438_gb300 import neuroute as nr
+
+        dev = torch.device("cuda", 0)
+        gix, _ = gpu_index(w, torch, nr, dev)
+        kw0 = op_params(w)
+        kw0["t_low"] = t_low
+        tmpdir = tempfile.TemporaryDirectory()
+        path = os.path.join(tmpdir.name, "sub.nrix")
+        per_step = max(8.0, 120.0 / max(1, args.steps + args.warmup))
+        nsub = calibrate_subindex(w, gix, qs, args.k, P, C, kw0, per_step, path, 100_000_000)
+        oracle_subindex(w, gix, qs[:nsub], P, kw0, path)
+        gix.close()
+        del gix
+        torch.cuda.empty_cache()
+        qs = qs[:nsub]
+        nq = nsub
+    else:
+        path = args.index or index_path(w)
+        build_or_load_index(w, path, 0, 1)
     orc = oracle.Index(path)
+    note = ("; sub-index of the buckets these queries probe, index built on the GPU"
+            if tmpdir is not None else "")
     kw = op_params(w)
     kw["t_low"] = t_low
     p = oracle.params(**kw)
@@ -281,21 +451,26 @@ def run_reference(args, w, rank, world):
             "vs_baseline": None, "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
             "config": {"workload": w.name, "nq_per_step": ns, "P": P, "C": C, "t_low": t_low, "k": args.k},
             "cpu_baseline": {"value": v, "unit": "queries/s", "cores": cores, "kind": "oracle",
-                             "sample": f"first {ns} of {nq} queries per step"},
+                             "sample": f"first {ns} of {nq} queries per step{note}"},
             "e2e": {"value": v, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+    orc.close()
+    if tmpdir is not None:
+        tmpdir.cleanup()
     return 0
 
 
 def encode_bench(args, w, torch, nr, dev):
     """Throughput of the encoder (K1, tensor cores) over a batch of base
     vectors, the operation an index build runs over the whole base."""
-    path = args.index or index_path(w)
-    build_or_load_index(w, path, 0, 1)
-    ix = nr.Index(path, dev.index or 0)
+    import dataclasses
+
     import synth
 
-    x = torch.from_numpy(synth.base(w, args.encode)).to(dev)
+    # the encoder does not depend on the index contents: a small index over
+    # the workload's first rows carries the same weights
+    ix, _ = gpu_index(dataclasses.replace(w, n=min(w.n, 100_000)), torch, nr, dev)
+    x = synth.DeviceRows(w, synth.SEED_DATA, device=dev.index or 0).rows(0, args.encode)
     out = torch.empty((args.encode, w.bits), dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
     L = nr.lib()
@@ -365,11 +540,17 @@ def main():
         return encode_bench(args, w, torch, nr, dev)
     P, C, t_low = op_point(args, w)
     k = args.k
-    path = args.index or index_path(w)
+    gpu_built = args.builder == "gpu" and not args.index
     t0 = time.time()
-    build_or_load_index(w, path, rank, world)
+    if gpu_built:
+        path = None
+        ix, build_info = gpu_index(w, torch, nr, dev)
+    else:
+        path = args.index or index_path(w)
+        build_or_load_index(w, path, rank, world)
+        ix = nr.Index(path, local)
+        build_info = None
     t_build = time.time() - t0
-    ix = nr.Index(path, local)
     nq = args.nq or w.nq
     # each rank searches its own batch of the query distribution
     qs = synth.mixture(w, synth.SEED_QUERIES, rank * nq, nq)
@@ -380,19 +561,43 @@ def main():
 
     # ground truth (outside any timed region)
     truth = None
+    t0 = time.time()
     if not args.no_gt:
-        base_np = synth.base(w)
-        base_t = torch.from_numpy(base_np).to(dev)
-        del base_np
-        truth = ground_truth(torch, base_t, dq, k, w.dtype)
-        del base_t
+        if gpu_built:
+            truth = ground_truth_rows(torch, w, dq, k, dev)
+        else:
+            base_np = synth.base(w)
+            base_t = torch.from_numpy(base_np).to(dev)
+            del base_np
+            truth = ground_truth(torch, base_t, dq, k, w.dtype)
+            del base_t
         torch.cuda.empty_cache()
+    t_gt = time.time() - t0
+    print(json.dumps({"setup_s": {"index_build": round(t_build, 2), "ground_truth": round(t_gt, 2)},
+                      "index": build_info, "n_clusters": ix.n_clusters}), file=sys.stderr, flush=True)
 
-    if args.sweep_gate:
-        for Pp in (128, 256, 512):
-            for Cc in (128, 256, 1024):
-                for tl in (0, 32, 64):
-                    for m1 in (None, 0.5, 1.0, 2.0, 4.0):
+    if args.sweep or args.sweep_gate or args.grid:
+        if args.grid:
+            g = dict(part.split("=") for part in args.grid.split(";"))
+            grid_p = [int(v) for v in g.get("P", "256").split(",")]
+            grid_c = [int(v) for v in g.get("C", "256").split(",")]
+            grid_t = [int(v) for v in g.get("t_low", "0").split(",")]
+            grid_m = [None if v == "none" else float(v) for v in g.get("m1", "none").split(",")]
+        elif args.sweep_gate:
+            grid_p, grid_c, grid_t, grid_m = (128, 256, 512), (128, 256, 1024), (0, 32, 64), \
+                (None, 0.5, 1.0, 2.0, 4.0)
+        else:
+            grid_p = (64, 128, 256, 512, 1024) if w.bits <= 20 else (256, 512, 1024)
+            grid_c = (256, 512, 1024, 2048) if w.bits <= 20 else (256, 1024)
+            if w.k_max == 1:  # no bucket-local clustering: C never binds
+                grid_p, grid_c = (64, 128, 256, 512, 1024, 2048), (256,)
+            grid_t, grid_m = (0, 8, 16, 32, 64), (None,)
+        for Pp in grid_p:
+            for Cc in grid_c:
+                if Pp * ix.k_max > 16384:
+                    continue
+                for tl in grid_t:
+                    for m1 in grid_m:
                         kw = {"t_low": tl}
                         if m1 is not None:
                             kw.update(gate_m0=0.0, gate_m1=m1)
@@ -406,31 +611,8 @@ def main():
                         st = ix.last_stats()
                         print(json.dumps({"P": Pp, "C": Cc, "t_low": tl, "gate_m1": m1,
                                           "recall": recall_at(ids.cpu().numpy(), truth, k),
-                                          "qps": nq / el, "cand_per_q": st.candidates / nq}), flush=True)
-        return 0
-
-    if args.sweep:
-        rows = []
-        grid_p = (64, 128, 256, 512, 1024) if w.bits <= 20 else (256, 512, 1024)
-        grid_c = (256, 512, 1024, 2048) if w.bits <= 20 else (256, 1024)
-        if w.k_max == 1:  # no bucket-local clustering: C never binds
-            grid_p, grid_c = (64, 128, 256, 512, 1024, 2048), (256,)
-        for Pp in grid_p:
-            for Cc in grid_c:
-                if Pp * ix.k_max > 16384:
-                    continue
-                for tl in (0, 8, 16, 32, 64):
-                    ix.set_params(t_low=tl)
-                    ix.search(dq, k, Pp, Cc, out=(ids, dd))
-                    torch.cuda.synchronize()
-                    t = time.perf_counter()
-                    ix.search(dq, k, Pp, Cc, out=(ids, dd))
-                    torch.cuda.synchronize()
-                    el = time.perf_counter() - t
-                    st = ix.last_stats()
-                    rows.append({"P": Pp, "C": Cc, "t_low": tl, "recall": recall_at(ids.cpu().numpy(), truth, k),
-                                 "qps": nq / el, "cand_per_q": st.candidates / nq})
-                    print(json.dumps(rows[-1]), flush=True)
+                                          "qps": nq / el, "cand_per_q": st.candidates / nq}),
+                              flush=True)
         return 0
 
     kw = op_params(w)
@@ -519,11 +701,16 @@ def main():
                 "d2h_bytes_per_step": nq * k * 12},
         "gpu_launches": launches,
         "clocks": clk.summary(),
-        "index_build_s": t_build,
+        "setup_s": {"index_build": t_build, "ground_truth": t_gt},
+        "index": {"builder": "gpu" if gpu_built else "host", "n_clusters": ix.n_clusters,
+                  **({} if build_info is None else build_info)},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cb, _ = cpu_baseline(w, path, qs, k, P, C, t_low, args.cpu_seconds)
-        out["cpu_baseline"] = cb
+        if gpu_built:
+            out["cpu_baseline"] = cpu_baseline_subindex(w, ix, qs, k, P, C, t_low, args.cpu_seconds)
+        else:
+            cb, _ = cpu_baseline(w, path, qs, k, P, C, t_low, args.cpu_seconds)
+            out["cpu_baseline"] = cb
     if rank == 0:
         print(json.dumps(out), flush=True)
     ix.close()

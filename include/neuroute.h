@@ -114,11 +114,28 @@ void nr_index_free(nr_index *ix);
 /* info[0..7] = N, D, H, b, n_clusters, dtype (0 uint8, 1 fp32), K_max, t */
 nr_status nr_index_info(const nr_index *ix, int64_t *info);
 
+/* Copy the per-bit thresholds tau [b] (Sec. 3.2.3) to host memory h_tau.
+ * Synchronous. Errors: NR_ERR_INVALID_ARG, NR_ERR_CUDA. */
+nr_status nr_index_thresholds(nr_index *ix, float *h_tau);
+
 /* Write the index to `path` in the file format above (the bytes nr_index_load
  * reads back). Waits for the device to finish its work first, then copies the
  * sections out through a pinned buffer. Errors: NR_ERR_IO (open or write),
  * NR_ERR_OOM, NR_ERR_CUDA. A failed call may leave a partial file. */
 nr_status nr_index_save(nr_index *ix, const char *path);
+
+/* Write to `path` a sub-index that holds only the buckets of the listed codes
+ * (every other bucket empty), in the file format above. Clusters and rows keep
+ * their order, so a query whose probe codes all lie in the list gets exactly
+ * the results and statistics it gets from the whole index (cluster ties are
+ * broken by cluster order, which is kept); it serves to check or time a CPU
+ * evaluation of sample queries against an index too large for host memory.
+ * h_codes: n host u32 codes < 2^b, any order, repeats allowed. info[0..1]
+ * (may be NULL) = rows and clusters written. Errors: NR_ERR_INVALID_ARG (a code
+ * out of range, or no row selected), NR_ERR_DEVICE_CHECK (inconsistent
+ * offsets), NR_ERR_IO, NR_ERR_OOM, NR_ERR_CUDA. */
+nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, const char *path,
+                           int64_t *info);
 
 /* Validate and set the query-time knobs (p = NULL restores the defaults).
  * NR_ERR_INVALID_ARG if a field is out of range. */

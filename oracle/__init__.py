@@ -41,6 +41,9 @@ def lib():
             getattr(L, name).argtypes = [vp]
             getattr(L, name).restype = vp
         L.or_encode.argtypes = [vp, vp, i64, vp, i32]
+        L.or_encode_weights.argtypes = [i32, i32, i32, i32, ctypes.c_float, vp, vp, vp, vp, vp, i64,
+                                        vp, i32]
+        L.or_encode_weights.restype = None
         L.or_probe_order.argtypes = [i32, vp, i32, ctypes.POINTER(Params), vp]
         L.or_probe_order.restype = i32
         L.or_probe_order_allsubsets.argtypes = [i32, vp, i32, ctypes.POINTER(Params), vp]
@@ -154,6 +157,19 @@ class Index:
         if rc != 0:
             raise RuntimeError("oracle: out-of-range index in file")
         return ids, d, st
+
+
+def encode_weights(weights, in_scale: float, x: np.ndarray, nthreads=None) -> np.ndarray:
+    """Logits of rows x under the encoder (W1, b1, W2, b2), without an index."""
+    W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights)
+    x = np.ascontiguousarray(x)
+    H, D = W1.shape
+    b = W2.shape[0]
+    out = np.empty((x.shape[0], b), np.float32)
+    lib().or_encode_weights(0 if x.dtype == np.uint8 else 1, D, H, b, in_scale, W1.ctypes.data,
+                            b1.ctypes.data, W2.ctypes.data, b2.ctypes.data, x.ctypes.data,
+                            x.shape[0], out.ctypes.data, nthreads or nthreads_default())
+    return out
 
 
 def probe_order(sd, P, p: Params):

@@ -183,6 +183,22 @@ extern "C" void or_encode(const or_index *ix, const void *x, int64_t nq, float *
   parallel_for(nq, nthreads, [&](int64_t i) { encode_one(ix, x, i, logits + (size_t)i * ix->b); });
 }
 
+extern "C" void or_encode_weights(int dtype, int D, int H, int b, float in_scale, const float *W1,
+                                  const float *b1, const float *W2, const float *b2, const void *x,
+                                  int64_t nq, float *logits, int nthreads) {
+  or_index e;  // an index holding only the encoder
+  e.dtype = dtype;
+  e.D = D;
+  e.H = H;
+  e.b = b;
+  e.in_scale = in_scale;
+  e.W1.assign(W1, W1 + (size_t)H * D);
+  e.b1.assign(b1, b1 + H);
+  e.W2.assign(W2, W2 + (size_t)b * H);
+  e.b2.assign(b2, b2 + b);
+  or_encode(&e, x, nq, logits, nthreads);
+}
+
 // ---------------------------------------------------------------- probe order
 // Algorithm 1: flip sets F over the least-certain bits, scored by the summed
 // deviation s = sum_{r in F} delta. Key = (cost, |F|, rank mask), cost added in

@@ -73,6 +73,11 @@ const float *or_index_cent(const or_index *ix);
 
 /* logits [nq x b] (fp32, rounded from a double-precision forward pass) */
 void or_encode(const or_index *ix, const void *x, int64_t nq, float *logits, int nthreads);
+/* the same forward pass from explicit weights W1 [H x D], b1 [H], W2 [b x H],
+ * b2 [b] (dtype 0 uint8 rows, 1 fp32 rows; inputs scaled by in_scale) */
+void or_encode_weights(int dtype, int D, int H, int b, float in_scale, const float *W1,
+                       const float *b1, const float *W2, const float *b2, const void *x,
+                       int64_t nq, float *logits, int nthreads);
 
 /* Probe order from a per-rank deviation vector sd[0..b-1] (sd sorted ascending
  * is NOT required here; rank r has cost sd[r]). Best-first over "add one rank"

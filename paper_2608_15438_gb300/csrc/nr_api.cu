@@ -6,6 +6,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <cmath>
 #include <new>
 #include <vector>
@@ -370,21 +371,20 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   return NR_OK;
 }
 
-nr_status nr_index_save(nr_index *ix, const char *path) {
-  if (!ix || !path) return NR_ERR_INVALID_ARG;
-  DeviceGuard g(ix->device);
-  if (cudaDeviceSynchronize() != cudaSuccess) {
-    cudaGetLastError();
-    return NR_ERR_CUDA;
-  }
+}  // extern "C"
+
+namespace {
+
+// Writes an index file: header fields from `ix` with N and n_cl given, the
+// ten sections from src[i] (device memory where dev[i], else host memory).
+nr_status write_nrix(const nr_index *ix, int64_t N, int64_t n_cl, const void *const src[10],
+                     const bool dev[10], const char *path) {
   const uint64_t nb = ((uint64_t)1 << ix->b) + 1;
   const uint64_t sz[10] = {(uint64_t)ix->H * ix->D * 4, (uint64_t)ix->H * 4,
                            (uint64_t)ix->b * ix->H * 4, (uint64_t)ix->b * 4,
                            (uint64_t)ix->b * 4,         nb * 4,
-                           (uint64_t)(ix->n_cl + 1) * 4, (uint64_t)ix->n_cl * ix->b * 4,
-                           (uint64_t)ix->N * 4,         (uint64_t)ix->N * ix->row_bytes};
-  const void *src[10] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->bkt_off,
-                         ix->cl_off, ix->cent, ix->ids, ix->vec};
+                           (uint64_t)(n_cl + 1) * 4,    (uint64_t)n_cl * ix->b * 4,
+                           (uint64_t)N * 4,             (uint64_t)N * ix->row_bytes};
   uint64_t off[10], cur = 256;
   for (int i = 0; i < 10; ++i) {
     off[i] = cur;
@@ -397,13 +397,13 @@ nr_status nr_index_save(nr_index *ix, const char *path) {
   auto w64 = [&](int o, uint64_t v) { memcpy(h + o, &v, 8); };
   w32(8, 1);
   w32(12, (uint32_t)ix->dtype);
-  w64(16, (uint64_t)ix->N);
+  w64(16, (uint64_t)N);
   w32(24, (uint32_t)ix->D);
   w32(28, (uint32_t)ix->H);
   w32(32, (uint32_t)ix->b);
   w32(36, (uint32_t)ix->K_max);
   w32(40, (uint32_t)ix->t);
-  w64(48, (uint64_t)ix->n_cl);
+  w64(48, (uint64_t)n_cl);
   memcpy(h + 56, &ix->in_scale, 4);
   for (int i = 0; i < 10; ++i) w64(64 + 8 * i, off[i]);
   w64(144, cur);
@@ -426,6 +426,10 @@ nr_status nr_index_save(nr_index *ix, const char *path) {
   put(h, 256);
   for (int i = 0; i < 10 && st == NR_OK; ++i) {
     put(zeros, (size_t)(off[i] - at));
+    if (!dev[i]) {
+      put(src[i], (size_t)sz[i]);
+      continue;
+    }
     for (uint64_t done = 0; done < sz[i] && st == NR_OK;) {
       const size_t n = (size_t)((sz[i] - done) < stage_bytes ? (sz[i] - done) : stage_bytes);
       if (cudaMemcpy(stage, (const char *)src[i] + done, n, cudaMemcpyDeviceToHost) != cudaSuccess) {
@@ -441,6 +445,124 @@ nr_status nr_index_save(nr_index *ix, const char *path) {
   cudaFreeHost(stage);
   if (fclose(f) != 0 && st == NR_OK) st = NR_ERR_IO;
   return st;
+}
+
+}  // namespace
+
+extern "C" {
+
+nr_status nr_index_save(nr_index *ix, const char *path) {
+  if (!ix || !path) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    cudaGetLastError();
+    return NR_ERR_CUDA;
+  }
+  const void *src[10] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->bkt_off,
+                         ix->cl_off, ix->cent, ix->ids, ix->vec};
+  const bool dev[10] = {true, true, true, true, true, true, true, true, true, true};
+  return write_nrix(ix, ix->N, ix->n_cl, src, dev, path);
+}
+
+nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, const char *path,
+                           int64_t *info) {
+  if (!ix || !path || n < 0 || (n > 0 && !h_codes)) return NR_ERR_INVALID_ARG;
+  const uint64_t nb = (uint64_t)1 << ix->b;
+  std::vector<uint32_t> codes(h_codes, h_codes + n);
+  for (uint32_t u : codes)
+    if (u >= nb) return NR_ERR_INVALID_ARG;
+  std::sort(codes.begin(), codes.end());
+  codes.erase(std::unique(codes.begin(), codes.end()), codes.end());
+  DeviceGuard g(ix->device);
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    cudaGetLastError();
+    return NR_ERR_CUDA;
+  }
+  auto d2h = [](void *dst, const void *src, size_t bytes) {
+    if (bytes == 0) return true;
+    if (cudaMemcpy(dst, src, bytes, cudaMemcpyDeviceToHost) == cudaSuccess) return true;
+    cudaGetLastError();
+    return false;
+  };
+  // cluster and row ranges of the listed buckets
+  std::vector<uint32_t> c0(codes.size()), c1(codes.size());
+  for (size_t i = 0; i < codes.size(); ++i) {
+    uint32_t pair[2];
+    if (!d2h(pair, ix->bkt_off + codes[i], 8)) return NR_ERR_CUDA;
+    if (pair[1] < pair[0] || pair[1] > (uint64_t)ix->n_cl) return NR_ERR_DEVICE_CHECK;
+    c0[i] = pair[0];
+    c1[i] = pair[1];
+  }
+  int64_t ncl = 0, nrow = 0;
+  std::vector<uint32_t> bkt(nb + 1, 0), cl(1, 0);
+  std::vector<std::vector<uint32_t>> clo(codes.size());
+  for (size_t i = 0; i < codes.size(); ++i) {
+    clo[i].resize((size_t)(c1[i] - c0[i]) + 1);
+    if (!d2h(clo[i].data(), ix->cl_off + c0[i], clo[i].size() * 4)) return NR_ERR_CUDA;
+    for (size_t k = 0; k + 1 < clo[i].size(); ++k) {
+      if (clo[i][k + 1] < clo[i][k] || clo[i][k + 1] > (uint64_t)ix->N) return NR_ERR_DEVICE_CHECK;
+      nrow += clo[i][k + 1] - clo[i][k];
+      cl.push_back((uint32_t)nrow);
+    }
+    ncl += c1[i] - c0[i];
+  }
+  if (nrow < 1 || ncl < 1) return NR_ERR_INVALID_ARG;  // the file format needs a row
+  {
+    size_t i = 0;
+    int64_t c = 0;
+    for (uint64_t u = 0; u < nb; ++u) {
+      bkt[u] = (uint32_t)c;
+      if (i < codes.size() && codes[i] == u) c += c1[i] - c0[i], ++i;
+    }
+    bkt[nb] = (uint32_t)c;
+  }
+  std::vector<float> cent((size_t)ncl * ix->b), W1((size_t)ix->H * ix->D), b1(ix->H),
+      W2((size_t)ix->b * ix->H), b2(ix->b), tau(ix->b);
+  std::vector<uint32_t> ids((size_t)nrow);
+  std::vector<unsigned char> vec;
+  try {
+    vec.resize((size_t)nrow * ix->row_bytes);
+  } catch (...) {
+    return NR_ERR_OOM;
+  }
+  int64_t ci = 0, ri = 0;
+  for (size_t i = 0; i < codes.size(); ++i) {
+    const size_t k = c1[i] - c0[i];
+    if (!d2h(&cent[(size_t)ci * ix->b], ix->cent + (size_t)c0[i] * ix->b, k * ix->b * 4))
+      return NR_ERR_CUDA;
+    const uint32_t r0 = clo[i].front(), r1 = clo[i].back();
+    if (r1 > r0) {
+      if (!d2h(&ids[(size_t)ri], ix->ids + r0, (size_t)(r1 - r0) * 4)) return NR_ERR_CUDA;
+      if (!d2h(&vec[(size_t)ri * ix->row_bytes], (const char *)ix->vec + (size_t)r0 * ix->row_bytes,
+               (size_t)(r1 - r0) * ix->row_bytes))
+        return NR_ERR_CUDA;
+    }
+    ci += k;
+    ri += r1 - r0;
+  }
+  if (!d2h(W1.data(), ix->W1, W1.size() * 4) || !d2h(b1.data(), ix->b1, b1.size() * 4) ||
+      !d2h(W2.data(), ix->W2, W2.size() * 4) || !d2h(b2.data(), ix->b2, b2.size() * 4) ||
+      !d2h(tau.data(), ix->tau, tau.size() * 4))
+    return NR_ERR_CUDA;
+  const void *src[10] = {W1.data(), b1.data(), W2.data(), b2.data(), tau.data(), bkt.data(),
+                         cl.data(), cent.data(), ids.data(), vec.data()};
+  const bool dev[10] = {false, false, false, false, false, false, false, false, false, false};
+  const nr_status st = write_nrix(ix, nrow, ncl, src, dev, path);
+  if (st == NR_OK && info) {
+    info[0] = nrow;
+    info[1] = ncl;
+  }
+  return st;
+}
+
+nr_status nr_index_thresholds(nr_index *ix, float *h_tau) {
+  if (!ix || !h_tau) return NR_ERR_INVALID_ARG;
+  DeviceGuard g(ix->device);
+  if (cudaMemcpy(h_tau, ix->tau, (size_t)ix->b * 4, cudaMemcpyDeviceToHost) != cudaSuccess) {
+    cudaGetLastError();
+    return NR_ERR_CUDA;
+  }
+  return NR_OK;
 }
 
 nr_status nr_index_info(const nr_index *ix, int64_t *info) {

@@ -23,7 +23,7 @@ EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_f
            "nr_index_info", "nr_set_params", "nr_encode", "nr_route", "nr_debug_clusters",
            "nr_search", "nr_search_logits", "nr_search_host", "nr_query_stats", "nr_last_stats",
            "nr_enable_timing", "nr_last_timing", "nr_kernel_launches", "nr_search_static",
-           "nr_index_save", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
+           "nr_index_save", "nr_index_extract", "nr_index_thresholds", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
            "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free"]
 
 
@@ -74,6 +74,8 @@ def lib():
         L.nr_kernel_launches.argtypes = [vp]
         L.nr_kernel_launches.restype = i64
         L.nr_index_save.argtypes = [vp, ctypes.c_char_p]
+        L.nr_index_thresholds.argtypes = [vp, vp]
+        L.nr_index_extract.argtypes = [vp, vp, i64, ctypes.c_char_p, vp]
         L.nr_build_begin.argtypes = [vp, i64, vp, vp, vp, vp, i32, ctypes.POINTER(vp)]
         L.nr_build_encode.argtypes = [vp, vp, i64, i64, vp]
         L.nr_build_set_logits.argtypes = [vp, vp, i64, i64, vp]
@@ -147,9 +149,24 @@ class Index:
     def row_bytes(self):
         return self.D * (1 if self.dtype_code == 0 else 4)
 
+    def thresholds(self) -> np.ndarray:
+        """The per-bit thresholds tau [b] (nr_index_thresholds)."""
+        tau = np.empty(self.b, np.float32)
+        _check("nr_index_thresholds", lib().nr_index_thresholds(self.h, tau.ctypes.data))
+        return tau
+
     def save(self, path: str):
         """Write the index file (nr_index_save)."""
         _check("nr_index_save", lib().nr_index_save(self.h, path.encode()))
+
+    def extract(self, codes, path: str):
+        """Write the sub-index of the buckets of `codes` (nr_index_extract);
+        returns (rows, clusters)."""
+        c = np.ascontiguousarray(np.asarray(codes).reshape(-1), np.uint32)
+        info = np.zeros(2, np.int64)
+        _check("nr_index_extract", lib().nr_index_extract(self.h, c.ctypes.data, c.size,
+                                                          path.encode(), info.ctypes.data))
+        return int(info[0]), int(info[1])
 
     def set_params(self, p: Params | None = None, **kw):
         if p is None:

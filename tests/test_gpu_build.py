@@ -160,3 +160,36 @@ def test_call_order_and_input_errors():
             setattr(c, k, v)
         with pytest.raises(nr.NRError):
             nr.Builder(c, 1000, weights, 0)
+
+
+def test_extract_gives_the_same_results(tmp_path):
+    """A sub-index of the buckets some queries probe: the oracle on it gives
+    those queries exactly the ids, distances and statistics the GPU gives on
+    the whole index."""
+    torch = need_cuda()
+    w, base, weights = tiny_inputs(100_000, 16)
+    cfg = config(w.dtype, w.dim, w.hidden, 16, w.k_max, w.t)
+    ix, _ = gpu_build(torch, cfg, base, None, weights)
+    qs = synth.queries(w, 64)
+    dq = torch.from_numpy(qs).cuda()
+    lg = ix.encode(dq)
+    P, C, kw = 32, 64, dict(t_low=2)
+    codes, nprobe = ix.route(lg, P)
+    ix.set_params(**kw)
+    ids, d = ix.search_logits(dq, lg, 10, P, C)
+    st = ix.query_stats(64)
+    torch.cuda.synchronize()
+    c = codes.cpu().numpy().view(np.uint32)
+    used = np.concatenate([c[i, :n] for i, n in enumerate(nprobe.cpu().numpy())])
+    sub = str(tmp_path / "sub.nrix")
+    rows, ncl = ix.extract(used, sub)
+    assert 0 < rows < base.shape[0] and 0 < ncl < ix.n_clusters
+    orc = oracle.Index(sub)
+    ids_o, d_o, st_o = orc.search(qs, 10, P, C, oracle.params(**kw), logits=lg.cpu().numpy())
+    assert np.array_equal(ids.cpu().numpy(), ids_o)
+    assert np.array_equal(d.cpu().numpy(), d_o)
+    assert np.array_equal(st.cpu().numpy(), st_o)
+    from paper_2608_15438_gb300 import neuroute as nr
+    with pytest.raises(nr.NRError):
+        ix.extract(np.array([1 << 16], np.uint32), sub)   # code out of range
+    ix.close()

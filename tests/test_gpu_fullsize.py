@@ -60,3 +60,52 @@ def test_full_batch_sampled_parity(name):
     r_orc = recall(ids_oe, truth)
     assert abs(r_gpu - r_orc) <= 0.002 + 1e-12, (r_gpu, r_orc)
     ix.close()
+
+
+def test_1b_sampled_parity():
+    """1e9 uint8 vectors, index built on the GPU, the whole 10,000-query batch in
+    one nr_search_logits call at the benchmark's operating point; 100 sampled
+    queries checked against the oracle, which answers them from the sub-index
+    of the buckets its own probe lists name (its own logits too). End to end
+    (GPU encoder), Recall@10 on the sample agrees with the oracle's within
+    0.002 against exact k-NN."""
+    torch = need_cuda()
+    import os
+    import tempfile
+
+    import bench
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    torch.cuda.empty_cache()
+    w = synth.WORKLOADS["u8-1b"]
+    P, C, _, _ = bench.OPERATING_POINTS["u8-1b"]
+    kw = bench.op_params(w)
+    dev = torch.device("cuda", 0)
+    ix, _ = bench.gpu_index(w, torch, nr, dev)
+    qs = synth.queries(w)
+    lg = oracle.encode_weights(synth.encoder_weights(w), w.in_scale, qs)
+    dq = torch.from_numpy(qs).cuda()
+    ix.set_params(**kw)
+    ids, d = ix.search_logits(dq, torch.from_numpy(lg).cuda(), 10, P, C)
+    st = ix.query_stats(w.nq)
+    torch.cuda.synchronize()
+    ids, d, st = ids.cpu().numpy(), d.cpu().numpy(), st.cpu().numpy()
+    sample = np.linspace(0, w.nq - 1, 100).astype(np.int64)
+    p = oracle.params(**kw)
+    with tempfile.TemporaryDirectory() as td:
+        sub = os.path.join(td, "sub.nrix")
+        bench.oracle_subindex(w, ix, qs[sample], P, kw, sub)
+        orc = oracle.Index(sub)
+        ids_o, d_o, st_o = orc.search(qs[sample], 10, P, C, p, logits=lg[sample])
+        assert np.array_equal(ids[sample], ids_o)
+        assert np.array_equal(d[sample], d_o)
+        assert np.array_equal(st[sample], st_o)
+        ids_oe, _, _ = orc.search(qs[sample], 10, P, C, p)
+        orc.close()
+    ids_e, _ = ix.search(dq, 10, P, C)
+    torch.cuda.synchronize()
+    truth = bench.ground_truth_rows(torch, w, dq[torch.from_numpy(sample).cuda()], 10, dev)
+    r_gpu = recall(ids_e.cpu().numpy()[sample], truth)
+    r_orc = recall(ids_oe, truth)
+    assert abs(r_gpu - r_orc) <= 0.002 + 1e-12, (r_gpu, r_orc)
+    ix.close()

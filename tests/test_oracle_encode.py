@@ -51,3 +51,26 @@ def test_matches_double_gemm(tmp_path):
     got = ix.encode(x).astype(np.float64)
     # fp32 rounding of a double result: half an ulp
     assert np.all(np.abs(got - ref) <= np.abs(ref) * 2.0 ** -24 + 1e-30)
+
+
+def test_encode_from_weights_equals_index_encode(tmp_path):
+    """The index-free entry point runs the same forward pass as the index's."""
+    from nrix_writer import write_nrix
+
+    rng = np.random.default_rng(3)
+    D, H, b = 16, 32, 6
+    W1 = rng.normal(size=(H, D)).astype(np.float32)
+    b1 = rng.normal(size=H).astype(np.float32)
+    W2 = rng.normal(size=(b, H)).astype(np.float32)
+    b2 = rng.normal(size=b).astype(np.float32)
+    vec = rng.integers(0, 256, (40, D), dtype=np.uint8)
+    path = str(tmp_path / "e.nrix")
+    bkt = np.zeros((1 << b) + 1, np.uint32)
+    bkt[1:] = 1
+    write_nrix(path, vec, np.arange(40, dtype=np.uint32), bkt, np.array([0, 40], np.uint32),
+               np.zeros((1, b), np.float32), np.zeros(b, np.float32), W1, b1, W2, b2,
+               in_scale=1.0 / 255.0)
+    ix = oracle.Index(path)
+    want = ix.encode(vec)
+    got = oracle.encode_weights((W1, b1, W2, b2), 1.0 / 255.0, vec)
+    assert np.array_equal(got, want)
