@@ -39,6 +39,7 @@ OPERATING_POINTS = {
     "f32-10m": (512, 256, 16, None),
     "u8-100m": (1024, 256, 32, None),
     "u8-1b": (1024, 1024, 64, 4.0),
+    "u8-30m": (1024, 1024, 64, 4.0),  # profiling proxy of u8-1b: its operating point
 }
 
 

@@ -238,6 +238,80 @@ __device__ __forceinline__ void bitonic_sort(uint64_t *k, int n) {
   __syncthreads();
 }
 
+// Block merge sort of k[0..n) ascending, for keys that are distinct apart
+// from kEmpty padding; n <= 16 * blockDim.x, blockDim.x a power of two.
+// Each thread sorts a run of E keys in registers (a bitonic network with
+// compile-time indices), then runs are merged pairwise through shared memory:
+// every thread finds where its E outputs start on the merge path of its pair
+// of runs by binary search and merges E keys. Leaves k[n..E*blockDim.x)
+// holding kEmpty.
+template <int E>
+__device__ __forceinline__ void merge_sort_e(uint64_t *k, int n) {
+  const int tid = threadIdx.x;
+  const int N = E * (int)blockDim.x;
+  uint64_t r[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = tid * E + e;
+    r[e] = i < n ? k[i] : kEmpty;
+  }
+#pragma unroll
+  for (int size = 2; size <= E; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool up = (i & size) == 0;
+          const uint64_t a = r[i], c = r[j];
+          if ((a > c) == up) {
+            r[i] = c;
+            r[j] = a;
+          }
+        }
+      }
+  __syncthreads();
+#pragma unroll
+  for (int e = 0; e < E; ++e) k[tid * E + e] = r[e];
+  __syncthreads();
+  for (int w = E; w < N; w <<= 1) {
+    const int lo = (tid * E) & ~(2 * w - 1);  // first key of my pair of runs
+    const int d = tid * E - lo;               // my first output on its merge path
+    const uint64_t *A = k + lo, *B = k + lo + w;
+    int a = d > w ? d - w : 0, hi = d < w ? d : w;
+    while (a < hi) {
+      const int mid = (a + hi) >> 1;
+      if (A[mid] > B[d - 1 - mid]) hi = mid;
+      else a = mid + 1;
+    }
+    int i = a, j = d - a;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const uint64_t x = i < w ? A[i] : kEmpty, y = j < w ? B[j] : kEmpty;
+      const bool takeA = j >= w || (i < w && x <= y);
+      r[e] = takeA ? x : y;
+      i += takeA ? 1 : 0;
+      j += takeA ? 0 : 1;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int e = 0; e < E; ++e) k[tid * E + e] = r[e];
+    __syncthreads();
+  }
+}
+
+// merge_sort_e with the smallest run length E (a power of two) that covers n;
+// returns the padded length E * blockDim.x.
+__device__ __forceinline__ int merge_sort(uint64_t *k, int n) {
+  const int nt = blockDim.x;
+  if (n <= nt) return merge_sort_e<1>(k, n), nt;
+  if (n <= 2 * nt) return merge_sort_e<2>(k, n), 2 * nt;
+  if (n <= 4 * nt) return merge_sort_e<4>(k, n), 4 * nt;
+  if (n <= 8 * nt) return merge_sort_e<8>(k, n), 8 * nt;
+  return merge_sort_e<16>(k, n), 16 * nt;
+}
+
 struct SelectParams {
   int b, K_max, P, C;
   int64_t n_cl, N;
@@ -258,9 +332,12 @@ __host__ __device__ inline int select_sort_cap(int P, int K_max) {
   while (s < P * K_max) s <<= 1;
   return s;
 }
+// at least one key per thread of the 128-thread select block (the merge
+// sort's shortest padded length), at most kSelectSmemKeys
+constexpr int kSelectMinKeys = 128;
 __host__ __device__ inline int select_smem_cap(int P, int K_max) {
   const int s = select_sort_cap(P, K_max);
-  return s < kSelectSmemKeys ? s : kSelectSmemKeys;
+  return s < kSelectMinKeys ? kSelectMinKeys : (s < kSelectSmemKeys ? s : kSelectSmemKeys);
 }
 __host__ __device__ inline size_t select_scratch_bytes(int P, int K_max) {
   const int S = select_smem_cap(P, K_max);
@@ -272,14 +349,66 @@ __host__ __device__ inline size_t select_slab_bytes(int P, int K_max) {
   return full > select_smem_cap(P, K_max) ? (size_t)full * 12 : 0;
 }
 
+// Centroid distance d_c = sum_j (l_j - mu_cj)^2 as a sequential fmaf chain.
+// When b is a multiple of 4 (rows 16-byte aligned) the row is loaded as
+// float4s up front; the arithmetic is the same chain either way.
+__device__ __forceinline__ float centroid_dist(const float *__restrict__ mu, const float *slog, int b) {
+  float acc = 0.0f;
+  if ((b & 3) == 0 && b <= 32) {
+#pragma unroll
+    for (int g = 0; g < 2; ++g) {
+      float4 v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (16 * g + 4 * q < b) v[q] = __ldg(reinterpret_cast<const float4 *>(mu) + 4 * g + q);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (16 * g + 4 * q < b) {
+          const float m[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float t = __fsub_rn(slog[16 * g + 4 * q + e], m[e]);
+            acc = __fmaf_rn(t, t, acc);
+          }
+        }
+    }
+    return acc;
+  }
+  for (int j = 0; j < b; ++j) {
+    const float t = __fsub_rn(slog[j], __ldg(&mu[j]));
+    acc = __fmaf_rn(t, t, acc);
+  }
+  return acc;
+}
+
+// Cluster of candidate slot s: slots are numbered probe by probe, off[i] the
+// first slot of probe i (nondecreasing), c0[i] the first cluster of probe i.
+__device__ __forceinline__ uint32_t slot_cluster(const int *off, const int *c0, int np, int s) {
+  int lo = 0, hi = np - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= s) lo = mid;
+    else hi = mid - 1;
+  }
+  return (uint32_t)(c0[lo] + (s - off[lo]));
+}
+
 // One query: codes[0..np) -> the kept clusters C^dir U C^cent in (d, cluster)
 // order and their refinement segments. Writes seg[i] = (first row, stream
 // position) for i < nl, and L[i] (cluster index, -1 padded to Lmax) when L is
 // not null. slog: the query's b logits in shared memory; scratch:
 // select_scratch_bytes(P, K_max) bytes of shared memory; slab: this query's
 // select_slab_bytes(P, K_max) bytes of global memory (null when that is 0);
-// warp_sums: 32 ints; sred: 1 unsigned. Returns nl; *total = stream length.
+// warp_sums: 32 ints; sred: 2 unsigned. Returns nl; *total = stream length.
 // Whole block calls.
+//
+// The keys to sort (C^dir and the gate's survivors) are collected straight
+// into shared memory: one pass over the candidate clusters computes their
+// distances, keeps the single-cluster buckets' and takes d_min over the rest;
+// a second pass recomputes the others' distances and keeps those within the
+// gate. Only when they do not fit does the query fall back to sorting all its
+// candidate keys in the global slab. Both give the same keys, and the sort
+// orders them by exact value.
 __device__ __forceinline__ int select_block(const SelectParams &sp, const float *slog,
                                             const uint32_t *codes, int np, unsigned char *scratch,
                                             unsigned char *slab, int *warp_sums, unsigned *sred,
@@ -289,7 +418,10 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   const int S_full = select_sort_cap(sp.P, sp.K_max);
   uint64_t *keys = reinterpret_cast<uint64_t *>(scratch);
   int *ibuf = reinterpret_cast<int *>(scratch + (size_t)S_smem * 8);
-  if (tid == 0) *sred = 0xffffffffu;
+  if (tid == 0) {
+    sred[0] = 0xffffffffu;  // d_min bits over non-singleton candidates
+    sred[1] = 0u;           // keys collected
+  }
   int *cnt = ibuf;        // [P] clusters per probe -> exclusive offsets
   int *c0s = ibuf + sp.P;  // [P] first cluster per probe
   const uint32_t nb = 1u << sp.b;
@@ -315,51 +447,124 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     c0s[i] = c0;
   }
   __syncthreads();
-  const int M = block_exclusive_scan(cnt, np, warp_sums);
-  int Sn = 1;
-  while (Sn < M) Sn <<= 1;
-  // many candidate clusters: keys and per-key integers move to the global slab
-  int *ints = ibuf;
-  if (M > S_smem && slab != nullptr && Sn <= S_full) {
-    keys = reinterpret_cast<uint64_t *>(slab);
-    ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
-  } else if (M > S_smem) {
-    if (tid == 0) set_err(sp.err, NR_DEV_TOO_MANY);
-    *total = 0;
-    return 0;
-  }
-  for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
-    const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
-    for (int j = 0; j < n; ++j) keys[o + j] = (uint64_t)(uint32_t)(c0s[i] + j);
-  }
+  int M = block_exclusive_scan(cnt, np, warp_sums);
+  // One pass over the candidates. C^dir keys are collected from the back of
+  // the key array; the other clusters from the front when they are within the
+  // gate of the running d_min (for m1 >= 0 that gate is never tighter than the
+  // final one: x + fmaf(m1, x, m0) does not decrease with x).
+  if (tid == 0) sred[2] = 0u;  // keys collected from the front
   __syncthreads();
-  // centroid distances d_c = sum_j (l_j - mu_cj)^2, sequential fmaf chain
+  const float m0 = sp.m0, m1 = sp.m1;
+  const bool prefilter = !sp.gate_off && m1 >= 0.0f;
   for (int s = tid; s < M; s += nt) {
-    const uint32_t c = (uint32_t)keys[s];
-    const float *mu = sp.cent + (size_t)c * sp.b;
-    float acc = 0.0f;
-    for (int j = 0; j < sp.b; ++j) {
-      const float t = __fsub_rn(slog[j], __ldg(&mu[j]));
-      acc = __fmaf_rn(t, t, acc);
+    const uint32_t c = slot_cluster(cnt, c0s, np, s);
+    const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
+    const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | c;
+    if (__ldg(&sp.single[c])) {
+      const unsigned pos = atomicAdd(&sred[1], 1u);
+      if (pos < (unsigned)S_smem) keys[S_smem - 1 - pos] = key;
+    } else {
+      const uint32_t db = __float_as_uint(d);
+      const uint32_t prev = atomicMin(&sred[0], db);  // d >= 0: bits order as values
+      bool maybe = true;
+      if (prefilter) {
+        const float dm = __uint_as_float(prev < db ? prev : db);
+        maybe = d <= __fadd_rn(dm, __fmaf_rn(m1, dm, m0));
+      }
+      if (maybe) {
+        const unsigned pos = atomicAdd(&sred[2], 1u);
+        if (pos < (unsigned)S_smem) keys[pos] = key;
+      }
     }
-    keys[s] = ((uint64_t)__float_as_uint(acc) << 32) | c;
-    if (!__ldg(&sp.single[c])) atomicMin(sred, __float_as_uint(acc));  // d >= 0: bits order as values
   }
-  for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
   __syncthreads();
-  const uint32_t dmin_bits = *sred;
+  const uint32_t dmin_bits = sred[0];
   float theta = __int_as_float(0x7f800000);
   if (!sp.gate_off && dmin_bits != 0xffffffffu) {
     const float dmin = __uint_as_float(dmin_bits);
-    theta = __fadd_rn(dmin, __fmaf_rn(sp.m1, dmin, sp.m0));  // theta = d_min + M(d_min)
+    theta = __fadd_rn(dmin, __fmaf_rn(m1, dmin, m0));  // theta = d_min + M(d_min)
   }
-  for (int s = tid; s < M; s += nt) {  // drop non-singleton clusters above the gate
-    const uint64_t kk = keys[s];
-    const uint32_t c = (uint32_t)kk;
-    if (!__ldg(&sp.single[c]) && !(__uint_as_float((uint32_t)(kk >> 32)) <= theta)) keys[s] = kEmpty;
+  const int nA = (int)sred[1], nB = (int)sred[2];
+  int Mk = nA + nB;
+  if (Mk <= S_smem) {
+    // keep the front keys within the final gate, compacted toward the front
+    // (a key never moves up, and each chunk reads before it writes), then move
+    // the C^dir keys down behind them
+    int *flag = ibuf;  // the probe offsets are no longer needed
+    __syncthreads();
+    for (int i = tid; i < nB; i += nt)
+      flag[i] = __uint_as_float((uint32_t)(keys[i] >> 32)) <= theta ? 1 : 0;
+    __syncthreads();
+    const int nS = block_exclusive_scan(flag, nB, warp_sums);
+    for (int i0 = 0; i0 < nB; i0 += 4 * nt) {
+      uint64_t kb[4];
+      int rk[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int i = i0 + e * nt + tid;
+        rk[e] = -1;
+        kb[e] = 0;
+        if (i < nB && (i + 1 < nB ? flag[i + 1] : nS) > flag[i]) {
+          rk[e] = flag[i];
+          kb[e] = keys[i];
+        }
+      }
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (rk[e] >= 0) keys[rk[e]] = kb[e];
+      __syncthreads();
+    }
+    for (int t0 = 0; t0 < nA; t0 += 4 * nt) {
+      uint64_t kb[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int t = t0 + e * nt + tid;
+        kb[e] = t < nA ? keys[S_smem - nA + t] : 0;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int t = t0 + e * nt + tid;
+        if (t < nA) keys[nS + t] = kb[e];
+      }
+      __syncthreads();
+    }
+    Mk = nS + nA;
+  } else {
+    Mk = S_smem + 1;  // does not fit: the slab path below
   }
-  __syncthreads();
-  bitonic_sort(keys, Sn);
+  int Sn = 1;
+  int *ints = ibuf;
+  if (Mk <= S_smem) {
+    M = Mk;
+    Sn = merge_sort(keys, M);  // keys[M..Sn) = kEmpty
+  } else {
+    // more keys than shared memory holds: all candidate keys in the global slab
+    // (slab is present: without it M <= S_full = S_smem)
+    while (Sn < M) Sn <<= 1;
+    if (slab == nullptr || Sn > S_full) {
+      if (tid == 0) set_err(sp.err, NR_DEV_TOO_MANY);
+      *total = 0;
+      return 0;
+    }
+    keys = reinterpret_cast<uint64_t *>(slab);
+    ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
+    for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
+      const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
+      for (int j = 0; j < n; ++j) keys[o + j] = (uint64_t)(uint32_t)(c0s[i] + j);
+    }
+    __syncthreads();
+    for (int s = tid; s < M; s += nt) {
+      const uint32_t c = (uint32_t)keys[s];
+      const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
+      const bool keep = __ldg(&sp.single[c]) || d <= theta;
+      keys[s] = keep ? (((uint64_t)__float_as_uint(d) << 32) | c) : kEmpty;
+    }
+    for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
+    __syncthreads();
+    bitonic_sort(keys, Sn);
+  }
   // keep C^dir and the first C survivors in key order
   int *keep = ints;  // [Sn]
   for (int s = tid; s < Sn; s += nt) {

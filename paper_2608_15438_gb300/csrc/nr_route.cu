@@ -61,7 +61,8 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
                                        (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t grid = (nq + wpb - 1) / wpb;
-  route_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(nr_route_params(ix, P), d_logits, nq,
+  const nrq::RouteParams rp = nr_route_params(ix, P);  // before the launch configuration
+  route_kernel<<<(unsigned)grid, 32 * wpb, smem, s>>>(rp, d_logits, nq,
                                                        d_codes, d_nprobe);
   ix->launches += 1;
   return cudaGetLastError();

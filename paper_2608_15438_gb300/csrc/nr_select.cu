@@ -5,7 +5,10 @@
 //   2. every cluster c of every probed bucket gets its centroid distance
 //      d_c = sum_j (l_j - mu_cj)^2 as a sequential fp32 fmaf chain over j;
 //   3. buckets holding exactly one cluster go to C^dir; over the other clusters
-//      d_min, the gate theta = d_min + fmaf(m1, d_min, m0), survivors d_c <= theta;
+//      d_min, the gate theta = d_min + fmaf(m1, d_min, m0), survivors d_c <= theta
+//      (keys of C^dir and the survivors collected in shared memory by two
+//      passes over the candidates, or, when they do not fit, all candidate
+//      keys sorted in the query's global slab);
 //   4. a bitonic sort of the 64-bit keys (d_c bits, c) of C^dir and the
 //      survivors, the first C survivors kept (top-C by (d_c, c)), and the kept
 //      list written in key order together with its refinement segments.
@@ -93,7 +96,8 @@ cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t
   cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
-  select_kernel<<<(unsigned)nq, kThreads, smem, s>>>(nr_select_params(ix, P, C), d_logits, d_codes,
+  const nrq::SelectParams sp = nr_select_params(ix, P, C);  // before the launch configuration
+  select_kernel<<<(unsigned)nq, kThreads, smem, s>>>(sp, d_logits, d_codes,
                                                       d_nprobe, d_L, d_nL, d_seg, d_slen, d_stats,
                                                       static_cast<unsigned char *>(d_slab),
                                                       nrq::select_slab_bytes(P, ix->K_max));

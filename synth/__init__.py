@@ -121,6 +121,9 @@ WORKLOADS = {
     # cluster per bucket): the analogue of the paper's bucket-clustering ablation
     "u8-10m-nocl": Workload("u8-10m-nocl", 10_000_000, 128, "u8", 256, 18.0, 10_000, 512, 20, 1, 64,
                             probe=(64, 256), clusters=(256,)),
+    # 3e7 uint8 x 128 with b = 19: the 1e9 workload's rows per code (~57) and
+    # rows per component, small enough for full kernel profiles
+    "u8-30m": Workload("u8-30m", 30_000_000, 128, "u8", 512, 18.0, 10_000, 512, 19, 16, 64),
     # 1e8 uint8 x 128, b = 24
     "u8-100m": Workload("u8-100m", 100_000_000, 128, "u8", 4096, 18.0, 10_000, 512, 24, 16, 64),
     # 1e9 uint8 x 128, b = 24

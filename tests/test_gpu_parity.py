@@ -83,8 +83,12 @@ def test_route_b4_hand_order(torch, tmp_path):
 
 
 @pytest.mark.parametrize("P,C", [(1, 1), (8, 32), (64, 16), (256, 1000), (1024, 4096)])
-@pytest.mark.parametrize("gate", [(float("inf"), 0.0), (2.0, 0.5), (0.0, 0.0)])
+@pytest.mark.parametrize("gate", [(float("inf"), 0.0), (2.0, 0.5), (0.0, 0.0), (0.0, 4.0),
+                                  (3.0, -0.5), (-0.5, 1.0), (float("-inf"), 1.0)])
 def test_cluster_list_bit_exact(tiny, torch, P, C, gate):
+    """Gates: off, affine, zero-width, the 1e9 operating point's M(x) = 4x, a
+    decreasing M (m1 < 0), a negative offset, and one that drops every
+    non-singleton cluster."""
     ix, orc = tiny["ix"], tiny["orc"]
     ix.set_params(gate_m0=gate[0], gate_m1=gate[1])
     try:
@@ -288,15 +292,21 @@ def many_clusters(torch, tmp_path_factory):
             "dq": torch.from_numpy(qs).cuda(), "dl": torch.from_numpy(lg).cuda()}
 
 
-@pytest.mark.parametrize("C", [64, 4096])
-def test_select_overflow_to_global_slab(many_clusters, torch, C):
+@pytest.mark.parametrize("C,m1", [(64, None), (4096, None), (64, 0.25), (4096, 0.25), (4096, 2.0),
+                                  (4096, -0.5), (64, 40.0)])
+def test_select_overflow_to_global_slab(many_clusters, torch, C, m1):
+    """More candidate clusters than shared memory holds: sorted in the global
+    slab (gate off), or, when the gate's survivors fit, moved back to shared
+    memory before the sort."""
     mc = many_clusters
     assert mc["info"]["n_clusters"] > 2048
     ix, orc = mc["ix"], mc["orc"]
+    kw = {} if m1 is None else dict(gate_m0=0.0, gate_m1=m1)
+    ix.set_params(**kw)
     cl, ncl = ix.debug_clusters(mc["dl"], 256, C)
     cl, ncl = cl.cpu().numpy(), ncl.cpu().numpy()
     tau = orc.tau()
-    p = oracle.params()
+    p = oracle.params(**kw)
     for i in range(0, len(mc["q"]), 7):
         codes, _, _ = oracle.probe_list(mc["lg"][i], tau, 256, p)
         L, _, _ = orc.cluster_list(mc["lg"][i], codes, C, p)
