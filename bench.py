@@ -294,7 +294,7 @@ def recall_at(found, truth, k=10):
 def refine_sources_digest():
     """sha256 over the sources that define the refine kernel."""
     h = hashlib.sha256()
-    for f in ("nr_refine.cu", "nr_query.cuh"):
+    for f in ("nr_refine.cu", "nrq_refine.cuh", "nrq_common.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2608_15438_gb300", "csrc", f), "rb").read())
     return h.hexdigest()
 

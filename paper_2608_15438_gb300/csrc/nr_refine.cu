@@ -10,7 +10,7 @@
 #include <stdint.h>
 
 #include "nr_internal.cuh"
-#include "nr_query.cuh"
+#include "nrq_refine.cuh"
 
 namespace {
 

@@ -4,7 +4,7 @@
 #include <stdint.h>
 
 #include "nr_internal.cuh"
-#include "nr_query.cuh"
+#include "nrq_route.cuh"
 
 namespace {
 

@@ -19,7 +19,7 @@
 #include <cmath>
 
 #include "nr_internal.cuh"
-#include "nr_query.cuh"
+#include "nrq_select.cuh"
 
 namespace {
 

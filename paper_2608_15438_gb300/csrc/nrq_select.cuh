@@ -1,0 +1,541 @@
+// select_block: one block per query looks up the probed buckets, scores
+// their centroids, applies the gate and top-C and lays out the refinement
+// segments of the kept clusters (Sec. 3.3, 3.4.2, Algorithm 2).
+#pragma once
+
+#include "nrq_common.cuh"
+
+namespace nrq {
+
+// ============================================================== select
+// Exclusive scan of a[0..n) in shared memory by the whole block (blockDim a
+// multiple of 32, at most 1024); returns the total.
+__device__ __forceinline__ int block_exclusive_scan(int *a, int n, int *warp_sums) {
+  const int nt = blockDim.x, tid = threadIdx.x, lane = tid & 31, wid = tid >> 5, nw = nt >> 5;
+  const int per = (n + nt - 1) / nt;
+  const int lo = tid * per, hi = min(n, lo + per);
+  int local = 0;
+  for (int i = lo; i < hi; ++i) local += a[i];
+  int incl = local;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(kFull, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) warp_sums[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    int ws = lane < nw ? warp_sums[lane] : 0;
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(kFull, ws, o);
+      if (lane >= o) ws += v;
+    }
+    if (lane < nw) warp_sums[lane] = ws;  // inclusive
+  }
+  __syncthreads();
+  int run = (wid > 0 ? warp_sums[wid - 1] : 0) + incl - local;
+  for (int i = lo; i < hi; ++i) {
+    const int v = a[i];
+    a[i] = run;
+    run += v;
+  }
+  const int total = warp_sums[nw - 1];
+  __syncthreads();
+  return total;
+}
+
+// Bitonic sort of k[0..n), n a power of two, by the whole block. Thread i
+// owns the pairs (lo, lo + stride) with lo = 2i - (i mod stride); for strides
+// up to 32 the pairs of one warp stay inside its own 64-element blocks, so
+// consecutive such stages need only a warp barrier.
+__device__ __forceinline__ void bitonic_sort(uint64_t *k, int n) {
+  const int nt = blockDim.x;
+  for (int size = 2; size <= n; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < n / 2; i += nt) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool up = (lo & size) == 0;
+        const uint64_t a = k[lo], c = k[hi];
+        if ((a > c) == up) {
+          k[lo] = c;
+          k[hi] = a;
+        }
+      }
+      const int next = stride > 1 ? stride >> 1 : size;
+      if (stride > 32 || next > 32 || nt <= 32) __syncthreads();
+      else __syncwarp();
+    }
+  }
+  __syncthreads();
+}
+
+// Exclusive prefix of v over the block's threads; *all = the sum. Starts
+// with a barrier (warp_sums may still be read by a previous call).
+__device__ __forceinline__ int block_thread_scan(int v, int *warp_sums, int *all) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  int x = v;
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(kFull, x, o);
+    if (lane >= o) x += y;
+  }
+  __syncthreads();
+  if (lane == 31) warp_sums[w] = x;
+  __syncthreads();
+  int before = 0, tot = 0;
+  for (int i = 0; i < nw; ++i) {
+    const int t = warp_sums[i];
+    before += i < w ? t : 0;
+    tot += t;
+  }
+  *all = tot;
+  return before + x - v;
+}
+
+// Shared-memory position of element i of the merge sort's runs: one 8-byte
+// gap every 16 keys, so that threads reading or writing their runs (a stride
+// of E keys) fall on different banks.
+__device__ __forceinline__ int pad16(int i) { return i + (i >> 4); }
+
+// Block merge sort of k[0..n) ascending, for keys that are distinct apart
+// from kEmpty padding; n <= E * blockDim.x, blockDim.x a power of two; k must
+// hold pad16(E * blockDim.x) keys. On return r[e] holds sorted element
+// threadIdx.x * E + e (kEmpty past n); k is clobbered.
+// The keys are read striped, each thread sorts its E keys in registers (a
+// bitonic network with compile-time indices), and runs are merged pairwise:
+// every thread finds where its E outputs start on the merge path of its pair
+// of runs by binary search and merges E keys.
+template <int E>
+__device__ __forceinline__ void merge_sort_regs(uint64_t *k, int n, uint64_t (&r)[E]) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int N = E * nt;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = e * nt + tid;
+    r[e] = i < n ? k[i] : kEmpty;
+  }
+#pragma unroll
+  for (int size = 2; size <= E; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+      for (int i = 0; i < E; ++i) {
+        const int j = i ^ stride;
+        if (j > i) {
+          const bool up = (i & size) == 0;
+          const uint64_t a = r[i], c = r[j];
+          if ((a > c) == up) {
+            r[i] = c;
+            r[j] = a;
+          }
+        }
+      }
+  __syncthreads();
+#pragma unroll
+  for (int e = 0; e < E; ++e) k[pad16(tid * E + e)] = r[e];
+  __syncthreads();
+  for (int w = E; w < N; w <<= 1) {
+    const int lo = (tid * E) & ~(2 * w - 1);  // first key of my pair of runs
+    const int d = tid * E - lo;               // my first output on its merge path
+    int a = d > w ? d - w : 0, hi = d < w ? d : w;
+    while (a < hi) {
+      const int mid = (a + hi) >> 1;
+      if (k[pad16(lo + mid)] > k[pad16(lo + w + d - 1 - mid)]) hi = mid;
+      else a = mid + 1;
+    }
+    int i = a, j = d - a;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const uint64_t x = i < w ? k[pad16(lo + i)] : kEmpty;
+      const uint64_t y = j < w ? k[pad16(lo + w + j)] : kEmpty;
+      const bool takeA = j >= w || (i < w && x <= y);
+      r[e] = takeA ? x : y;
+      i += takeA ? 1 : 0;
+      j += takeA ? 0 : 1;
+    }
+    if (2 * w < N) {  // the last level's outputs stay in registers
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < E; ++e) k[pad16(tid * E + e)] = r[e];
+      __syncthreads();
+    }
+  }
+}
+
+struct SelectParams {
+  int b, K_max, P, C;
+  int64_t n_cl, N;
+  const uint32_t *bkt_off, *cl_off;
+  const float *cent;
+  const uint8_t *single;  // [n_cl] 1 if the cluster's bucket holds one cluster
+  bool gate_off;
+  float m0, m1;
+  int *err;
+};
+
+// Sort capacity for probe budget P: all clusters of P buckets. Shared memory
+// holds at most kSelectSmemKeys keys; a query with more candidate clusters
+// sorts in its slab of global memory (select_slab_bytes, 0 when unneeded).
+constexpr int kSelectSmemKeys = 2048;
+__host__ __device__ inline int select_sort_cap(int P, int K_max) {
+  int s = 1;
+  while (s < P * K_max) s <<= 1;
+  return s;
+}
+// at least one key per thread of the 128-thread select block (the merge
+// sort's shortest padded length), at most kSelectSmemKeys
+constexpr int kSelectMinKeys = 128;
+__host__ __device__ inline int select_smem_cap(int P, int K_max) {
+  const int s = select_sort_cap(P, K_max);
+  return s < kSelectMinKeys ? kSelectMinKeys : (s < kSelectSmemKeys ? s : kSelectSmemKeys);
+}
+// key capacity of the shared-memory scratch: S keys plus the merge sort's gaps
+__host__ __device__ inline int select_smem_keys(int S) { return S + S / 16; }
+__host__ __device__ inline size_t select_scratch_bytes(int P, int K_max) {
+  const int S = select_smem_cap(P, K_max);
+  const int ib = S > 2 * P + 1 ? S : 2 * P + 1;
+  return (size_t)select_smem_keys(S) * 8 + (size_t)ib * 4;
+}
+__host__ __device__ inline size_t select_slab_bytes(int P, int K_max) {
+  const int full = select_sort_cap(P, K_max);
+  return full > select_smem_cap(P, K_max) ? (size_t)full * 12 : 0;
+}
+
+// Centroid distance d_c = sum_j (l_j - mu_cj)^2 as a sequential fmaf chain.
+// When b is a multiple of 4 (rows 16-byte aligned) the row is loaded as
+// float4s up front; the arithmetic is the same chain either way.
+__device__ __forceinline__ float centroid_dist(const float *__restrict__ mu, const float *slog, int b) {
+  float acc = 0.0f;
+  if ((b & 3) == 0 && b <= 32) {
+#pragma unroll
+    for (int g = 0; g < 2; ++g) {
+      float4 v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (16 * g + 4 * q < b) v[q] = __ldg(reinterpret_cast<const float4 *>(mu) + 4 * g + q);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if (16 * g + 4 * q < b) {
+          const float m[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float t = __fsub_rn(slog[16 * g + 4 * q + e], m[e]);
+            acc = __fmaf_rn(t, t, acc);
+          }
+        }
+    }
+    return acc;
+  }
+  for (int j = 0; j < b; ++j) {
+    const float t = __fsub_rn(slog[j], __ldg(&mu[j]));
+    acc = __fmaf_rn(t, t, acc);
+  }
+  return acc;
+}
+
+// Cluster of candidate slot s: slots are numbered probe by probe, off[i] the
+// first slot of probe i (nondecreasing), c0[i] the first cluster of probe i.
+__device__ __forceinline__ uint32_t slot_cluster(const int *off, const int *c0, int np, int s) {
+  int lo = 0, hi = np - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (off[mid] <= s) lo = mid;
+    else hi = mid - 1;
+  }
+  return (uint32_t)(c0[lo] + (s - off[lo]));
+}
+
+// The kept list from the collected keys k[0..n) (n <= E * blockDim.x), sorted
+// into registers: C^dir keys always, the others while their rank among the
+// others is below C, in key order; then their segments (first row, stream
+// position) and, when L is not null, their cluster indices (-1 padded to
+// Lmax). Returns the list length; *total = stream length.
+template <int E>
+__device__ __forceinline__ int select_tail_regs(const SelectParams &sp, uint64_t *k, int n,
+                                                int *warp_sums, nr_seg *seg, int32_t *L, int Lmax,
+                                                uint32_t *total) {
+  uint64_t r[E];
+  merge_sort_regs<E>(k, n, r);
+  uint32_t sg = 0, kp = 0;
+  int ns = 0;
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if (r[e] != kEmpty) {
+      if (__ldg(&sp.single[(uint32_t)r[e]])) sg |= 1u << e;
+      else ++ns;
+    }
+  int all;
+  int rank = block_thread_scan(ns, warp_sums, &all);  // rank among the non-C^dir keys
+  int nk = 0;
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if (r[e] != kEmpty) {
+      bool keep = (sg >> e) & 1u;
+      if (!keep) {
+        keep = rank < sp.C;
+        ++rank;
+      }
+      if (keep) {
+        kp |= 1u << e;
+        ++nk;
+      }
+    }
+  int nl;
+  int pos = block_thread_scan(nk, warp_sums, &nl);  // output position
+  int lsum = 0;
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if ((kp >> e) & 1u) {
+      const uint32_t c = (uint32_t)r[e];
+      const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
+      if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
+      else lsum += (int)(r1 - r0);
+    }
+  int tot;
+  int spos = block_thread_scan(lsum, warp_sums, &tot);  // stream position
+#pragma unroll
+  for (int e = 0; e < E; ++e)
+    if ((kp >> e) & 1u) {
+      const uint32_t c = (uint32_t)r[e];
+      const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
+      const int ln = (r1 < r0 || (int64_t)r1 > sp.N) ? 0 : (int)(r1 - r0);
+      seg[pos].row0 = r0;
+      seg[pos].pos = (uint32_t)spos;
+      if (L) L[pos] = (int32_t)c;
+      spos += ln;
+      ++pos;
+    }
+  if (L)
+    for (int i = nl + threadIdx.x; i < Lmax; i += blockDim.x) L[i] = -1;
+  *total = (uint32_t)tot;
+  return nl;
+}
+
+// select_tail_regs with the smallest run length E (a power of two) that covers n
+__device__ __forceinline__ int select_tail_smem(const SelectParams &sp, uint64_t *k, int n,
+                                                int *warp_sums, nr_seg *seg, int32_t *L, int Lmax,
+                                                uint32_t *total) {
+  const int nt = blockDim.x;
+  if (n <= nt) return select_tail_regs<1>(sp, k, n, warp_sums, seg, L, Lmax, total);
+  if (n <= 2 * nt) return select_tail_regs<2>(sp, k, n, warp_sums, seg, L, Lmax, total);
+  if (n <= 4 * nt) return select_tail_regs<4>(sp, k, n, warp_sums, seg, L, Lmax, total);
+  if (n <= 8 * nt) return select_tail_regs<8>(sp, k, n, warp_sums, seg, L, Lmax, total);
+  return select_tail_regs<16>(sp, k, n, warp_sums, seg, L, Lmax, total);
+}
+
+// One query: codes[0..np) -> the kept clusters C^dir U C^cent in (d, cluster)
+// order and their refinement segments. Writes seg[i] = (first row, stream
+// position) for i < nl, and L[i] (cluster index, -1 padded to Lmax) when L is
+// not null. slog: the query's b logits in shared memory; scratch:
+// select_scratch_bytes(P, K_max) bytes of shared memory; slab: this query's
+// select_slab_bytes(P, K_max) bytes of global memory (null when that is 0);
+// warp_sums: 32 ints; sred: 2 unsigned. Returns nl; *total = stream length.
+// Whole block calls.
+//
+// The keys to sort (C^dir and the gate's survivors) are collected straight
+// into shared memory: one pass over the candidate clusters computes their
+// distances, keeps the single-cluster buckets' and takes d_min over the rest;
+// a second pass recomputes the others' distances and keeps those within the
+// gate. Only when they do not fit does the query fall back to sorting all its
+// candidate keys in the global slab. Both give the same keys, and the sort
+// orders them by exact value.
+__device__ __forceinline__ int select_block(const SelectParams &sp, const float *slog,
+                                            const uint32_t *codes, int np, unsigned char *scratch,
+                                            unsigned char *slab, int *warp_sums, unsigned *sred,
+                                            nr_seg *seg, int32_t *L, int Lmax, uint32_t *total) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int S_smem = select_smem_cap(sp.P, sp.K_max);
+  const int S_full = select_sort_cap(sp.P, sp.K_max);
+  uint64_t *keys = reinterpret_cast<uint64_t *>(scratch);
+  int *ibuf = reinterpret_cast<int *>(scratch + (size_t)select_smem_keys(S_smem) * 8);
+  if (tid == 0) {
+    sred[0] = 0xffffffffu;  // d_min bits over non-singleton candidates
+    sred[1] = 0u;           // keys collected
+  }
+  int *cnt = ibuf;        // [P] clusters per probe -> exclusive offsets
+  int *c0s = ibuf + sp.P;  // [P] first cluster per probe
+  const uint32_t nb = 1u << sp.b;
+  for (int i = tid; i < np; i += nt) {
+    const uint32_t u = codes[i];
+    int n = 0, c0 = 0;
+    if (u >= nb) {
+      set_err(sp.err, NR_DEV_BAD_CODE);
+    } else {
+      const uint32_t lo = __ldg(&sp.bkt_off[u]), hi = __ldg(&sp.bkt_off[u + 1]);
+      if (hi < lo || (int64_t)hi > sp.n_cl) {
+        set_err(sp.err, NR_DEV_BAD_BUCKET);
+      } else {
+        n = (int)(hi - lo);
+        c0 = (int)lo;
+        if (n > sp.K_max) {
+          set_err(sp.err, NR_DEV_TOO_MANY);
+          n = sp.K_max;
+        }
+      }
+    }
+    cnt[i] = n;
+    c0s[i] = c0;
+  }
+  __syncthreads();
+  int M = block_exclusive_scan(cnt, np, warp_sums);
+  // One pass over the candidates. C^dir keys are collected from the back of
+  // the key array; the other clusters from the front when they are within the
+  // gate of the running d_min (for m1 >= 0 that gate is never tighter than the
+  // final one: x + fmaf(m1, x, m0) does not decrease with x).
+  if (tid == 0) sred[2] = 0u;  // keys collected from the front
+  __syncthreads();
+  const float m0 = sp.m0, m1 = sp.m1;
+  const bool prefilter = !sp.gate_off && m1 >= 0.0f;
+  for (int s = tid; s < M; s += nt) {
+    const uint32_t c = slot_cluster(cnt, c0s, np, s);
+    const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
+    const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | c;
+    if (__ldg(&sp.single[c])) {
+      const unsigned pos = atomicAdd(&sred[1], 1u);
+      if (pos < (unsigned)S_smem) keys[S_smem - 1 - pos] = key;
+    } else {
+      const uint32_t db = __float_as_uint(d);
+      const uint32_t prev = atomicMin(&sred[0], db);  // d >= 0: bits order as values
+      bool maybe = true;
+      if (prefilter) {
+        const float dm = __uint_as_float(prev < db ? prev : db);
+        maybe = d <= __fadd_rn(dm, __fmaf_rn(m1, dm, m0));
+      }
+      if (maybe) {
+        const unsigned pos = atomicAdd(&sred[2], 1u);
+        if (pos < (unsigned)S_smem) keys[pos] = key;
+      }
+    }
+  }
+  __syncthreads();
+  const uint32_t dmin_bits = sred[0];
+  float theta = __int_as_float(0x7f800000);
+  if (!sp.gate_off && dmin_bits != 0xffffffffu) {
+    const float dmin = __uint_as_float(dmin_bits);
+    theta = __fadd_rn(dmin, __fmaf_rn(m1, dmin, m0));  // theta = d_min + M(d_min)
+  }
+  const int nA = (int)sred[1], nB = (int)sred[2];
+  int Mk = nA + nB;
+  if (Mk <= S_smem) {
+    // keep the front keys within the final gate, compacted toward the front
+    // (a key never moves up, and each chunk reads before it writes), then move
+    // the C^dir keys down behind them
+    int *flag = ibuf;  // the probe offsets are no longer needed
+    __syncthreads();
+    for (int i = tid; i < nB; i += nt)
+      flag[i] = __uint_as_float((uint32_t)(keys[i] >> 32)) <= theta ? 1 : 0;
+    __syncthreads();
+    const int nS = block_exclusive_scan(flag, nB, warp_sums);
+    for (int i0 = 0; i0 < nB; i0 += 4 * nt) {
+      uint64_t kb[4];
+      int rk[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int i = i0 + e * nt + tid;
+        rk[e] = -1;
+        kb[e] = 0;
+        if (i < nB && (i + 1 < nB ? flag[i + 1] : nS) > flag[i]) {
+          rk[e] = flag[i];
+          kb[e] = keys[i];
+        }
+      }
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (rk[e] >= 0) keys[rk[e]] = kb[e];
+      __syncthreads();
+    }
+    for (int t0 = 0; t0 < nA; t0 += 4 * nt) {
+      uint64_t kb[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int t = t0 + e * nt + tid;
+        kb[e] = t < nA ? keys[S_smem - nA + t] : 0;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int t = t0 + e * nt + tid;
+        if (t < nA) keys[nS + t] = kb[e];
+      }
+      __syncthreads();
+    }
+    Mk = nS + nA;
+  } else {
+    Mk = S_smem + 1;  // does not fit: the slab path below
+  }
+  if (Mk <= S_smem) return select_tail_smem(sp, keys, Mk, warp_sums, seg, L, Lmax, total);
+  int Sn = 1;
+  int *ints = ibuf;
+  {
+    // more keys than shared memory holds: all candidate keys in the global slab
+    // (slab is present: without it M <= S_full = S_smem)
+    while (Sn < M) Sn <<= 1;
+    if (slab == nullptr || Sn > S_full) {
+      if (tid == 0) set_err(sp.err, NR_DEV_TOO_MANY);
+      *total = 0;
+      return 0;
+    }
+    keys = reinterpret_cast<uint64_t *>(slab);
+    ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
+    for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
+      const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
+      for (int j = 0; j < n; ++j) keys[o + j] = (uint64_t)(uint32_t)(c0s[i] + j);
+    }
+    __syncthreads();
+    for (int s = tid; s < M; s += nt) {
+      const uint32_t c = (uint32_t)keys[s];
+      const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
+      const bool keep = __ldg(&sp.single[c]) || d <= theta;
+      keys[s] = keep ? (((uint64_t)__float_as_uint(d) << 32) | c) : kEmpty;
+    }
+    for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
+    __syncthreads();
+    bitonic_sort(keys, Sn);
+  }
+  // keep C^dir and the first C survivors in key order
+  int *keep = ints;  // [Sn]
+  for (int s = tid; s < Sn; s += nt) {
+    const uint64_t kk = keys[s];
+    keep[s] = (s < M && kk != kEmpty && !__ldg(&sp.single[(uint32_t)kk])) ? 1 : 0;
+  }
+  __syncthreads();
+  block_exclusive_scan(keep, Sn, warp_sums);  // survivor rank in key order
+  for (int s = tid; s < Sn; s += nt) {
+    const uint64_t kk = keys[s];
+    int kp = 0;
+    if (s < M && kk != kEmpty) kp = __ldg(&sp.single[(uint32_t)kk]) ? 1 : (keep[s] < sp.C ? 1 : 0);
+    keep[s] = kp;
+  }
+  __syncthreads();
+  const int nl = block_exclusive_scan(keep, Sn, warp_sums);  // output positions
+  for (int s = tid; s < Sn; s += nt) {
+    const uint64_t kk = keys[s];
+    if (s < M && kk != kEmpty) {
+      const int pos = keep[s];
+      const bool kept = (s + 1 < Sn ? keep[s + 1] : nl) > pos;
+      if (kept) seg[pos].row0 = (uint32_t)kk;  // cluster index for now
+    }
+  }
+  __syncthreads();
+  int *len = ints;  // [nl]
+  for (int i = tid; i < nl; i += nt) {
+    const uint32_t c = seg[i].row0;
+    if (L) L[i] = (int32_t)c;
+    const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
+    int ln = 0;
+    if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
+    else ln = (int)(r1 - r0);
+    len[i] = ln;
+    seg[i].row0 = r0;
+  }
+  if (L)
+    for (int i = nl + tid; i < Lmax; i += nt) L[i] = -1;
+  __syncthreads();
+  const int tot = block_exclusive_scan(len, nl, warp_sums);
+  for (int i = tid; i < nl; i += nt) seg[i].pos = (uint32_t)len[i];
+  __syncthreads();
+  *total = (uint32_t)tot;
+  return nl;
+}
+
+}  // namespace nrq
