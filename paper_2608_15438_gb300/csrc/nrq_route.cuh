@@ -34,7 +34,9 @@ struct RouteParams {
 };
 
 // Bytes of shared memory route_warp needs for probe budget P.
-__host__ __device__ inline size_t route_heap_bytes(int P) { return (size_t)(P + 2) * 8 + 128; }
+// heap keys [(P + 2) x 8 B], deviations by rank [32 x 4 B], and the table of
+// left-to-right sums over subsets of ranks 0..7 [256 x 4 B]
+__host__ __device__ inline size_t route_heap_bytes(int P) { return (size_t)(P + 2) * 8 + 128 + 1024; }
 
 // Writes codes[0..n) (any address space) and returns n, uniform in the warp.
 // Must be called by a whole warp. heap: route_heap_bytes(P) bytes of shared
@@ -66,6 +68,18 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
   }
   if (lane < b) ssd[rank] = dj;
   __syncwarp();
+  // psum[s] = left-to-right fp32 sum of ssd over the ranks in s (s over ranks
+  // 0..7), built by adding each s's highest rank to psum of the rest: the
+  // same order as summing the ranks one by one from 0.0f
+  float *psum = ssd + 32;
+  const int lo_ranks = b < 8 ? b : 8;
+  if (lane == 0) psum[0] = 0.0f;
+  __syncwarp();
+  for (int j = 0; j < lo_ranks; ++j) {
+    const float sj = ssd[j];
+    for (int t = lane; t < (1 << j); t += 32) psum[(1 << j) + t] = __fadd_rn(psum[t], sj);
+    __syncwarp();
+  }
   if (lane == 0) codes[0] = u0;
   int n = 1, hs = 0;
   if (rp.P > 1 && rp.bsel >= 1 && ssd[0] <= rp.smax) {
@@ -88,8 +102,10 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
     if (m + 1 < rp.bsel) {
       const float sdn = ssd[m + 1];
       // cost without rank m: fp32 sum from 0 over the other ranks, ascending
-      float costp = 0.0f;
-      for (uint32_t mm = rmask & ~(1u << m); mm; mm &= mm - 1) costp = __fadd_rn(costp, ssd[__ffs(mm) - 1]);
+      // (ranks below 8 from the table, the rest one by one)
+      const uint32_t rest = rmask & ~(1u << m);
+      float costp = psum[rest & 0xffu];
+      for (uint32_t mm = rest >> 8; mm; mm &= mm - 1) costp = __fadd_rn(costp, ssd[7 + __ffs(mm)]);
       const float c1 = __fadd_rn(costp, sdn);  // shift: rank m -> m + 1
       if (c1 <= rp.smax) {
         v1 = true;
