@@ -131,6 +131,10 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
     if (x != kEmpty) {  // sift-down of x from the root
       int i = 0;
       for (;;) {
+        if (32 * i + 1 >= hs) {  // a leaf (warp-uniform)
+          if (lane == 0) hkey[i] = x;
+          break;
+        }
         const int c = 32 * i + 1 + lane;
         const uint64_t ck = c < hs ? hkey[c] : kEmpty;
         const uint32_t chi = (uint32_t)(ck >> 32), clo = (uint32_t)ck;
