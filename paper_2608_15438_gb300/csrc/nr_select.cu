@@ -25,7 +25,7 @@ namespace {
 
 constexpr int kThreads = 128;
 
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 6)
     select_kernel(nrq::SelectParams sp, const float *__restrict__ logits,
                   const uint32_t *__restrict__ codes, const int32_t *__restrict__ nprobe,
                   int32_t *L, int32_t *nL, nr_seg *seg, uint32_t *slen, int64_t *stats,
