@@ -20,7 +20,10 @@ class Params(ctypes.Structure):
     _fields_ = [("l_sel", ctypes.c_int), ("r_max", ctypes.c_int), ("s_max", ctypes.c_float),
                 ("gate_m0", ctypes.c_float), ("gate_m1", ctypes.c_float),
                 ("round_size", ctypes.c_int), ("t_low", ctypes.c_int), ("u_min", ctypes.c_int),
-                ("f_min", ctypes.c_int), ("r_min", ctypes.c_int), ("alpha_front", ctypes.c_float)]
+                ("f_min", ctypes.c_int), ("r_min", ctypes.c_int), ("alpha_front", ctypes.c_float),
+                ("cent_mode", ctypes.c_int), ("n_bins", ctypes.c_int), ("b_batch", ctypes.c_int),
+                ("b_min", ctypes.c_int), ("c_t_low", ctypes.c_int), ("c_u_min", ctypes.c_int),
+                ("c_f_min", ctypes.c_int), ("c_alpha_front", ctypes.c_float)]
 
 
 def lib():
@@ -51,6 +54,9 @@ def lib():
         L.or_probe_list.argtypes = [i32, vp, vp, i32, ctypes.POINTER(Params), vp, vp, vp]
         L.or_probe_list.restype = i32
         L.or_cluster_list.argtypes = [vp, vp, vp, i32, i32, ctypes.POINTER(Params), vp, vp, vp]
+        L.or_cluster_list_seq.argtypes = [vp, vp, vp, vp, i32, i32, ctypes.POINTER(Params), vp, vp,
+                                          vp, vp]
+        L.or_cluster_list_seq.restype = i32
         L.or_cluster_list.restype = i32
         L.or_refine_stream.argtypes = [i32, i32, vp, vp, vp, i64, i32, ctypes.POINTER(Params),
                                        vp, vp, vp]
@@ -143,6 +149,24 @@ class Index:
         if n < 0:
             raise RuntimeError("oracle: out-of-range index in file")
         return L[:n].copy(), dL[:n].copy(), int(ndir[0])
+
+    def cluster_list_seq(self, logit, codes, scores, C, p: Params):
+        """The sequential centroid stage (Algorithm 2): returns (L, dL, n_dir,
+        n_batches)."""
+        logit = np.ascontiguousarray(logit, np.float32)
+        codes = np.ascontiguousarray(codes, np.uint32)
+        scores = np.ascontiguousarray(scores, np.float32)
+        L = np.empty(len(codes) + C, np.int32)
+        dL = np.empty(len(codes) + C, np.float32)
+        ndir = np.zeros(1, np.int32)
+        nbat = np.zeros(1, np.int32)
+        n = lib().or_cluster_list_seq(self.h, logit.ctypes.data, codes.ctypes.data,
+                                      scores.ctypes.data, len(codes), C, ctypes.byref(p),
+                                      L.ctypes.data, dL.ctypes.data, ndir.ctypes.data,
+                                      nbat.ctypes.data)
+        if n < 0:
+            raise RuntimeError("oracle: out-of-range index in file")
+        return L[:n].copy(), dL[:n].copy(), int(ndir[0]), int(nbat[0])
 
     def search(self, queries, k, P, C, p: Params, logits=None, nthreads=None):
         queries = np.ascontiguousarray(queries)

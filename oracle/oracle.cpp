@@ -42,6 +42,14 @@ extern "C" void or_params_default(or_params *p) {
   p->f_min = 1;
   p->r_min = 1;
   p->alpha_front = 0.5f;
+  p->cent_mode = 0;
+  p->n_bins = 1;
+  p->b_batch = 256;
+  p->b_min = 1;
+  p->c_t_low = 0;
+  p->c_u_min = 1;
+  p->c_f_min = 1;
+  p->c_alpha_front = 0.5f;
 }
 
 // ---------------------------------------------------------------- index file
@@ -365,6 +373,95 @@ extern "C" int or_cluster_list(const or_index *ix, const float *logit, const uin
   return (int)all.size();
 }
 
+// Algorithm 2 in its own order (Sec. 3.4.2): bins from Algorithm 1 in
+// increasing score, each bin's single-cluster buckets to C^dir, its other
+// clusters in batches; per batch the running d_min, the gate, the bounded
+// heap kept under the gate, the heap/front update counts and the stop test.
+extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const uint32_t *codes,
+                                   const float *score, int nprobe, int C, const or_params *p,
+                                   int32_t *L, float *dL, int32_t *n_dir, int32_t *n_batches) {
+  const int b = ix->b;
+  const uint64_t nbuckets = (uint64_t)1 << b;
+  const int nbins = p->n_bins > 1 ? p->n_bins : 1;
+  const bool binned = nbins > 1 && p->s_max < kInf;
+  auto bin_of = [&](float s) {
+    if (!binned) return 0;
+    const float z = (s * (float)nbins) / p->s_max;  // Bin(s; N_bins, S_max)
+    const int zi = (int)z;
+    return zi < nbins - 1 ? zi : nbins - 1;
+  };
+  const bool gate_off = std::isinf(p->gate_m0) && p->gate_m0 > 0.0f;
+  const int B = p->b_batch > 0 ? p->b_batch : 1;
+  std::vector<std::pair<float, int64_t>> dir, H;
+  float dmin = kInf;
+  int b_proc = 0, t_low = 0, batches = 0;
+  bool stop = false;
+  int i = 0;
+  while (i < nprobe && !stop) {
+    const int z = bin_of(score[i]);
+    int j = i;
+    while (j < nprobe && bin_of(score[j]) == z) ++j;  // the bin: probes [i, j)
+    b_proc += 1;
+    std::vector<int64_t> cz;  // MapBucketsToClusters
+    for (int t = i; t < j; ++t) {
+      const uint64_t u = codes[t];
+      if (u >= nbuckets) return -1;
+      const uint32_t c0 = ix->bkt_off[u], c1 = ix->bkt_off[u + 1];
+      if (c1 < c0 || (int64_t)c1 > ix->n_cl) return -1;
+      if (c1 - c0 == 1) {
+        dir.push_back({centroid_distance(logit, &ix->cent[(size_t)c0 * b], b), (int64_t)c0});
+      } else {
+        for (uint32_t c = c0; c < c1; ++c) cz.push_back((int64_t)c);
+      }
+    }
+    for (size_t s0 = 0; s0 < cz.size() && !stop; s0 += (size_t)B) {
+      const size_t s1 = std::min(cz.size(), s0 + (size_t)B);
+      std::vector<std::pair<float, int64_t>> batch;
+      for (size_t t = s0; t < s1; ++t)
+        batch.push_back({centroid_distance(logit, &ix->cent[(size_t)cz[t] * b], b), cz[t]});
+      for (auto &e : batch) dmin = std::min(dmin, e.first);
+      float theta = kInf, front_th = kInf;
+      if (!gate_off) {
+        const float m = std::fmaf(p->gate_m1, dmin, p->gate_m0);  // M(d_min)
+        theta = dmin + m;
+        front_th = dmin + p->c_alpha_front * m;
+      }
+      // KeepTopKUnderGate: the C smallest of H U batch within the gate
+      std::vector<std::pair<float, int64_t>> all;
+      for (auto &e : H)
+        if (e.first <= theta) all.push_back(e);
+      for (auto &e : batch)
+        if (e.first <= theta) all.push_back(e);
+      std::sort(all.begin(), all.end(), dc_less);
+      if ((int)all.size() > C) all.resize((size_t)C);
+      int updates = 0, front = 0;
+      for (auto &e : batch)
+        for (auto &h : all)
+          if (h == e) {
+            updates += 1;
+            if (e.first <= front_th) front += 1;
+          }
+      H.swap(all);
+      batches += 1;
+      const bool lowq = updates < p->c_u_min && front < p->c_f_min;
+      t_low = lowq ? t_low + 1 : 0;
+      if (p->c_t_low > 0 && (int)H.size() == C && b_proc >= p->b_min && t_low >= p->c_t_low)
+        stop = true;
+    }
+    i = j;
+  }
+  std::vector<std::pair<float, int64_t>> out(dir);
+  out.insert(out.end(), H.begin(), H.end());
+  std::sort(out.begin(), out.end(), dc_less);
+  for (size_t t = 0; t < out.size(); ++t) {
+    L[t] = (int32_t)out[t].second;
+    if (dL) dL[t] = out[t].first;
+  }
+  if (n_dir) *n_dir = (int32_t)dir.size();
+  if (n_batches) *n_batches = batches;
+  return (int)out.size();
+}
+
 // ---------------------------------------------------------------- refinement
 // Exact squared L2 in the original space (uint8 kept as integers, Sec. 4.1.1),
 // top-k by (dist, id), candidates processed in rounds of R with the
@@ -494,9 +591,21 @@ extern "C" int or_search(const or_index *ix, const void *queries, const float *l
     else
       encode_one(ix, queries, qi, lg.data());
     std::vector<uint32_t> codes((size_t)P);
-    int np = or_probe_list(b, lg.data(), ix->tau.data(), P, p, codes.data(), nullptr, nullptr);
+    std::vector<uint64_t> keys((size_t)P);
+    int np = or_probe_list(b, lg.data(), ix->tau.data(), P, p, codes.data(), keys.data(), nullptr);
     std::vector<int32_t> L((size_t)np + (size_t)C);
-    int nl = or_cluster_list(ix, lg.data(), codes.data(), np, C, p, L.data(), nullptr, nullptr);
+    int nl;
+    if (p->cent_mode == 1) {
+      std::vector<float> score((size_t)np);  // summed deviation of each probe's flip set
+      for (int t = 0; t < np; ++t) {
+        const uint32_t cb = (uint32_t)(keys[t] >> 32);
+        memcpy(&score[t], &cb, 4);
+      }
+      nl = or_cluster_list_seq(ix, lg.data(), codes.data(), score.data(), np, C, p, L.data(),
+                               nullptr, nullptr, nullptr);
+    } else {
+      nl = or_cluster_list(ix, lg.data(), codes.data(), np, C, p, L.data(), nullptr, nullptr);
+    }
     if (nl < 0) {
       bad = 1;
       nl = 0;

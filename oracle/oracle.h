@@ -16,6 +16,8 @@
  *   or_cluster_list    bucket -> clusters (Sec. 3.3), singleton buckets to C^dir,
  *                      centroid distances, calibrated gate theta = d + M(d) and
  *                      top-C (Algorithm 2, Sec. 3.4.2)
+ *   or_cluster_list_seq  the same stage in Algorithm 2's sequence: score bins,
+ *                      centroid batches, running d_min, heap-quality early stop
  *   or_refine_stream   exact squared-L2 refinement into a top-k with heap-quality
  *                      early stopping counted in fixed rounds (Sec. 3.4.2, Alg. 2)
  *   or_search          all of the above per query, threads across queries
@@ -55,6 +57,16 @@ typedef struct {
   int f_min;
   int r_min;          /* no stop before r_min completed rounds */
   float alpha_front;  /* front = first ceil(alpha_front * k) slots of the top-k */
+  /* centroid stage: 0 = order-independent (final d_min gate, top-C); 1 = the
+   * sequential stage of Algorithm 2 (score bins, centroid batches, running
+   * d_min gate, a bounded heap of C, early stop on heap quality) */
+  int cent_mode;
+  int n_bins;          /* score bins over [0, s_max] (Algorithm 1); one bin if s_max = +inf */
+  int b_batch;         /* clusters per centroid batch (B_batch) */
+  int b_min;           /* bins started before a stop is allowed (B_min) */
+  int c_t_low;         /* stop after c_t_low consecutive low-quality batches; 0: never */
+  int c_u_min, c_f_min; /* batch low quality iff updates < c_u_min and front < c_f_min */
+  float c_alpha_front; /* front threshold d_min + c_alpha_front * M(d_min) */
 } or_params;
 
 void or_params_default(or_params *p);
@@ -98,6 +110,21 @@ int or_probe_list(int b, const float *logit, const float *tau, int P, const or_p
  * n_dir (optional) gets |C^dir|. Returns |L|, or -1 on an out-of-range index. */
 int or_cluster_list(const or_index *ix, const float *logit, const uint32_t *codes, int nprobe,
                     int C, const or_params *p, int32_t *L, float *dL, int32_t *n_dir);
+
+/* The sequential centroid stage (Algorithm 2) of one query: probes in order
+ * with scores score[i] (the summed deviation of their flip set), binned by
+ * Bin(s) = min(n_bins - 1, floor(s n_bins / s_max)); bins processed in order;
+ * single-cluster buckets of every bin entered go to C^dir; the other clusters
+ * of a bin, in probe order, in batches of b_batch: d_min <- min(d_min, batch
+ * min), theta = d_min + M(d_min), H <- the C smallest (d, c) of H U batch with
+ * d <= theta; updates = batch entries in H, front = those with
+ * d <= d_min + c_alpha_front M(d_min); stop when |H| = C, at least b_min bins
+ * were entered and c_t_low consecutive batches had updates < c_u_min and
+ * front < c_f_min. L = C^dir U H in (d, c) order. n_batches (optional) gets
+ * the batches processed. Returns |L|, or -1 on an out-of-range index. */
+int or_cluster_list_seq(const or_index *ix, const float *logit, const uint32_t *codes,
+                        const float *score, int nprobe, int C, const or_params *p, int32_t *L,
+                        float *dL, int32_t *n_dir, int32_t *n_batches);
 
 /* Refinement over an explicit candidate stream: rows [n x D] (u8 or f32 by
  * dtype), ids [n]. out_ids/out_d [k] sorted by (dist, id), padded (-1, +inf).
