@@ -84,6 +84,27 @@ typedef struct {
   int f_min;          /* default 1 */
   int r_min;          /* default 1 */
   float alpha_front;  /* in [0, 1]; default 0.5 */
+  /* Centroid stage. cent_mode 0 (default): order independent, the gate uses
+   * the final d_min over all probed non-singleton clusters and C^cent is the
+   * top-C of the survivors. cent_mode 1: Algorithm 2's sequence: probes in
+   * score bins Bin(s) = min(n_bins - 1, floor(s n_bins / s_max)) (one bin when
+   * s_max = +inf); bins in order; single-cluster buckets of every bin entered
+   * to C^dir; the other clusters of a bin, in probe order, in batches of
+   * b_batch: d_min <- min(d_min, batch minimum), theta = d_min + M(d_min),
+   * H <- the C smallest (d, c) of H U batch with d <= theta; a batch is low
+   * quality iff fewer than c_u_min of its clusters are in H and fewer than
+   * c_f_min of those have d <= d_min + c_alpha_front M(d_min); stop when
+   * |H| = C, at least b_min bins were entered and c_t_low consecutive batches
+   * were low quality (c_t_low = 0: never). C^cent = H. */
+  int cent_mode;        /* 0 or 1; default 0. Mode 1 needs probe_budget <= 2048 and
+                         * its shared memory (about 16 C + 12 P + 8 b_batch bytes)
+                         * within 220 KB; searches outside are NR_ERR_INVALID_ARG */
+  int n_bins;           /* >= 1; default 1 */
+  int b_batch;          /* in [1, 2048]; default 256 */
+  int b_min;            /* >= 0; default 1 */
+  int c_t_low;          /* >= 0; default 0 */
+  int c_u_min, c_f_min; /* >= 0; default 1, 1 */
+  float c_alpha_front;  /* in [0, 1]; default 0.5 */
 } nr_params;
 
 /* Per-search statistics (sums over the queries of the last search call). */

@@ -107,6 +107,10 @@ nr_status check_params(const nr_params *p) {
   if (p->t_low < 0 || p->r_min < 0 || p->u_min < 0 || p->f_min < 0) return NR_ERR_INVALID_ARG;
   if (!(p->alpha_front >= 0.0f && p->alpha_front <= 1.0f)) return NR_ERR_INVALID_ARG;
   if (std::isnan(p->s_max) || std::isnan(p->gate_m0) || std::isnan(p->gate_m1)) return NR_ERR_INVALID_ARG;
+  if ((p->cent_mode != 0 && p->cent_mode != 1) || p->n_bins < 1 || p->b_batch < 1 ||
+      p->b_batch > 2048 || p->b_min < 0 || p->c_t_low < 0 || p->c_u_min < 0 || p->c_f_min < 0 ||
+      !(p->c_alpha_front >= 0.0f && p->c_alpha_front <= 1.0f))
+    return NR_ERR_INVALID_ARG;
   return NR_OK;
 }
 
@@ -218,6 +222,14 @@ nr_status nr_params_default(nr_params *p) {
   p->f_min = 1;
   p->r_min = 1;
   p->alpha_front = 0.5f;
+  p->cent_mode = 0;
+  p->n_bins = 1;
+  p->b_batch = 256;
+  p->b_min = 1;
+  p->c_t_low = 0;
+  p->c_u_min = 1;
+  p->c_f_min = 1;
+  p->c_alpha_front = 0.5f;
   return NR_OK;
 }
 
@@ -611,6 +623,10 @@ static nr_status check_budgets(const nr_index *ix, int64_t nq, int k, int P, int
   if (nq < 0 || P < 1 || P > kMaxProbe || C < 1 || C > kMaxClusterBudget) return NR_ERR_INVALID_ARG;
   if ((int64_t)P * ix->K_max > kMaxSelect) return NR_ERR_INVALID_ARG;
   if (k < 1 || k > kMaxTopK || nq > ((int64_t)1 << 31) - 1) return NR_ERR_INVALID_ARG;
+  // the sequential centroid stage sorts C^dir in one block and keeps H in
+  // shared memory
+  if (ix->params.cent_mode == 1 && (P > 2048 || nr_select_smem_bytes(ix, P, C) > (size_t)220 * 1024))
+    return NR_ERR_INVALID_ARG;
   return NR_OK;
 }
 

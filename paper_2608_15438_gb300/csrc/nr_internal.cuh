@@ -69,7 +69,9 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
                              cudaStream_t s);
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s);
-size_t nr_select_smem_bytes(int P, int C, int K_max);
+// dynamic shared memory of the select kernel for budgets (P, C) under the
+// index's current parameters
+size_t nr_select_smem_bytes(const nr_index *ix, int P, int C);
 // global scratch per query that select needs for probe budget P (0: none)
 size_t nr_select_slab_bytes(int P, int K_max);
 cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t *d_codes,

@@ -25,7 +25,9 @@ namespace {
 
 constexpr int kThreads = 128;
 
-__global__ void __launch_bounds__(kThreads, 6)
+// MODE 0: the order-independent stage; MODE 1: the sequential stage
+template <int MODE>
+__global__ void __launch_bounds__(kThreads, MODE == 0 ? 6 : 1)
     select_kernel(nrq::SelectParams sp, const float *__restrict__ logits,
                   const uint32_t *__restrict__ codes, const int32_t *__restrict__ nprobe,
                   int32_t *L, int32_t *nL, nr_seg *seg, uint32_t *slen, int64_t *stats,
@@ -34,7 +36,9 @@ __global__ void __launch_bounds__(kThreads, 6)
   const int q = blockIdx.x, tid = threadIdx.x;
   const int Lmax = sp.P + sp.C;
   unsigned char *scratch = smem;
-  float *slog = reinterpret_cast<float *>(smem + nrq::select_scratch_bytes(sp.P, sp.K_max));
+  const size_t sbytes = MODE == 1 ? nrq::select_seq_bytes(sp.P, sp.C, sp.b_batch)
+                                   : nrq::select_scratch_bytes(sp.P, sp.K_max);
+  float *slog = reinterpret_cast<float *>(smem + sbytes);
   int *warp_sums = reinterpret_cast<int *>(slog + 32);
   unsigned *sred = reinterpret_cast<unsigned *>(warp_sums + 32);
   const int np = nprobe[q];
@@ -42,9 +46,14 @@ __global__ void __launch_bounds__(kThreads, 6)
   __syncthreads();
   uint32_t total = 0;
   unsigned char *qslab = slab ? slab + (size_t)q * slab_bytes : nullptr;
-  const int nl = nrq::select_block(sp, slog, codes + (size_t)q * sp.P, np, scratch, qslab, warp_sums, sred,
-                                   seg + (size_t)q * Lmax, L ? L + (size_t)q * Lmax : nullptr,
-                                   Lmax, &total);
+  const int nl =
+      MODE == 1
+          ? nrq::select_block_seq(sp, slog, codes + (size_t)q * sp.P, np, scratch, warp_sums, sred,
+                                  seg + (size_t)q * Lmax, L ? L + (size_t)q * Lmax : nullptr, Lmax,
+                                  &total)
+          : nrq::select_block(sp, slog, codes + (size_t)q * sp.P, np, scratch, qslab, warp_sums,
+                              sred, seg + (size_t)q * Lmax, L ? L + (size_t)q * Lmax : nullptr,
+                              Lmax, &total);
   if (tid == 0) {
     nL[q] = nl;
     slen[q] = total;
@@ -77,14 +86,26 @@ nrq::SelectParams nr_select_params(nr_index *ix, int P, int C) {
   sp.m0 = m0;
   sp.m1 = ix->params.gate_m1;
   sp.err = ix->d_err;
+  sp.mode = ix->params.cent_mode;
+  sp.n_bins = ix->params.n_bins;
+  sp.b_batch = ix->params.b_batch;
+  sp.b_min = ix->params.b_min;
+  sp.c_t_low = ix->params.c_t_low;
+  sp.c_u_min = ix->params.c_u_min;
+  sp.c_f_min = ix->params.c_f_min;
+  sp.s_max = ix->params.s_max;
+  sp.c_alpha_front = ix->params.c_alpha_front;
+  sp.tau = ix->tau;
   return sp;
 }
 
 size_t nr_select_slab_bytes(int P, int K_max) { return nrq::select_slab_bytes(P, K_max); }
 
-size_t nr_select_smem_bytes(int P, int C, int K_max) {
-  (void)C;
-  return nrq::select_scratch_bytes(P, K_max) + 32 * 4 + 32 * 4 + 16;
+size_t nr_select_smem_bytes(const nr_index *ix, int P, int C) {
+  const nr_params &p = ix->params;
+  const size_t s = p.cent_mode == 1 ? nrq::select_seq_bytes(P, C, p.b_batch)
+                                    : nrq::select_scratch_bytes(P, ix->K_max);
+  return s + 32 * 4 + 32 * 4 + 16;
 }
 
 cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t *d_codes,
@@ -92,15 +113,22 @@ cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t
                              int32_t *d_nL, nr_seg *d_seg, uint32_t *d_slen, int64_t *d_stats,
                              void *d_slab, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
-  const size_t smem = nr_select_smem_bytes(P, C, ix->K_max);
-  cudaError_t e = cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)smem);
-  if (e != cudaSuccess) return e;
+  const size_t smem = nr_select_smem_bytes(ix, P, C);
   const nrq::SelectParams sp = nr_select_params(ix, P, C);  // before the launch configuration
-  select_kernel<<<(unsigned)nq, kThreads, smem, s>>>(sp, d_logits, d_codes,
-                                                      d_nprobe, d_L, d_nL, d_seg, d_slen, d_stats,
-                                                      static_cast<unsigned char *>(d_slab),
-                                                      nrq::select_slab_bytes(P, ix->K_max));
+  const size_t slab_bytes = nrq::select_slab_bytes(P, ix->K_max);
+  unsigned char *slab = static_cast<unsigned char *>(d_slab);
+  cudaError_t e;
+  if (sp.mode == 1) {
+    e = cudaFuncSetAttribute(select_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    select_kernel<1><<<(unsigned)nq, kThreads, smem, s>>>(sp, d_logits, d_codes, d_nprobe, d_L, d_nL,
+                                                          d_seg, d_slen, d_stats, slab, slab_bytes);
+  } else {
+    e = cudaFuncSetAttribute(select_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    select_kernel<0><<<(unsigned)nq, kThreads, smem, s>>>(sp, d_logits, d_codes, d_nprobe, d_L, d_nL,
+                                                          d_seg, d_slen, d_stats, slab, slab_bytes);
+  }
   ix->launches += 1;
   return cudaGetLastError();
 }

@@ -170,6 +170,10 @@ struct SelectParams {
   bool gate_off;
   float m0, m1;
   int *err;
+  // the sequential centroid stage (mode 1)
+  int mode, n_bins, b_batch, b_min, c_t_low, c_u_min, c_f_min;
+  float s_max, c_alpha_front;
+  const float *tau;
 };
 
 // Sort capacity for probe budget P: all clusters of P buckets. Shared memory
@@ -536,6 +540,308 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   __syncthreads();
   *total = (uint32_t)tot;
   return nl;
+}
+
+// ============================================================== select, mode 1
+// The sequential centroid stage of Algorithm 2 (cent_mode 1), one block per
+// query: probe scores and score bins (Algorithm 1), bins in order, C^dir of
+// every bin entered, the other clusters in batches of b_batch with the
+// running d_min gate, a bounded heap H of C kept sorted by (d, c), the
+// heap-quality stop. Limits: P <= 2048 (C^dir is sorted by one block merge
+// sort), b_batch <= 2048.
+
+__host__ __device__ inline int seq_pow2(int v) {
+  int p = 128;
+  while (p < v) p <<= 1;
+  return p;
+}
+// shared memory of select_block_seq
+__host__ __device__ inline size_t select_seq_bytes(int P, int C, int B) {
+  return (size_t)2 * C * 8                               // H, two buffers
+         + (size_t)select_smem_keys(seq_pow2(B)) * 8     // one batch
+         + (size_t)select_smem_keys(seq_pow2(P)) * 8     // C^dir keys
+         + (size_t)(4 * P + 1) * 4                       // clusters, first cluster, slots, bin per probe
+         + 32 * 4 * 2 + 64;                              // deviations and bits by rank, state
+}
+
+// Bin(s; n_bins, s_max) of Algorithm 1: min(n_bins - 1, floor(s n_bins / s_max)),
+// or 0 when there is one bin or no finite s_max
+__device__ __forceinline__ int score_bin(float s, int n_bins, float s_max) {
+  if (n_bins <= 1 || !(s_max < __int_as_float(0x7f800000))) return 0;
+  const int z = (int)__fdiv_rn(__fmul_rn(s, (float)n_bins), s_max);
+  return z < n_bins - 1 ? z : n_bins - 1;
+}
+
+// Index of the last element of the nondecreasing off[lo..hi) that is <= v.
+__device__ __forceinline__ int last_le(const int *off, int lo, int hi, int v) {
+  int a = lo, b = hi - 1;
+  while (a < b) {
+    const int mid = (a + b + 1) >> 1;
+    if (off[mid] <= v) a = mid;
+    else b = mid - 1;
+  }
+  return a;
+}
+
+// Merge path: how many of the first d outputs of merging A[0..na) and
+// B[0..nb) (ascending, ties to A) come from A. A is read through pad16 when
+// a_pad, B when b_pad.
+__device__ __forceinline__ int merge_split(const uint64_t *A, int na, bool a_pad, const uint64_t *B,
+                                           int nb, bool b_pad, int d) {
+  int a = d > nb ? d - nb : 0, hi = d < na ? d : na;
+  while (a < hi) {
+    const int mid = (a + hi) >> 1;
+    const uint64_t x = A[a_pad ? pad16(mid) : mid], y = B[b_pad ? pad16(d - 1 - mid) : d - 1 - mid];
+    if (x > y) hi = mid;
+    else a = mid + 1;
+  }
+  return a;
+}
+
+template <int E>
+__device__ __forceinline__ void sort_to_padded(uint64_t *k, int n) {
+  uint64_t r[E];
+  merge_sort_regs<E>(k, n, r);
+  __syncthreads();
+#pragma unroll
+  for (int e = 0; e < E; ++e) k[pad16(threadIdx.x * E + e)] = r[e];
+  __syncthreads();
+}
+// Sorts k[0..n) (n <= 16 blockDim.x) into k's padded layout (pad16(i) holds
+// the i-th smallest; kEmpty past n).
+__device__ __forceinline__ void sort_padded(uint64_t *k, int n) {
+  const int nt = blockDim.x;
+  if (n <= nt) sort_to_padded<1>(k, n);
+  else if (n <= 2 * nt) sort_to_padded<2>(k, n);
+  else if (n <= 4 * nt) sort_to_padded<4>(k, n);
+  else if (n <= 8 * nt) sort_to_padded<8>(k, n);
+  else sort_to_padded<16>(k, n);
+}
+
+__device__ __forceinline__ int select_block_seq(const SelectParams &sp, const float *slog,
+                                                const uint32_t *codes, int np, unsigned char *seq,
+                                                int *warp_sums, unsigned *sred, nr_seg *seg,
+                                                int32_t *L, int Lmax, uint32_t *total) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int C = sp.C, B = sp.b_batch, b = sp.b;
+  uint64_t *Hb0 = reinterpret_cast<uint64_t *>(seq);
+  uint64_t *Hb1 = Hb0 + C;
+  uint64_t *Bk = Hb1 + C;
+  uint64_t *dirk = Bk + select_smem_keys(seq_pow2(B));
+  int *cnt = reinterpret_cast<int *>(dirk + select_smem_keys(seq_pow2(sp.P)));
+  int *c0s = cnt + sp.P;
+  int *nsoff = c0s + sp.P;  // [P + 1]
+  int *zb = nsoff + sp.P + 1;
+  float *sdr = reinterpret_cast<float *>(zb + sp.P);  // deviation of rank r
+  int *bitr = reinterpret_cast<int *>(sdr + 32);      // bit index of rank r
+  unsigned *st = reinterpret_cast<unsigned *>(bitr + 32);  // [0] u0, [1] |C^dir|
+  const uint32_t nbk = 1u << b;
+  // bucket lookups
+  for (int i = tid; i < np; i += nt) {
+    const uint32_t u = codes[i];
+    int n = 0, c0 = 0;
+    if (u >= nbk) {
+      set_err(sp.err, NR_DEV_BAD_CODE);
+    } else {
+      const uint32_t lo = __ldg(&sp.bkt_off[u]), hi = __ldg(&sp.bkt_off[u + 1]);
+      if (hi < lo || (int64_t)hi > sp.n_cl) {
+        set_err(sp.err, NR_DEV_BAD_BUCKET);
+      } else {
+        n = (int)(hi - lo);
+        c0 = (int)lo;
+        if (n > sp.K_max) {
+          set_err(sp.err, NR_DEV_TOO_MANY);
+          n = sp.K_max;
+        }
+      }
+    }
+    cnt[i] = n;
+    c0s[i] = c0;
+  }
+  // the base code and the rank order of the bits (Eq. 10, Algorithm 1)
+  if (tid == 0) {
+    uint32_t u0 = 0;
+    for (int j = 0; j < b; ++j) {
+      const float l = slog[j], t = __ldg(&sp.tau[j]);
+      if (l >= t) u0 |= 1u << j;
+      sdr[j] = fabsf(__fsub_rn(l, t));
+      bitr[j] = j;
+    }
+    for (int r = 1; r < b; ++r) {  // insertion sort by (deviation, bit)
+      const float dv = sdr[r];
+      const int bj = bitr[r];
+      int q = r - 1;
+      while (q >= 0 && (sdr[q] > dv || (sdr[q] == dv && bitr[q] > bj))) {
+        sdr[q + 1] = sdr[q];
+        bitr[q + 1] = bitr[q];
+        --q;
+      }
+      sdr[q + 1] = dv;
+      bitr[q + 1] = bj;
+    }
+    st[0] = u0;
+    st[1] = 0u;
+  }
+  __syncthreads();
+  // each probe's score (summed deviation of its flip set, ranks ascending),
+  // its bin, and its clusters outside C^dir
+  const uint32_t u0 = st[0];
+  for (int i = tid; i < np; i += nt) {
+    const uint32_t flips = codes[i] ^ u0;
+    float s = 0.0f;
+    for (int r = 0; r < b; ++r)
+      if ((flips >> bitr[r]) & 1u) s = __fadd_rn(s, sdr[r]);
+    zb[i] = score_bin(s, sp.n_bins, sp.s_max);
+    nsoff[i] = cnt[i] >= 2 ? cnt[i] : 0;
+  }
+  __syncthreads();
+  const int NS = block_exclusive_scan(nsoff, np, warp_sums);
+  if (tid == 0) nsoff[np] = NS;
+  __syncthreads();
+  const bool gate_off = sp.gate_off;
+  float dmin = __int_as_float(0x7f800000);
+  int hN = 0, t_low = 0, b_proc = 0;
+  bool stop = false;
+  uint64_t *H = Hb0, *Hn = Hb1;
+  int i = 0;
+  while (i < np && !stop) {
+    const int z = zb[i];
+    int a = i + 1, e = np;  // first probe of a later bin
+    while (a < e) {
+      const int mid = (a + e) >> 1;
+      if (zb[mid] <= z) a = mid + 1;
+      else e = mid;
+    }
+    const int j = a;
+    b_proc += 1;
+    for (int p = i + tid; p < j; p += nt)  // C^dir of this bin
+      if (cnt[p] == 1) {
+        const uint32_t c = (uint32_t)c0s[p];
+        const float d = centroid_dist(sp.cent + (size_t)c * b, slog, b);
+        const unsigned pos = atomicAdd(&st[1], 1u);
+        dirk[pos] = ((uint64_t)__float_as_uint(d) << 32) | c;
+      }
+    const int sa = nsoff[i], sb = nsoff[j];
+    for (int x = sa; x < sb && !stop; x += B) {
+      const int nb = sb - x < B ? sb - x : B;
+      if (tid == 0) sred[0] = 0xffffffffu;
+      __syncthreads();
+      for (int t = tid; t < nb; t += nt) {
+        const int slot = x + t;
+        const int p = last_le(nsoff, i, j, slot);
+        const uint32_t c = (uint32_t)(c0s[p] + (slot - nsoff[p]));
+        const float d = centroid_dist(sp.cent + (size_t)c * b, slog, b);
+        Bk[t] = ((uint64_t)__float_as_uint(d) << 32) | c;
+        atomicMin(&sred[0], __float_as_uint(d));
+      }
+      __syncthreads();
+      const float bmin = __uint_as_float(sred[0]);
+      if (bmin < dmin) dmin = bmin;
+      float theta = __int_as_float(0x7f800000), front_th = theta;
+      if (!gate_off) {
+        const float m = __fmaf_rn(sp.m1, dmin, sp.m0);  // M(d_min)
+        theta = __fadd_rn(dmin, m);
+        front_th = __fadd_rn(dmin, __fmul_rn(sp.c_alpha_front, m));
+      }
+      for (int t = tid; t < nb; t += nt)  // the gate
+        if (!(__uint_as_float((uint32_t)(Bk[t] >> 32)) <= theta)) Bk[t] = kEmpty;
+      __syncthreads();
+      sort_padded(Bk, nb);
+      // gated keys of the batch (sorted, kEmpty last) and of H (a prefix)
+      int bk = 0;
+      {
+        int lo = 0, hi = nb;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (Bk[pad16(mid)] != kEmpty) lo = mid + 1;
+          else hi = mid;
+        }
+        bk = lo;
+      }
+      int hf = 0;
+      {
+        int lo = 0, hi = hN;
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (__uint_as_float((uint32_t)(H[mid] >> 32)) <= theta) lo = mid + 1;
+          else hi = mid;
+        }
+        hf = lo;
+      }
+      const int hn = hf + bk < C ? hf + bk : C;
+      // the first hn of merge(H[0..hf), batch[0..bk)) into Hn
+      const int Q = (hn + nt - 1) / nt;
+      const int o0 = tid * Q < hn ? tid * Q : hn, o1 = o0 + Q < hn ? o0 + Q : hn;
+      int ia = merge_split(H, hf, false, Bk, bk, true, o0);
+      int ib = o0 - ia;
+      int upd = 0, fr = 0;
+      for (int o = o0; o < o1; ++o) {
+        const uint64_t xa = ia < hf ? H[ia] : kEmpty, xb = ib < bk ? Bk[pad16(ib)] : kEmpty;
+        const bool takeA = ib >= bk || (ia < hf && xa <= xb);
+        if (takeA) {
+          Hn[o] = xa;
+          ++ia;
+        } else {
+          Hn[o] = xb;
+          ++ib;
+          ++upd;
+          if (__uint_as_float((uint32_t)(xb >> 32)) <= front_th) ++fr;
+        }
+      }
+      int updates, front;
+      block_thread_scan(upd, warp_sums, &updates);
+      block_thread_scan(fr, warp_sums, &front);
+      uint64_t *tmp = H;
+      H = Hn;
+      Hn = tmp;
+      hN = hn;
+      t_low = (updates < sp.c_u_min && front < sp.c_f_min) ? t_low + 1 : 0;
+      stop = sp.c_t_low > 0 && hN == C && b_proc >= sp.b_min && t_low >= sp.c_t_low;
+      __syncthreads();
+    }
+    i = j;
+  }
+  // L = C^dir U H in (d, c) order, with the clusters' segments
+  __syncthreads();
+  const int nd = (int)st[1];
+  sort_padded(dirk, nd);
+  const int n = nd + hN;
+  const int Q = (n + nt - 1) / nt;
+  const int o0 = tid * Q < n ? tid * Q : n, o1 = o0 + Q < n ? o0 + Q : n;
+  const int ia0 = merge_split(dirk, nd, true, H, hN, false, o0);
+  int ia = ia0, ib = o0 - ia0;
+  int lsum = 0;
+  for (int o = o0; o < o1; ++o) {
+    const uint64_t xa = ia < nd ? dirk[pad16(ia)] : kEmpty, xb = ib < hN ? H[ib] : kEmpty;
+    const bool takeA = ib >= hN || (ia < nd && xa <= xb);
+    const uint32_t c = (uint32_t)(takeA ? xa : xb);
+    if (takeA) ++ia;
+    else ++ib;
+    const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
+    if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
+    else lsum += (int)(r1 - r0);
+  }
+  int tot;
+  int spos = block_thread_scan(lsum, warp_sums, &tot);
+  ia = ia0;
+  ib = o0 - ia0;
+  for (int o = o0; o < o1; ++o) {
+    const uint64_t xa = ia < nd ? dirk[pad16(ia)] : kEmpty, xb = ib < hN ? H[ib] : kEmpty;
+    const bool takeA = ib >= hN || (ia < nd && xa <= xb);
+    const uint32_t c = (uint32_t)(takeA ? xa : xb);
+    if (takeA) ++ia;
+    else ++ib;
+    const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
+    const int ln = (r1 < r0 || (int64_t)r1 > sp.N) ? 0 : (int)(r1 - r0);
+    seg[o].row0 = r0;
+    seg[o].pos = (uint32_t)spos;
+    if (L) L[o] = (int32_t)c;
+    spos += ln;
+  }
+  if (L)
+    for (int t = n + tid; t < Lmax; t += nt) L[t] = -1;
+  *total = (uint32_t)tot;
+  return n;
 }
 
 }  // namespace nrq

@@ -37,7 +37,10 @@ class Params(ctypes.Structure):
     _fields_ = [("l_sel", ctypes.c_int), ("r_max", ctypes.c_int), ("s_max", ctypes.c_float),
                 ("gate_m0", ctypes.c_float), ("gate_m1", ctypes.c_float),
                 ("round_size", ctypes.c_int), ("t_low", ctypes.c_int), ("u_min", ctypes.c_int),
-                ("f_min", ctypes.c_int), ("r_min", ctypes.c_int), ("alpha_front", ctypes.c_float)]
+                ("f_min", ctypes.c_int), ("r_min", ctypes.c_int), ("alpha_front", ctypes.c_float),
+                ("cent_mode", ctypes.c_int), ("n_bins", ctypes.c_int), ("b_batch", ctypes.c_int),
+                ("b_min", ctypes.c_int), ("c_t_low", ctypes.c_int), ("c_u_min", ctypes.c_int),
+                ("c_f_min", ctypes.c_int), ("c_alpha_front", ctypes.c_float)]
 
 
 class Stats(ctypes.Structure):

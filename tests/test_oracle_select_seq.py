@@ -53,20 +53,13 @@ BASE = dict(cent_mode=1, s_max=1.0, n_bins=2, b_batch=2, b_min=2, c_t_low=1, c_u
     (dict(b_min=3), 2, [9, 2], [0.0625, 9.0], 5),
     # C = 3: the heap is never full, no stop
     (dict(), 3, [9, 2], [0.0625, 9.0], 5),
-    # gate off: H keeps the C smallest of everything seen
-    (dict(gate_m0=float("inf"), c_t_low=0), 2, [5, 9, 2], [0.25, 0.0625, 9.0], 5),
+    # gate off: H keeps the C smallest of everything seen: (0.0625, 9), (0.25, 3)
+    (dict(gate_m0=float("inf"), c_t_low=0), 2, [9, 3, 2], [0.0625, 0.25, 9.0], 5),
 ])
 def test_hand_worked_sequence(tmp_path, kw, C, want_L, want_d, want_batches):
     ix = hand_index(tmp_path)
     logit, codes, scores = hand_probes()
     L, dL, ndir, nb = ix.cluster_list_seq(logit, codes, scores, C, oracle.params(**{**BASE, **kw}))
-    order = np.lexsort((L, dL))
-    assert list(L[order]) == list(L), "list ordered by (d, cluster)"
-    if kw.get("gate_m0") == float("inf"):
-        # gate off: the two smallest non-singleton keys over all batches, (0.0625, 9)
-        # and (0.25, 3), plus C^dir; re-derive the order
-        want = sorted([(0.0625, 9), (0.25, 3), (9.0, 2)])
-        want_L, want_d = [c for _, c in want], [d for d, _ in want]
     assert list(L) == want_L and list(dL) == want_d
     assert ndir == 1 and nb == want_batches
 
