@@ -578,42 +578,51 @@ def main():
                       "index": build_info, "n_clusters": ix.n_clusters}), file=sys.stderr, flush=True)
 
     if args.sweep or args.sweep_gate or args.grid:
+        import itertools
+
+        def num(v):
+            return None if v == "none" else (float(v) if ("." in v or "e" in v or v == "inf") else int(v))
+
         if args.grid:
-            g = dict(part.split("=") for part in args.grid.split(";"))
-            grid_p = [int(v) for v in g.get("P", "256").split(",")]
-            grid_c = [int(v) for v in g.get("C", "256").split(",")]
-            grid_t = [int(v) for v in g.get("t_low", "0").split(",")]
-            grid_m = [None if v == "none" else float(v) for v in g.get("m1", "none").split(",")]
+            # "P=..;C=..;t_low=..;m1=..;<any nr_params field>=.." (comma lists)
+            g = {k: [num(v) for v in vals.split(",")]
+                 for k, vals in (part.split("=") for part in args.grid.split(";"))}
         elif args.sweep_gate:
-            grid_p, grid_c, grid_t, grid_m = (128, 256, 512), (128, 256, 1024), (0, 32, 64), \
-                (None, 0.5, 1.0, 2.0, 4.0)
+            g = {"P": [128, 256, 512], "C": [128, 256, 1024], "t_low": [0, 32, 64],
+                 "m1": [None, 0.5, 1.0, 2.0, 4.0]}
         else:
-            grid_p = (64, 128, 256, 512, 1024) if w.bits <= 20 else (256, 512, 1024)
-            grid_c = (256, 512, 1024, 2048) if w.bits <= 20 else (256, 1024)
+            g = {"P": [64, 128, 256, 512, 1024] if w.bits <= 20 else [256, 512, 1024],
+                 "C": [256, 512, 1024, 2048] if w.bits <= 20 else [256, 1024],
+                 "t_low": [0, 8, 16, 32, 64], "m1": [None]}
             if w.k_max == 1:  # no bucket-local clustering: C never binds
-                grid_p, grid_c = (64, 128, 256, 512, 1024, 2048), (256,)
-            grid_t, grid_m = (0, 8, 16, 32, 64), (None,)
-        for Pp in grid_p:
-            for Cc in grid_c:
-                if Pp * ix.k_max > 16384:
-                    continue
-                for tl in grid_t:
-                    for m1 in grid_m:
-                        kw = {"t_low": tl}
-                        if m1 is not None:
-                            kw.update(gate_m0=0.0, gate_m1=m1)
-                        ix.set_params(**kw)
-                        ix.search(dq, k, Pp, Cc, out=(ids, dd))
-                        torch.cuda.synchronize()
-                        t = time.perf_counter()
-                        ix.search(dq, k, Pp, Cc, out=(ids, dd))
-                        torch.cuda.synchronize()
-                        el = time.perf_counter() - t
-                        st = ix.last_stats()
-                        print(json.dumps({"P": Pp, "C": Cc, "t_low": tl, "gate_m1": m1,
-                                          "recall": recall_at(ids.cpu().numpy(), truth, k),
-                                          "qps": nq / el, "cand_per_q": st.candidates / nq}),
-                              flush=True)
+                g["P"], g["C"] = [64, 128, 256, 512, 1024, 2048], [256]
+        g.setdefault("P", [P])
+        g.setdefault("C", [C])
+        g.setdefault("m1", [None])
+        names = list(g)
+        for combo in itertools.product(*(g[k] for k in names)):
+            cfg = dict(zip(names, combo))
+            Pp, Cc, m1 = cfg["P"], cfg["C"], cfg["m1"]
+            if Pp * ix.k_max > 16384:
+                continue
+            kw = {k: v for k, v in cfg.items() if k not in ("P", "C", "m1")}
+            if m1 is not None:
+                kw.update(gate_m0=0.0, gate_m1=m1)
+            try:
+                ix.set_params(**kw)
+                ix.search(dq, k, Pp, Cc, out=(ids, dd))
+            except nr.NRError as ex:
+                print(json.dumps({**cfg, "error": str(ex)}), flush=True)
+                continue
+            torch.cuda.synchronize()
+            t = time.perf_counter()
+            ix.search(dq, k, Pp, Cc, out=(ids, dd))
+            torch.cuda.synchronize()
+            el = time.perf_counter() - t
+            st = ix.last_stats()
+            print(json.dumps({**cfg, "recall": recall_at(ids.cpu().numpy(), truth, k), "qps": nq / el,
+                              "cand_per_q": st.candidates / nq, "clusters_per_q": st.clusters / nq}),
+                  flush=True)
         return 0
 
     kw = op_params(w)
