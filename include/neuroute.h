@@ -105,6 +105,14 @@ typedef struct {
   int c_t_low;          /* >= 0; default 0 */
   int c_u_min, c_f_min; /* >= 0; default 1, 1 */
   float c_alpha_front;  /* in [0, 1]; default 0.5 */
+  /* Calibrated gate (Sec. 3.4): when gate_n >= 2 (at most 16), M is the
+   * piecewise-linear curve through (gate_x[i], gate_y[i]), flat beyond its
+   * ends: on segment i (the last breakpoint with gate_x[i] <= x),
+   * M(x) = fmaf(x - x_i, (y_{i+1} - y_i) / (x_{i+1} - x_i), y_i) in fp32; the
+   * gate is then on and gate_m0 / gate_m1 are unused. gate_x strictly
+   * increasing, gate_y non-decreasing, all finite. gate_n = 0: M(x) = m0 + m1 x. */
+  int gate_n;           /* 0, or 2..16; default 0 */
+  float gate_x[16], gate_y[16];
 } nr_params;
 
 /* Per-search statistics (sums over the queries of the last search call). */

@@ -50,6 +50,25 @@ extern "C" void or_params_default(or_params *p) {
   p->c_u_min = 1;
   p->c_f_min = 1;
   p->c_alpha_front = 0.5f;
+  p->gate_n = 0;
+  for (int i = 0; i < 16; ++i) p->gate_x[i] = p->gate_y[i] = 0.0f;
+}
+
+// The gate margin M(x) (Sec. 3.4): m0 + m1 x, or the calibrated monotone
+// piecewise-linear curve: flat beyond its ends, on segment i (the last
+// breakpoint with x_i <= x) y_i + (x - x_i) (y_{i+1} - y_i) / (x_{i+1} - x_i)
+// in fp32, the last step fused.
+static float gate_margin(const or_params *p, float x) {
+  if (p->gate_n < 2) return std::fmaf(p->gate_m1, x, p->gate_m0);
+  int i = 0;
+  while (i + 1 < p->gate_n && p->gate_x[i + 1] <= x) ++i;
+  if (x <= p->gate_x[0]) return p->gate_y[0];
+  if (i == p->gate_n - 1) return p->gate_y[i];
+  const float s = (p->gate_y[i + 1] - p->gate_y[i]) / (p->gate_x[i + 1] - p->gate_x[i]);
+  return std::fmaf(x - p->gate_x[i], s, p->gate_y[i]);
+}
+static bool gate_is_off(const or_params *p) {
+  return p->gate_n < 2 && std::isinf(p->gate_m0) && p->gate_m0 > 0.0f;
 }
 
 // ---------------------------------------------------------------- index file
@@ -354,9 +373,9 @@ extern "C" int or_cluster_list(const or_index *ix, const float *logit, const uin
   }
   float dmin = kInf;
   for (auto &e : cand) dmin = std::min(dmin, e.first);
-  const bool gate_off = std::isinf(p->gate_m0) && p->gate_m0 > 0.0f;
+  const bool gate_off = gate_is_off(p);
   float theta = kInf;
-  if (!gate_off && !cand.empty()) theta = dmin + std::fmaf(p->gate_m1, dmin, p->gate_m0);
+  if (!gate_off && !cand.empty()) theta = dmin + gate_margin(p, dmin);
   std::vector<std::pair<float, int64_t>> surv;
   for (auto &e : cand)
     if (e.first <= theta) surv.push_back(e);
@@ -390,7 +409,7 @@ extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const
     const int zi = (int)z;
     return zi < nbins - 1 ? zi : nbins - 1;
   };
-  const bool gate_off = std::isinf(p->gate_m0) && p->gate_m0 > 0.0f;
+  const bool gate_off = gate_is_off(p);
   const int B = p->b_batch > 0 ? p->b_batch : 1;
   std::vector<std::pair<float, int64_t>> dir, H;
   float dmin = kInf;
@@ -422,7 +441,7 @@ extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const
       for (auto &e : batch) dmin = std::min(dmin, e.first);
       float theta = kInf, front_th = kInf;
       if (!gate_off) {
-        const float m = std::fmaf(p->gate_m1, dmin, p->gate_m0);  // M(d_min)
+        const float m = gate_margin(p, dmin);  // M(d_min)
         theta = dmin + m;
         front_th = dmin + p->c_alpha_front * m;
       }

@@ -67,6 +67,11 @@ typedef struct {
   int c_t_low;         /* stop after c_t_low consecutive low-quality batches; 0: never */
   int c_u_min, c_f_min; /* batch low quality iff updates < c_u_min and front < c_f_min */
   float c_alpha_front; /* front threshold d_min + c_alpha_front * M(d_min) */
+  /* calibrated gate (Sec. 3.4): when gate_n >= 2, M is the piecewise-linear
+   * curve through (gate_x[i], gate_y[i]) (x increasing, y non-decreasing),
+   * flat beyond its ends, instead of gate_m0 + gate_m1 x */
+  int gate_n;
+  float gate_x[16], gate_y[16];
 } or_params;
 
 void or_params_default(or_params *p);

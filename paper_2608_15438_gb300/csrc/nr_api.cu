@@ -111,6 +111,14 @@ nr_status check_params(const nr_params *p) {
       p->b_batch > 2048 || p->b_min < 0 || p->c_t_low < 0 || p->c_u_min < 0 || p->c_f_min < 0 ||
       !(p->c_alpha_front >= 0.0f && p->c_alpha_front <= 1.0f))
     return NR_ERR_INVALID_ARG;
+  if (p->gate_n != 0) {
+    if (p->gate_n < 2 || p->gate_n > 16) return NR_ERR_INVALID_ARG;
+    for (int i = 0; i < p->gate_n; ++i) {
+      if (!std::isfinite(p->gate_x[i]) || !std::isfinite(p->gate_y[i])) return NR_ERR_INVALID_ARG;
+      if (i > 0 && !(p->gate_x[i] > p->gate_x[i - 1] && p->gate_y[i] >= p->gate_y[i - 1]))
+        return NR_ERR_INVALID_ARG;
+    }
+  }
   return NR_OK;
 }
 
@@ -230,6 +238,8 @@ nr_status nr_params_default(nr_params *p) {
   p->c_u_min = 1;
   p->c_f_min = 1;
   p->c_alpha_front = 0.5f;
+  p->gate_n = 0;
+  for (int i = 0; i < 16; ++i) p->gate_x[i] = p->gate_y[i] = 0.0f;
   return NR_OK;
 }
 

@@ -82,7 +82,12 @@ nrq::SelectParams nr_select_params(nr_index *ix, int P, int C) {
   sp.cent = ix->cent;
   sp.single = nr_single_table(ix);
   const float m0 = ix->params.gate_m0;
-  sp.gate_off = std::isinf(m0) && m0 > 0.0f;
+  sp.gate_n = ix->params.gate_n;
+  for (int i = 0; i < 16; ++i) {
+    sp.gate_x[i] = ix->params.gate_x[i];
+    sp.gate_y[i] = ix->params.gate_y[i];
+  }
+  sp.gate_off = sp.gate_n < 2 && std::isinf(m0) && m0 > 0.0f;
   sp.m0 = m0;
   sp.m1 = ix->params.gate_m1;
   sp.err = ix->d_err;

@@ -174,7 +174,23 @@ struct SelectParams {
   int mode, n_bins, b_batch, b_min, c_t_low, c_u_min, c_f_min;
   float s_max, c_alpha_front;
   const float *tau;
+  // calibrated gate curve (gate_n >= 2), else M(x) = m0 + m1 x
+  int gate_n;
+  float gate_x[16], gate_y[16];
 };
+
+// The gate margin M(x): m0 + m1 x, or the calibrated monotone piecewise-linear
+// curve, flat beyond its ends (the definition of the oracle's gate_margin).
+__device__ __forceinline__ float gate_margin(const SelectParams &sp, float x) {
+  if (sp.gate_n < 2) return __fmaf_rn(sp.m1, x, sp.m0);
+  int i = 0;
+  while (i + 1 < sp.gate_n && sp.gate_x[i + 1] <= x) ++i;
+  if (x <= sp.gate_x[0]) return sp.gate_y[0];
+  if (i == sp.gate_n - 1) return sp.gate_y[i];
+  const float s = __fdiv_rn(__fsub_rn(sp.gate_y[i + 1], sp.gate_y[i]),
+                            __fsub_rn(sp.gate_x[i + 1], sp.gate_x[i]));
+  return __fmaf_rn(__fsub_rn(x, sp.gate_x[i]), s, sp.gate_y[i]);
+}
 
 // Sort capacity for probe budget P: all clusters of P buckets. Shared memory
 // holds at most kSelectSmemKeys keys; a query with more candidate clusters
@@ -388,7 +404,9 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   if (tid == 0) sred[2] = 0u;  // keys collected from the front
   __syncthreads();
   const float m0 = sp.m0, m1 = sp.m1;
-  const bool prefilter = !sp.gate_off && m1 >= 0.0f;
+  // (with a calibrated curve, fp32 rounding at its breakpoints could make the
+  // gate decrease by an ulp: no prefilter then)
+  const bool prefilter = !sp.gate_off && sp.gate_n < 2 && m1 >= 0.0f;
   for (int s = tid; s < M; s += nt) {
     const uint32_t c = slot_cluster(cnt, c0s, np, s);
     const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
@@ -415,7 +433,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   float theta = __int_as_float(0x7f800000);
   if (!sp.gate_off && dmin_bits != 0xffffffffu) {
     const float dmin = __uint_as_float(dmin_bits);
-    theta = __fadd_rn(dmin, __fmaf_rn(m1, dmin, m0));  // theta = d_min + M(d_min)
+    theta = __fadd_rn(dmin, gate_margin(sp, dmin));  // theta = d_min + M(d_min)
   }
   const int nA = (int)sred[1], nB = (int)sred[2];
   int Mk = nA + nB;
@@ -739,7 +757,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
       if (bmin < dmin) dmin = bmin;
       float theta = __int_as_float(0x7f800000), front_th = theta;
       if (!gate_off) {
-        const float m = __fmaf_rn(sp.m1, dmin, sp.m0);  // M(d_min)
+        const float m = gate_margin(sp, dmin);  // M(d_min)
         theta = __fadd_rn(dmin, m);
         front_th = __fadd_rn(dmin, __fmul_rn(sp.c_alpha_front, m));
       }

@@ -40,7 +40,9 @@ class Params(ctypes.Structure):
                 ("f_min", ctypes.c_int), ("r_min", ctypes.c_int), ("alpha_front", ctypes.c_float),
                 ("cent_mode", ctypes.c_int), ("n_bins", ctypes.c_int), ("b_batch", ctypes.c_int),
                 ("b_min", ctypes.c_int), ("c_t_low", ctypes.c_int), ("c_u_min", ctypes.c_int),
-                ("c_f_min", ctypes.c_int), ("c_alpha_front", ctypes.c_float)]
+                ("c_f_min", ctypes.c_int), ("c_alpha_front", ctypes.c_float),
+                ("gate_n", ctypes.c_int), ("gate_x", ctypes.c_float * 16),
+                ("gate_y", ctypes.c_float * 16)]
 
 
 class Stats(ctypes.Structure):
@@ -104,6 +106,15 @@ def params(**kw) -> Params:
     p = Params()
     lib().nr_params_default(ctypes.byref(p))
     for k, v in kw.items():
+        if k == "gate_curve":  # (xs, ys): the calibrated piecewise-linear M, or None
+            xs, ys = (v if v is not None else ((), ()))
+            if len(xs) != len(ys) or len(xs) > 16:
+                raise ValueError("gate_curve: up to 16 (x, y) points")
+            p.gate_n = len(xs)
+            for i in range(16):
+                p.gate_x[i] = float(xs[i]) if i < len(xs) else 0.0
+                p.gate_y[i] = float(ys[i]) if i < len(ys) else 0.0
+            continue
         if not hasattr(p, k):
             raise KeyError(k)
         setattr(p, k, v)

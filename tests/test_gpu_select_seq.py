@@ -167,3 +167,49 @@ def test_argument_checks(tiny, torch):
     with pytest.raises(nr.NRError):
         ix.search_logits(tiny["dq"], tiny["dl"], 10, 4096, 64)   # P > 2048 in mode 1
     ix.set_params()
+
+
+CURVES = [((0.0, 2.0, 6.0, 20.0), (0.5, 2.0, 3.0, 3.5)),
+          ((1.0, 3.0), (0.0, 4.0)),
+          ((0.5, 1.0, 1.5, 2.0, 2.5, 3.0, 3.5, 4.0, 5.0, 6.0, 7.0, 8.0, 9.0, 10.0, 12.0, 14.0),
+           (0.1, 0.2, 0.4, 0.8, 1.0, 1.2, 1.3, 1.4, 1.5, 1.6, 1.7, 1.8, 1.9, 2.0, 2.1, 2.2))]
+
+
+@pytest.mark.parametrize("curve", CURVES, ids=["4pt", "2pt", "16pt"])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_calibrated_gate_curve_matches_oracle(tiny, torch, curve, mode):
+    ix, orc = tiny["ix"], tiny["orc"]
+    kw = dict(gate_curve=curve, cent_mode=mode)
+    if mode == 1:
+        kw.update(n_bins=8, s_max=0.6, b_batch=16, c_t_low=2)
+    ix.set_params(**kw)
+    try:
+        cl, ncl = ix.debug_clusters(tiny["dl"], 256, 128)
+        ids, d = ix.search_logits(tiny["dq"], tiny["dl"], 10, 256, 128)
+        torch.cuda.synchronize()
+    finally:
+        ix.set_params()
+    cl, ncl = cl.cpu().numpy(), ncl.cpu().numpy()
+    p = oracle.params(**kw)
+    tau = orc.tau()
+    for i in range(len(tiny["q"])):
+        codes, keys, _ = oracle.probe_list(tiny["lg"][i], tau, 256, p)
+        if mode == 1:
+            scores = (keys >> np.uint64(32)).astype(np.uint32).view(np.float32)
+            L = orc.cluster_list_seq(tiny["lg"][i], codes, scores, 128, p)[0]
+        else:
+            L = orc.cluster_list(tiny["lg"][i], codes, 128, p)[0]
+        assert ncl[i] == len(L) and np.array_equal(cl[i, : len(L)], L), i
+    ids_o, d_o, _ = orc.search(tiny["q"], 10, 256, 128, p, logits=tiny["lg"])
+    assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
+
+
+def test_gate_curve_argument_checks(tiny, torch):
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    ix = tiny["ix"]
+    for bad in (((1.0,), (1.0,)), ((1.0, 1.0), (0.0, 1.0)), ((1.0, 2.0), (1.0, 0.5)),
+                ((0.0, float("inf")), (0.0, 1.0)), ((0.0, 1.0), (float("nan"), 1.0))):
+        with pytest.raises(nr.NRError):
+            ix.set_params(gate_curve=bad)
+    ix.set_params()

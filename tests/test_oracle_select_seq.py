@@ -122,3 +122,28 @@ def test_search_uses_the_sequential_stage(tmp_path):
         scores = (keys >> np.uint64(32)).astype(np.uint32).view(np.float32)
         L, _, _, _ = ix.cluster_list_seq(lg[i], codes, scores, 4, p)
         assert st[i, 2] == len(L)
+
+
+@pytest.mark.parametrize("curve,want", [
+    # inside the curve: M(0.0625) = 0.5 + 0.0625 * 1 = 0.5625, theta 0.625: 9, 3, 5 pass
+    (((0.0, 1.0), (0.5, 1.5)), [9, 3, 5, 2]),
+    # d_min below the first point: M = y_0 = 0.25, theta 0.3125: 9, 3, 5 pass
+    (((0.5, 1.0), (0.25, 2.0)), [9, 3, 5, 2]),
+    # d_min past the last point: M = y_last = 1, theta 1.0625: 0 (d 1) and 7 (d 1) join
+    (((0.01, 0.05), (1.0, 1.0)), [9, 3, 5, 0, 7, 2]),
+    # three points, d_min on the second: segment 1, M = 0 + (0.0625 - 0.0625) s = 0,
+    # theta 0.0625: only 9 passes
+    (((0.0, 0.0625, 4.0), (0.0, 0.0, 8.0)), [9, 2]),
+])
+def test_calibrated_gate_curve(tmp_path, curve, want):
+    """The piecewise-linear M of Sec. 3.4 on the hand-worked index (d_min over
+    the non-singleton clusters = 0.0625): flat beyond its ends, linear inside,
+    in both centroid stages."""
+    ix = hand_index(tmp_path)
+    logit, codes, scores = hand_probes()
+    p0 = oracle.params(gate_curve=curve)
+    L0, _, _ = ix.cluster_list(logit, codes, 8, p0)
+    assert list(L0) == want
+    p1 = oracle.params(gate_curve=curve, cent_mode=1, b_batch=1 << 20, c_t_low=0)
+    L1, _, _, _ = ix.cluster_list_seq(logit, codes, scores, 8, p1)
+    assert list(L1) == want
