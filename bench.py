@@ -77,6 +77,16 @@ def parse():
     ap.add_argument("--encode", type=int, default=0,
                     help="time only the tensor-core encoder over this many base vectors")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--calibrate", type=int, default=0,
+                    help="calibrate M(x) and S_max on this many held-out queries (Sec. 3.4); "
+                         "grid keys cq=<quantile> and cov=<coverage> then select the fitted "
+                         "curve and cutoff")
+    ap.add_argument("--calib-budget", default=None, help="'P,C' of the high-recall target run")
+    ap.add_argument("--calib-bins", type=int, default=16)
+    ap.add_argument("--cq", type=float, default=None,
+                    help="timed run: calibrated gate at this quantile (needs --calibrate)")
+    ap.add_argument("--cov", type=float, default=None,
+                    help="timed run: calibrated S_max at this coverage (needs --calibrate)")
     return ap.parse_args()
 
 
@@ -313,12 +323,11 @@ def traffic_from_profile(workload, P, C):
         return None
 
 
-def cpu_baseline(w, path, queries, k, P, C, t_low, seconds, truth=None):
+def cpu_baseline(w, path, queries, k, P, C, kw, seconds, truth=None):
     import oracle
 
     orc = oracle.Index(path)
-    kw = op_params(w)
-    kw["t_low"] = t_low
+    t_low = kw.get("t_low")
     p = oracle.params(**kw)
     cores = os.cpu_count() or 1
     n = 16
@@ -353,14 +362,13 @@ def calibrate_subindex(w, ix, queries, k, P, C, kw, seconds, path, row_budget):
     return int(min(len(queries), max(n, row_budget / per_q), max(n, n * seconds / dt)))
 
 
-def cpu_baseline_subindex(w, ix, queries, k, P, C, t_low, seconds, row_budget=100_000_000):
+def cpu_baseline_subindex(w, ix, queries, k, P, C, kw, seconds, row_budget=100_000_000):
     """The oracle timed on the host cores for a bounded query sample, on the
     sub-index of the buckets those queries probe (the index may be too large
-    for host memory)."""
+    for host memory), with the timed run's parameters kw."""
     import oracle
 
-    kw = op_params(w)
-    kw["t_low"] = t_low
+    t_low = kw.get("t_low")
     p = oracle.params(**kw)
     cores = os.cpu_count() or 1
     with tempfile.TemporaryDirectory() as td:
@@ -505,6 +513,52 @@ def encode_bench(args, w, torch, nr, dev):
     return 0
 
 
+def run_calibration(args, w, torch, ix, dev, P, C, k):
+    """Observations for the calibrated gate and cutoff (Sec. 3.4) from held-out
+    calibration queries: targets from a high-recall run of the search."""
+    import synth
+    from paper_2608_15438_gb300 import calibrate as cal
+
+    t0 = time.time()
+    cq = torch.from_numpy(synth.calib_queries(w, args.calibrate)).to(dev)
+    if args.calib_budget:
+        cP, cC = (int(v) for v in args.calib_budget.split(","))
+    else:
+        cP, cC = min(4096, 2 * P, 16384 // ix.k_max), min(4096, 4 * C)
+    lg = ix.encode(cq)
+    targets = cal.targets_high_recall(ix, cq, lg, k, cP, cC)
+    scores, x, y = cal.observations(ix, lg, targets)
+    torch.cuda.synchronize()
+    res = {"scores": scores, "x": x, "y": y}
+    summary = {"nq": args.calibrate, "budget": [cP, cC], "seconds": round(time.time() - t0, 2),
+               "n_gated": int((~np.isnan(x)).sum()),
+               "curves": {q: cal.fit_gate(x, y, args.calib_bins, q) for q in (0.9, 0.95, 0.99)},
+               "s_max": {c: [float(v) for v in cal.fit_s_max(scores, c)] for c in (0.95, 0.99, 0.999)}}
+    print(json.dumps({"calibration": summary}), file=sys.stderr, flush=True)
+    return res
+
+
+def calibrated_params(args, calib, cq, cov):
+    """nr_params keywords of the calibrated gate (quantile cq) and cutoff
+    (coverage cov); either may be None."""
+    from paper_2608_15438_gb300 import calibrate as cal
+
+    kw = {}
+    if cq is None and cov is None:
+        return kw
+    if calib is None:
+        raise SystemExit("cq/cov need --calibrate")
+    if cq is not None:
+        curve = cal.fit_gate(calib["x"], calib["y"], args.calib_bins, cq)
+        if curve is not None:
+            kw["gate_curve"] = curve
+    if cov is not None:
+        s_max = cal.fit_s_max(calib["scores"], cov)[0]
+        if s_max is not None:
+            kw["s_max"] = float(s_max)
+    return kw
+
+
 def op_point(args, w):
     P, C, t_low, _ = OPERATING_POINTS.get(w.name, (64, 128, 4, None))
     return (args.P or P, args.C or C, t_low if args.t_low is None else args.t_low)
@@ -577,6 +631,10 @@ def main():
     print(json.dumps({"setup_s": {"index_build": round(t_build, 2), "ground_truth": round(t_gt, 2)},
                       "index": build_info, "n_clusters": ix.n_clusters}), file=sys.stderr, flush=True)
 
+    calib = None
+    if args.calibrate:
+        calib = run_calibration(args, w, torch, ix, dev, P, C, k)
+
     if args.sweep or args.sweep_gate or args.grid:
         import itertools
 
@@ -605,9 +663,10 @@ def main():
             Pp, Cc, m1 = cfg["P"], cfg["C"], cfg["m1"]
             if Pp * ix.k_max > 16384:
                 continue
-            kw = {k: v for k, v in cfg.items() if k not in ("P", "C", "m1")}
+            kw = {k: v for k, v in cfg.items() if k not in ("P", "C", "m1", "cq", "cov")}
             if m1 is not None:
                 kw.update(gate_m0=0.0, gate_m1=m1)
+            kw.update(calibrated_params(args, calib, cfg.get("cq"), cfg.get("cov")))
             try:
                 ix.set_params(**kw)
                 ix.search(dq, k, Pp, Cc, out=(ids, dd))
@@ -627,6 +686,12 @@ def main():
 
     kw = op_params(w)
     kw["t_low"] = t_low
+    if args.cq is not None or args.cov is not None:
+        if calib is None:
+            raise SystemExit("--cq/--cov need --calibrate")
+        kw.update(calibrated_params(args, calib, args.cq, args.cov))
+        kw.pop("gate_m0", None)
+        kw.pop("gate_m1", None)
     ix.set_params(**kw)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     for _ in range(max(3, args.warmup)):
@@ -696,7 +761,11 @@ def main():
         "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
         "config": {"workload": w.name, "N": w.n, "D": w.dim, "nq": nq, "k": k, "bits": w.bits,
                    "hidden": w.hidden, "K_max": w.k_max, "P": P, "C": C, "t_low": t_low,
-                   "gate_m1": kw.get("gate_m1"),
+                   "gate_m1": kw.get("gate_m1"), "gate_curve": kw.get("gate_curve"),
+                   "s_max": kw.get("s_max"),
+                   "calibration": (None if args.cq is None and args.cov is None else
+                                   {"queries": args.calibrate, "quantile": args.cq,
+                                    "coverage": args.cov, "bins": args.calib_bins}),
                    "round": 256, "recall_at_10": rec, "cand_per_query": cand / nq,
                    "l2": "flushed between timed steps (256 MB write)",
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},
@@ -717,9 +786,9 @@ def main():
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         if gpu_built:
-            out["cpu_baseline"] = cpu_baseline_subindex(w, ix, qs, k, P, C, t_low, args.cpu_seconds)
+            out["cpu_baseline"] = cpu_baseline_subindex(w, ix, qs, k, P, C, kw, args.cpu_seconds)
         else:
-            cb, _ = cpu_baseline(w, path, qs, k, P, C, t_low, args.cpu_seconds)
+            cb, _ = cpu_baseline(w, path, qs, k, P, C, kw, args.cpu_seconds)
             out["cpu_baseline"] = cb
     if rank == 0:
         print(json.dumps(out), flush=True)

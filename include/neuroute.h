@@ -166,6 +166,25 @@ nr_status nr_index_save(nr_index *ix, const char *path);
 nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, const char *path,
                            int64_t *info);
 
+/* Where rows are stored, for calibrating the gate M and the score cutoff
+ * S_max (Sec. 3.4: both are fitted on where a query's true neighbours lie).
+ * d_ids: n device int64 row ids (any order, repeats allowed). d_out: n x 4
+ * device int32, per id (cluster, bucket code, first cluster of that bucket,
+ * clusters in that bucket), or (-1, -1, -1, 0) for an id not in the index.
+ * Allocates O(n) device scratch; synchronous on `stream`. 0 <= n < 2^31.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_OOM, NR_ERR_CUDA. */
+nr_status nr_index_locate(nr_index *ix, const int64_t *d_ids, int64_t n, int32_t *d_out,
+                          void *stream);
+
+/* Centroid distances (Eq. 12): d_out[q * m + j] = sum_i (l_qi - mu_ci)^2 with
+ * c = d_clusters[q * m + j], evaluated as the query path evaluates it (fp32,
+ * one fused multiply-add per coordinate in coordinate order), +inf where c is
+ * out of range (-1 pads). d_logits [nq x b] fp32, d_clusters [nq x m] int32,
+ * d_out [nq x m] fp32, all device. Asynchronous on `stream`.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_CUDA. */
+nr_status nr_centroid_dists(nr_index *ix, const float *d_logits, int64_t nq,
+                            const int32_t *d_clusters, int m, float *d_out, void *stream);
+
 /* Validate and set the query-time knobs (p = NULL restores the defaults).
  * NR_ERR_INVALID_ARG if a field is out of range. */
 nr_status nr_set_params(nr_index *ix, const nr_params *p);

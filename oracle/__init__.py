@@ -66,6 +66,8 @@ def lib():
                                 vp, i32]
         L.or_search.restype = i32
         L.or_bruteforce.argtypes = [i32, i32, vp, i64, vp, i64, i32, vp, vp, i32]
+        L.or_centroid_dist.argtypes = [vp, vp, i64]
+        L.or_centroid_dist.restype = ctypes.c_float
         _LIB = L
     return _LIB
 
@@ -178,6 +180,12 @@ class Index:
         if n < 0:
             raise RuntimeError("oracle: out-of-range index in file")
         return L[:n].copy(), dL[:n].copy(), int(ndir[0]), int(nbat[0])
+
+    def centroid_dist(self, logit, c: int) -> np.float32:
+        """Distance of cluster c's centroid from the logits (the centroid
+        stage's fmaf chain); +inf for c out of range."""
+        logit = np.ascontiguousarray(logit, np.float32)
+        return np.float32(lib().or_centroid_dist(self.h, logit.ctypes.data, int(c)))
 
     def search(self, queries, k, P, C, p: Params, logits=None, nthreads=None):
         queries = np.ascontiguousarray(queries)

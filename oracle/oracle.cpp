@@ -349,6 +349,11 @@ static float centroid_distance(const float *logit, const float *mu, int b) {
   return acc;
 }
 
+extern "C" float or_centroid_dist(const or_index *ix, const float *logit, int64_t c) {
+  if (c < 0 || c >= ix->n_cl) return kInf;
+  return centroid_distance(logit, &ix->cent[(size_t)c * ix->b], ix->b);
+}
+
 static bool dc_less(const std::pair<float, int64_t> &a, const std::pair<float, int64_t> &c) {
   return a.first < c.first || (a.first == c.first && a.second < c.second);
 }

@@ -131,6 +131,10 @@ int or_cluster_list_seq(const or_index *ix, const float *logit, const uint32_t *
                         const float *score, int nprobe, int C, const or_params *p, int32_t *L,
                         float *dL, int32_t *n_dir, int32_t *n_batches);
 
+/* Centroid distance (Eq. 12) of cluster c from one query's logits, the fmaf
+ * chain of the centroid stage; +inf when c is out of range. */
+float or_centroid_dist(const or_index *ix, const float *logit, int64_t c);
+
 /* Refinement over an explicit candidate stream: rows [n x D] (u8 or f32 by
  * dtype), ids [n]. out_ids/out_d [k] sorted by (dist, id), padded (-1, +inf).
  * stats[0..1] = candidates scored, rounds. */

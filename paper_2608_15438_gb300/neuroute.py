@@ -23,7 +23,8 @@ EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_f
            "nr_index_info", "nr_set_params", "nr_encode", "nr_route", "nr_debug_clusters",
            "nr_search", "nr_search_logits", "nr_search_host", "nr_query_stats", "nr_last_stats",
            "nr_enable_timing", "nr_last_timing", "nr_kernel_launches", "nr_search_static",
-           "nr_index_save", "nr_index_extract", "nr_index_thresholds", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
+           "nr_index_save", "nr_index_extract", "nr_index_thresholds", "nr_index_locate",
+           "nr_centroid_dists", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
            "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free"]
 
 
@@ -81,6 +82,8 @@ def lib():
         L.nr_index_save.argtypes = [vp, ctypes.c_char_p]
         L.nr_index_thresholds.argtypes = [vp, vp]
         L.nr_index_extract.argtypes = [vp, vp, i64, ctypes.c_char_p, vp]
+        L.nr_index_locate.argtypes = [vp, vp, i64, vp, vp]
+        L.nr_centroid_dists.argtypes = [vp, vp, i64, vp, i32, vp, vp]
         L.nr_build_begin.argtypes = [vp, i64, vp, vp, vp, vp, i32, ctypes.POINTER(vp)]
         L.nr_build_encode.argtypes = [vp, vp, i64, i64, vp]
         L.nr_build_set_logits.argtypes = [vp, vp, i64, i64, vp]
@@ -181,6 +184,30 @@ class Index:
         _check("nr_index_extract", lib().nr_index_extract(self.h, c.ctypes.data, c.size,
                                                           path.encode(), info.ctypes.data))
         return int(info[0]), int(info[1])
+
+    def locate(self, ids, stream=None):
+        """Where the rows `ids` (device int64) are stored (nr_index_locate):
+        int32 [n x 4] = (cluster, bucket code, first cluster of the bucket,
+        clusters in the bucket), (-1, -1, -1, 0) for an unknown id."""
+        import torch
+
+        ids = ids.reshape(-1).to(torch.int64).contiguous()
+        out = torch.empty((ids.numel(), 4), dtype=torch.int32, device=self._dev())
+        _check("nr_index_locate", lib().nr_index_locate(self.h, _ptr(ids), ids.numel(), _ptr(out),
+                                                        _stream(stream)))
+        return out
+
+    def centroid_dists(self, logits, clusters, stream=None):
+        """Distances of each query's logits to its listed clusters
+        (nr_centroid_dists): fp32 [nq x m], +inf for -1 pads."""
+        import torch
+
+        clusters = clusters.to(torch.int32).contiguous()
+        nq, m = clusters.shape
+        out = torch.empty((nq, m), dtype=torch.float32, device=self._dev())
+        _check("nr_centroid_dists", lib().nr_centroid_dists(self.h, _ptr(logits), nq, _ptr(clusters), m,
+                                                            _ptr(out), _stream(stream)))
+        return out
 
     def set_params(self, p: Params | None = None, **kw):
         if p is None:

@@ -25,6 +25,7 @@ SEED_DATA = 1
 SEED_QUERIES = 2
 SEED_ENCODER = 3
 SEED_KMEANS = 4
+SEED_CALIB = 5    # held-out calibration queries
 STREAM_W1 = 1
 STREAM_W2 = 2
 
@@ -149,6 +150,11 @@ def base(w: Workload, n: int | None = None, nthreads: int | None = None) -> np.n
 
 def queries(w: Workload, nq: int | None = None, nthreads: int | None = None) -> np.ndarray:
     return mixture(w, SEED_QUERIES, 0, w.nq if nq is None else nq, nthreads)
+
+
+def calib_queries(w: Workload, nq: int, nthreads: int | None = None) -> np.ndarray:
+    """Held-out calibration queries: the query distribution on its own stream."""
+    return mixture(w, SEED_CALIB, 0, nq, nthreads)
 
 
 def components(w: Workload, seed_rows: int, row0: int, n: int) -> np.ndarray:
