@@ -31,24 +31,38 @@ sys.path.insert(0, ROOT)
 
 METRIC = "QPS at Recall@10~0.90 (batched query path); refine-scan HBM GB/s"
 
-# operating points (P, C, t_low, gate m1) with Recall@10 in [0.88, 0.92], from
-# `--sweep` / `--sweep-gate`; gate m1 = None: gate off, else M(x) = m1 x
+# operating points with Recall@10 in [0.88, 0.92], from `--sweep`, `--grid`
+# and `--calibrate`: budgets P and C, early-stop t_low, and the centroid gate:
+# m1 gives M(x) = m1 x; cq the calibrated curve at that quantile and cov the
+# calibrated S_max at that coverage (Sec. 3.4), both fitted on CALIB_QUERIES
+# held-out queries; neither: gate off
 OPERATING_POINTS = {
-    "tiny": (128, 256, 4, None),
-    "u8-10m": (256, 256, 0, 4.0),
-    "f32-10m": (512, 256, 16, None),
-    "u8-100m": (1024, 256, 32, None),
-    "u8-1b": (1024, 1024, 64, 4.0),
-    "u8-30m": (1024, 1024, 64, 4.0),  # profiling proxy of u8-1b: its operating point
+    "tiny": dict(P=128, C=256, t_low=4),
+    "u8-10m": dict(P=256, C=256, t_low=0, m1=4.0),
+    "f32-10m": dict(P=512, C=256, t_low=16),
+    "u8-100m": dict(P=1024, C=256, t_low=32),
+    "u8-1b": dict(P=1024, C=1024, t_low=80, cq=0.9, cov=0.99),
+    "u8-30m": dict(P=1024, C=1024, t_low=80, cq=0.9, cov=0.99),  # profiling proxy of u8-1b
 }
+DEFAULT_POINT = dict(P=64, C=128, t_low=4)
+CALIB_QUERIES = 10000
+CALIB_BINS = 16
 
 
-def op_params(w):
-    """nr_params keyword arguments of the workload's operating point."""
-    _, _, t_low, m1 = OPERATING_POINTS.get(w.name, (64, 128, 4, None))
-    kw = {"t_low": t_low}
-    if m1 is not None:
-        kw.update(gate_m0=0.0, gate_m1=m1)
+def op_params(w, ix=None, t_low=None, calib=None, k=10):
+    """nr_params keyword arguments of the workload's operating point. A
+    calibrated point fits its curve and cutoff on the GPU index ix (or on
+    given observations), outside any timed region."""
+    op = OPERATING_POINTS.get(w.name, DEFAULT_POINT)
+    kw = {"t_low": op["t_low"] if t_low is None else t_low}
+    if op.get("m1") is not None:
+        kw.update(gate_m0=0.0, gate_m1=op["m1"])
+    if op.get("cq") is not None or op.get("cov") is not None:
+        if calib is None:
+            if ix is None:
+                raise SystemExit(f"{w.name}: the calibrated operating point needs the GPU index")
+            calib = calibration_observations(w, ix, op["P"], op["C"], k)
+        kw.update(calibrated_params(calib, op.get("cq"), op.get("cov"), CALIB_BINS))
     return kw
 
 
@@ -78,11 +92,11 @@ def parse():
                     help="time only the tensor-core encoder over this many base vectors")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--calibrate", type=int, default=0,
-                    help="calibrate M(x) and S_max on this many held-out queries (Sec. 3.4); "
-                         "grid keys cq=<quantile> and cov=<coverage> then select the fitted "
-                         "curve and cutoff")
+                    help="calibrate M(x) and S_max on this many held-out queries (Sec. 3.4; "
+                         "default 10,000 when the operating point is calibrated); grid keys "
+                         "cq=<quantile> and cov=<coverage> select the fitted curve and cutoff")
     ap.add_argument("--calib-budget", default=None, help="'P,C' of the high-recall target run")
-    ap.add_argument("--calib-bins", type=int, default=16)
+    ap.add_argument("--calib-bins", type=int, default=CALIB_BINS)
     ap.add_argument("--cq", type=float, default=None,
                     help="timed run: calibrated gate at this quantile (needs --calibrate)")
     ap.add_argument("--cov", type=float, default=None,
@@ -309,16 +323,20 @@ def refine_sources_digest():
     return h.hexdigest()
 
 
-def traffic_from_profile(workload, P, C):
+def traffic_from_profile(workload, P, C, algorithmic_bytes):
     """Per-launch DRAM bytes of the refine kernel from a committed ncu summary,
-    valid only while the kernel source is unchanged since the capture."""
+    valid only while the kernel source is unchanged since the capture and the
+    capture scanned the same candidates (its algorithmic bytes per launch equal
+    this run's: same operating point)."""
     path = os.path.join(ROOT, "profiles", "refine_traffic.json")
     try:
         rec = json.load(open(path))
         if rec.get("sources_sha256") != refine_sources_digest():
             return None
         e = rec.get("captures", {}).get(f"{workload}/P{P}/C{C}")
-        return None if e is None else e.get("bytes_per_launch")
+        if e is None or e.get("algorithmic_bytes_per_launch") != algorithmic_bytes:
+            return None
+        return e.get("bytes_per_launch")
     except Exception:
         return None
 
@@ -417,8 +435,7 @@ def run_reference(args, w, rank, world):
 
         dev = torch.device("cuda", 0)
         gix, _ = gpu_index(w, torch, nr, dev)
-        kw0 = op_params(w)
-        kw0["t_low"] = t_low
+        kw0 = op_params(w, gix, t_low, k=args.k)
         tmpdir = tempfile.TemporaryDirectory()
         path = os.path.join(tmpdir.name, "sub.nrix")
         per_step = max(8.0, 120.0 / max(1, args.steps + args.warmup))
@@ -435,8 +452,7 @@ def run_reference(args, w, rank, world):
     orc = oracle.Index(path)
     note = ("; sub-index of the buckets these queries probe, index built on the GPU"
             if tmpdir is not None else "")
-    kw = op_params(w)
-    kw["t_low"] = t_low
+    kw = kw0 if tmpdir is not None else op_params(w, t_low=t_low)
     p = oracle.params(**kw)
     cores = os.cpu_count() or 1
     n = 16
@@ -513,32 +529,32 @@ def encode_bench(args, w, torch, nr, dev):
     return 0
 
 
-def run_calibration(args, w, torch, ix, dev, P, C, k):
-    """Observations for the calibrated gate and cutoff (Sec. 3.4) from held-out
-    calibration queries: targets from a high-recall run of the search."""
+def calibration_observations(w, ix, P, C, k, nq=CALIB_QUERIES, budget=None, bins=CALIB_BINS):
+    """Observations for the calibrated gate and cutoff (Sec. 3.4) from nq
+    held-out calibration queries, targets from a high-recall run of the search
+    (budgets 2P and 4C by default, gate and early stop off)."""
+    import torch
+
     import synth
     from paper_2608_15438_gb300 import calibrate as cal
 
     t0 = time.time()
-    cq = torch.from_numpy(synth.calib_queries(w, args.calibrate)).to(dev)
-    if args.calib_budget:
-        cP, cC = (int(v) for v in args.calib_budget.split(","))
-    else:
-        cP, cC = min(4096, 2 * P, 16384 // ix.k_max), min(4096, 4 * C)
+    dev = torch.device("cuda", ix.device)
+    cq = torch.from_numpy(synth.calib_queries(w, nq)).to(dev)
+    cP, cC = budget or (min(4096, 2 * P, 16384 // ix.k_max), min(4096, 4 * C))
     lg = ix.encode(cq)
     targets = cal.targets_high_recall(ix, cq, lg, k, cP, cC)
     scores, x, y = cal.observations(ix, lg, targets)
     torch.cuda.synchronize()
-    res = {"scores": scores, "x": x, "y": y}
-    summary = {"nq": args.calibrate, "budget": [cP, cC], "seconds": round(time.time() - t0, 2),
+    summary = {"nq": nq, "budget": [cP, cC], "seconds": round(time.time() - t0, 2),
                "n_gated": int((~np.isnan(x)).sum()),
-               "curves": {q: cal.fit_gate(x, y, args.calib_bins, q) for q in (0.9, 0.95, 0.99)},
+               "curves": {q: cal.fit_gate(x, y, bins, q) for q in (0.9, 0.95, 0.99)},
                "s_max": {c: [float(v) for v in cal.fit_s_max(scores, c)] for c in (0.95, 0.99, 0.999)}}
     print(json.dumps({"calibration": summary}), file=sys.stderr, flush=True)
-    return res
+    return {"scores": scores, "x": x, "y": y, "nq": nq, "budget": [cP, cC]}
 
 
-def calibrated_params(args, calib, cq, cov):
+def calibrated_params(calib, cq, cov, bins=CALIB_BINS):
     """nr_params keywords of the calibrated gate (quantile cq) and cutoff
     (coverage cov); either may be None."""
     from paper_2608_15438_gb300 import calibrate as cal
@@ -547,9 +563,9 @@ def calibrated_params(args, calib, cq, cov):
     if cq is None and cov is None:
         return kw
     if calib is None:
-        raise SystemExit("cq/cov need --calibrate")
+        raise SystemExit("cq/cov need calibration observations (--calibrate)")
     if cq is not None:
-        curve = cal.fit_gate(calib["x"], calib["y"], args.calib_bins, cq)
+        curve = cal.fit_gate(calib["x"], calib["y"], bins, cq)
         if curve is not None:
             kw["gate_curve"] = curve
     if cov is not None:
@@ -560,8 +576,8 @@ def calibrated_params(args, calib, cq, cov):
 
 
 def op_point(args, w):
-    P, C, t_low, _ = OPERATING_POINTS.get(w.name, (64, 128, 4, None))
-    return (args.P or P, args.C or C, t_low if args.t_low is None else args.t_low)
+    op = OPERATING_POINTS.get(w.name, DEFAULT_POINT)
+    return (args.P or op["P"], args.C or op["C"], op["t_low"] if args.t_low is None else args.t_low)
 
 
 def main():
@@ -631,9 +647,13 @@ def main():
     print(json.dumps({"setup_s": {"index_build": round(t_build, 2), "ground_truth": round(t_gt, 2)},
                       "index": build_info, "n_clusters": ix.n_clusters}), file=sys.stderr, flush=True)
 
+    op = OPERATING_POINTS.get(w.name, DEFAULT_POINT)
+    calibrated_op = op.get("cq") is not None or op.get("cov") is not None
     calib = None
-    if args.calibrate:
-        calib = run_calibration(args, w, torch, ix, dev, P, C, k)
+    if args.calibrate or calibrated_op or args.cq is not None or args.cov is not None:
+        budget = tuple(int(v) for v in args.calib_budget.split(",")) if args.calib_budget else None
+        calib = calibration_observations(w, ix, P, C, k, nq=args.calibrate or CALIB_QUERIES,
+                                         budget=budget, bins=args.calib_bins)
 
     if args.sweep or args.sweep_gate or args.grid:
         import itertools
@@ -666,7 +686,7 @@ def main():
             kw = {k: v for k, v in cfg.items() if k not in ("P", "C", "m1", "cq", "cov")}
             if m1 is not None:
                 kw.update(gate_m0=0.0, gate_m1=m1)
-            kw.update(calibrated_params(args, calib, cfg.get("cq"), cfg.get("cov")))
+            kw.update(calibrated_params(calib, cfg.get("cq"), cfg.get("cov"), args.calib_bins))
             try:
                 ix.set_params(**kw)
                 ix.search(dq, k, Pp, Cc, out=(ids, dd))
@@ -684,14 +704,12 @@ def main():
                   flush=True)
         return 0
 
-    kw = op_params(w)
-    kw["t_low"] = t_low
     if args.cq is not None or args.cov is not None:
-        if calib is None:
-            raise SystemExit("--cq/--cov need --calibrate")
-        kw.update(calibrated_params(args, calib, args.cq, args.cov))
-        kw.pop("gate_m0", None)
-        kw.pop("gate_m1", None)
+        cq, cov, bins = args.cq, args.cov, args.calib_bins
+        kw = {"t_low": t_low, **calibrated_params(calib, cq, cov, bins)}
+    else:
+        cq, cov, bins = op.get("cq"), op.get("cov"), CALIB_BINS
+        kw = op_params(w, ix, t_low, calib=calib, k=k)
     ix.set_params(**kw)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     for _ in range(max(3, args.warmup)):
@@ -752,7 +770,7 @@ def main():
     refine_avg_ms = sum(refine_ms) / len(refine_ms)
     achieved = cand * row_bytes / (refine_avg_ms / 1e3) / 1e9
     peaks, peak_src = measured_peaks()
-    traffic = traffic_from_profile(w.name, P, C)
+    traffic = traffic_from_profile(w.name, P, C, cand * row_bytes)
     out = {
         "metric": METRIC,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
@@ -763,9 +781,10 @@ def main():
                    "hidden": w.hidden, "K_max": w.k_max, "P": P, "C": C, "t_low": t_low,
                    "gate_m1": kw.get("gate_m1"), "gate_curve": kw.get("gate_curve"),
                    "s_max": kw.get("s_max"),
-                   "calibration": (None if args.cq is None and args.cov is None else
-                                   {"queries": args.calibrate, "quantile": args.cq,
-                                    "coverage": args.cov, "bins": args.calib_bins}),
+                   "calibration": (None if cq is None and cov is None else
+                                   {"queries": calib["nq"], "target_budget": calib["budget"],
+                                    "quantile": cq, "coverage": cov, "bins": bins,
+                                    "held_out": "synthetic query stream of its own seed"}),
                    "round": 256, "recall_at_10": rec, "cand_per_query": cand / nq,
                    "l2": "flushed between timed steps (256 MB write)",
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},

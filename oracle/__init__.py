@@ -68,6 +68,8 @@ def lib():
         L.or_bruteforce.argtypes = [i32, i32, vp, i64, vp, i64, i32, vp, vp, i32]
         L.or_centroid_dist.argtypes = [vp, vp, i64]
         L.or_centroid_dist.restype = ctypes.c_float
+        L.or_gate_margin.argtypes = [ctypes.POINTER(Params), ctypes.c_float]
+        L.or_gate_margin.restype = ctypes.c_float
         _LIB = L
     return _LIB
 
@@ -213,6 +215,11 @@ def encode_weights(weights, in_scale: float, x: np.ndarray, nthreads=None) -> np
                             b1.ctypes.data, W2.ctypes.data, b2.ctypes.data, x.ctypes.data,
                             x.shape[0], out.ctypes.data, nthreads or nthreads_default())
     return out
+
+
+def gate_margin(p: Params, x) -> np.float32:
+    """M(x) under the parameters p."""
+    return np.float32(lib().or_gate_margin(ctypes.byref(p), float(np.float32(x))))
 
 
 def probe_order(sd, P, p: Params):

@@ -57,7 +57,8 @@ extern "C" void or_params_default(or_params *p) {
 // The gate margin M(x) (Sec. 3.4): m0 + m1 x, or the calibrated monotone
 // piecewise-linear curve: flat beyond its ends, on segment i (the last
 // breakpoint with x_i <= x) y_i + (x - x_i) (y_{i+1} - y_i) / (x_{i+1} - x_i)
-// in fp32, the last step fused.
+// in fp32, the last step fused, then held within [y_i, y_{i+1}]: the paper
+// asks for a monotone curve, and this keeps it monotone after fp32 rounding.
 static float gate_margin(const or_params *p, float x) {
   if (p->gate_n < 2) return std::fmaf(p->gate_m1, x, p->gate_m0);
   int i = 0;
@@ -65,8 +66,10 @@ static float gate_margin(const or_params *p, float x) {
   if (x <= p->gate_x[0]) return p->gate_y[0];
   if (i == p->gate_n - 1) return p->gate_y[i];
   const float s = (p->gate_y[i + 1] - p->gate_y[i]) / (p->gate_x[i + 1] - p->gate_x[i]);
-  return std::fmaf(x - p->gate_x[i], s, p->gate_y[i]);
+  const float v = std::fmaf(x - p->gate_x[i], s, p->gate_y[i]);
+  return std::min(std::max(v, p->gate_y[i]), p->gate_y[i + 1]);
 }
+extern "C" float or_gate_margin(const or_params *p, float x) { return gate_margin(p, x); }
 static bool gate_is_off(const or_params *p) {
   return p->gate_n < 2 && std::isinf(p->gate_m0) && p->gate_m0 > 0.0f;
 }

@@ -131,6 +131,9 @@ int or_cluster_list_seq(const or_index *ix, const float *logit, const uint32_t *
                         const float *score, int nprobe, int C, const or_params *p, int32_t *L,
                         float *dL, int32_t *n_dir, int32_t *n_batches);
 
+/* The gate margin M(x) of the parameters p (linear, or the calibrated curve). */
+float or_gate_margin(const or_params *p, float x);
+
 /* Centroid distance (Eq. 12) of cluster c from one query's logits, the fmaf
  * chain of the centroid stage; +inf when c is out of range. */
 float or_centroid_dist(const or_index *ix, const float *logit, int64_t c);

@@ -180,7 +180,9 @@ struct SelectParams {
 };
 
 // The gate margin M(x): m0 + m1 x, or the calibrated monotone piecewise-linear
-// curve, flat beyond its ends (the definition of the oracle's gate_margin).
+// curve, flat beyond its ends, each segment's value held within its end values
+// so that M never decreases in fp32 (the definition of the oracle's
+// gate_margin).
 __device__ __forceinline__ float gate_margin(const SelectParams &sp, float x) {
   if (sp.gate_n < 2) return __fmaf_rn(sp.m1, x, sp.m0);
   int i = 0;
@@ -189,7 +191,8 @@ __device__ __forceinline__ float gate_margin(const SelectParams &sp, float x) {
   if (i == sp.gate_n - 1) return sp.gate_y[i];
   const float s = __fdiv_rn(__fsub_rn(sp.gate_y[i + 1], sp.gate_y[i]),
                             __fsub_rn(sp.gate_x[i + 1], sp.gate_x[i]));
-  return __fmaf_rn(__fsub_rn(x, sp.gate_x[i]), s, sp.gate_y[i]);
+  const float v = __fmaf_rn(__fsub_rn(x, sp.gate_x[i]), s, sp.gate_y[i]);
+  return fminf(fmaxf(v, sp.gate_y[i]), sp.gate_y[i + 1]);
 }
 
 // Sort capacity for probe budget P: all clusters of P buckets. Shared memory
@@ -399,14 +402,14 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   int M = block_exclusive_scan(cnt, np, warp_sums);
   // One pass over the candidates. C^dir keys are collected from the back of
   // the key array; the other clusters from the front when they are within the
-  // gate of the running d_min (for m1 >= 0 that gate is never tighter than the
-  // final one: x + fmaf(m1, x, m0) does not decrease with x).
+  // gate of the running d_min. That gate is never tighter than the final one
+  // when theta(x) = x + M(x) does not decrease with x: for m1 >= 0
+  // (x + fmaf(m1, x, m0)) and for a calibrated curve (non-decreasing y, each
+  // segment held within its end values).
   if (tid == 0) sred[2] = 0u;  // keys collected from the front
   __syncthreads();
-  const float m0 = sp.m0, m1 = sp.m1;
-  // (with a calibrated curve, fp32 rounding at its breakpoints could make the
-  // gate decrease by an ulp: no prefilter then)
-  const bool prefilter = !sp.gate_off && sp.gate_n < 2 && m1 >= 0.0f;
+  const float m1 = sp.m1;
+  const bool prefilter = !sp.gate_off && (sp.gate_n >= 2 || m1 >= 0.0f);
   for (int s = tid; s < M; s += nt) {
     const uint32_t c = slot_cluster(cnt, c0s, np, s);
     const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
@@ -420,7 +423,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
       bool maybe = true;
       if (prefilter) {
         const float dm = __uint_as_float(prev < db ? prev : db);
-        maybe = d <= __fadd_rn(dm, __fmaf_rn(m1, dm, m0));
+        maybe = d <= __fadd_rn(dm, gate_margin(sp, dm));
       }
       if (maybe) {
         const unsigned pos = atomicAdd(&sred[2], 1u);

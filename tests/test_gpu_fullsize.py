@@ -25,10 +25,11 @@ def test_full_batch_sampled_parity(name):
     from paper_2608_15438_gb300 import neuroute as nr
 
     w = synth.WORKLOADS[name]
-    P, C, _, _ = bench.OPERATING_POINTS[name]
-    kw = bench.op_params(w)
+    op = bench.OPERATING_POINTS[name]
+    P, C = op["P"], op["C"]
     path = cached_index(name)
     ix = nr.Index(path, 0)
+    kw = bench.op_params(w, ix)
     orc = oracle.Index(path)
     qs = synth.queries(w)
     lg = orc.encode(qs)
@@ -78,10 +79,11 @@ def test_1b_sampled_parity():
 
     torch.cuda.empty_cache()
     w = synth.WORKLOADS["u8-1b"]
-    P, C, _, _ = bench.OPERATING_POINTS["u8-1b"]
-    kw = bench.op_params(w)
+    op = bench.OPERATING_POINTS["u8-1b"]
+    P, C = op["P"], op["C"]
     dev = torch.device("cuda", 0)
     ix, _ = bench.gpu_index(w, torch, nr, dev)
+    kw = bench.op_params(w, ix)       # the calibrated gate and S_max, fitted on this index
     qs = synth.queries(w)
     lg = oracle.encode_weights(synth.encoder_weights(w), w.in_scale, qs)
     dq = torch.from_numpy(qs).cuda()

@@ -147,3 +147,35 @@ def test_calibrated_gate_curve(tmp_path, curve, want):
     p1 = oracle.params(gate_curve=curve, cent_mode=1, b_batch=1 << 20, c_t_low=0)
     L1, _, _, _ = ix.cluster_list_seq(logit, codes, scores, 8, p1)
     assert list(L1) == want
+
+
+def test_gate_margin_closed_form_and_monotone():
+    """M on dyadic breakpoints is the exact linear interpolation; an fp32 slope
+    that rounds up (here (0.7287708 - 0.1917987) / (0.2216479 - 0.0459872))
+    would put M one ulp above y_1 just left of x_1, so each segment is held
+    within its end values; over random curves M never decreases, so the gate
+    theta = x + M(x) does not either."""
+    p = oracle.params(gate_curve=((0.0, 1.0, 3.0), (0.5, 1.0, 2.0)))
+    for x, want in [(-1.0, 0.5), (0.0, 0.5), (0.25, 0.625), (1.0, 1.0), (2.0, 1.5), (2.5, 1.75),
+                    (3.0, 2.0), (100.0, 2.0)]:
+        assert oracle.gate_margin(p, x) == np.float32(want), x
+    f = np.float32
+    x0, x1, y0, y1 = f(0.04598718), f(0.22164789), f(0.19179872), f(0.72877085)
+    p = oracle.params(gate_curve=((x0, x1), (y0, y1)))
+    s = f(f(y1 - y0) / f(x1 - x0))
+    just_left = np.nextafter(x1, f(0))
+    assert f(np.float64(f(just_left - x0)) * np.float64(s) + np.float64(y0)) > y1  # would overshoot
+    assert oracle.gate_margin(p, just_left) == y1
+    rng = np.random.default_rng(9)
+    for _ in range(200):
+        n = int(rng.integers(2, 17))
+        xs = np.sort(rng.choice(np.arange(1, 4000), n, replace=False)).astype(np.float32) * f(1e-4)
+        ys = np.sort(rng.random(n).astype(np.float32))
+        p = oracle.params(gate_curve=(xs, ys))
+        probe = np.concatenate([xs, [np.nextafter(v, f(0)) for v in xs], [np.nextafter(v, f(1)) for v in xs],
+                                rng.random(64).astype(np.float32) * f(0.5)])
+        probe = np.sort(probe.astype(np.float32))
+        m = np.array([oracle.gate_margin(p, v) for v in probe], np.float32)
+        assert np.all(np.diff(m) >= 0)
+        theta = (probe + m).astype(np.float32)
+        assert np.all(np.diff(theta) >= 0)
