@@ -418,6 +418,7 @@ def run_reference(args, w, rank, world):
 
     P, C, t_low = op_point(args, w)
     nq = args.nq or w.nq
+    nq_all = nq
     qs = synth.queries(w, nq)
     import oracle
 
@@ -474,9 +475,11 @@ def run_reference(args, w, rank, world):
             "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
-            "config": {"workload": w.name, "nq_per_step": ns, "P": P, "C": C, "t_low": t_low, "k": args.k},
+            "config": {"workload": w.name, "nq_per_step": ns, "P": P, "C": C, "t_low": t_low, "k": args.k,
+                       "gate_m1": kw.get("gate_m1"), "gate_curve": kw.get("gate_curve"),
+                       "s_max": kw.get("s_max")},
             "cpu_baseline": {"value": v, "unit": "queries/s", "cores": cores, "kind": "oracle",
-                             "sample": f"first {ns} of {nq} queries per step{note}"},
+                             "sample": f"first {ns} of {nq_all} queries per step{note}"},
             "e2e": {"value": v, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     orc.close()
