@@ -49,6 +49,15 @@ CALIB_QUERIES = 10000
 CALIB_BINS = 16
 
 
+EXEC_KEYS = ("pipe_chunk", "refine_ctas")  # nr_params fields that change no result
+
+
+def method_kw(kw):
+    """The parameters of the method itself (the oracle's), without the
+    library's execution settings."""
+    return {k: v for k, v in kw.items() if k not in EXEC_KEYS}
+
+
 def op_params(w, ix=None, t_low=None, calib=None, k=10):
     """nr_params keyword arguments of the workload's operating point. A
     calibrated point fits its curve and cutoff on the GPU index ix (or on
@@ -284,7 +293,7 @@ def oracle_subindex(w, ix, qs, P, kw, path):
 
     lg = oracle.encode_weights(synth.encoder_weights(w), w.in_scale, qs)
     tau = ix.thresholds()
-    p = oracle.params(**kw)
+    p = oracle.params(**method_kw(kw))
     codes = np.concatenate([oracle.probe_list(lg[i], tau, P, p)[0] for i in range(len(qs))])
     rows, _ = ix.extract(codes, path)
     return lg, rows
@@ -323,18 +332,21 @@ def refine_sources_digest():
     return h.hexdigest()
 
 
-def traffic_from_profile(workload, P, C, algorithmic_bytes):
-    """Per-launch DRAM bytes of the refine kernel from a committed ncu summary,
-    valid only while the kernel source is unchanged since the capture and the
-    capture scanned the same candidates (its algorithmic bytes per launch equal
-    this run's: same operating point)."""
+def traffic_from_profile(workload, P, C, algorithmic_bytes, launches=1):
+    """Per-launch DRAM bytes of the refine kernel from a committed ncu summary
+    of the `launches` refine launches of one step, valid only while the kernel
+    source is unchanged since the capture and the capture scanned the same
+    candidates (the algorithmic bytes of the step equal this run's: same
+    operating point)."""
     path = os.path.join(ROOT, "profiles", "refine_traffic.json")
     try:
         rec = json.load(open(path))
         if rec.get("sources_sha256") != refine_sources_digest():
             return None
         e = rec.get("captures", {}).get(f"{workload}/P{P}/C{C}")
-        if e is None or e.get("algorithmic_bytes_per_launch") != algorithmic_bytes:
+        if e is None or e.get("launches", 1) != launches:
+            return None
+        if e.get("algorithmic_bytes_per_launch") * launches != algorithmic_bytes:
             return None
         return e.get("bytes_per_launch")
     except Exception:
@@ -346,7 +358,7 @@ def cpu_baseline(w, path, queries, k, P, C, kw, seconds, truth=None):
 
     orc = oracle.Index(path)
     t_low = kw.get("t_low")
-    p = oracle.params(**kw)
+    p = oracle.params(**method_kw(kw))
     cores = os.cpu_count() or 1
     n = 16
     t = time.perf_counter()
@@ -373,7 +385,7 @@ def calibrate_subindex(w, ix, queries, k, P, C, kw, seconds, path, row_budget):
     lg, rows = oracle_subindex(w, ix, queries[:n], P, kw, path)
     orc = oracle.Index(path)
     t = time.perf_counter()
-    orc.search(queries[:n], k, P, C, oracle.params(**kw), logits=lg, nthreads=os.cpu_count() or 1)
+    orc.search(queries[:n], k, P, C, oracle.params(**method_kw(kw)), logits=lg, nthreads=os.cpu_count() or 1)
     dt = max(time.perf_counter() - t, 1e-6)
     orc.close()
     per_q = max(1.0, rows / n)
@@ -387,7 +399,7 @@ def cpu_baseline_subindex(w, ix, queries, k, P, C, kw, seconds, row_budget=100_0
     import oracle
 
     t_low = kw.get("t_low")
-    p = oracle.params(**kw)
+    p = oracle.params(**method_kw(kw))
     cores = os.cpu_count() or 1
     with tempfile.TemporaryDirectory() as td:
         sub = os.path.join(td, "sub.nrix")
@@ -454,7 +466,7 @@ def run_reference(args, w, rank, world):
     note = ("; sub-index of the buckets these queries probe, index built on the GPU"
             if tmpdir is not None else "")
     kw = kw0 if tmpdir is not None else op_params(w, t_low=t_low)
-    p = oracle.params(**kw)
+    p = oracle.params(**method_kw(kw))
     cores = os.cpu_count() or 1
     n = 16
     t = time.perf_counter()
@@ -697,10 +709,13 @@ def main():
                 print(json.dumps({**cfg, "error": str(ex)}), flush=True)
                 continue
             torch.cuda.synchronize()
-            t = time.perf_counter()
-            ix.search(dq, k, Pp, Cc, out=(ids, dd))
-            torch.cuda.synchronize()
-            el = time.perf_counter() - t
+            els = []
+            for _ in range(3):  # median of three
+                t = time.perf_counter()
+                ix.search(dq, k, Pp, Cc, out=(ids, dd))
+                torch.cuda.synchronize()
+                els.append(time.perf_counter() - t)
+            el = statistics.median(els)
             st = ix.last_stats()
             print(json.dumps({**cfg, "recall": recall_at(ids.cpu().numpy(), truth, k), "qps": nq / el,
                               "cand_per_q": st.candidates / nq, "clusters_per_q": st.clusters / nq}),
@@ -770,10 +785,13 @@ def main():
 
     cand = st.candidates
     row_bytes = w.row_bytes
-    refine_avg_ms = sum(refine_ms) / len(refine_ms)
-    achieved = cand * row_bytes / (refine_avg_ms / 1e3) / 1e9
+    # refinement launches per step: one per pipelined chunk
+    pc = kw.get("pipe_chunk", 0) or 0
+    n_ref = -(-nq // pc) if 0 < pc < nq else 1
+    refine_avg_ms = sum(refine_ms) / len(refine_ms) / n_ref
+    achieved = cand * row_bytes / n_ref / (refine_avg_ms / 1e3) / 1e9
     peaks, peak_src = measured_peaks()
-    traffic = traffic_from_profile(w.name, P, C, cand * row_bytes)
+    traffic = traffic_from_profile(w.name, P, C, cand * row_bytes, n_ref)
     out = {
         "metric": METRIC,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
@@ -795,8 +813,8 @@ def main():
                      "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
                      "frac": achieved / peaks.get("hbm_gbs"), "peak_source": peak_src,
                      "traffic": traffic,
-                     "algorithmic_bytes_per_launch": cand * row_bytes,
-                     "avg_launch_ms": refine_avg_ms},
+                     "algorithmic_bytes_per_launch": cand * row_bytes / n_ref,
+                     "avg_launch_ms": refine_avg_ms, "launches_per_step": n_ref},
         "stage_ms_per_step": {kk: v / args.steps for kk, v in stage_ms.items()},
         "e2e": {"value": e2e_v, "unit": "queries/s", "h2d_bytes_per_step": nq * row_bytes,
                 "d2h_bytes_per_step": nq * k * 12},

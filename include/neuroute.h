@@ -108,11 +108,22 @@ typedef struct {
   /* Calibrated gate (Sec. 3.4): when gate_n >= 2 (at most 16), M is the
    * piecewise-linear curve through (gate_x[i], gate_y[i]), flat beyond its
    * ends: on segment i (the last breakpoint with gate_x[i] <= x),
-   * M(x) = fmaf(x - x_i, (y_{i+1} - y_i) / (x_{i+1} - x_i), y_i) in fp32; the
-   * gate is then on and gate_m0 / gate_m1 are unused. gate_x strictly
-   * increasing, gate_y non-decreasing, all finite. gate_n = 0: M(x) = m0 + m1 x. */
+   * M(x) = fmaf(x - x_i, (y_{i+1} - y_i) / (x_{i+1} - x_i), y_i) in fp32, held
+   * within [y_i, y_{i+1}] so that M never decreases; the gate is then on and
+   * gate_m0 / gate_m1 are unused. gate_x strictly increasing, gate_y
+   * non-decreasing, all finite. gate_n = 0: M(x) = m0 + m1 x. */
   int gate_n;           /* 0, or 2..16; default 0 */
   float gate_x[16], gate_y[16];
+  /* Execution only (results do not depend on these). pipe_chunk > 0: a batch
+   * larger than pipe_chunk queries runs in chunks of pipe_chunk, the
+   * refinement of a chunk (on a library-owned stream) overlapping encode,
+   * route and select of the next chunks (on another), in up to three chunk
+   * buffers; the caller's stream waits for both at the end of the call.
+   * 0 (default): every stage on the caller's stream, one after the other.
+   * refine_ctas: refinement blocks resident per SM, capped (0: as many as fit),
+   * which leaves SM room to the overlapping stages. */
+  int pipe_chunk;       /* >= 0; default 0 */
+  int refine_ctas;      /* in [0, 32]; default 0 */
 } nr_params;
 
 /* Per-search statistics (sums over the queries of the last search call). */

@@ -77,6 +77,9 @@ Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
 nr_status ensure_ws(nr_index *ix, size_t bytes) {
   if (bytes <= ix->ws_cap) return NR_OK;
   if (ix->ws) {
+    // earlier calls' kernels (on the caller's or the library's streams) may
+    // still read the old workspace
+    cudaDeviceSynchronize();
     cudaFree(ix->ws);
     ix->ws = nullptr;
     ix->ws_cap = 0;
@@ -111,6 +114,7 @@ nr_status check_params(const nr_params *p) {
       p->b_batch > 2048 || p->b_min < 0 || p->c_t_low < 0 || p->c_u_min < 0 || p->c_f_min < 0 ||
       !(p->c_alpha_front >= 0.0f && p->c_alpha_front <= 1.0f))
     return NR_ERR_INVALID_ARG;
+  if (p->pipe_chunk < 0 || p->refine_ctas < 0 || p->refine_ctas > 32) return NR_ERR_INVALID_ARG;
   if (p->gate_n != 0) {
     if (p->gate_n < 2 || p->gate_n > 16) return NR_ERR_INVALID_ARG;
     for (int i = 0; i < p->gate_n; ++i) {
@@ -127,11 +131,23 @@ nr_status check_params(const nr_params *p) {
 // Host-side extras of an index: the per-cluster "bucket holds one cluster"
 // table used by K3, stage timers, and the device staging buffer of
 // nr_search_host.
+constexpr int kPipeSlots = 3;  // chunk buffers of the pipelined search
+
+// Streams and events of the pipelined search (created on first use):
+// a runs encode, route and select, b the refinement; sel[s] / ref[s] mark the
+// end of select and of refinement in chunk buffer s.
+struct PipeStreams {
+  cudaStream_t a = nullptr, b = nullptr;
+  cudaEvent_t fork = nullptr, join_a = nullptr, join_b = nullptr;
+  cudaEvent_t sel[kPipeSlots] = {}, ref[kPipeSlots] = {};
+};
+
 struct nr_index_ext {
   uint8_t *single = nullptr;
   std::vector<TimedStage> timers;
   void *io = nullptr;
   size_t io_cap = 0;
+  PipeStreams pipe;
 };
 
 // The extension lives right after the index object (allocated together).
@@ -240,6 +256,8 @@ nr_status nr_params_default(nr_params *p) {
   p->c_alpha_front = 0.5f;
   p->gate_n = 0;
   for (int i = 0; i < 16; ++i) p->gate_x[i] = p->gate_y[i] = 0.0f;
+  p->pipe_chunk = 0;
+  p->refine_ctas = 0;
   return NR_OK;
 }
 
@@ -251,6 +269,15 @@ void nr_index_free(nr_index *ix) {
     cudaEventDestroy(t.a);
     cudaEventDestroy(t.b);
   }
+  PipeStreams &ps = e->pipe;
+  for (cudaEvent_t ev : {ps.fork, ps.join_a, ps.join_b})
+    if (ev) cudaEventDestroy(ev);
+  for (int i = 0; i < kPipeSlots; ++i) {
+    if (ps.sel[i]) cudaEventDestroy(ps.sel[i]);
+    if (ps.ref[i]) cudaEventDestroy(ps.ref[i]);
+  }
+  if (ps.a) cudaStreamDestroy(ps.a);
+  if (ps.b) cudaStreamDestroy(ps.b);
   void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
                   ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->single, e->io};
   for (void *p : ptrs)
@@ -663,29 +690,58 @@ nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int
   return cuda_status(e);
 }
 
+// Streams and events of the pipelined search, created once per index.
+static nr_status ensure_pipe(nr_index *ix) {
+  PipeStreams &ps = ext_of(ix)->pipe;
+  if (ps.a) return NR_OK;
+  int lo = 0, hi = 0;
+  cudaError_t e = cudaDeviceGetStreamPriorityRange(&lo, &hi);
+  // encode, route and select at the higher priority: their blocks are
+  // scheduled first whenever refinement blocks leave room
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&ps.a, cudaStreamNonBlocking, hi);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&ps.b, cudaStreamNonBlocking, lo);
+  cudaEvent_t *evs[] = {&ps.fork, &ps.join_a, &ps.join_b};
+  for (cudaEvent_t *ev : evs)
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+  for (int i = 0; i < kPipeSlots && e == cudaSuccess; ++i) {
+    e = cudaEventCreateWithFlags(&ps.sel[i], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ps.ref[i], cudaEventDisableTiming);
+  }
+  return cuda_status(e);
+}
+
 static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logits_in, int64_t nq,
                              int k, int P, int C, int64_t *d_ids, float *d_d, cudaStream_t s) {
   nr_status st = check_budgets(ix, nq, k, P, C);
   if (st != NR_OK) return st;
-  // workspace: [per-query stats][query counter][per-chunk buffers]
-  const size_t stats_off = 0;
-  const size_t cnt_off = align256(stats_off + (size_t)nq * 4 * 8);
-  const size_t chunk_off = align256(cnt_off + 16);
+  // chunks of qc queries: as many as the workspace budget allows, or
+  // pipe_chunk when pipelined (refinement of chunk i on stream b while stream
+  // a encodes, routes and selects chunk i + 1, i + 2 into other buffers)
+  const int64_t pc = ix->params.pipe_chunk;
+  const bool pipe = pc > 0 && nq > pc;
+  const int slots = pipe ? kPipeSlots : 1;
   Layout one = chunk_layout(ix, 1, P, C);
-  int64_t qc = (int64_t)(kChunkBudget / (one.total > 0 ? one.total : 1));
+  int64_t qc = (int64_t)(kChunkBudget / slots / (one.total > 0 ? one.total : 1));
   if (qc < 1) qc = 1;
+  if (pipe && qc > pc) qc = pc;
   if (qc > nq) qc = nq;
   Layout l = chunk_layout(ix, qc, P, C);
-  if ((st = ensure_ws(ix, chunk_off + l.total)) != NR_OK) return st;
+  const size_t slot_bytes = align256(l.total);
+  // workspace: [per-query stats][one query counter per buffer][chunk buffers]
+  const size_t stats_off = 0;
+  const size_t cnt_off = align256(stats_off + (size_t)nq * 4 * 8);
+  const size_t chunk_off = align256(cnt_off + 16 * (size_t)slots);
+  if ((st = ensure_ws(ix, chunk_off + slot_bytes * (size_t)slots)) != NR_OK) return st;
+  if (pipe && (st = ensure_pipe(ix)) != NR_OK) return st;
   char *w = (char *)ix->ws;
   int64_t *stats = (int64_t *)(w + stats_off);
   ix->d_stats = stats;
   ix->last_nq = nq;
-  unsigned int *counter = (unsigned int *)(w + cnt_off);
-  char *cw = w + chunk_off;
   nr_index_ext *ex = ext_of(ix);
+  PipeStreams &ps = ex->pipe;
+  cudaStream_t sa = pipe ? ps.a : s, sb = pipe ? ps.b : s;
   size_t tslot = 0;
-  auto tstart = [&](int stage) -> size_t {
+  auto tstart = [&](int stage, cudaStream_t st) -> size_t {
     if (!ix->timing) return 0;
     if (tslot >= ex->timers.size()) {
       TimedStage t{stage, nullptr, nullptr};
@@ -694,46 +750,70 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
       ex->timers.push_back(t);
     }
     ex->timers[tslot].stage = stage;
-    cudaEventRecord(ex->timers[tslot].a, s);
+    cudaEventRecord(ex->timers[tslot].a, st);
     return tslot;
   };
-  auto tend = [&](size_t slot) {
+  auto tend = [&](size_t slot, cudaStream_t st) {
     if (!ix->timing) return;
-    cudaEventRecord(ex->timers[slot].b, s);
+    cudaEventRecord(ex->timers[slot].b, st);
     ++tslot;
   };
   cudaError_t e = cudaSuccess;
+  if (pipe) {  // both library streams start after the caller's earlier work
+    e = cudaEventRecord(ps.fork, s);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(sa, ps.fork, 0);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(sb, ps.fork, 0);
+  }
   const int64_t RB = ix->row_bytes;
-  for (int64_t q0 = 0; q0 < nq && e == cudaSuccess; q0 += qc) {
+  int64_t i = 0;
+  for (int64_t q0 = 0; q0 < nq && e == cudaSuccess; q0 += qc, ++i) {
     const int64_t n = (nq - q0) < qc ? (nq - q0) : qc;
+    const int slot = (int)(i % slots);
+    char *cw = w + chunk_off + slot_bytes * (size_t)slot;
+    unsigned int *counter = (unsigned int *)(w + cnt_off + 16 * (size_t)slot);
+    // buffer `slot` is free again once the refinement that last read it ended
+    if (pipe && i >= slots && (e = cudaStreamWaitEvent(sa, ps.ref[slot], 0)) != cudaSuccess) break;
     const void *qp = (const char *)d_q + q0 * RB;
     const float *lg = d_logits_in ? d_logits_in + q0 * ix->b : (const float *)(cw + l.logits);
     size_t ev;
     if (!d_logits_in) {
-      ev = tstart(0);
-      e = nr_launch_encode(ix, qp, n, (float *)(cw + l.logits), s);
-      tend(ev);
+      ev = tstart(0, sa);
+      e = nr_launch_encode(ix, qp, n, (float *)(cw + l.logits), sa);
+      tend(ev, sa);
       if (e != cudaSuccess) break;
     }
-    ev = tstart(1);
-    e = nr_launch_route(ix, lg, n, P, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), s);
-    tend(ev);
+    ev = tstart(1, sa);
+    e = nr_launch_route(ix, lg, n, P, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), sa);
+    tend(ev, sa);
     if (e != cudaSuccess) break;
-    ev = tstart(2);
+    ev = tstart(2, sa);
     e = nr_launch_select(ix, lg, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), n, P, C,
                          (int32_t *)(cw + l.L), (int32_t *)(cw + l.nL), (nr_seg *)(cw + l.seg),
                          (uint32_t *)(cw + l.slen), stats + q0 * 4,
-                         nr_select_slab_bytes(P, ix->K_max) ? cw + l.slab : nullptr, s);
-    tend(ev);
+                         nr_select_slab_bytes(P, ix->K_max) ? cw + l.slab : nullptr, sa);
+    tend(ev, sa);
     if (e != cudaSuccess) break;
-    ev = tstart(3);
+    if (pipe) {
+      e = cudaEventRecord(ps.sel[slot], sa);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(sb, ps.sel[slot], 0);
+      if (e != cudaSuccess) break;
+    }
+    ev = tstart(3, sb);
     e = nr_launch_refine(ix, qp, n, k, P + C, (nr_seg *)(cw + l.seg), (int32_t *)(cw + l.nL),
                          (uint32_t *)(cw + l.slen), d_ids + q0 * k, d_d + q0 * k, stats + q0 * 4,
-                         counter, (int32_t *)(cw + l.perm), s);
-    tend(ev);
+                         counter, (int32_t *)(cw + l.perm), sb);
+    tend(ev, sb);
+    if (pipe && e == cudaSuccess) e = cudaEventRecord(ps.ref[slot], sb);
+  }
+  if (pipe) {  // the caller's stream waits for everything enqueued above, even after an error
+    cudaError_t j = cudaEventRecord(ps.join_a, sa);
+    if (j == cudaSuccess) j = cudaEventRecord(ps.join_b, sb);
+    if (j == cudaSuccess) j = cudaStreamWaitEvent(s, ps.join_a, 0);
+    if (j == cudaSuccess) j = cudaStreamWaitEvent(s, ps.join_b, 0);
+    if (e == cudaSuccess) e = j;
   }
   ix->timed_last = ix->timing;
-  for (size_t i = tslot; i < ex->timers.size(); ++i) ex->timers[i].stage = -1;
+  for (size_t t = tslot; t < ex->timers.size(); ++t) ex->timers[t].stage = -1;
   return cuda_status(e);
 }
 

@@ -101,6 +101,7 @@ cudaError_t persistent_launch(nr_index *ix, K kern, int threads, size_t smem, in
   e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
   if (e != cudaSuccess) return e;
   if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  if (ix->params.refine_ctas > 0 && per_sm > ix->params.refine_ctas) per_sm = ix->params.refine_ctas;
   int64_t grid = (int64_t)per_sm * ix->num_sms;
   if (grid > nq) grid = nq;
   go(kern, (int)grid, threads, smem, s, args);

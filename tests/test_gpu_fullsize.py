@@ -40,7 +40,7 @@ def test_full_batch_sampled_parity(name):
     torch.cuda.synchronize()
     ids, d, st = ids.cpu().numpy(), d.cpu().numpy(), st.cpu().numpy()
     sample = np.linspace(0, w.nq - 1, SAMPLE).astype(np.int64)
-    p = oracle.params(**kw)
+    p = oracle.params(**bench.method_kw(kw))
     ids_o, d_o, st_o = orc.search(qs[sample], 10, P, C, p, logits=lg[sample])
     assert np.array_equal(ids[sample], ids_o)
     if w.dtype == "u8":
@@ -93,7 +93,7 @@ def test_1b_sampled_parity():
     torch.cuda.synchronize()
     ids, d, st = ids.cpu().numpy(), d.cpu().numpy(), st.cpu().numpy()
     sample = np.linspace(0, w.nq - 1, 100).astype(np.int64)
-    p = oracle.params(**kw)
+    p = oracle.params(**bench.method_kw(kw))
     with tempfile.TemporaryDirectory() as td:
         sub = os.path.join(td, "sub.nrix")
         bench.oracle_subindex(w, ix, qs[sample], P, kw, sub)
