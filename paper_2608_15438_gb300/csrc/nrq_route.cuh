@@ -2,7 +2,7 @@
 // lists the probe codes (Eq. 10, Algorithm 1).
 #pragma once
 
-#include "nrq_common.cuh"
+#include "nrq_block.cuh"
 
 namespace nrq {
 
@@ -170,6 +170,247 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
     __syncwarp();
   }
   return n;
+}
+
+// ============================================================== route_block
+// The same probe list by a threshold enumeration, one 128-thread block per
+// query. The flip sets with cost <= T form a subtree of the tree above (costs
+// never decrease along an edge), so for any T with at least P - 1 of them, the
+// first P - 1 sets in key order are the P - 1 smallest keys of that subtree:
+// enumerate it breadth first, sort it, keep the front. T comes from counting
+// subsets by cost on a grid of kRouteBins steps D over [0, T_range], T_range
+// the cost of ranks {0..m-1} with 2^m >= P (its 2^m - 1 subsets cost no more,
+// so the P - 1-th set does not either): each deviation rounded up to
+// s_r = floor(delta_r / D) + 1 steps, the number of subsets with sum of steps
+// <= c is a dynamic program over the ranks, and every such subset costs at most
+// c D in exact arithmetic, below c D (1 + 2^-16) after fp32 rounding. The
+// smallest c whose count reaches P (the empty set included) gives T. Keys,
+// ties and codes are those of route_warp; a subtree larger than the capacity,
+// the R_max filter, or P above 1024 take route_warp (warp 0 of the block).
+constexpr int kRouteThreads = 128;
+constexpr int kRouteBins = 512;
+constexpr int kRouteDp = kRouteBins + 32;  // sums of rounded-up steps overshoot by < 1 per rank
+
+// Keys a thread holds in the final sort: the smallest power of two E with
+// 128 E >= 2 P, or 0 when P > 1024 (route_warp only).
+__host__ __device__ inline int route_block_e(int P) {
+  int E = 1;
+  while (E * kRouteThreads < 2 * P && E < 16) E <<= 1;
+  return E * kRouteThreads >= 2 * P ? E : 0;
+}
+
+struct RouteSmem {
+  uint64_t *keys;   // subtree keys, then the sort's padded runs; or route_warp's heap
+  float *costp;     // per subtree key: its cost without the largest rank
+  uint32_t *dp;     // two count arrays of kRouteDp
+  float *ssd;       // deviation of rank r
+  int *bitidx;      // bit index of rank r
+  int *ctl;         // [0] tail, [1] chosen bin, [2] u0, [3] route_warp's count
+};
+
+__host__ __device__ inline size_t route_region_bytes(int E, int P) {
+  const size_t sort = (size_t)(E * kRouteThreads + (E * kRouteThreads) / 16) * 8;
+  const size_t heap = route_heap_bytes(P);
+  return ((sort > heap ? sort : heap) + 15) & ~(size_t)15;
+}
+
+__host__ __device__ inline size_t route_block_bytes(int E, int P) {
+  return route_region_bytes(E, P) + (size_t)E * kRouteThreads * 4 + (size_t)2 * kRouteDp * 4 +
+         32 * 4 + 32 * 4 + 16 * 4;
+}
+
+__device__ __forceinline__ RouteSmem route_carve(unsigned char *base, int E, int P) {
+  RouteSmem m;
+  m.keys = reinterpret_cast<uint64_t *>(base);
+  m.costp = reinterpret_cast<float *>(base + route_region_bytes(E, P));
+  m.dp = reinterpret_cast<uint32_t *>(m.costp + E * kRouteThreads);
+  m.ssd = reinterpret_cast<float *>(m.dp + 2 * kRouteDp);
+  m.bitidx = reinterpret_cast<int *>(m.ssd + 32);
+  m.ctl = m.bitidx + 32;
+  return m;
+}
+
+// Writes codes[0..n) (any address space) and returns n, uniform in the block.
+// Called by the whole 128-thread block; smem: route_block_bytes(E, P) bytes.
+template <int E>
+__device__ __forceinline__ int route_block(const RouteParams &rp, const float *__restrict__ logit,
+                                           unsigned char *smem, uint32_t *codes) {
+  constexpr int cap = E * kRouteThreads;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int b = rp.b, bsel = rp.bsel, P = rp.P;
+  const RouteSmem m = route_carve(smem, E, P);
+  if (warp == 0) {  // deviations, base code and ranks (Eq. 10, Sec. 3.2.3)
+    float dj = __int_as_float(0x7f800000);
+    bool bit = false;
+    if (lane < b) {
+      const float l = logit[lane];
+      const float tj = rp.tau[lane];
+      bit = l >= tj;
+      dj = fabsf(__fsub_rn(l, tj));
+    }
+    const uint32_t u0 = __ballot_sync(kFull, bit);
+    int rank = 0;
+    for (int i = 0; i < b; ++i) {
+      const float di = __shfl_sync(kFull, dj, i);
+      if (di < dj || (di == dj && i < lane)) ++rank;
+    }
+    if (lane < b) {
+      m.ssd[rank] = dj;
+      m.bitidx[rank] = lane;
+    }
+    if (lane == 0) {
+      m.ctl[0] = 0;
+      m.ctl[1] = -1;
+      m.ctl[2] = (int)u0;
+    }
+  }
+  __syncthreads();
+  const uint32_t u0 = (uint32_t)m.ctl[2];
+  bool use_heap = rp.rmax > 0;
+  float T = __int_as_float(0x7f800000);  // the whole tree
+  const bool none = P <= 1 || bsel < 1;
+  if (!use_heap && !none && P - 1 < (1 << bsel) - 1) {
+    int mr = 0;
+    while ((1 << mr) < P) ++mr;  // mr <= bsel here
+    float thi = 0.0f;
+    for (int r = 0; r < mr; ++r) thi = __fadd_rn(thi, m.ssd[r]);
+    const float trange = fminf(thi, rp.smax);
+    if (!(trange > 0.0f)) {
+      T = trange;
+    } else {
+      const double step = (double)trange / kRouteBins;
+      uint32_t *d0 = m.dp, *d1 = m.dp + kRouteDp;
+      for (int c = tid; c < kRouteDp; c += kRouteThreads) d0[c] = c == 0 ? 1u : 0u;
+      __syncthreads();
+      for (int r = 0; r < bsel; ++r) {
+        const double qv = (double)m.ssd[r] / step;
+        if (qv >= (double)(kRouteDp - 1)) break;  // this rank and all later ones fit no bin
+        const int sr = (int)qv + 1;
+        for (int c = tid; c < kRouteDp; c += kRouteThreads) d1[c] = d0[c] + (c >= sr ? d0[c - sr] : 0u);
+        __syncthreads();
+        uint32_t *t = d0;
+        d0 = d1;
+        d1 = t;
+      }
+      if (warp == 0) {  // smallest c with count(sum of steps <= c) >= P
+        constexpr int per = kRouteDp / 32;
+        uint32_t loc = 0;
+        for (int i = 0; i < per; ++i) loc += d0[lane * per + i];
+        uint32_t incl = loc;
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t v = __shfl_up_sync(kFull, incl, o);
+          if (lane >= o) incl += v;
+        }
+        const unsigned hit = __ballot_sync(kFull, incl >= (uint32_t)P);
+        if (hit) {
+          const int src = __ffs(hit) - 1;
+          if (lane == src) {
+            uint32_t run = incl - loc;
+            int c = lane * per;
+            for (;; ++c) {
+              run += d0[c];
+              if (run >= (uint32_t)P) break;
+            }
+            m.ctl[1] = c;
+          }
+        }
+      }
+      __syncthreads();
+      const int c = m.ctl[1];
+      T = c < 0 ? rp.smax
+                : __double2float_ru((double)c * step * (1.0 + 1.0 / 65536.0));
+    }
+  }
+  const float teff = fminf(T, rp.smax);
+  // breadth-first enumeration of the subtree with cost <= teff
+  int tail = 0;
+  if (!use_heap && !none) {
+    if (tid == 0 && m.ssd[0] <= teff) {
+      m.keys[0] = pack_key(m.ssd[0], 1u, 1u);
+      m.costp[0] = 0.0f;
+      m.ctl[0] = 1;
+    }
+    __syncthreads();
+    int head = 0;
+    tail = m.ctl[0];
+    __syncthreads();  // every thread has read the tail before the first appends
+    while (head < tail && tail <= cap) {
+      const int nb = min(tail - head, kRouteThreads);
+      uint64_t k1 = kEmpty, k2 = kEmpty;
+      float p1 = 0.0f, p2 = 0.0f;
+      if (tid < nb) {
+        const uint64_t key = m.keys[head + tid];
+        const float cp = m.costp[head + tid];
+        const uint32_t mask = (uint32_t)key & 0xffffffu;
+        const uint32_t size = ((uint32_t)key >> 24) & 0xffu;
+        const float cost = __uint_as_float((uint32_t)(key >> 32));
+        const int mx = 31 - __clz((int)mask);
+        if (mx + 1 < bsel) {
+          const float sdn = m.ssd[mx + 1];
+          const float c1 = __fadd_rn(cp, sdn);  // shift: rank mx -> mx + 1
+          if (c1 <= teff) {
+            k1 = pack_key(c1, size, mask + (1u << mx));
+            p1 = cp;
+          }
+          const float c2 = __fadd_rn(cost, sdn);  // expand: add rank mx + 1
+          if (c2 <= teff) {
+            k2 = pack_key(c2, size + 1, mask | (1u << (mx + 1)));
+            p2 = cost;
+          }
+        }
+      }
+      const int cnt = (k1 != kEmpty ? 1 : 0) + (k2 != kEmpty ? 1 : 0);
+      int incl = cnt;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int v = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += v;
+      }
+      int base = 0;
+      if (lane == 31 && incl > 0) base = atomicAdd(&m.ctl[0], incl);
+      base = __shfl_sync(kFull, base, 31);
+      int pos = base + incl - cnt;
+      if (k1 != kEmpty) {
+        if (pos < cap) {
+          m.keys[pos] = k1;
+          m.costp[pos] = p1;
+        }
+        ++pos;
+      }
+      if (k2 != kEmpty && pos < cap) {
+        m.keys[pos] = k2;
+        m.costp[pos] = p2;
+      }
+      __syncthreads();
+      head += nb;
+      tail = m.ctl[0];
+      __syncthreads();  // every thread has read the tail before the next appends
+    }
+    if (tail > cap) use_heap = true;  // uniform: every thread read the same tail
+  }
+  if (use_heap) {
+    __syncthreads();
+    if (warp == 0) {
+      const int n = route_warp(rp, logit, reinterpret_cast<unsigned char *>(m.keys), codes);
+      if (lane == 0) m.ctl[3] = n;
+    }
+    __syncthreads();
+    return m.ctl[3];
+  }
+  const int nout = min(P - 1, tail);
+  uint64_t r[E];
+  merge_sort_regs<E>(m.keys, tail, r);
+  if (tid == 0) codes[0] = u0;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = tid * E + e;
+    if (i < nout) {
+      uint32_t flips = 0;
+      for (uint32_t mk = (uint32_t)r[e] & 0xffffffu; mk; mk &= mk - 1)
+        flips |= 1u << m.bitidx[__ffs(mk) - 1];
+      codes[1 + i] = u0 ^ flips;
+    }
+  }
+  return 1 + nout;
 }
 
 }  // namespace nrq

@@ -67,6 +67,50 @@ def test_route_filters_bit_exact(tiny, torch, kw):
         assert np.array_equal(codes[i, : len(exp)], exp)
 
 
+@pytest.mark.parametrize("P", [2, 63, 64, 65, 128, 129, 256, 257, 512, 513, 777, 1024, 1025])
+@pytest.mark.parametrize("kind", ["encoded", "ties"])
+def test_route_threshold_enumeration_bit_exact(tiny, torch, P, kind):
+    """Probe budgets up to 1024 take the block-wide threshold enumeration
+    (each capacity of its final sort and both sides of every boundary), 1025
+    the heap; logits on a grid of 1/8 around tau give deviations with many
+    ties and zeros, whose subtrees often outgrow the capacity (the block then
+    falls back to the heap)."""
+    ix, orc = tiny["ix"], tiny["orc"]
+    tau = orc.tau()
+    lg = tiny["lg"][:200]
+    if kind == "ties":
+        rng = np.random.default_rng(P)
+        lg = (tau[None, :] + rng.integers(-3, 4, lg.shape) / 8).astype(np.float32)
+    codes, nprobe = ix.route(torch.from_numpy(lg).cuda(), P)
+    codes = codes.cpu().numpy().view(np.uint32)
+    nprobe = nprobe.cpu().numpy()
+    p = oracle.params()
+    for i in range(len(lg)):
+        exp, _, _ = oracle.probe_list(lg[i], tau, P, p)
+        assert nprobe[i] == len(exp), i
+        assert np.array_equal(codes[i, : len(exp)], exp), i
+        assert np.all(codes[i, len(exp):] == 0xFFFFFFFF)
+
+
+@pytest.mark.parametrize("kw", [dict(s_max=0.0), dict(s_max=-1.0), dict(s_max=0.3), dict(l_sel=5),
+                                dict(l_sel=11, s_max=0.5), dict(l_sel=1)])
+@pytest.mark.parametrize("P", [64, 1024])
+def test_route_threshold_filters_bit_exact(tiny, torch, kw, P):
+    ix = tiny["ix"]
+    ix.set_params(**kw)
+    try:
+        codes, nprobe = ix.route(tiny["dl"][:150], P)
+    finally:
+        ix.set_params()
+    codes = codes.cpu().numpy().view(np.uint32)
+    tau = tiny["orc"].tau()
+    p = oracle.params(**kw)
+    for i in range(150):
+        exp, _, _ = oracle.probe_list(tiny["lg"][i], tau, P, p)
+        assert int(nprobe[i]) == len(exp), i
+        assert np.array_equal(codes[i, : len(exp)], exp), i
+
+
 def test_route_b4_hand_order(torch, tmp_path):
     from paper_2608_15438_gb300 import neuroute as nr
 
