@@ -278,14 +278,17 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
     if (!(trange > 0.0f)) {
       T = trange;
     } else {
-      const double step = (double)trange / kRouteBins;
+      // step D = T_range / 512 (exact in fp32); s_r = floor(q + 0.001) + 1 with
+      // q = delta_r / D rounded, whose error (< 1e-4 for q below 544) the 0.001
+      // covers, so s_r D >= delta_r exactly
+      const float step = __fdiv_rn(trange, (float)kRouteBins);
       uint32_t *d0 = m.dp, *d1 = m.dp + kRouteDp;
       for (int c = tid; c < kRouteDp; c += kRouteThreads) d0[c] = c == 0 ? 1u : 0u;
       __syncthreads();
       for (int r = 0; r < bsel; ++r) {
-        const double qv = (double)m.ssd[r] / step;
-        if (qv >= (double)(kRouteDp - 1)) break;  // this rank and all later ones fit no bin
-        const int sr = (int)qv + 1;
+        const float qv = __fdiv_rn(m.ssd[r], step);
+        if (!(qv < (float)(kRouteDp - 2))) break;  // this rank and all later ones fit no bin
+        const int sr = (int)__fadd_rn(qv, 0.001f) + 1;
         for (int c = tid; c < kRouteDp; c += kRouteThreads) d1[c] = d0[c] + (c >= sr ? d0[c - sr] : 0u);
         __syncthreads();
         uint32_t *t = d0;
@@ -317,8 +320,8 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
       }
       __syncthreads();
       const int c = m.ctl[1];
-      T = c < 0 ? rp.smax
-                : __double2float_ru((double)c * step * (1.0 + 1.0 / 65536.0));
+      // T >= c D (1 + 2^-16): products rounded up
+      T = c < 0 ? rp.smax : __fmul_ru(__fmul_ru((float)c, step), 1.0f + 1.0f / 65536.0f);
     }
   }
   const float teff = fminf(T, rp.smax);
