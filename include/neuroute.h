@@ -31,7 +31,8 @@
  *
  * Index file (little-endian), written by the package's builder:
  *   header 256 B: "NRIXv001", u32 version=1, u32 dtype (0 uint8, 1 fp32),
- *     u64 N, u32 D, H, b, K_max, t, u32 0, u64 n_clusters, f32 in_scale,
+ *     u64 N (< 2^32 - 1), u32 D, H, b, K_max, t, u32 0, u64 n_clusters (< 2^31),
+ *     f32 in_scale,
  *     u32 0, u64 section offsets[10], u64 file size
  *   sections (256-byte aligned): W1 f32[H][D], b1 f32[H], W2 f32[b][H],
  *     b2 f32[b], tau f32[b], bkt_off u32[2^b + 1] (code -> cluster range),

@@ -143,7 +143,6 @@ struct PipeStreams {
 };
 
 struct nr_index_ext {
-  uint8_t *single = nullptr;
   std::vector<TimedStage> timers;
   void *io = nullptr;
   size_t io_cap = 0;
@@ -158,7 +157,6 @@ struct nr_index_full {
 
 static nr_index_ext *ext_of(nr_index *ix) { return &reinterpret_cast<nr_index_full *>(ix)->ext; }
 
-const uint8_t *nr_single_table(nr_index *ix) { return ext_of(ix)->single; }
 
 nr_index *nr_index_alloc() {
   auto *full = new (std::nothrow) nr_index_full();
@@ -167,7 +165,6 @@ nr_index *nr_index_alloc() {
   return &full->ix;
 }
 
-void nr_index_set_single(nr_index *ix, uint8_t *d_single) { ext_of(ix)->single = d_single; }
 
 nr_status nr_index_init_device(nr_index *ix) {
   cudaDeviceProp prop;
@@ -279,7 +276,7 @@ void nr_index_free(nr_index *ix) {
   if (ps.a) cudaStreamDestroy(ps.a);
   if (ps.b) cudaStreamDestroy(ps.b);
   void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
-                  ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->single, e->io};
+                  ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->io};
   for (void *p : ptrs)
     if (p) cudaFree(p);
   delete reinterpret_cast<nr_index_full *>(ix);
@@ -336,7 +333,7 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   };
   if ((ix->dtype != 0 && ix->dtype != 1) || ix->b < 1 || ix->b > 24 || ix->D < 1 || ix->H < 1 ||
       ix->H > 4096 || ix->N < 1 || ix->N >= (int64_t)0xFFFFFFFFll || ix->n_cl < 1 ||
-      ix->n_cl >= (int64_t)0xFFFFFFFFll || ix->row_bytes % 16 != 0 || ix->row_bytes > 1024 ||
+      ix->n_cl >= ((int64_t)1 << 31) || ix->row_bytes % 16 != 0 || ix->row_bytes > 1024 ||
       ix->K_max < 0)
     return bad(NR_ERR_FORMAT);
   const uint64_t nb = ((uint64_t)1 << ix->b) + 1;
@@ -359,12 +356,10 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
     return bad(NR_ERR_IO);
   // clusters per bucket: K_max from the header, else from the directory
   int kmax_dir = 1;
-  std::vector<uint8_t> single((size_t)ix->n_cl, 0);
   for (uint64_t u = 0; u + 1 < nb; ++u) {
     if (bkt[u + 1] >= bkt[u]) {
       const uint32_t n = bkt[u + 1] - bkt[u];
       if ((int64_t)n > kmax_dir && n <= 65536) kmax_dir = (int)n;
-      if (n == 1 && bkt[u] < (uint64_t)ix->n_cl) single[bkt[u]] = 1;
     }
   }
   if (ix->K_max < 1) ix->K_max = kmax_dir;
@@ -385,7 +380,6 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   };
   if ((st = up((void **)&ix->tau, tau.data(), sz[4])) != NR_OK) return bad(st);
   if ((st = up((void **)&ix->bkt_off, bkt.data(), sz[5])) != NR_OK) return bad(st);
-  if ((st = up((void **)&ext_of(ix)->single, single.data(), single.size())) != NR_OK) return bad(st);
   // large sections streamed through a pinned staging buffer
   const size_t stage_bytes = (size_t)64 << 20;
   void *stage = nullptr;

@@ -574,7 +574,7 @@ __global__ void csr_kernel(const uint32_t *__restrict__ ne_code, const uint32_t 
                            const uint32_t *__restrict__ bstart,
                            const uint32_t *__restrict__ slot_cnt,
                            const float *__restrict__ slot_cent, int64_t ne, int b, uint32_t *cl_off,
-                           float *cent, uint8_t *single, unsigned int *stats) {
+                           float *cent, unsigned int *stats) {
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < ne;
        e += (int64_t)gridDim.x * blockDim.x) {
     const uint32_t u = ne_code[e];
@@ -586,7 +586,6 @@ __global__ void csr_kernel(const uint32_t *__restrict__ ne_code, const uint32_t 
       cl_off[g0 + k] = r;
       r += slot_cnt[sl + k];
       atomicMax(&stats[1], slot_cnt[sl + k]);
-      single[g0 + k] = nk == 1 ? 1 : 0;
       for (int j = 0; j < b; ++j) cent[(size_t)(g0 + k) * b + j] = slot_cent[(size_t)(sl + k) * b + j];
     }
   }
@@ -873,15 +872,13 @@ nr_status finish_impl(nr_builder *bd, int64_t *info, cudaStream_t s) {
   uint32_t ncl_total = 0;
   NRB_TRY(cudaMemcpy(&ncl_total, ix->bkt_off + nb, 4, cudaMemcpyDeviceToHost));
   ix->n_cl = ncl_total;
-  uint8_t *single;
+  if (ix->n_cl >= ((int64_t)1 << 31)) return NR_ERR_INVALID_ARG;  // cluster indices fill 31 bits of a sort key
   NRB_TRY(cudaMalloc((void **)&ix->cl_off, ((size_t)ix->n_cl + 1) * 4));
   NRB_TRY(cudaMalloc((void **)&ix->cent, (size_t)ix->n_cl * b * 4 + 16));
-  NRB_TRY(cudaMalloc((void **)&single, (size_t)ix->n_cl + 16));
-  nr_index_set_single(ix, single);
   NRB_TRY(cudaMemsetAsync(d_small, 0, 64, s));
   csr_kernel<<<grid_for(ne, 128, nsm), 128, 0, s>>>(ne_code, a.ncl, kslot, ix->bkt_off, bstart,
                                                     a.slot_cnt, a.slot_cent, ne, b, ix->cl_off,
-                                                    ix->cent, single, d_small);
+                                                    ix->cent, d_small);
   NRB_TRY(cudaGetLastError());
   {
     const uint32_t nn = (uint32_t)N;

@@ -61,7 +61,6 @@ nr_status nr_index_init_device(nr_index *ix);  // num_sms and the device check f
 // derived forms; needs D, H and b set
 nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1, const float *W2,
                                   const float *b2);
-void nr_index_set_single(nr_index *ix, uint8_t *d_single);  // takes ownership
 
 // kernel launchers (each returns cudaGetLastError() after the launch)
 bool nr_encode_uses_tensor_cores(const nr_index *ix);

@@ -66,8 +66,6 @@ __global__ void __launch_bounds__(kThreads, MODE == 0 ? 6 : 1)
 
 }  // namespace
 
-// defined in nr_api.cu: per-cluster flag "its bucket holds exactly one cluster"
-const uint8_t *nr_single_table(nr_index *ix);
 
 nrq::SelectParams nr_select_params(nr_index *ix, int P, int C) {
   nrq::SelectParams sp;
@@ -80,7 +78,6 @@ nrq::SelectParams nr_select_params(nr_index *ix, int P, int C) {
   sp.bkt_off = ix->bkt_off;
   sp.cl_off = ix->cl_off;
   sp.cent = ix->cent;
-  sp.single = nr_single_table(ix);
   const float m0 = ix->params.gate_m0;
   sp.gate_n = ix->params.gate_n;
   for (int i = 0; i < 16; ++i) {

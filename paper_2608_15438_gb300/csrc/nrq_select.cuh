@@ -13,7 +13,6 @@ struct SelectParams {
   int64_t n_cl, N;
   const uint32_t *bkt_off, *cl_off;
   const float *cent;
-  const uint8_t *single;  // [n_cl] 1 if the cluster's bucket holds one cluster
   bool gate_off;
   float m0, m1;
   int *err;
@@ -102,17 +101,27 @@ __device__ __forceinline__ float centroid_dist(const float *__restrict__ mu, con
   return acc;
 }
 
-// Cluster of candidate slot s: slots are numbered probe by probe, off[i] the
-// first slot of probe i (nondecreasing), c0[i] the first cluster of probe i.
-__device__ __forceinline__ uint32_t slot_cluster(const int *off, const int *c0, int np, int s) {
+// Probe of candidate slot s: slots are numbered probe by probe, off[i] the
+// first slot of probe i (nondecreasing).
+__device__ __forceinline__ int slot_probe(const int *off, int np, int s) {
   int lo = 0, hi = np - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
     if (off[mid] <= s) lo = mid;
     else hi = mid - 1;
   }
-  return (uint32_t)(c0[lo] + (s - off[lo]));
+  return lo;
 }
+
+// Sort keys of the order-independent stage: ((d bits) << 32) | (c << 1) |
+// single, single = the cluster's bucket holds only it (C^dir). For distinct
+// clusters (c < 2^31) they order exactly as (d, c) does; the flag rides along
+// so that no lookup is needed to tell C^dir apart after the sort.
+__device__ __forceinline__ uint64_t tagged_key(float d, uint32_t c, bool single) {
+  return ((uint64_t)__float_as_uint(d) << 32) | ((uint64_t)c << 1) | (single ? 1u : 0u);
+}
+__device__ __forceinline__ uint32_t key_cluster(uint64_t k) { return (uint32_t)k >> 1; }
+__device__ __forceinline__ bool key_single(uint64_t k) { return (k & 1u) != 0; }
 
 // The kept list from the collected keys k[0..n) (n <= E * blockDim.x), sorted
 // into registers: C^dir keys always, the others while their rank among the
@@ -130,7 +139,7 @@ __device__ __forceinline__ int select_tail_regs(const SelectParams &sp, uint64_t
 #pragma unroll
   for (int e = 0; e < E; ++e)
     if (r[e] != kEmpty) {
-      if (__ldg(&sp.single[(uint32_t)r[e]])) sg |= 1u << e;
+      if (key_single(r[e])) sg |= 1u << e;
       else ++ns;
     }
   int all;
@@ -155,7 +164,7 @@ __device__ __forceinline__ int select_tail_regs(const SelectParams &sp, uint64_t
 #pragma unroll
   for (int e = 0; e < E; ++e)
     if ((kp >> e) & 1u) {
-      const uint32_t c = (uint32_t)r[e];
+      const uint32_t c = key_cluster(r[e]);
       const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
       if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
       else lsum += (int)(r1 - r0);
@@ -165,7 +174,7 @@ __device__ __forceinline__ int select_tail_regs(const SelectParams &sp, uint64_t
 #pragma unroll
   for (int e = 0; e < E; ++e)
     if ((kp >> e) & 1u) {
-      const uint32_t c = (uint32_t)r[e];
+      const uint32_t c = key_cluster(r[e]);
       const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
       const int ln = (r1 < r0 || (int64_t)r1 > sp.N) ? 0 : (int)(r1 - r0);
       seg[pos].row0 = r0;
@@ -258,10 +267,12 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   const float m1 = sp.m1;
   const bool prefilter = !sp.gate_off && (sp.gate_n >= 2 || m1 >= 0.0f);
   for (int s = tid; s < M; s += nt) {
-    const uint32_t c = slot_cluster(cnt, c0s, np, s);
+    const int pi = slot_probe(cnt, np, s);
+    const uint32_t c = (uint32_t)(c0s[pi] + (s - cnt[pi]));
+    const bool single = (pi + 1 < np ? cnt[pi + 1] : M) - cnt[pi] == 1;  // C^dir
     const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
-    const uint64_t key = ((uint64_t)__float_as_uint(d) << 32) | c;
-    if (__ldg(&sp.single[c])) {
+    const uint64_t key = tagged_key(d, c, single);
+    if (single) {
       const unsigned pos = atomicAdd(&sred[1], 1u);
       if (pos < (unsigned)S_smem) keys[S_smem - 1 - pos] = key;
     } else {
@@ -351,14 +362,15 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
     for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
       const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
-      for (int j = 0; j < n; ++j) keys[o + j] = (uint64_t)(uint32_t)(c0s[i] + j);
+      for (int j = 0; j < n; ++j) keys[o + j] = ((uint64_t)(uint32_t)(c0s[i] + j) << 1) | (n == 1 ? 1u : 0u);
     }
     __syncthreads();
     for (int s = tid; s < M; s += nt) {
-      const uint32_t c = (uint32_t)keys[s];
+      const uint64_t kc = keys[s];
+      const uint32_t c = key_cluster(kc);
       const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
-      const bool keep = __ldg(&sp.single[c]) || d <= theta;
-      keys[s] = keep ? (((uint64_t)__float_as_uint(d) << 32) | c) : kEmpty;
+      const bool keep = key_single(kc) || d <= theta;
+      keys[s] = keep ? tagged_key(d, c, key_single(kc)) : kEmpty;
     }
     for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
     __syncthreads();
@@ -368,14 +380,14 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   int *keep = ints;  // [Sn]
   for (int s = tid; s < Sn; s += nt) {
     const uint64_t kk = keys[s];
-    keep[s] = (s < M && kk != kEmpty && !__ldg(&sp.single[(uint32_t)kk])) ? 1 : 0;
+    keep[s] = (s < M && kk != kEmpty && !key_single(kk)) ? 1 : 0;
   }
   __syncthreads();
   block_exclusive_scan(keep, Sn, warp_sums);  // survivor rank in key order
   for (int s = tid; s < Sn; s += nt) {
     const uint64_t kk = keys[s];
     int kp = 0;
-    if (s < M && kk != kEmpty) kp = __ldg(&sp.single[(uint32_t)kk]) ? 1 : (keep[s] < sp.C ? 1 : 0);
+    if (s < M && kk != kEmpty) kp = key_single(kk) ? 1 : (keep[s] < sp.C ? 1 : 0);
     keep[s] = kp;
   }
   __syncthreads();
@@ -385,7 +397,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     if (s < M && kk != kEmpty) {
       const int pos = keep[s];
       const bool kept = (s + 1 < Sn ? keep[s + 1] : nl) > pos;
-      if (kept) seg[pos].row0 = (uint32_t)kk;  // cluster index for now
+      if (kept) seg[pos].row0 = key_cluster(kk);  // cluster index for now
     }
   }
   __syncthreads();
