@@ -182,55 +182,6 @@ nr_status nr_index_init_device(nr_index *ix) {
   return NR_OK;
 }
 
-namespace {
-
-__global__ void pack_clusters_kernel(const float *__restrict__ cent, const uint32_t *__restrict__ cl_off,
-                                     int64_t n_cl, int b, int stride, float *__restrict__ crec) {
-  for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < n_cl;
-       c += (int64_t)gridDim.x * blockDim.x) {
-    float *r = crec + (size_t)c * stride;
-    for (int j = 0; j < stride - 2; ++j) r[j] = j < b ? cent[(size_t)c * b + j] : 0.0f;
-    reinterpret_cast<uint2 *>(r)[stride / 2 - 1] = make_uint2(cl_off[c], cl_off[c + 1]);
-  }
-}
-
-__global__ void unpack_centroids_kernel(const float *__restrict__ crec, int64_t c0, int64_t n, int b,
-                                        int stride, float *__restrict__ cent) {
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n * b;
-       i += (int64_t)gridDim.x * blockDim.x)
-    cent[i] = crec[(size_t)(c0 + i / b) * stride + (size_t)(i % b)];
-}
-
-int grid_of(int64_t work, int sms) {
-  int64_t g = (work + 255) / 256;
-  const int64_t cap = (int64_t)(sms > 0 ? sms : 1) * 32;
-  return (int)(g < 1 ? 1 : (g > cap ? cap : g));
-}
-
-}  // namespace
-
-nr_status nr_index_pack_clusters(nr_index *ix, const float *d_cent) {
-  ix->crec_stride = nr_crec_stride(ix->b);
-  if (cudaMalloc((void **)&ix->crec, (size_t)ix->n_cl * ix->crec_stride * 4 + 16) != cudaSuccess) {
-    cudaGetLastError();
-    ix->crec = nullptr;
-    return NR_ERR_OOM;
-  }
-  pack_clusters_kernel<<<grid_of(ix->n_cl, ix->num_sms), 256>>>(d_cent, ix->cl_off, ix->n_cl, ix->b,
-                                                                 ix->crec_stride, ix->crec);
-  cudaError_t e = cudaGetLastError();
-  if (e == cudaSuccess) e = cudaDeviceSynchronize();
-  return cuda_status(e);
-}
-
-cudaError_t nr_unpack_centroids(const nr_index *ix, int64_t c0, int64_t n, float *d_cent,
-                                cudaStream_t s) {
-  if (n <= 0) return cudaSuccess;
-  unpack_centroids_kernel<<<grid_of(n * ix->b, ix->num_sms), 256, 0, s>>>(ix->crec, c0, n, ix->b,
-                                                                         ix->crec_stride, d_cent);
-  return cudaGetLastError();
-}
-
 nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1, const float *W2,
                                   const float *b2) {
   const int D = ix->D, H = ix->H, b = ix->b;
@@ -324,7 +275,7 @@ void nr_index_free(nr_index *ix) {
   }
   if (ps.a) cudaStreamDestroy(ps.a);
   if (ps.b) cudaStreamDestroy(ps.b);
-  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->crec, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
+  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
                   ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->io};
   for (void *p : ptrs)
     if (p) cudaFree(p);
@@ -452,11 +403,8 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
     }
     return NR_OK;
   };
-  float *d_cent = nullptr;  // [n_cl][b], packed into the cluster records below
   st = stream_up(6, (void **)&ix->cl_off);
-  if (st == NR_OK) st = stream_up(7, (void **)&d_cent);
-  if (st == NR_OK) st = nr_index_pack_clusters(ix, d_cent);
-  if (d_cent) cudaFree(d_cent);
+  if (st == NR_OK) st = stream_up(7, (void **)&ix->cent);
   if (st == NR_OK) st = stream_up(8, (void **)&ix->ids);
   if (st == NR_OK) st = stream_up(9, &ix->vec);
   cudaFreeHost(stage);
@@ -553,23 +501,10 @@ nr_status nr_index_save(nr_index *ix, const char *path) {
     cudaGetLastError();
     return NR_ERR_CUDA;
   }
-  float *d_cent = nullptr;  // the centroids out of the cluster records
-  if (cudaMalloc((void **)&d_cent, (size_t)ix->n_cl * ix->b * 4 + 16) != cudaSuccess) {
-    cudaGetLastError();
-    return NR_ERR_OOM;
-  }
-  cudaError_t e = nr_unpack_centroids(ix, 0, ix->n_cl, d_cent, nullptr);
-  if (e == cudaSuccess) e = cudaDeviceSynchronize();
-  if (e != cudaSuccess) {
-    cudaFree(d_cent);
-    return cuda_status(e);
-  }
   const void *src[10] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->bkt_off,
-                         ix->cl_off, d_cent, ix->ids, ix->vec};
+                         ix->cl_off, ix->cent, ix->ids, ix->vec};
   const bool dev[10] = {true, true, true, true, true, true, true, true, true, true};
-  const nr_status st = write_nrix(ix, ix->N, ix->n_cl, src, dev, path);
-  cudaFree(d_cent);
-  return st;
+  return write_nrix(ix, ix->N, ix->n_cl, src, dev, path);
 }
 
 nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, const char *path,
@@ -636,12 +571,8 @@ nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, con
   int64_t ci = 0, ri = 0;
   for (size_t i = 0; i < codes.size(); ++i) {
     const size_t k = c1[i] - c0[i];
-    if (k > 0 && cudaMemcpy2D(&cent[(size_t)ci * ix->b], (size_t)ix->b * 4,
-                              ix->crec + (size_t)c0[i] * ix->crec_stride, (size_t)ix->crec_stride * 4,
-                              (size_t)ix->b * 4, k, cudaMemcpyDeviceToHost) != cudaSuccess) {
-      cudaGetLastError();
+    if (!d2h(&cent[(size_t)ci * ix->b], ix->cent + (size_t)c0[i] * ix->b, k * ix->b * 4))
       return NR_ERR_CUDA;
-    }
     const uint32_t r0 = clo[i].front(), r1 = clo[i].back();
     if (r1 > r0) {
       if (!d2h(&ids[(size_t)ri], ix->ids + r0, (size_t)(r1 - r0) * 4)) return NR_ERR_CUDA;

@@ -573,8 +573,8 @@ __global__ void csr_kernel(const uint32_t *__restrict__ ne_code, const uint32_t 
                            const uint32_t *__restrict__ kslot, const uint32_t *__restrict__ bkt_off,
                            const uint32_t *__restrict__ bstart,
                            const uint32_t *__restrict__ slot_cnt,
-                           const float *__restrict__ slot_cent, int64_t ne, int b, int stride,
-                           uint32_t *cl_off, float *crec, unsigned int *stats) {
+                           const float *__restrict__ slot_cent, int64_t ne, int b, uint32_t *cl_off,
+                           float *cent, unsigned int *stats) {
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < ne;
        e += (int64_t)gridDim.x * blockDim.x) {
     const uint32_t u = ne_code[e];
@@ -584,11 +584,9 @@ __global__ void csr_kernel(const uint32_t *__restrict__ ne_code, const uint32_t 
     if (nk == 1) atomicAdd(&stats[2], 1u);
     for (uint32_t k = 0; k < nk; ++k) {
       cl_off[g0 + k] = r;
-      float *rec = crec + (size_t)(g0 + k) * stride;  // cluster record: centroid, zeros, row range
-      for (int j = 0; j < stride - 2; ++j) rec[j] = j < b ? slot_cent[(size_t)(sl + k) * b + j] : 0.0f;
-      reinterpret_cast<uint2 *>(rec)[stride / 2 - 1] = make_uint2(r, r + slot_cnt[sl + k]);
       r += slot_cnt[sl + k];
       atomicMax(&stats[1], slot_cnt[sl + k]);
+      for (int j = 0; j < b; ++j) cent[(size_t)(g0 + k) * b + j] = slot_cent[(size_t)(sl + k) * b + j];
     }
   }
 }
@@ -876,12 +874,11 @@ nr_status finish_impl(nr_builder *bd, int64_t *info, cudaStream_t s) {
   ix->n_cl = ncl_total;
   if (ix->n_cl >= ((int64_t)1 << 31)) return NR_ERR_INVALID_ARG;  // cluster indices fill 31 bits of a sort key
   NRB_TRY(cudaMalloc((void **)&ix->cl_off, ((size_t)ix->n_cl + 1) * 4));
-  ix->crec_stride = nr_crec_stride(b);
-  NRB_TRY(cudaMalloc((void **)&ix->crec, (size_t)ix->n_cl * ix->crec_stride * 4 + 16));
+  NRB_TRY(cudaMalloc((void **)&ix->cent, (size_t)ix->n_cl * b * 4 + 16));
   NRB_TRY(cudaMemsetAsync(d_small, 0, 64, s));
   csr_kernel<<<grid_for(ne, 128, nsm), 128, 0, s>>>(ne_code, a.ncl, kslot, ix->bkt_off, bstart,
-                                                    a.slot_cnt, a.slot_cent, ne, b, ix->crec_stride,
-                                                    ix->cl_off, ix->crec, d_small);
+                                                    a.slot_cnt, a.slot_cent, ne, b, ix->cl_off,
+                                                    ix->cent, d_small);
   NRB_TRY(cudaGetLastError());
   {
     const uint32_t nn = (uint32_t)N;

@@ -97,8 +97,7 @@ __global__ void locate_kernel(const uint32_t *__restrict__ ids, int64_t N,
 // d_c = sum_j (l_j - mu_cj)^2 as a sequential fmaf chain (the select kernel's)
 __global__ void cent_dist_kernel(const float *__restrict__ logits, int64_t nq, int b,
                                  const int32_t *__restrict__ clusters, int m,
-                                 const float *__restrict__ crec, int stride, int64_t n_cl,
-                                 float *out) {
+                                 const float *__restrict__ cent, int64_t n_cl, float *out) {
   const int64_t total = nq * (int64_t)m;
   for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
        t += (int64_t)gridDim.x * blockDim.x) {
@@ -107,7 +106,7 @@ __global__ void cent_dist_kernel(const float *__restrict__ logits, int64_t nq, i
     float acc = __int_as_float(0x7f800000);
     if (c >= 0 && c < n_cl) {
       acc = 0.0f;
-      const float *mu = crec + (size_t)c * stride;
+      const float *mu = cent + (size_t)c * b;
       const float *l = logits + (size_t)q * b;
       for (int j = 0; j < b; ++j) {
         const float d = __fsub_rn(l[j], mu[j]);
@@ -172,7 +171,7 @@ nr_status nr_centroid_dists(nr_index *ix, const float *d_logits, int64_t nq,
   DeviceGuard g(ix->device);
   const int sms = ix->num_sms > 0 ? ix->num_sms : 1;
   cent_dist_kernel<<<grid_for(nq * (int64_t)m, sms), 256, 0, (cudaStream_t)stream>>>(
-      d_logits, nq, ix->b, d_clusters, m, ix->crec, ix->crec_stride, ix->n_cl, d_out);
+      d_logits, nq, ix->b, d_clusters, m, ix->cent, ix->n_cl, d_out);
   return cuda_status(cudaGetLastError());
 }
 

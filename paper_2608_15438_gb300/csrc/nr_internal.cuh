@@ -26,11 +26,7 @@ struct nr_index {
   int64_t row_bytes = 0;
   // device arrays
   float *W1 = nullptr, *b1 = nullptr, *W2 = nullptr, *b2 = nullptr, *tau = nullptr;
-  // cluster records [n_cl][crec_stride floats]: the centroid (b floats), zeros,
-  // then the cluster's row range (u32 first row, u32 end row) in the last two
-  // slots; 64 or 128 bytes, so a centroid read and its row range share lines
-  float *crec = nullptr;
-  int crec_stride = 0;
+  float *cent = nullptr;
   float *W1T = nullptr;  // [D][H]
   void *W1h = nullptr;   // fp16 [H][D] (tensor-core encoder)
   void *W2h = nullptr;   // fp16 [16 or 32][H], rows >= b zero
@@ -56,15 +52,6 @@ struct nr_seg {
   uint32_t row0;
   uint32_t pos;
 };
-
-// Floats per cluster record for b-bit codes (64 bytes up to b = 14, else 128).
-inline int nr_crec_stride(int b) { return b + 2 <= 16 ? 16 : 32; }
-// Fills ix->crec (allocated here) from centroids d_cent [n_cl][b] and
-// ix->cl_off (both on the device); synchronous.
-nr_status nr_index_pack_clusters(nr_index *ix, const float *d_cent);
-// Copies the centroids of clusters [c0, c0 + n) into d_cent [n][b] on stream s.
-cudaError_t nr_unpack_centroids(const nr_index *ix, int64_t c0, int64_t n, float *d_cent,
-                                cudaStream_t s);
 
 // Index object helpers shared by the file loader and the GPU builder
 // (nr_api.cu). The device must be current.

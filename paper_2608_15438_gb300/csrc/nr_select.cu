@@ -76,8 +76,8 @@ nrq::SelectParams nr_select_params(nr_index *ix, int P, int C) {
   sp.n_cl = ix->n_cl;
   sp.N = ix->N;
   sp.bkt_off = ix->bkt_off;
-  sp.crec = ix->crec;
-  sp.stride = ix->crec_stride;
+  sp.cl_off = ix->cl_off;
+  sp.cent = ix->cent;
   const float m0 = ix->params.gate_m0;
   sp.gate_n = ix->params.gate_n;
   for (int i = 0; i < 16; ++i) {

@@ -11,9 +11,8 @@ namespace nrq {
 struct SelectParams {
   int b, K_max, P, C;
   int64_t n_cl, N;
-  const uint32_t *bkt_off;
-  const float *crec;  // cluster records: centroid, then (first row, end row) in the last two slots
-  int stride;         // floats per record
+  const uint32_t *bkt_off, *cl_off;
+  const float *cent;
   bool gate_off;
   float m0, m1;
   int *err;
@@ -25,14 +24,6 @@ struct SelectParams {
   int gate_n;
   float gate_x[16], gate_y[16];
 };
-
-// Cluster c's record: its centroid, then its row range
-__device__ __forceinline__ const float *cluster_rec(const SelectParams &sp, uint32_t c) {
-  return sp.crec + (size_t)c * sp.stride;
-}
-__device__ __forceinline__ uint2 cluster_rows(const SelectParams &sp, uint32_t c) {
-  return __ldg(reinterpret_cast<const uint2 *>(cluster_rec(sp, c)) + (sp.stride / 2 - 1));
-}
 
 // The gate margin M(x): m0 + m1 x, or the calibrated monotone piecewise-linear
 // curve, flat beyond its ends, each segment's value held within its end values
@@ -174,8 +165,7 @@ __device__ __forceinline__ int select_tail_regs(const SelectParams &sp, uint64_t
   for (int e = 0; e < E; ++e)
     if ((kp >> e) & 1u) {
       const uint32_t c = key_cluster(r[e]);
-      const uint2 rr = cluster_rows(sp, c);
-      const uint32_t r0 = rr.x, r1 = rr.y;
+      const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
       if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
       else lsum += (int)(r1 - r0);
     }
@@ -185,8 +175,7 @@ __device__ __forceinline__ int select_tail_regs(const SelectParams &sp, uint64_t
   for (int e = 0; e < E; ++e)
     if ((kp >> e) & 1u) {
       const uint32_t c = key_cluster(r[e]);
-      const uint2 rr = cluster_rows(sp, c);
-      const uint32_t r0 = rr.x, r1 = rr.y;
+      const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
       const int ln = (r1 < r0 || (int64_t)r1 > sp.N) ? 0 : (int)(r1 - r0);
       seg[pos].row0 = r0;
       seg[pos].pos = (uint32_t)spos;
@@ -281,7 +270,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     const int pi = slot_probe(cnt, np, s);
     const uint32_t c = (uint32_t)(c0s[pi] + (s - cnt[pi]));
     const bool single = (pi + 1 < np ? cnt[pi + 1] : M) - cnt[pi] == 1;  // C^dir
-    const float d = centroid_dist(cluster_rec(sp, c), slog, sp.b);
+    const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
     const uint64_t key = tagged_key(d, c, single);
     if (single) {
       const unsigned pos = atomicAdd(&sred[1], 1u);
@@ -379,7 +368,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     for (int s = tid; s < M; s += nt) {
       const uint64_t kc = keys[s];
       const uint32_t c = key_cluster(kc);
-      const float d = centroid_dist(cluster_rec(sp, c), slog, sp.b);
+      const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
       const bool keep = key_single(kc) || d <= theta;
       keys[s] = keep ? tagged_key(d, c, key_single(kc)) : kEmpty;
     }
@@ -416,8 +405,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   for (int i = tid; i < nl; i += nt) {
     const uint32_t c = seg[i].row0;
     if (L) L[i] = (int32_t)c;
-    const uint2 rr = cluster_rows(sp, c);
-    const uint32_t r0 = rr.x, r1 = rr.y;
+    const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
     int ln = 0;
     if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
     else ln = (int)(r1 - r0);
@@ -609,7 +597,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
     for (int p = i + tid; p < j; p += nt)  // C^dir of this bin
       if (cnt[p] == 1) {
         const uint32_t c = (uint32_t)c0s[p];
-        const float d = centroid_dist(cluster_rec(sp, c), slog, b);
+        const float d = centroid_dist(sp.cent + (size_t)c * b, slog, b);
         const unsigned pos = atomicAdd(&st[1], 1u);
         dirk[pos] = ((uint64_t)__float_as_uint(d) << 32) | c;
       }
@@ -622,7 +610,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
         const int slot = x + t;
         const int p = last_le(nsoff, i, j, slot);
         const uint32_t c = (uint32_t)(c0s[p] + (slot - nsoff[p]));
-        const float d = centroid_dist(cluster_rec(sp, c), slog, b);
+        const float d = centroid_dist(sp.cent + (size_t)c * b, slog, b);
         Bk[t] = ((uint64_t)__float_as_uint(d) << 32) | c;
         atomicMin(&sred[0], __float_as_uint(d));
       }
@@ -709,8 +697,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
     const uint32_t c = (uint32_t)(takeA ? xa : xb);
     if (takeA) ++ia;
     else ++ib;
-    const uint2 rr = cluster_rows(sp, c);
-    const uint32_t r0 = rr.x, r1 = rr.y;
+    const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
     if (r1 < r0 || (int64_t)r1 > sp.N) set_err(sp.err, NR_DEV_BAD_CLUSTER);
     else lsum += (int)(r1 - r0);
   }
@@ -724,8 +711,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
     const uint32_t c = (uint32_t)(takeA ? xa : xb);
     if (takeA) ++ia;
     else ++ib;
-    const uint2 rr = cluster_rows(sp, c);
-    const uint32_t r0 = rr.x, r1 = rr.y;
+    const uint32_t r0 = __ldg(&sp.cl_off[c]), r1 = __ldg(&sp.cl_off[c + 1]);
     const int ln = (r1 < r0 || (int64_t)r1 > sp.N) ? 0 : (int)(r1 - r0);
     seg[o].row0 = r0;
     seg[o].pos = (uint32_t)spos;
