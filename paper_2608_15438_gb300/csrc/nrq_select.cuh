@@ -103,6 +103,11 @@ __device__ __forceinline__ float centroid_dist(const float *__restrict__ mu, con
 
 // Probe of candidate slot s: slots are numbered probe by probe, off[i] the
 // first slot of probe i (nondecreasing).
+// Requests the 128-byte line holding p into L2 (no register result).
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ int slot_probe(const int *off, int np, int s) {
   int lo = 0, hi = np - 1;
   while (lo < hi) {
@@ -233,26 +238,43 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   int *cnt = ibuf;        // [P] clusters per probe -> exclusive offsets
   int *c0s = ibuf + sp.P;  // [P] first cluster per probe
   const uint32_t nb = 1u << sp.b;
-  for (int i = tid; i < np; i += nt) {
-    const uint32_t u = codes[i];
-    int n = 0, c0 = 0;
-    if (u >= nb) {
-      set_err(sp.err, NR_DEV_BAD_CODE);
-    } else {
-      const uint32_t lo = __ldg(&sp.bkt_off[u]), hi = __ldg(&sp.bkt_off[u + 1]);
-      if (hi < lo || (int64_t)hi > sp.n_cl) {
+  // directory lookups four probes a thread at a time, all loads issued before
+  // any is used (they are independent random reads)
+  for (int i0 = tid; i0 < np; i0 += 4 * nt) {
+    uint32_t u[4], lo[4], hi[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int i = i0 + e * nt;
+      u[e] = i < np ? codes[i] : 0u;
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      lo[e] = hi[e] = 0u;
+      if (i0 + e * nt < np && u[e] < nb) {
+        lo[e] = __ldg(&sp.bkt_off[u[e]]);
+        hi[e] = __ldg(&sp.bkt_off[u[e] + 1]);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int i = i0 + e * nt;
+      if (i >= np) break;
+      int n = 0, c0 = 0;
+      if (u[e] >= nb) {
+        set_err(sp.err, NR_DEV_BAD_CODE);
+      } else if (hi[e] < lo[e] || (int64_t)hi[e] > sp.n_cl) {
         set_err(sp.err, NR_DEV_BAD_BUCKET);
       } else {
-        n = (int)(hi - lo);
-        c0 = (int)lo;
+        n = (int)(hi[e] - lo[e]);
+        c0 = (int)lo[e];
         if (n > sp.K_max) {
           set_err(sp.err, NR_DEV_TOO_MANY);
           n = sp.K_max;
         }
       }
+      cnt[i] = n;
+      c0s[i] = c0;
     }
-    cnt[i] = n;
-    c0s[i] = c0;
   }
   __syncthreads();
   int M = block_exclusive_scan(cnt, np, warp_sums);
@@ -266,10 +288,18 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   __syncthreads();
   const float m1 = sp.m1;
   const bool prefilter = !sp.gate_off && (sp.gate_n >= 2 || m1 >= 0.0f);
+  int pi = tid < M ? slot_probe(cnt, np, tid) : 0;
   for (int s = tid; s < M; s += nt) {
-    const int pi = slot_probe(cnt, np, s);
     const uint32_t c = (uint32_t)(c0s[pi] + (s - cnt[pi]));
     const bool single = (pi + 1 < np ? cnt[pi + 1] : M) - cnt[pi] == 1;  // C^dir
+    // the next slot's centroid is requested into L2 before this one is read
+    const int sn = s + nt;
+    if (sn < M) {
+      pi = slot_probe(cnt, np, sn);
+      const float *mn = sp.cent + (size_t)(uint32_t)(c0s[pi] + (sn - cnt[pi])) * sp.b;
+      prefetch_l2(mn);
+      prefetch_l2(mn + sp.b - 1);
+    }
     const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
     const uint64_t key = tagged_key(d, c, single);
     if (single) {
