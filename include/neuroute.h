@@ -125,7 +125,15 @@ typedef struct {
    * which leaves SM room to the overlapping stages. */
   int pipe_chunk;       /* >= 0; default 0 */
   int refine_ctas;      /* in [0, 32]; default 0 */
+  /* 1: probe_budget counts non-empty buckets: flip sets in key order whose
+   * buckets hold no cluster are skipped (not listed, not counted), the first
+   * probe_budget non-empty ones listed, at most NR_NONEMPTY_SCAN *
+   * probe_budget flip sets examined, the base code included. 0 (default):
+   * probe_budget counts codes, empty buckets included. */
+  int nonempty_budget;  /* 0 or 1; default 0 */
 } nr_params;
+
+#define NR_NONEMPTY_SCAN 4
 
 /* Per-search statistics (sums over the queries of the last search call). */
 typedef struct {

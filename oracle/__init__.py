@@ -25,7 +25,7 @@ class Params(ctypes.Structure):
                 ("b_min", ctypes.c_int), ("c_t_low", ctypes.c_int), ("c_u_min", ctypes.c_int),
                 ("c_f_min", ctypes.c_int), ("c_alpha_front", ctypes.c_float),
                 ("gate_n", ctypes.c_int), ("gate_x", ctypes.c_float * 16),
-                ("gate_y", ctypes.c_float * 16)]
+                ("gate_y", ctypes.c_float * 16), ("nonempty_budget", ctypes.c_int)]
 
 
 def lib():
@@ -66,6 +66,8 @@ def lib():
                                 vp, i32]
         L.or_search.restype = i32
         L.or_bruteforce.argtypes = [i32, i32, vp, i64, vp, i64, i32, vp, vp, i32]
+        L.or_probe_list_index.argtypes = [vp, vp, i32, ctypes.POINTER(Params), vp, vp]
+        L.or_probe_list_index.restype = i32
         L.or_centroid_dist.argtypes = [vp, vp, i64]
         L.or_centroid_dist.restype = ctypes.c_float
         L.or_gate_margin.argtypes = [ctypes.POINTER(Params), ctypes.c_float]
@@ -182,6 +184,16 @@ class Index:
         if n < 0:
             raise RuntimeError("oracle: out-of-range index in file")
         return L[:n].copy(), dL[:n].copy(), int(ndir[0]), int(nbat[0])
+
+    def probe_list(self, logit, P, p: Params):
+        """(codes, keys) of one query's probe list against this index (the
+        non-empty budget skips empty buckets)."""
+        logit = np.ascontiguousarray(logit, np.float32)
+        codes = np.empty(max(P, 1), np.uint32)
+        keys = np.empty(max(P, 1), np.uint64)
+        n = lib().or_probe_list_index(self.h, logit.ctypes.data, P, ctypes.byref(p), codes.ctypes.data,
+                                      keys.ctypes.data)
+        return codes[:n].copy(), keys[:n].copy()
 
     def centroid_dist(self, logit, c: int) -> np.float32:
         """Distance of cluster c's centroid from the logits (the centroid

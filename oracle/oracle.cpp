@@ -52,6 +52,7 @@ extern "C" void or_params_default(or_params *p) {
   p->c_alpha_front = 0.5f;
   p->gate_n = 0;
   for (int i = 0; i < 16; ++i) p->gate_x[i] = p->gate_y[i] = 0.0f;
+  p->nonempty_budget = 0;
 }
 
 // The gate margin M(x) (Sec. 3.4): m0 + m1 x, or the calibrated monotone
@@ -339,6 +340,28 @@ extern "C" int or_probe_list(int b, const float *logit, const float *tau, int P,
   return n;
 }
 
+// The probe list against the index: with the non-empty budget, the first P
+// codes in key order whose buckets hold a cluster, among the first
+// OR_NONEMPTY_SCAN * P flip sets (plain reading of the D3 variant: empty
+// buckets are enumerated but not spent).
+extern "C" int or_probe_list_index(const or_index *ix, const float *logit, int P, const or_params *p,
+                                   uint32_t *codes, uint64_t *keys) {
+  if (!p->nonempty_budget)
+    return or_probe_list(ix->b, logit, ix->tau.data(), P, p, codes, keys, nullptr);
+  const int scan = OR_NONEMPTY_SCAN * P;
+  std::vector<uint32_t> c((size_t)scan);
+  std::vector<uint64_t> k((size_t)scan);
+  const int m = or_probe_list(ix->b, logit, ix->tau.data(), scan, p, c.data(), k.data(), nullptr);
+  int n = 0;
+  for (int i = 0; i < m && n < P; ++i) {
+    if (ix->bkt_off[(size_t)c[i] + 1] == ix->bkt_off[c[i]]) continue;  // empty bucket
+    codes[n] = c[i];
+    if (keys) keys[n] = k[i];
+    ++n;
+  }
+  return n;
+}
+
 // ---------------------------------------------------------------- centroid stage
 // Sec. 3.4.2 / Algorithm 2: buckets holding one cluster go straight to C^dir;
 // the other buckets' centroids are scored by squared L2 in logit space, gated
@@ -619,7 +642,7 @@ extern "C" int or_search(const or_index *ix, const void *queries, const float *l
       encode_one(ix, queries, qi, lg.data());
     std::vector<uint32_t> codes((size_t)P);
     std::vector<uint64_t> keys((size_t)P);
-    int np = or_probe_list(b, lg.data(), ix->tau.data(), P, p, codes.data(), keys.data(), nullptr);
+    int np = or_probe_list_index(ix, lg.data(), P, p, codes.data(), keys.data());
     std::vector<int32_t> L((size_t)np + (size_t)C);
     int nl;
     if (p->cent_mode == 1) {

@@ -72,7 +72,14 @@ typedef struct {
    * flat beyond its ends, instead of gate_m0 + gate_m1 x */
   int gate_n;
   float gate_x[16], gate_y[16];
+  /* 1: the probe budget counts non-empty buckets (the D3 variant): flip sets
+   * in key order whose buckets hold no cluster are skipped, the first P
+   * non-empty ones listed, at most OR_NONEMPTY_SCAN * P flip sets examined
+   * (the base code included). 0 (default): P counts codes. */
+  int nonempty_budget;
 } or_params;
+
+#define OR_NONEMPTY_SCAN 4
 
 void or_params_default(or_params *p);
 
@@ -109,6 +116,11 @@ int or_probe_order_allsubsets(int b, const float *sd, int P, const or_params *p,
  * keys (optional) as above; perm (optional) [b] = bit index of each rank. */
 int or_probe_list(int b, const float *logit, const float *tau, int P, const or_params *p,
                   uint32_t *codes, uint64_t *keys, int32_t *perm);
+
+/* The probe list of one query under p, against the index (for the
+ * non-empty budget): codes [P], keys [P] (optional). Returns its length. */
+int or_probe_list_index(const or_index *ix, const float *logit, int P, const or_params *p,
+                        uint32_t *codes, uint64_t *keys);
 
 /* Ordered cluster list L = C^dir U C^cent of one query. L has room for
  * nprobe + C entries; dL (optional) gets each entry's centroid distance.

@@ -115,6 +115,7 @@ nr_status check_params(const nr_params *p) {
       !(p->c_alpha_front >= 0.0f && p->c_alpha_front <= 1.0f))
     return NR_ERR_INVALID_ARG;
   if (p->pipe_chunk < 0 || p->refine_ctas < 0 || p->refine_ctas > 32) return NR_ERR_INVALID_ARG;
+  if (p->nonempty_budget != 0 && p->nonempty_budget != 1) return NR_ERR_INVALID_ARG;
   if (p->gate_n != 0) {
     if (p->gate_n < 2 || p->gate_n > 16) return NR_ERR_INVALID_ARG;
     for (int i = 0; i < p->gate_n; ++i) {
@@ -255,6 +256,7 @@ nr_status nr_params_default(nr_params *p) {
   for (int i = 0; i < 16; ++i) p->gate_x[i] = p->gate_y[i] = 0.0f;
   p->pipe_chunk = 0;
   p->refine_ctas = 0;
+  p->nonempty_budget = 0;
   return NR_OK;
 }
 

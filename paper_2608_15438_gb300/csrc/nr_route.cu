@@ -16,7 +16,7 @@ __global__ void route_kernel(nrq::RouteParams rp, const float *__restrict__ logi
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, wpb = blockDim.x >> 5;
   const int64_t q = (int64_t)blockIdx.x * wpb + warp;
   if (q >= nq) return;  // uniform per warp
-  unsigned char *heap = smem + (size_t)warp * nrq::route_heap_bytes(rp.P);
+  unsigned char *heap = smem + (size_t)warp * nrq::route_heap_bytes(rp.Q);
   uint32_t *out = codes + (size_t)q * rp.P;
   const int n = nrq::route_warp(rp, logits + q * rp.b, heap, out);
   for (int t = n + lane; t < rp.P; t += 32) out[t] = 0xffffffffu;
@@ -60,16 +60,19 @@ nrq::RouteParams nr_route_params(const nr_index *ix, int P) {
   rp.rmax = p.r_max;
   rp.smax = p.s_max;
   rp.P = P;
+  rp.bkt_off = ix->bkt_off;
+  rp.nonempty = p.nonempty_budget;
+  rp.Q = p.nonempty_budget ? NR_NONEMPTY_SCAN * P : P;
   return rp;
 }
 
-size_t nr_route_heap_bytes(int P) { return nrq::route_heap_bytes(P); }
+size_t nr_route_heap_bytes(int Q) { return nrq::route_heap_bytes(Q); }
 
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
   const nrq::RouteParams rpb = nr_route_params(ix, P);  // before the launch configuration
-  if (ix->params.r_max <= 0) {  // the threshold enumeration (P <= 1024)
+  if (ix->params.r_max <= 0 && !ix->params.nonempty_budget) {  // threshold enumeration (P <= 1024)
     cudaError_t e = cudaSuccess;
     bool done = true;
     switch (nrq::route_block_e(P)) {
@@ -85,7 +88,7 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
       return e;
     }
   }
-  const size_t per_warp = nr_route_heap_bytes(P);
+  const size_t per_warp = nr_route_heap_bytes(rpb.Q);
   // warps per block: the choice that packs the most warps into an SM's
   // shared memory (the heap is the limit at large probe budgets)
   const size_t sm_bytes = (size_t)227 * 1024;

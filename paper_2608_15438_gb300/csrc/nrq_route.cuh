@@ -31,12 +31,16 @@ struct RouteParams {
   int b, bsel, rmax;
   float smax;
   int P;
+  // non-empty budget: bucket directory, and Q = the most flip sets examined
+  // (NR_NONEMPTY_SCAN P); without it Q = P and bkt_off is unused
+  const uint32_t *bkt_off;
+  int nonempty, Q;
 };
 
-// Bytes of shared memory route_warp needs for probe budget P.
-// heap keys [(P + 2) x 8 B], deviations by rank [32 x 4 B], and the table of
+// Bytes of shared memory route_warp needs to examine at most Q flip sets:
+// heap keys [(Q + 2) x 8 B], deviations by rank [32 x 4 B], and the table of
 // left-to-right sums over subsets of ranks 0..7 [256 x 4 B]
-__host__ __device__ inline size_t route_heap_bytes(int P) { return (size_t)(P + 2) * 8 + 128 + 1024; }
+__host__ __device__ inline size_t route_heap_bytes(int Q) { return (size_t)(Q + 2) * 8 + 128 + 1024; }
 
 // Writes codes[0..n) (any address space) and returns n, uniform in the warp.
 // Must be called by a whole warp. heap: route_heap_bytes(P) bytes of shared
@@ -46,7 +50,7 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
   const int lane = threadIdx.x & 31;
   const int b = rp.b;
   uint64_t *hkey = reinterpret_cast<uint64_t *>(heap);
-  float *ssd = reinterpret_cast<float *>(heap + (size_t)(rp.P + 2) * 8);
+  float *ssd = reinterpret_cast<float *>(heap + (size_t)(rp.Q + 2) * 8);
   float dj = __int_as_float(0x7f800000);
   bool bit = false;
   if (lane < b) {
@@ -80,22 +84,36 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
     for (int t = lane; t < (1 << j); t += 32) psum[(1 << j) + t] = __fadd_rn(psum[t], sj);
     __syncwarp();
   }
-  if (lane == 0) codes[0] = u0;
-  int n = 1, hs = 0;
+  // with the non-empty budget a code is listed only when its bucket holds a
+  // cluster; every examined flip set counts toward Q
+  auto listed = [&](uint32_t code) {
+    if (!rp.nonempty) return true;
+    uint32_t occ = 0;
+    if (lane == 0) occ = __ldg(&rp.bkt_off[code + 1]) - __ldg(&rp.bkt_off[code]);
+    return __shfl_sync(kFull, occ, 0) != 0u;
+  };
+  int n = 0, seen = 1, hs = 0;
+  if (listed(u0)) {
+    if (lane == 0) codes[0] = u0;
+    n = 1;
+  }
   if (rp.P > 1 && rp.bsel >= 1 && ssd[0] <= rp.smax) {
     if (lane == 0) hkey[0] = pack_key(ssd[0], 1u, 1u);
     hs = 1;
   }
   __syncwarp();
-  while (n < rp.P && hs > 0) {
+  while (n < rp.P && hs > 0 && seen < rp.Q) {
     const uint64_t top = hkey[0];
     const uint32_t rmask = (uint32_t)top & 0xffffffu;
     const uint32_t size = ((uint32_t)top >> 24) & 0xffu;
     const float cost = __uint_as_float((uint32_t)(top >> 32));
     // ApplyFlips: code = u0 XOR (bits of the ranks in F)
     const uint32_t flips = __reduce_or_sync(kFull, ((rmask >> lane) & 1u) ? rbit : 0u);
-    if (lane == 0) codes[n] = u0 ^ flips;
-    ++n;
+    ++seen;
+    if (listed(u0 ^ flips)) {
+      if (lane == 0) codes[n] = u0 ^ flips;
+      ++n;
+    }
     const int m = 31 - __clz((int)rmask);
     bool v1 = false, v2 = false;
     uint64_t k1 = kEmpty, k2 = kEmpty;
@@ -210,7 +228,7 @@ struct RouteSmem {
 
 __host__ __device__ inline size_t route_region_bytes(int E, int P) {
   const size_t sort = (size_t)(E * kRouteThreads + (E * kRouteThreads) / 16) * 8;
-  const size_t heap = route_heap_bytes(P);
+  const size_t heap = route_heap_bytes(P);  // route_warp with Q = P
   return ((sort > heap ? sort : heap) + 15) & ~(size_t)15;
 }
 

@@ -111,6 +111,48 @@ def test_route_threshold_filters_bit_exact(tiny, torch, kw, P):
         assert np.array_equal(codes[i, : len(exp)], exp), i
 
 
+@pytest.mark.parametrize("P", [1, 8, 100, 1024, 4096])
+@pytest.mark.parametrize("kw", [dict(), dict(s_max=0.3), dict(l_sel=9, r_max=3)])
+def test_route_nonempty_budget_bit_exact(tiny, torch, P, kw):
+    """The non-empty budget (D3 variant) skips empty buckets without spending
+    the budget, examining at most 4 P flip sets (the tiny index has many
+    empty buckets)."""
+    ix, orc = tiny["ix"], tiny["orc"]
+    ix.set_params(nonempty_budget=1, **kw)
+    try:
+        codes, nprobe = ix.route(tiny["dl"][:100], P)
+    finally:
+        ix.set_params()
+    codes = codes.cpu().numpy().view(np.uint32)
+    nprobe = nprobe.cpu().numpy()
+    p = oracle.params(nonempty_budget=1, **kw)
+    bkt = orc.bkt_off()
+    for i in range(100):
+        exp, _ = orc.probe_list(tiny["lg"][i], P, p)
+        assert nprobe[i] == len(exp), i
+        assert np.array_equal(codes[i, : len(exp)], exp), i
+        assert np.all(codes[i, len(exp):] == 0xFFFFFFFF)
+        assert np.all(bkt[exp.astype(np.int64) + 1] > bkt[exp])
+
+
+@pytest.mark.parametrize("kw", [dict(t_low=4), dict(t_low=0, gate_m0=0.0, gate_m1=2.0),
+                                dict(t_low=4, cent_mode=1, n_bins=4, s_max=1.0, c_t_low=2)])
+def test_search_nonempty_budget_bit_exact(tiny, torch, kw):
+    ix, orc = tiny["ix"], tiny["orc"]
+    ix.set_params(nonempty_budget=1, **kw)
+    try:
+        ids, d = ix.search_logits(tiny["dq"], tiny["dl"], 10, 64, 128)
+        st = ix.query_stats(len(tiny["q"]))
+        torch.cuda.synchronize()
+    finally:
+        ix.set_params()
+    ids_o, d_o, st_o = orc.search(tiny["q"], 10, 64, 128, oracle.params(nonempty_budget=1, **kw),
+                                  logits=tiny["lg"])
+    assert np.array_equal(ids.cpu().numpy(), ids_o)
+    assert np.array_equal(d.cpu().numpy(), d_o)
+    assert np.array_equal(st.cpu().numpy(), st_o)
+
+
 def test_route_b4_hand_order(torch, tmp_path):
     from paper_2608_15438_gb300 import neuroute as nr
 
