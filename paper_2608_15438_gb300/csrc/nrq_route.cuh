@@ -97,7 +97,7 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
     if (lane == 0) codes[0] = u0;
     n = 1;
   }
-  if (rp.P > 1 && rp.bsel >= 1 && ssd[0] <= rp.smax) {
+  if (rp.Q > 1 && rp.bsel >= 1 && ssd[0] <= rp.smax) {  // Q > 1: a flip set may be examined
     if (lane == 0) hkey[0] = pack_key(ssd[0], 1u, 1u);
     hs = 1;
   }
