@@ -49,6 +49,11 @@ def lib():
         L.or_encode_weights.argtypes = [i32, i32, i32, i32, ctypes.c_float, vp, vp, vp, vp, vp, i64,
                                         vp, i32]
         L.or_encode_weights.restype = None
+        L.or_encode_mlp.argtypes = [i32, i32, i32, i32, i32, vp, ctypes.c_float, vp, vp, vp, vp, vp,
+                                    vp, i64, vp, i32]
+        L.or_encode_mlp.restype = None
+        L.or_index_mid.argtypes = [vp, vp]
+        L.or_index_mid.restype = i32
         L.or_probe_order.argtypes = [i32, vp, i32, ctypes.POINTER(Params), vp]
         L.or_probe_order.restype = i32
         L.or_probe_order_allsubsets.argtypes = [i32, vp, i32, ctypes.POINTER(Params), vp]
@@ -116,6 +121,8 @@ class Index:
         lib().or_index_info(h, info.ctypes.data)
         (self.N, self.D, self.H, self.b, self.n_clusters, self.dtype_code, self.k_max,
          self.t) = (int(v) for v in info)
+        w = np.zeros(8, np.int32)
+        self.mid = tuple(int(v) for v in w[: lib().or_index_mid(h, w.ctypes.data)])
 
     def close(self):
         if self.h:
@@ -216,16 +223,31 @@ class Index:
         return ids, d, st
 
 
+def mid_layers(weights):
+    """The hidden layers after the first of an encoder given as (W1, b1, W2,
+    b2) or (W1, b1, W2, b2, ((W, b), ...)): (widths, the concatenated W then b
+    of each layer as the file stores them)."""
+    mid = weights[4] if len(weights) > 4 else ()
+    widths = [int(np.asarray(W).shape[0]) for W, _ in mid]
+    flat = [np.concatenate([np.asarray(W, np.float32).ravel(), np.asarray(bb, np.float32).ravel()])
+            for W, bb in mid]
+    return widths, (np.concatenate(flat) if flat else np.zeros(0, np.float32))
+
+
 def encode_weights(weights, in_scale: float, x: np.ndarray, nthreads=None) -> np.ndarray:
-    """Logits of rows x under the encoder (W1, b1, W2, b2), without an index."""
-    W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights)
+    """Logits of rows x under the encoder (W1, b1, W2, b2[, middle layers]),
+    without an index."""
+    W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights[:4])
+    widths, Wm = mid_layers(weights)
     x = np.ascontiguousarray(x)
     H, D = W1.shape
     b = W2.shape[0]
     out = np.empty((x.shape[0], b), np.float32)
-    lib().or_encode_weights(0 if x.dtype == np.uint8 else 1, D, H, b, in_scale, W1.ctypes.data,
-                            b1.ctypes.data, W2.ctypes.data, b2.ctypes.data, x.ctypes.data,
-                            x.shape[0], out.ctypes.data, nthreads or nthreads_default())
+    w = (ctypes.c_int * max(1, len(widths)))(*widths)
+    lib().or_encode_mlp(0 if x.dtype == np.uint8 else 1, D, H, b, len(widths), w, in_scale,
+                        W1.ctypes.data, b1.ctypes.data, W2.ctypes.data, b2.ctypes.data,
+                        Wm.ctypes.data, x.ctypes.data, x.shape[0], out.ctypes.data,
+                        nthreads or nthreads_default())
     return out
 
 

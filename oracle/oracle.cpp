@@ -24,6 +24,11 @@ struct or_index {
   int64_t n_cl = 0;
   float in_scale = 1.0f;
   std::vector<float> W1, b1, W2, b2, tau, cent;
+  // hidden layers after the first (file version 2): widths, and per layer
+  // W [width x previous width] then its bias, concatenated as in the file
+  int n_mid = 0;
+  std::vector<int> mid_w;
+  std::vector<float> Wm;
   std::vector<uint32_t> bkt_off, cl_off, ids;
   std::vector<uint8_t> vec;  // N * D * elem bytes
 };
@@ -109,7 +114,8 @@ extern "C" or_index *or_index_load(const char *path, char *err, int errlen) {
     fclose(f);
     return fail("truncated header");
   }
-  if (memcmp(h, "NRIXv001", 8) != 0 || rd32(h, 8) != 1) {
+  const uint32_t version = rd32(h, 8);
+  if (memcmp(h, "NRIXv001", 8) != 0 || (version != 1 && version != 2)) {
     fclose(f);
     return fail("bad magic or version");
   }
@@ -125,16 +131,29 @@ extern "C" or_index *or_index_load(const char *path, char *err, int errlen) {
   memcpy(&ix->in_scale, h + 56, 4);
   uint64_t off[10];
   for (int i = 0; i < 10; ++i) off[i] = rd64(h, 64 + 8 * i);
-  if (ix->dtype < 0 || ix->dtype > 1 || ix->b < 1 || ix->b > 24 || ix->D < 1 || ix->H < 1) {
+  ix->n_mid = version == 2 ? (int)rd32(h, 152) : 0;
+  bool widths_ok = ix->n_mid >= 0 && ix->n_mid <= 7;
+  for (int i = 0; widths_ok && i < ix->n_mid; ++i) {
+    ix->mid_w.push_back((int)rd32(h, 156 + 4 * i));
+    widths_ok = ix->mid_w.back() >= 1;
+  }
+  const uint64_t mid_off = rd64(h, 192);
+  if (ix->dtype < 0 || ix->dtype > 1 || ix->b < 1 || ix->b > 24 || ix->D < 1 || ix->H < 1 ||
+      !widths_ok) {
     fclose(f);
     delete ix;
     return fail("bad header fields");
   }
+  const int h_last = ix->n_mid > 0 ? ix->mid_w.back() : ix->H;
+  size_t mid_n = 0;
+  for (int i = 0, prev = ix->H; i < ix->n_mid; prev = ix->mid_w[i], ++i)
+    mid_n += (size_t)ix->mid_w[i] * prev + ix->mid_w[i];
   size_t esz = ix->dtype == 0 ? 1 : 4;
   size_t nb = ((size_t)1 << ix->b) + 1;
   bool ok = read_section(f, off[0], (size_t)ix->H * ix->D, ix->W1) &&
             read_section(f, off[1], (size_t)ix->H, ix->b1) &&
-            read_section(f, off[2], (size_t)ix->b * ix->H, ix->W2) &&
+            read_section(f, off[2], (size_t)ix->b * h_last, ix->W2) &&
+            (ix->n_mid == 0 || read_section(f, mid_off, mid_n, ix->Wm)) &&
             read_section(f, off[3], (size_t)ix->b, ix->b2) &&
             read_section(f, off[4], (size_t)ix->b, ix->tau) &&
             read_section(f, off[5], nb, ix->bkt_off) &&
@@ -151,6 +170,11 @@ extern "C" or_index *or_index_load(const char *path, char *err, int errlen) {
 }
 
 extern "C" void or_index_free(or_index *ix) { delete ix; }
+
+extern "C" int or_index_mid(const or_index *ix, int32_t *widths) {
+  for (int i = 0; i < ix->n_mid; ++i) widths[i] = ix->mid_w[i];
+  return ix->n_mid;
+}
 
 extern "C" void or_index_info(const or_index *ix, int64_t *info) {
   info[0] = ix->N;
@@ -188,8 +212,11 @@ static void parallel_for(int64_t n, int nthreads, const std::function<void(int64
 }
 
 // ---------------------------------------------------------------- encoder
-// Sec. 3.2.1: l = E(x). One hidden layer: h = max(0, W1 (s x) + b1),
-// l = W2 h + b2, in double, rounded to fp32 at the end.
+// Sec. 3.2.1 and the encoder table of the appendix: l = E(x), an MLP whose
+// hidden layers are linear then ReLU (BatchNorm folded into the linear map)
+// and whose last layer is linear: h_1 = max(0, W1 (s x) + b1), h_i =
+// max(0, W_i h_{i-1} + b_i), l = W2 h_L + b2, in double, rounded to fp32 at
+// the end.
 static void encode_one(const or_index *ix, const void *x, int64_t i, float *out) {
   const int D = ix->D, H = ix->H, b = ix->b;
   std::vector<double> xin(D), h(H);
@@ -203,10 +230,24 @@ static void encode_one(const or_index *ix, const void *x, int64_t i, float *out)
     for (int j = 0; j < D; ++j) acc += (double)ix->W1[(size_t)u * D + j] * xin[j];
     h[u] = acc > 0.0 ? acc : 0.0;
   }
-  for (int o = 0; o < b; ++o) {
-    double acc = (double)ix->b2[o];
-    for (int u = 0; u < H; ++u) acc += (double)ix->W2[(size_t)o * H + u] * h[u];
-    out[o] = (float)acc;
+  size_t o = 0;  // walks the middle layers' weights and biases
+  for (int l = 0; l < ix->n_mid; ++l) {
+    const int prev = (int)h.size(), w = ix->mid_w[l];
+    std::vector<double> g(w);
+    const float *W = ix->Wm.data() + o, *bias = W + (size_t)w * prev;
+    for (int u = 0; u < w; ++u) {
+      double acc = (double)bias[u];
+      for (int j = 0; j < prev; ++j) acc += (double)W[(size_t)u * prev + j] * h[j];
+      g[u] = acc > 0.0 ? acc : 0.0;
+    }
+    o += (size_t)w * prev + w;
+    h.swap(g);
+  }
+  const int hl = (int)h.size();
+  for (int q = 0; q < b; ++q) {
+    double acc = (double)ix->b2[q];
+    for (int u = 0; u < hl; ++u) acc += (double)ix->W2[(size_t)q * hl + u] * h[u];
+    out[q] = (float)acc;
   }
 }
 
@@ -214,20 +255,36 @@ extern "C" void or_encode(const or_index *ix, const void *x, int64_t nq, float *
   parallel_for(nq, nthreads, [&](int64_t i) { encode_one(ix, x, i, logits + (size_t)i * ix->b); });
 }
 
-extern "C" void or_encode_weights(int dtype, int D, int H, int b, float in_scale, const float *W1,
-                                  const float *b1, const float *W2, const float *b2, const void *x,
-                                  int64_t nq, float *logits, int nthreads) {
+extern "C" void or_encode_mlp(int dtype, int D, int H, int b, int n_mid, const int *mid_w,
+                              float in_scale, const float *W1, const float *b1, const float *W2,
+                              const float *b2, const float *Wm, const void *x, int64_t nq,
+                              float *logits, int nthreads) {
   or_index e;  // an index holding only the encoder
   e.dtype = dtype;
   e.D = D;
   e.H = H;
   e.b = b;
   e.in_scale = in_scale;
+  e.n_mid = n_mid;
+  size_t mid_n = 0;
+  for (int i = 0, prev = H; i < n_mid; prev = mid_w[i], ++i) {
+    e.mid_w.push_back(mid_w[i]);
+    mid_n += (size_t)mid_w[i] * prev + mid_w[i];
+  }
+  const int hl = n_mid > 0 ? mid_w[n_mid - 1] : H;
   e.W1.assign(W1, W1 + (size_t)H * D);
   e.b1.assign(b1, b1 + H);
-  e.W2.assign(W2, W2 + (size_t)b * H);
+  e.W2.assign(W2, W2 + (size_t)b * hl);
   e.b2.assign(b2, b2 + b);
+  if (n_mid > 0) e.Wm.assign(Wm, Wm + mid_n);
   or_encode(&e, x, nq, logits, nthreads);
+}
+
+extern "C" void or_encode_weights(int dtype, int D, int H, int b, float in_scale, const float *W1,
+                                  const float *b1, const float *W2, const float *b2, const void *x,
+                                  int64_t nq, float *logits, int nthreads) {
+  or_encode_mlp(dtype, D, H, b, 0, nullptr, in_scale, W1, b1, W2, b2, nullptr, x, nq, logits,
+                nthreads);
 }
 
 // ---------------------------------------------------------------- probe order

@@ -97,6 +97,17 @@ const float *or_index_cent(const or_index *ix);
 
 /* logits [nq x b] (fp32, rounded from a double-precision forward pass) */
 void or_encode(const or_index *ix, const void *x, int64_t nq, float *logits, int nthreads);
+
+/* Widths of the hidden layers after the first (widths[0..n_mid), at most 7);
+ * returns n_mid. */
+int or_index_mid(const or_index *ix, int32_t *widths);
+
+/* Logits of rows x under an encoder given by its weights: W1 [H x D], b1 [H],
+ * then n_mid hidden layers of widths mid_w (Wm: per layer W [w x previous]
+ * followed by its bias [w], concatenated), W2 [b x last hidden width], b2 [b]. */
+void or_encode_mlp(int dtype, int D, int H, int b, int n_mid, const int *mid_w, float in_scale,
+                   const float *W1, const float *b1, const float *W2, const float *b2,
+                   const float *Wm, const void *x, int64_t nq, float *logits, int nthreads);
 /* the same forward pass from explicit weights W1 [H x D], b1 [H], W2 [b x H],
  * b2 [b] (dtype 0 uint8 rows, 1 fp32 rows; inputs scaled by in_scale) */
 void or_encode_weights(int dtype, int D, int H, int b, float in_scale, const float *W1,

@@ -35,6 +35,8 @@ typedef struct {
   int lloyd_iters;  // Lloyd passes on the whole bucket
   int sample_per_cluster;  // k-means++ sample size per cluster
   uint64_t seed;    // k-means seed
+  int n_mid;        // hidden layers after the first (0..7)
+  int mid_w[7];     // their widths; the last layer maps the last hidden width to b
 } nrb_config;
 }
 
@@ -65,12 +67,22 @@ uint64_t splitmix64(uint64_t &s) {
   return z ^ (z >> 31);
 }
 
+// Widths of the hidden layers: H, then the middle layers'.
+int hidden_last(const nrb_config &c) { return c.n_mid > 0 ? c.mid_w[c.n_mid - 1] : c.H; }
+size_t mid_floats(const nrb_config &c) {
+  size_t n = 0;
+  for (int i = 0, prev = c.H; i < c.n_mid; prev = c.mid_w[i], ++i) n += (size_t)c.mid_w[i] * prev + c.mid_w[i];
+  return n;
+}
+
 // Encoder forward over rows [r0, r0 + n): blocks of 16 rows so the inner loop
-// runs over independent accumulators.
+// runs over independent accumulators. Hidden layers linear then ReLU, the
+// last linear; Wm holds each middle layer's W [w x previous] then its bias.
 void encode_block(const nrb_config &c, const void *x, int64_t r0, int n, const float *W1,
-                  const float *b1, const float *W2, const float *b2, float *out) {
+                  const float *b1, const float *W2, const float *b2, const float *Wm, float *out) {
   constexpr int BR = 16;
-  const int D = c.D, H = c.H, B = c.b;
+  const int D = c.D, B = c.b;
+  int H = c.H;
   std::vector<float> xt((size_t)D * BR, 0.0f), h((size_t)H * BR, 0.0f);
   for (int r = 0; r < n; ++r)
     for (int j = 0; j < D; ++j) {
@@ -88,6 +100,26 @@ void encode_block(const nrb_config &c, const void *x, int64_t r0, int n, const f
       for (int r = 0; r < BR; ++r) acc[r] += wj * xr[r];
     }
     for (int r = 0; r < BR; ++r) h[(size_t)u * BR + r] = acc[r] > 0.0f ? acc[r] : 0.0f;
+  }
+  const float *wl = Wm;
+  for (int l = 0; l < c.n_mid; ++l) {
+    const int w = c.mid_w[l];
+    const float *bias = wl + (size_t)w * H;
+    std::vector<float> g((size_t)w * BR, 0.0f);
+    for (int u = 0; u < w; ++u) {
+      float acc[BR];
+      for (int r = 0; r < BR; ++r) acc[r] = bias[u];
+      const float *wr = wl + (size_t)u * H;
+      for (int j = 0; j < H; ++j) {
+        const float wj = wr[j];
+        const float *hr = &h[(size_t)j * BR];
+        for (int r = 0; r < BR; ++r) acc[r] += wj * hr[r];
+      }
+      for (int r = 0; r < BR; ++r) g[(size_t)u * BR + r] = acc[r] > 0.0f ? acc[r] : 0.0f;
+    }
+    wl = bias + w;
+    h.swap(g);
+    H = w;
   }
   for (int o = 0; o < B; ++o) {
     float acc[BR];
@@ -285,13 +317,13 @@ extern "C" {
 
 // Encode n rows with the builder's encoder (fp32). out: [n x b].
 int nrb_encode(const nrb_config *c, const void *x, int64_t n, const float *W1, const float *b1,
-               const float *W2, const float *b2, float *out, int nthreads) {
-  if (!c || !x || !out || n < 0) return -1;
+               const float *W2, const float *b2, const float *Wm, float *out, int nthreads) {
+  if (!c || !x || !out || n < 0 || c->n_mid < 0 || c->n_mid > 7 || (c->n_mid > 0 && !Wm)) return -1;
   const int64_t nblk = (n + 15) / 16;
   parallel_for(nblk, nthreads, [&](int64_t blk) {
     int64_t r0 = blk * 16;
     int cnt = (int)std::min<int64_t>(16, n - r0);
-    encode_block(*c, x, r0, cnt, W1, b1, W2, b2, out + (size_t)r0 * c->b);
+    encode_block(*c, x, r0, cnt, W1, b1, W2, b2, Wm, out + (size_t)r0 * c->b);
   });
   return 0;
 }
@@ -301,11 +333,14 @@ int nrb_encode(const nrb_config *c, const void *x, int64_t n, const float *W1, c
 // logits), -2 I/O error.
 int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float *logits_in,
                      const float *W1, const float *b1, const float *W2, const float *b2,
-                     const char *path, int nthreads, int64_t *info_out) {
+                     const float *Wm, const char *path, int nthreads, int64_t *info_out) {
   if (!c || !x || !logits_in || !path || N < 1 || N >= (int64_t)0xFFFFFFFFll || c->b < 1 ||
       c->b > 24 || c->D < 1 || c->H < 1 || c->K_max < 1 || c->K_max > 64 || c->t < 1 ||
-      c->sample_per_cluster < 1 || (c->dtype != 0 && c->dtype != 1))
+      c->sample_per_cluster < 1 || (c->dtype != 0 && c->dtype != 1) || c->n_mid < 0 ||
+      c->n_mid > 7 || (c->n_mid > 0 && !Wm))
     return -1;
+  for (int i = 0; i < c->n_mid; ++i)
+    if (c->mid_w[i] < 1) return -1;
   const int b = c->b, D = c->D;
   const size_t esz = c->dtype == 0 ? 1 : 4;
   const float *logits = logits_in;
@@ -414,7 +449,8 @@ int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float 
   FILE *f = fopen(path, "wb");
   if (!f) return -2;
   auto align = [](uint64_t v) { return (v + 255) & ~(uint64_t)255; };
-  uint64_t sz[10] = {(uint64_t)c->H * D * 4,  (uint64_t)c->H * 4, (uint64_t)b * c->H * 4,
+  const int hl = hidden_last(*c);
+  uint64_t sz[10] = {(uint64_t)c->H * D * 4,  (uint64_t)c->H * 4, (uint64_t)b * hl * 4,
                      (uint64_t)b * 4,         (uint64_t)b * 4,    (uint64_t)(nb + 1) * 4,
                      (uint64_t)(n_cl + 1) * 4, (uint64_t)n_cl * b * 4, (uint64_t)N * 4,
                      (uint64_t)N * D * esz};
@@ -424,12 +460,15 @@ int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float 
     off[i] = cur;
     cur = align(cur + sz[i]);
   }
+  // the middle hidden layers (version 2): one more section after the vectors
+  const uint64_t mid_sz = (uint64_t)mid_floats(*c) * 4, mid_off = c->n_mid > 0 ? cur : 0;
+  if (c->n_mid > 0) cur = align(cur + mid_sz);
   unsigned char h[256];
   memset(h, 0, sizeof(h));
   memcpy(h, "NRIXv001", 8);
   uint32_t u32;
   uint64_t u64;
-  u32 = 1; memcpy(h + 8, &u32, 4);
+  u32 = c->n_mid > 0 ? 2 : 1; memcpy(h + 8, &u32, 4);
   u32 = (uint32_t)c->dtype; memcpy(h + 12, &u32, 4);
   u64 = (uint64_t)N; memcpy(h + 16, &u64, 8);
   u32 = (uint32_t)D; memcpy(h + 24, &u32, 4);
@@ -441,6 +480,14 @@ int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float 
   memcpy(h + 56, &c->in_scale, 4);
   for (int i = 0; i < 10; ++i) memcpy(h + 64 + 8 * i, &off[i], 8);
   memcpy(h + 144, &cur, 8);
+  if (c->n_mid > 0) {
+    u32 = (uint32_t)c->n_mid; memcpy(h + 152, &u32, 4);
+    for (int i = 0; i < c->n_mid; ++i) {
+      u32 = (uint32_t)c->mid_w[i];
+      memcpy(h + 156 + 4 * i, &u32, 4);
+    }
+    memcpy(h + 192, &mid_off, 8);
+  }
   bool ok = write_all(f, h, 256);
   const void *secs[9] = {W1, b1, W2, b2, tau.data(), bkt_off.data(), cl_off.data(), cent.data(), ids.data()};
   static const unsigned char zeros[256] = {0};
@@ -465,6 +512,11 @@ int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float 
     }
     at += sz[i];
   }
+  if (c->n_mid > 0) {
+    ok = ok && write_all(f, zeros, (size_t)(mid_off - at));
+    ok = ok && write_all(f, Wm, (size_t)mid_sz);
+    at = mid_off + mid_sz;
+  }
   ok = ok && write_all(f, zeros, (size_t)(cur - at));
   ok = (fclose(f) == 0) && ok;
   if (!ok) return -2;
@@ -487,7 +539,8 @@ int nrb_build_logits(const nrb_config *c, const void *x, int64_t N, const float 
 // Build the index over base x [N x D] with the builder's fp32 encoder and
 // write it to path (nrb_build_logits on the encoded base).
 int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, const float *b1,
-              const float *W2, const float *b2, const char *path, int nthreads, int64_t *info_out) {
+              const float *W2, const float *b2, const float *Wm, const char *path, int nthreads,
+              int64_t *info_out) {
   if (!c || !x || N < 1 || N >= (int64_t)0xFFFFFFFFll || c->b < 1 || c->b > 24) return -1;
   std::vector<float> logits;
   try {
@@ -495,8 +548,8 @@ int nrb_build(const nrb_config *c, const void *x, int64_t N, const float *W1, co
   } catch (...) {
     return -1;
   }
-  nrb_encode(c, x, N, W1, b1, W2, b2, logits.data(), nthreads);
-  return nrb_build_logits(c, x, N, logits.data(), W1, b1, W2, b2, path, nthreads, info_out);
+  if (nrb_encode(c, x, N, W1, b1, W2, b2, Wm, logits.data(), nthreads) != 0) return -1;
+  return nrb_build_logits(c, x, N, logits.data(), W1, b1, W2, b2, Wm, path, nthreads, info_out);
 }
 
 }  // extern "C"
