@@ -63,13 +63,18 @@ typedef struct {
   int lloyd_iters;        /* Lloyd passes per bucket (< 1 means 1) */
   int sample_per_cluster; /* k-means++ sample per cluster (>= 1) */
   uint64_t seed;          /* k-means++ seed */
+  int n_mid;              /* encoder hidden layers after the first (0..7) */
+  int mid_w[7];           /* their widths */
 } nr_build_config;
 
-/* Start a build of N rows on `device`. W1 [H x D], b1 [H], W2 [b x H], b2 [b]
- * are host fp32 encoder weights, copied. Errors: NR_ERR_INVALID_ARG (a field
- * out of range), NR_ERR_OOM, NR_ERR_CUDA. */
+/* Start a build of N rows on `device`. W1 [H x D], b1 [H], W2 [b x H_last],
+ * b2 [b] are host fp32 encoder weights, copied; H_last is the last hidden
+ * width. Wm (NULL when n_mid = 0): the hidden layers after the first, for
+ * each W [mid_w[i] x previous width] then its bias [mid_w[i]], concatenated.
+ * Errors: NR_ERR_INVALID_ARG (a field out of range), NR_ERR_OOM, NR_ERR_CUDA. */
 nr_status nr_build_begin(const nr_build_config *cfg, int64_t N, const float *W1, const float *b1,
-                         const float *W2, const float *b2, int device, nr_builder **out);
+                         const float *W2, const float *b2, const float *Wm, int device,
+                         nr_builder **out);
 
 /* Pass 1, encoder: logits of rows [row0, row0 + n) from d_rows [n x D]
  * (uint8 or fp32, cfg.dtype). Enqueued on `stream`. */

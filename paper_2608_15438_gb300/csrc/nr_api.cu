@@ -183,9 +183,18 @@ nr_status nr_index_init_device(nr_index *ix) {
   return NR_OK;
 }
 
+int nr_hidden_last(const nr_index *ix) { return ix->n_mid > 0 ? ix->mid_w[ix->n_mid - 1] : ix->H; }
+
+size_t nr_mid_floats(const nr_index *ix) {
+  size_t n = 0;
+  for (int i = 0, prev = ix->H; i < ix->n_mid; prev = ix->mid_w[i], ++i)
+    n += (size_t)ix->mid_w[i] * prev + ix->mid_w[i];
+  return n;
+}
+
 nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1, const float *W2,
-                                  const float *b2) {
-  const int D = ix->D, H = ix->H, b = ix->b;
+                                  const float *b2, const float *Wm) {
+  const int D = ix->D, H = ix->H, b = ix->b, HL = nr_hidden_last(ix);
   auto up = [&](void **dptr, const void *src, size_t bytes) -> nr_status {
     if (cudaMalloc(dptr, bytes > 0 ? bytes : 16) != cudaSuccess) {
       cudaGetLastError();
@@ -199,18 +208,34 @@ nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1
   std::vector<float> W1T((size_t)D * H);
   for (int u = 0; u < H; ++u)
     for (int j = 0; j < D; ++j) W1T[(size_t)j * H + u] = W1[(size_t)u * D + j];
+  nr_status st;
+  if ((st = up((void **)&ix->W1, W1, (size_t)H * D * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->b1, b1, (size_t)H * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->W2, W2, (size_t)b * HL * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->b2, b2, (size_t)b * 4)) != NR_OK) return st;
+  if ((st = up((void **)&ix->W1T, W1T.data(), W1T.size() * 4)) != NR_OK) return st;
+  if (ix->n_mid > 0) {
+    // the middle layers as stored, and transposed per layer for the kernel
+    const size_t n = nr_mid_floats(ix);
+    std::vector<float> t(n);
+    size_t o = 0;
+    for (int l = 0, prev = H; l < ix->n_mid; prev = ix->mid_w[l], ++l) {
+      const int w = ix->mid_w[l];
+      for (int u = 0; u < w; ++u)
+        for (int j = 0; j < prev; ++j) t[o + (size_t)j * w + u] = Wm[o + (size_t)u * prev + j];
+      for (int u = 0; u < w; ++u) t[o + (size_t)w * prev + u] = Wm[o + (size_t)w * prev + u];
+      o += (size_t)w * prev + w;
+    }
+    if ((st = up((void **)&ix->Wm, Wm, n * 4)) != NR_OK) return st;
+    if ((st = up((void **)&ix->WmT, t.data(), n * 4)) != NR_OK) return st;
+    return NR_OK;  // the tensor-core encoder covers one hidden layer only
+  }
   // fp16 operands of the tensor-core encoder; layer 2 padded to 16 or 32 rows
   const int n2 = b <= 16 ? 16 : 32;
   std::vector<__half> w1h((size_t)H * D), w2h((size_t)n2 * H, __float2half_rn(0.0f));
   for (size_t i = 0; i < w1h.size(); ++i) w1h[i] = __float2half_rn(W1[i]);
   for (int o = 0; o < b; ++o)
     for (int u = 0; u < H; ++u) w2h[(size_t)o * H + u] = __float2half_rn(W2[(size_t)o * H + u]);
-  nr_status st;
-  if ((st = up((void **)&ix->W1, W1, (size_t)H * D * 4)) != NR_OK) return st;
-  if ((st = up((void **)&ix->b1, b1, (size_t)H * 4)) != NR_OK) return st;
-  if ((st = up((void **)&ix->W2, W2, (size_t)b * H * 4)) != NR_OK) return st;
-  if ((st = up((void **)&ix->b2, b2, (size_t)b * 4)) != NR_OK) return st;
-  if ((st = up((void **)&ix->W1T, W1T.data(), W1T.size() * 4)) != NR_OK) return st;
   if ((st = up(&ix->W1h, w1h.data(), w1h.size() * 2)) != NR_OK) return st;
   if ((st = up(&ix->W2h, w2h.data(), w2h.size() * 2)) != NR_OK) return st;
   return NR_OK;
@@ -277,7 +302,7 @@ void nr_index_free(nr_index *ix) {
   }
   if (ps.a) cudaStreamDestroy(ps.a);
   if (ps.b) cudaStreamDestroy(ps.b);
-  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
+  void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->Wm, ix->WmT, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
                   ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->io};
   for (void *p : ptrs)
     if (p) cudaFree(p);
@@ -305,7 +330,8 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
     return NR_ERR_IO;
   }
   const uint64_t fsize = (uint64_t)ftello(f);
-  if (memcmp(h, "NRIXv001", 8) != 0 || rd32(h, 8) != 1) {
+  const uint32_t version = rd32(h, 8);
+  if (memcmp(h, "NRIXv001", 8) != 0 || (version != 1 && version != 2)) {
     fclose(f);
     return NR_ERR_FORMAT;
   }
@@ -326,6 +352,14 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   memcpy(&ix->in_scale, h + 56, 4);
   uint64_t off[10];
   for (int i = 0; i < 10; ++i) off[i] = rd64(h, 64 + 8 * i);
+  // version 2: the encoder's hidden layers after the first
+  ix->n_mid = version == 2 ? (int)rd32(h, 152) : 0;
+  bool mid_ok = ix->n_mid >= 0 && ix->n_mid <= 7;
+  for (int i = 0; mid_ok && i < ix->n_mid; ++i) {
+    ix->mid_w[i] = (int)rd32(h, 156 + 4 * i);
+    mid_ok = ix->mid_w[i] >= 1 && ix->mid_w[i] <= 4096;
+  }
+  const uint64_t mid_off = rd64(h, 192);
   const size_t esz = ix->dtype == 0 ? 1 : 4;
   ix->row_bytes = (int64_t)ix->D * (int64_t)esz;
   auto bad = [&](nr_status st) {
@@ -336,25 +370,30 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   if ((ix->dtype != 0 && ix->dtype != 1) || ix->b < 1 || ix->b > 24 || ix->D < 1 || ix->H < 1 ||
       ix->H > 4096 || ix->N < 1 || ix->N >= (int64_t)0xFFFFFFFFll || ix->n_cl < 1 ||
       ix->n_cl >= ((int64_t)1 << 31) || ix->row_bytes % 16 != 0 || ix->row_bytes > 1024 ||
-      ix->K_max < 0)
+      ix->K_max < 0 || !mid_ok)
     return bad(NR_ERR_FORMAT);
   const uint64_t nb = ((uint64_t)1 << ix->b) + 1;
   const uint64_t sz[10] = {(uint64_t)ix->H * ix->D * 4, (uint64_t)ix->H * 4,
-                           (uint64_t)ix->b * ix->H * 4, (uint64_t)ix->b * 4,
+                           (uint64_t)ix->b * nr_hidden_last(ix) * 4, (uint64_t)ix->b * 4,
                            (uint64_t)ix->b * 4,         nb * 4,
                            (uint64_t)(ix->n_cl + 1) * 4, (uint64_t)ix->n_cl * ix->b * 4,
                            (uint64_t)ix->N * 4,         (uint64_t)ix->N * ix->D * esz};
   for (int i = 0; i < 10; ++i)
     if (off[i] < 256 || off[i] + sz[i] > fsize) return bad(NR_ERR_FORMAT);
+  const uint64_t mid_sz = (uint64_t)nr_mid_floats(ix) * 4;
+  if (ix->n_mid > 0 && (mid_off < 256 || mid_off + mid_sz > fsize)) return bad(NR_ERR_FORMAT);
   // host copies of the small sections
-  std::vector<float> W1((size_t)ix->H * ix->D), b1(ix->H), W2((size_t)ix->b * ix->H), b2(ix->b),
-      tau(ix->b);
+  std::vector<float> W1((size_t)ix->H * ix->D), b1(ix->H), W2((size_t)ix->b * nr_hidden_last(ix)),
+      b2(ix->b), tau(ix->b), Wm(mid_sz / 4);
   std::vector<uint32_t> bkt(nb);
   auto rd = [&](int i, void *dst) {
     return fseeko(f, (off_t)off[i], SEEK_SET) == 0 && fread(dst, 1, sz[i], f) == sz[i];
   };
   if (!rd(0, W1.data()) || !rd(1, b1.data()) || !rd(2, W2.data()) || !rd(3, b2.data()) ||
       !rd(4, tau.data()) || !rd(5, bkt.data()))
+    return bad(NR_ERR_IO);
+  if (ix->n_mid > 0 && (fseeko(f, (off_t)mid_off, SEEK_SET) != 0 ||
+                        fread(Wm.data(), 1, mid_sz, f) != mid_sz))
     return bad(NR_ERR_IO);
   // clusters per bucket: K_max from the header, else from the directory
   int kmax_dir = 1;
@@ -368,7 +407,8 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   DeviceGuard g(device);
   nr_status st = nr_index_init_device(ix);
   if (st != NR_OK) return bad(st);
-  if ((st = nr_index_upload_encoder(ix, W1.data(), b1.data(), W2.data(), b2.data())) != NR_OK)
+  if ((st = nr_index_upload_encoder(ix, W1.data(), b1.data(), W2.data(), b2.data(),
+                                    ix->n_mid > 0 ? Wm.data() : nullptr)) != NR_OK)
     return bad(st);
   auto up = [&](void **dptr, const void *src, size_t bytes) -> nr_status {
     if (cudaMalloc(dptr, bytes > 0 ? bytes : 16) != cudaSuccess) {
@@ -421,12 +461,14 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
 namespace {
 
 // Writes an index file: header fields from `ix` with N and n_cl given, the
-// ten sections from src[i] (device memory where dev[i], else host memory).
+// ten sections from src[i] (device memory where dev[i], else host memory),
+// and with middle encoder layers (version 2) an eleventh section from mid
+// (device memory where mid_dev).
 nr_status write_nrix(const nr_index *ix, int64_t N, int64_t n_cl, const void *const src[10],
-                     const bool dev[10], const char *path) {
+                     const bool dev[10], const void *mid, bool mid_dev, const char *path) {
   const uint64_t nb = ((uint64_t)1 << ix->b) + 1;
   const uint64_t sz[10] = {(uint64_t)ix->H * ix->D * 4, (uint64_t)ix->H * 4,
-                           (uint64_t)ix->b * ix->H * 4, (uint64_t)ix->b * 4,
+                           (uint64_t)ix->b * nr_hidden_last(ix) * 4, (uint64_t)ix->b * 4,
                            (uint64_t)ix->b * 4,         nb * 4,
                            (uint64_t)(n_cl + 1) * 4,    (uint64_t)n_cl * ix->b * 4,
                            (uint64_t)N * 4,             (uint64_t)N * ix->row_bytes};
@@ -435,12 +477,19 @@ nr_status write_nrix(const nr_index *ix, int64_t N, int64_t n_cl, const void *co
     off[i] = cur;
     cur = (cur + sz[i] + 255) & ~(uint64_t)255;
   }
+  const uint64_t mid_sz = (uint64_t)nr_mid_floats(ix) * 4, mid_off = ix->n_mid > 0 ? cur : 0;
+  if (ix->n_mid > 0) cur = (cur + mid_sz + 255) & ~(uint64_t)255;
   unsigned char h[256];
   memset(h, 0, sizeof(h));
   memcpy(h, "NRIXv001", 8);
   auto w32 = [&](int o, uint32_t v) { memcpy(h + o, &v, 4); };
   auto w64 = [&](int o, uint64_t v) { memcpy(h + o, &v, 8); };
-  w32(8, 1);
+  w32(8, ix->n_mid > 0 ? 2 : 1);
+  if (ix->n_mid > 0) {
+    w32(152, (uint32_t)ix->n_mid);
+    for (int i = 0; i < ix->n_mid; ++i) w32(156 + 4 * i, (uint32_t)ix->mid_w[i]);
+    w64(192, mid_off);
+  }
   w32(12, (uint32_t)ix->dtype);
   w64(16, (uint64_t)N);
   w32(24, (uint32_t)ix->D);
@@ -486,6 +535,20 @@ nr_status write_nrix(const nr_index *ix, int64_t N, int64_t n_cl, const void *co
       done += n;
     }
   }
+  if (ix->n_mid > 0 && st == NR_OK) {
+    put(zeros, (size_t)(mid_off - at));
+    if (!mid_dev) put(mid, (size_t)mid_sz);
+    for (uint64_t done = 0; mid_dev && done < mid_sz && st == NR_OK;) {
+      const size_t n = (size_t)((mid_sz - done) < stage_bytes ? (mid_sz - done) : stage_bytes);
+      if (cudaMemcpy(stage, (const char *)mid + done, n, cudaMemcpyDeviceToHost) != cudaSuccess) {
+        cudaGetLastError();
+        st = NR_ERR_CUDA;
+        break;
+      }
+      put(stage, n);
+      done += n;
+    }
+  }
   put(zeros, (size_t)(cur - at));
   cudaFreeHost(stage);
   if (fclose(f) != 0 && st == NR_OK) st = NR_ERR_IO;
@@ -506,7 +569,7 @@ nr_status nr_index_save(nr_index *ix, const char *path) {
   const void *src[10] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->tau, ix->bkt_off,
                          ix->cl_off, ix->cent, ix->ids, ix->vec};
   const bool dev[10] = {true, true, true, true, true, true, true, true, true, true};
-  return write_nrix(ix, ix->N, ix->n_cl, src, dev, path);
+  return write_nrix(ix, ix->N, ix->n_cl, src, dev, ix->Wm, true, path);
 }
 
 nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, const char *path,
@@ -562,7 +625,7 @@ nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, con
     bkt[nb] = (uint32_t)c;
   }
   std::vector<float> cent((size_t)ncl * ix->b), W1((size_t)ix->H * ix->D), b1(ix->H),
-      W2((size_t)ix->b * ix->H), b2(ix->b), tau(ix->b);
+      W2((size_t)ix->b * nr_hidden_last(ix)), b2(ix->b), tau(ix->b), Wm(nr_mid_floats(ix));
   std::vector<uint32_t> ids((size_t)nrow);
   std::vector<unsigned char> vec;
   try {
@@ -587,12 +650,13 @@ nr_status nr_index_extract(nr_index *ix, const uint32_t *h_codes, int64_t n, con
   }
   if (!d2h(W1.data(), ix->W1, W1.size() * 4) || !d2h(b1.data(), ix->b1, b1.size() * 4) ||
       !d2h(W2.data(), ix->W2, W2.size() * 4) || !d2h(b2.data(), ix->b2, b2.size() * 4) ||
-      !d2h(tau.data(), ix->tau, tau.size() * 4))
+      !d2h(tau.data(), ix->tau, tau.size() * 4) ||
+      (ix->n_mid > 0 && !d2h(Wm.data(), ix->Wm, Wm.size() * 4)))
     return NR_ERR_CUDA;
   const void *src[10] = {W1.data(), b1.data(), W2.data(), b2.data(), tau.data(), bkt.data(),
                          cl.data(), cent.data(), ids.data(), vec.data()};
   const bool dev[10] = {false, false, false, false, false, false, false, false, false, false};
-  const nr_status st = write_nrix(ix, nrow, ncl, src, dev, path);
+  const nr_status st = write_nrix(ix, nrow, ncl, src, dev, Wm.data(), false, path);
   if (st == NR_OK && info) {
     info[0] = nrow;
     info[1] = ncl;

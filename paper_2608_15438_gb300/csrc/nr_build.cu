@@ -907,8 +907,12 @@ nr_status finish_impl(nr_builder *bd, int64_t *info, cudaStream_t s) {
 extern "C" {
 
 nr_status nr_build_begin(const nr_build_config *cfg, int64_t N, const float *W1, const float *b1,
-                         const float *W2, const float *b2, int device, nr_builder **out) {
+                         const float *W2, const float *b2, const float *Wm, int device,
+                         nr_builder **out) {
   if (!cfg || !out || !W1 || !b1 || !W2 || !b2) return NR_ERR_INVALID_ARG;
+  if (cfg->n_mid < 0 || cfg->n_mid > 7 || (cfg->n_mid > 0 && !Wm)) return NR_ERR_INVALID_ARG;
+  for (int i = 0; i < cfg->n_mid; ++i)
+    if (cfg->mid_w[i] < 1 || cfg->mid_w[i] > 4096) return NR_ERR_INVALID_ARG;
   *out = nullptr;
   const int64_t esz = cfg->dtype == 0 ? 1 : 4;
   const int64_t row_bytes = (int64_t)cfg->D * esz;
@@ -943,8 +947,10 @@ nr_status nr_build_begin(const nr_build_config *cfg, int64_t N, const float *W1,
   ix->t = cfg->t;
   ix->in_scale = cfg->in_scale;
   ix->row_bytes = row_bytes;
+  ix->n_mid = cfg->n_mid;
+  for (int i = 0; i < 7; ++i) ix->mid_w[i] = i < cfg->n_mid ? cfg->mid_w[i] : 0;
   nr_status st = nr_index_init_device(ix);
-  if (st == NR_OK) st = nr_index_upload_encoder(ix, W1, b1, W2, b2);
+  if (st == NR_OK) st = nr_index_upload_encoder(ix, W1, b1, W2, b2, Wm);
   if (st == NR_OK) st = cuda_status(cudaMalloc((void **)&ix->tau, (size_t)cfg->b * 4));
   if (st == NR_OK)
     st = cuda_status(cudaMalloc((void **)&ix->bkt_off, (((size_t)1 << cfg->b) + 1) * 4));

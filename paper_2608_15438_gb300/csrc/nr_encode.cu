@@ -324,6 +324,83 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// Encoders with hidden layers after the first: kQB queries a block, every
+// layer's activations for them in shared memory (two buffers of kQB x the
+// widest layer), one thread per output unit; layer weights transposed
+// [previous x width] so that a warp's loads are contiguous.
+__global__ void __launch_bounds__(kThreads)
+    encode_mlp_kernel(const void *__restrict__ x, int dtype, int D, int H, int b, float s,
+                      const float *__restrict__ W1T, const float *__restrict__ b1, int n_mid,
+                      int4 mid_lo, int4 mid_hi, const float *__restrict__ WmT,
+                      const float *__restrict__ W2, const float *__restrict__ b2, int maxw,
+                      int64_t nq, float *__restrict__ out) {
+  extern __shared__ float sm[];
+  float *A = sm, *B = sm + (size_t)kQB * maxw;  // [kQB][width] each
+  const int tid = threadIdx.x;
+  const int64_t q0 = (int64_t)blockIdx.x * kQB;
+  for (int i = tid; i < kQB * D; i += kThreads) {
+    const int qi = i / D, j = i - qi * D;
+    const int64_t qq = q0 + qi;
+    float v = 0.0f;
+    if (qq < nq)
+      v = dtype == 0 ? (float)static_cast<const uint8_t *>(x)[qq * D + j]
+                     : static_cast<const float *>(x)[qq * D + j];
+    A[qi * D + j] = v;
+  }
+  __syncthreads();
+  for (int u = tid; u < H; u += kThreads) {  // first hidden layer, input scale s
+    float acc[kQB];
+#pragma unroll
+    for (int qi = 0; qi < kQB; ++qi) acc[qi] = 0.0f;
+    for (int j = 0; j < D; ++j) {
+      const float w = W1T[(size_t)j * H + u];
+#pragma unroll
+      for (int qi = 0; qi < kQB; ++qi) acc[qi] = __fmaf_rn(w, A[qi * D + j], acc[qi]);
+    }
+#pragma unroll
+    for (int qi = 0; qi < kQB; ++qi) {
+      const float h = __fmaf_rn(s, acc[qi], b1[u]);
+      B[qi * H + u] = h > 0.0f ? h : 0.0f;
+    }
+  }
+  __syncthreads();
+  const int widths[8] = {mid_lo.x, mid_lo.y, mid_lo.z, mid_lo.w, mid_hi.x, mid_hi.y, mid_hi.z, 0};
+  int prev = H;
+  const float *wl = WmT;
+  float *cur = B, *nxt = A;
+  for (int l = 0; l < n_mid; ++l) {
+    const int w = widths[l];
+    const float *bias = wl + (size_t)w * prev;
+    for (int u = tid; u < w; u += kThreads) {
+      float acc[kQB];
+#pragma unroll
+      for (int qi = 0; qi < kQB; ++qi) acc[qi] = bias[u];
+      for (int j = 0; j < prev; ++j) {
+        const float wj = wl[(size_t)j * w + u];
+#pragma unroll
+        for (int qi = 0; qi < kQB; ++qi) acc[qi] = __fmaf_rn(wj, cur[qi * prev + j], acc[qi]);
+      }
+#pragma unroll
+      for (int qi = 0; qi < kQB; ++qi) nxt[qi * w + u] = acc[qi] > 0.0f ? acc[qi] : 0.0f;
+    }
+    __syncthreads();
+    wl = bias + w;
+    prev = w;
+    float *t = cur;
+    cur = nxt;
+    nxt = t;
+  }
+  for (int o = tid; o < kQB * b; o += kThreads) {  // last layer, linear
+    const int qi = o / b, j = o - qi * b;
+    const int64_t qq = q0 + qi;
+    if (qq >= nq) continue;
+    float acc = b2[j];
+    const float *w = W2 + (size_t)j * prev;
+    for (int u = 0; u < prev; ++u) acc = __fmaf_rn(w[u], cur[qi * prev + u], acc);
+    out[qq * b + j] = acc;
+  }
+}
+
 }  // namespace
 
 bool nr_encode_uses_tensor_cores(const nr_index *ix) {
@@ -345,6 +422,22 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
                                            static_cast<const __half *>(ix->W1h), ix->b1,
                                            static_cast<const __half *>(ix->W2h), ix->b2, nq,
                                            d_logits, ix->d_err);
+    ix->launches += 1;
+    return cudaGetLastError();
+  }
+  if (ix->n_mid > 0) {
+    int maxw = ix->D > ix->H ? ix->D : ix->H;
+    for (int i = 0; i < ix->n_mid; ++i) maxw = ix->mid_w[i] > maxw ? ix->mid_w[i] : maxw;
+    const size_t smem = (size_t)2 * kQB * maxw * sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(encode_mlp_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int *mw = ix->mid_w;
+    const int64_t grid = (nq + kQB - 1) / kQB;
+    encode_mlp_kernel<<<(unsigned)grid, kThreads, smem, s>>>(
+        d_x, ix->dtype, ix->D, ix->H, ix->b, ix->in_scale, ix->W1T, ix->b1, ix->n_mid,
+        make_int4(mw[0], mw[1], mw[2], mw[3]), make_int4(mw[4], mw[5], mw[6], 0), ix->WmT, ix->W2,
+        ix->b2, maxw, nq, d_logits);
     ix->launches += 1;
     return cudaGetLastError();
   }

@@ -21,6 +21,12 @@ struct nr_index {
   int dtype = 0;  // 0 uint8, 1 fp32
   int64_t N = 0;
   int D = 0, H = 0, b = 0, K_max = 0, t = 0;
+  // encoder hidden layers after the first: widths, weights as the file
+  // stores them (W [w x previous] then bias, per layer) and, for the kernel,
+  // each layer's W transposed [previous x w] followed by its bias
+  int n_mid = 0;
+  int mid_w[7] = {0, 0, 0, 0, 0, 0, 0};
+  float *Wm = nullptr, *WmT = nullptr;
   int64_t n_cl = 0;
   float in_scale = 1.0f;
   int64_t row_bytes = 0;
@@ -57,10 +63,14 @@ struct nr_seg {
 // (nr_api.cu). The device must be current.
 nr_index *nr_index_alloc();  // zeroed object with default params and host extras
 nr_status nr_index_init_device(nr_index *ix);  // num_sms and the device check flag
-// uploads fp32 W1 [H x D], b1 [H], W2 [b x H], b2 [b] (host) and the encoder's
-// derived forms; needs D, H and b set
+// uploads fp32 W1 [H x D], b1 [H], W2 [b x H_last], b2 [b] and the middle
+// layers Wm (host; NULL without any) and the encoder's derived forms; needs
+// D, H, b, n_mid and mid_w set
 nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1, const float *W2,
-                                  const float *b2);
+                                  const float *b2, const float *Wm);
+// last hidden width and the number of floats of the middle layers
+int nr_hidden_last(const nr_index *ix);
+size_t nr_mid_floats(const nr_index *ix);
 
 // kernel launchers (each returns cudaGetLastError() after the launch)
 bool nr_encode_uses_tensor_cores(const nr_index *ix);

@@ -85,7 +85,7 @@ def lib():
         L.nr_index_extract.argtypes = [vp, vp, i64, ctypes.c_char_p, vp]
         L.nr_index_locate.argtypes = [vp, vp, i64, vp, vp]
         L.nr_centroid_dists.argtypes = [vp, vp, i64, vp, i32, vp, vp]
-        L.nr_build_begin.argtypes = [vp, i64, vp, vp, vp, vp, i32, ctypes.POINTER(vp)]
+        L.nr_build_begin.argtypes = [vp, i64, vp, vp, vp, vp, vp, i32, ctypes.POINTER(vp)]
         L.nr_build_encode.argtypes = [vp, vp, i64, i64, vp]
         L.nr_build_set_logits.argtypes = [vp, vp, i64, i64, vp]
         L.nr_build_finish.argtypes = [vp, vp]
@@ -320,14 +320,19 @@ class Builder:
     the CSR levels, pass 2 places the rows, end() returns the Index.
 
     cfg is a ctypes structure with the fields of nr_build_config (the host
-    builder's Config has the same layout); weights = (W1, b1, W2, b2) fp32."""
+    builder's Config has the same layout); weights = (W1, b1, W2, b2[, middle
+    layers ((W, b), ...)]) fp32."""
 
     def __init__(self, cfg, N: int, weights, device: int = 0):
-        W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights)
+        W1, b1, W2, b2 = (np.ascontiguousarray(w, np.float32) for w in weights[:4])
+        mid = weights[4] if len(weights) > 4 else ()
+        Wm = np.ascontiguousarray(np.concatenate(
+            [np.concatenate([np.asarray(W, np.float32).ravel(), np.asarray(bb, np.float32).ravel()])
+             for W, bb in mid]) if mid else np.zeros(1, np.float32))
         h = ctypes.c_void_p()
         _check("nr_build_begin", lib().nr_build_begin(
             ctypes.byref(cfg), N, W1.ctypes.data, b1.ctypes.data, W2.ctypes.data, b2.ctypes.data,
-            device, ctypes.byref(h)))
+            Wm.ctypes.data if mid else None, device, ctypes.byref(h)))
         self.h, self.N, self.device, self.b = h, N, device, cfg.b
 
     def encode(self, rows, row0: int, stream=None):
