@@ -369,7 +369,7 @@ nr_status nr_index_load(const char *path, int device, nr_index **out) {
   };
   if ((ix->dtype != 0 && ix->dtype != 1) || ix->b < 1 || ix->b > 24 || ix->D < 1 || ix->H < 1 ||
       ix->H > 4096 || ix->N < 1 || ix->N >= (int64_t)0xFFFFFFFFll || ix->n_cl < 1 ||
-      ix->n_cl >= ((int64_t)1 << 31) || ix->row_bytes % 16 != 0 || ix->row_bytes > 1024 ||
+      ix->n_cl >= ((int64_t)1 << 31) || !nr_row_bytes_ok(ix->dtype, ix->row_bytes) ||
       ix->K_max < 0 || !mid_ok)
     return bad(NR_ERR_FORMAT);
   const uint64_t nb = ((uint64_t)1 << ix->b) + 1;

@@ -919,7 +919,7 @@ nr_status nr_build_begin(const nr_build_config *cfg, int64_t N, const float *W1,
   if ((cfg->dtype != 0 && cfg->dtype != 1) || cfg->D < 1 || cfg->H < 1 || cfg->H > 4096 ||
       cfg->b < 1 || cfg->b > kBMax || cfg->K_max < 1 || cfg->K_max > kKMax || cfg->t < 1 ||
       cfg->sample_per_cluster < 1 || cfg->sample_per_cluster > kMaxSample || N < 1 ||
-      N >= (int64_t)0xFFFFFFFFll || row_bytes % 16 != 0 || row_bytes > 1024)
+      N >= (int64_t)0xFFFFFFFFll || !nr_row_bytes_ok(cfg->dtype, row_bytes))
     return NR_ERR_INVALID_ARG;
   int ndev = 0;
   if (cudaGetDeviceCount(&ndev) != cudaSuccess) {

@@ -59,6 +59,15 @@ struct nr_seg {
   uint32_t pos;
 };
 
+// Row sizes the query path supports: a multiple of 16 bytes up to 1 KB, and
+// for fp32 rows a multiple of 64 bytes up to 8 KB (D up to 2048, the long-row
+// refinement).
+inline bool nr_row_bytes_ok(int dtype, int64_t row_bytes) {
+  if (row_bytes < 16 || row_bytes % 16 != 0) return false;
+  if (row_bytes <= 1024) return true;
+  return dtype == 1 && row_bytes % 64 == 0 && row_bytes <= 8192;
+}
+
 // Index object helpers shared by the file loader and the GPU builder
 // (nr_api.cu). The device must be current.
 nr_index *nr_index_alloc();  // zeroed object with default params and host extras

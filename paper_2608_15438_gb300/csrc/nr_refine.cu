@@ -91,6 +91,30 @@ __global__ void __launch_bounds__(TR, MINB) refine_kernel(RefineArgs a) {
   }
 }
 
+// fp32 rows longer than 1 KB: tiles staged in pieces (refine_block_split)
+template <int TR, int STAGES, int KCC, int MINB>
+__global__ void __launch_bounds__(TR, MINB) refine_split_kernel(RefineArgs a) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  const int tid = threadIdx.x;
+  const int k = a.rf.k;
+  const nrq::RefineSmem m = nrq::refine_split_carve<TR, STAGES, KCC>(smem, a.row_bytes, k);
+  int *qslot = m.sctl + 4;
+  for (;;) {
+    if (tid == 0) {
+      const unsigned int slot = atomicAdd(a.counter, 1u);
+      *qslot = slot < a.nq ? (a.perm ? a.perm[slot] : (int)slot) : -1;
+    }
+    __syncthreads();
+    const int64_t q = *qslot;
+    if (q < 0) break;
+    for (int c = tid; c * 16 < a.row_bytes; c += TR)
+      reinterpret_cast<uint4 *>(m.sq)[c] = reinterpret_cast<const uint4 *>(a.q + q * a.row_bytes)[c];
+    nrq::refine_block_split<TR, STAGES, KCC>(a.rf, m, a.slen[q], a.nL[q],
+                                             a.seg + (size_t)q * a.Lmax, a.out_ids + q * k,
+                                             a.out_d + q * k, a.stats ? a.stats + q * 4 : nullptr);
+  }
+}
+
 template <typename K>
 cudaError_t persistent_launch(nr_index *ix, K kern, int threads, size_t smem, int64_t nq,
                               const void *args, cudaStream_t s, void (*go)(K, int, int, size_t,
@@ -113,6 +137,17 @@ template <int DT, int TR, int STAGES, int CPR, int MINB = 1>
 cudaError_t launch_refine(nr_index *ix, const RefineArgs &a, cudaStream_t s) {
   const size_t smem = nrq::refine_smem_bytes<DT, TR, STAGES>(a.row_bytes, a.rf.k) + 16;
   auto kern = refine_kernel<DT, TR, STAGES, CPR, MINB>;
+  return persistent_launch(ix, kern, TR, smem, a.nq, &a, s,
+                           +[](decltype(kern) kk, int g, int t, size_t sm, cudaStream_t st,
+                               const void *p) {
+                             kk<<<g, t, sm, st>>>(*static_cast<const RefineArgs *>(p));
+                           });
+}
+
+template <int TR, int STAGES, int KCC, int MINB>
+cudaError_t launch_refine_split(nr_index *ix, const RefineArgs &a, cudaStream_t s) {
+  const size_t smem = nrq::refine_split_smem_bytes<TR, STAGES, KCC>(a.row_bytes, a.rf.k) + 16;
+  auto kern = refine_split_kernel<TR, STAGES, KCC, MINB>;
   return persistent_launch(ix, kern, TR, smem, a.nq, &a, s,
                            +[](decltype(kern) kk, int g, int t, size_t sm, cudaStream_t st,
                                const void *p) {
@@ -175,6 +210,11 @@ cudaError_t nr_launch_refine(nr_index *ix, const void *d_q, int64_t nq, int k, i
     if (a.rf.cpr == 8) return launch_refine<0, 128, 2, 8, 6>(ix, a, s);  // uint8, D = 128
     if (ix->row_bytes <= 512) return launch_refine<0, 128, 2, 0, 4>(ix, a, s);
     return launch_refine<0, 64, 2, 0, 4>(ix, a, s);
+  }
+  if (ix->row_bytes > 1024) {  // fp32, D above 256: rows staged in pieces
+    if (ix->row_bytes % 256 == 0) return launch_refine_split<128, 2, 16, 3>(ix, a, s);
+    if (ix->row_bytes % 128 == 0) return launch_refine_split<128, 2, 8, 3>(ix, a, s);
+    return launch_refine_split<128, 2, 4, 3>(ix, a, s);  // row_bytes % 64 == 0 (load check)
   }
   if (a.rf.cpr == 24) return launch_refine<1, 32, 2, 24, 12>(ix, a, s);  // fp32, D = 96
   if (ix->row_bytes <= 512) return launch_refine<1, 64, 2, 0, 4>(ix, a, s);

@@ -270,4 +270,204 @@ __device__ __forceinline__ void refine_block(const RefineParams &a, const Refine
   __syncthreads();
 }
 
+// ============================================================== refine, long rows
+// fp32 rows too long for whole-row stages (D above 256): each tile of TR rows
+// is staged in pieces of KCC 16-byte chunks of every row (TR x 16 KCC bytes a
+// stage), and each thread carries its row's distance from piece to piece, so
+// the sum over j stays the sequential fmaf chain of refine_block; the merge,
+// rounds and stop rule are refine_block's. row_bytes is a multiple of 16 KCC.
+template <int TR, int STAGES, int KCC>
+__host__ __device__ inline size_t refine_split_smem_bytes(int64_t row_bytes, int k) {
+  return (size_t)STAGES * TR * KCC * 16 + (size_t)row_bytes + (size_t)2 * TR * 4 +
+         (size_t)2 * k * 8 + (size_t)2 * TR * 8 + (size_t)2 * k * 4 + 16;
+}
+
+template <int TR, int STAGES, int KCC>
+__device__ __forceinline__ RefineSmem refine_split_carve(unsigned char *base, int64_t row_bytes,
+                                                         int k) {
+  RefineSmem m;
+  m.stage = base;
+  m.sq = base + (size_t)STAGES * TR * KCC * 16;
+  m.srow = reinterpret_cast<uint32_t *>(m.sq + row_bytes);  // 2 x TR: rows of the open tiles
+  m.hkey = reinterpret_cast<uint64_t *>(m.srow + 2 * TR);
+  m.skey = m.hkey + 2 * k;
+  m.htag = reinterpret_cast<int *>(m.skey + 2 * TR);
+  m.sctl = m.htag + 2 * k;
+  return m;
+}
+
+template <int TR, int STAGES, int KCC>
+__device__ __forceinline__ void refine_block_split(const RefineParams &a, const RefineSmem &m,
+                                                   uint32_t n, int nl, const nr_seg *segs,
+                                                   int64_t *out_ids, float *out_d, int64_t *stats) {
+  constexpr int swz = KCC % 8 == 0 ? 7 : KCC % 4 == 0 ? 3 : KCC % 2 == 0 ? 1 : 0;
+  constexpr uint32_t PB = KCC * 16;  // bytes of one row in one stage
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t RB = (int64_t)a.cpr * 16;
+  const int nk = a.cpr / KCC;  // pieces per row
+  const uint32_t stage_s = (uint32_t)__cvta_generic_to_shared(m.stage);
+  const int k = a.k;
+  const int chunk = a.R < TR ? a.R : TR;
+  const uint32_t ntiles = (uint32_t)(((uint64_t)n + TR - 1) / TR);
+  const uint32_t nitems = ntiles * (uint32_t)nk;
+  if (tid == 0) m.sctl[1] = m.sctl[2] = m.sctl[3] = 0;
+  __syncthreads();  // the caller's copy of the query row into m.sq is visible after this
+
+  int seg_i = 0;       // this thread's segment cursor (positions only grow)
+  uint32_t grow = 0;   // this thread's row in the tile being issued
+  auto issue = [&](uint32_t it, int st) {
+    if (it < nitems) {
+      const uint32_t t = it / (uint32_t)nk;
+      const int kk = (int)(it - t * (uint32_t)nk);
+      if (kk == 0) {  // a new tile: find this thread's row
+        const uint32_t p = t * TR + tid;
+        grow = 0;
+        if (p < n) {
+          int step = 1;
+          while (seg_i + step < nl && segs[seg_i + step].pos <= p) {
+            seg_i += step;
+            step <<= 1;
+          }
+          for (step >>= 1; step > 0; step >>= 1)
+            if (seg_i + step < nl && segs[seg_i + step].pos <= p) seg_i += step;
+          grow = segs[seg_i].row0 + (p - segs[seg_i].pos);
+          m.srow[(t & 1) * TR + tid] = grow;
+        }
+      }
+      const uint32_t wbase = t * TR + warp * 32;
+      const uint32_t sbase = stage_s + (uint32_t)((size_t)st * TR * PB);
+#pragma unroll 4
+      for (int f = lane; f < 32 * KCC; f += 32) {
+        const int rr = f / KCC;
+        const int c = f - rr * KCC;
+        const uint32_t gr = __shfl_sync(kFull, grow, rr);
+        if (wbase + rr < n) {
+          const int r = warp * 32 + rr;
+          const uint32_t dst = sbase + (uint32_t)(r * PB) + (uint32_t)((c ^ (r & swz)) << 4);
+          cp_async16(dst, a.vec + (size_t)gr * RB + (size_t)kk * PB + ((size_t)c << 4));
+        }
+      }
+    }
+    cp_async_commit();
+  };
+
+  for (int s = 0; s < STAGES - 1; ++s) issue((uint32_t)s, s);
+  int cur = 0, hn = 0, rounds = 0, low = 0, ci = 0;
+  bool stop = false;
+  uint32_t done = 0;
+  const uint32_t rmask_round = (uint32_t)a.R - 1u;
+  int st = 0;
+  float acc = 0.0f;  // sequential over j across the pieces of a row
+  for (uint32_t it = 0; it < nitems && !stop; ++it) {
+    issue(it + STAGES - 1, st == 0 ? STAGES - 1 : st - 1);
+    cp_async_wait<STAGES - 1>();
+    __syncwarp();
+    const uint32_t t = it / (uint32_t)nk;
+    const int kk = (int)(it - t * (uint32_t)nk);
+    const uint32_t p = t * TR + tid;
+    if (p < n) {
+      const unsigned char *row = m.stage + (size_t)st * TR * PB + (size_t)tid * PB;
+      const float4 *q4 = reinterpret_cast<const float4 *>(m.sq + (size_t)kk * PB);
+#pragma unroll 4
+      for (int c = 0; c < KCC; ++c) {
+        const float4 v = *reinterpret_cast<const float4 *>(row + ((c ^ (tid & swz)) << 4));
+        const float4 w = q4[c];
+        float d;
+        d = __fsub_rn(v.x, w.x); acc = __fmaf_rn(d, d, acc);
+        d = __fsub_rn(v.y, w.y); acc = __fmaf_rn(d, d, acc);
+        d = __fsub_rn(v.z, w.z); acc = __fmaf_rn(d, d, acc);
+        d = __fsub_rn(v.w, w.w); acc = __fmaf_rn(d, d, acc);
+      }
+    }
+    st = st + 1 == STAGES ? 0 : st + 1;
+    if (kk + 1 < nk) continue;  // the row is not complete yet
+    const uint32_t dkey = p < n ? __float_as_uint(acc) : 0xffffffffu;
+    acc = 0.0f;
+    for (int cs = 0; cs < TR && !stop; cs += chunk, ++ci) {
+      const uint32_t cstart = t * TR + cs;
+      if (cstart >= n) break;
+      int *cnt = &m.sctl[1 + ci % 3];
+      uint64_t *sk_buf = m.skey + (ci & 1) * TR;
+      const uint64_t thr = hn == k ? m.hkey[cur * k + k - 1] : kEmpty;
+      const uint32_t thr_hi = (uint32_t)(thr >> 32);
+      if (tid >= cs && tid < cs + chunk && p < n && dkey <= thr_hi) {
+        const uint32_t id = __ldg(&a.ids[m.srow[(t & 1) * TR + tid]]);
+        const uint64_t key = ((uint64_t)dkey << 32) | id;
+        if (key < thr) sk_buf[atomicAdd(cnt, 1)] = key;
+      }
+      if (tid == 0) m.sctl[1 + (ci + 1) % 3] = 0;
+      __syncthreads();
+      const int ns = *cnt;
+      const int roundno = rounds + 1;
+      if (ns > 0) {
+        const int nxt = cur ^ 1;
+        const uint64_t *H = m.hkey + cur * k;
+        for (int i = tid; i < ns; i += TR) {
+          const uint64_t sk = sk_buf[i];
+          int lo = 0, hi = hn;
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (H[mid] <= sk) lo = mid + 1; else hi = mid;
+          }
+          int r = lo;
+          for (int j = 0; j < ns; ++j) r += (sk_buf[j] < sk || (sk_buf[j] == sk && j < i)) ? 1 : 0;
+          if (r < k) {
+            m.hkey[nxt * k + r] = sk;
+            m.htag[nxt * k + r] = roundno;
+          }
+        }
+        for (int j = tid; j < hn; j += TR) {
+          const uint64_t hk = H[j];
+          int r = j;
+          for (int i = 0; i < ns; ++i) r += sk_buf[i] < hk ? 1 : 0;
+          if (r < k) {
+            m.hkey[nxt * k + r] = hk;
+            m.htag[nxt * k + r] = m.htag[cur * k + j];
+          }
+        }
+        __syncthreads();
+        cur = nxt;
+        hn = hn + ns < k ? hn + ns : k;
+      }
+      const uint32_t cend = n - cstart > (uint32_t)chunk ? cstart + chunk : n;
+      if ((cend & rmask_round) == 0 || cend >= n) {
+        rounds = roundno;
+        done = cend;
+        int newc = 0, frontc = 0;
+        for (int i = lane; i < hn; i += 32) {
+          const bool nw = m.htag[cur * k + i] == roundno;
+          newc += nw ? 1 : 0;
+          frontc += (nw && i < a.nfront) ? 1 : 0;
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+          newc += __shfl_xor_sync(kFull, newc, o);
+          frontc += __shfl_xor_sync(kFull, frontc, o);
+        }
+        const bool lowq = newc < a.u_min && frontc < a.f_min;
+        low = lowq ? low + 1 : 0;
+        stop = a.t_low > 0 && hn == k && roundno >= a.r_min && low >= a.t_low;
+      }
+    }
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+  const uint64_t *H = m.hkey + cur * k;
+  for (int i = tid; i < k; i += TR) {
+    int64_t id = -1;
+    float d = __int_as_float(0x7f800000);
+    if (i < hn) {
+      const uint64_t kk2 = H[i];
+      id = (int64_t)(uint32_t)kk2;
+      d = __uint_as_float((uint32_t)(kk2 >> 32));
+    }
+    out_ids[i] = id;
+    out_d[i] = d;
+  }
+  if (tid == 0 && stats) {
+    stats[0] = (int64_t)done;
+    stats[1] = rounds;
+  }
+  __syncthreads();
+}
+
 }  // namespace nrq

@@ -36,12 +36,20 @@ def mlp_case(D=48, widths=(64, 32, 24, 16), b=12, n=20_000, seed=1):
     return base, q, weights, widths, b
 
 
-@pytest.fixture(scope="module")
-def built(torch, tmp_path_factory):
+# (D, hidden widths, b, rows): one hidden-layer chain per case; D = 272, 288,
+# 512 and 1536 fp32 rows (1,088 to 6,144 bytes) take the long-row refinement
+# with 4, 8 and 16 chunks a piece
+CASES = [(48, (64, 32, 24, 16), 12, 20_000), (272, (128, 64), 12, 12_000), (288, (128, 64), 12, 12_000),
+         (512, (256, 128, 64), 12, 12_000), (1536, (512, 256, 128, 64), 16, 6_000)]
+
+
+@pytest.fixture(scope="module", params=CASES, ids=[f"D{c[0]}" for c in CASES])
+def built(torch, tmp_path_factory, request):
     from paper_2608_15438_gb300 import neuroute as nr
     from paper_2608_15438_gb300.builder import build_index, config
 
-    base, q, weights, widths, b = mlp_case()
+    D, widths, b, n = request.param
+    base, q, weights, widths, b = mlp_case(D, widths, b, n)
     cfg = config("f32", base.shape[1], widths[0], b, 4, 16, mid=widths[1:])
     path = str(tmp_path_factory.mktemp("mlp") / "m.nrix")
     build_index(cfg, base, weights, path)
