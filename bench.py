@@ -200,7 +200,7 @@ def build_or_load_index(w, path, rank, world):
 
     if rank == 0 and not os.path.exists(path):
         base = synth.base(w)
-        info = build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t), base,
+        info = build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t, mid=w.mid), base,
                            synth.encoder_weights(w), path + ".tmp")
         os.replace(path + ".tmp", path)
         del base
@@ -219,7 +219,7 @@ def gpu_index(w, torch, nr, dev):
 
     d = dev.index or 0
     gen = synth.DeviceRows(w, synth.SEED_DATA, device=d)
-    bd = nr.Builder(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t), w.n,
+    bd = nr.Builder(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t, mid=w.mid), w.n,
                     synth.encoder_weights(w), d)
     chunk = min(w.n, (4 << 30) // w.row_bytes)
     buf = torch.empty((chunk, w.dim), dtype=torch.uint8 if w.dtype == "u8" else torch.float32,
@@ -248,6 +248,8 @@ def ground_truth_rows(torch, w, dq, k, dev, chunk=1 << 22, qblock=2500, group=10
     import synth
 
     gen = synth.DeviceRows(w, synth.SEED_DATA, device=dev.index or 0)
+    # at most about 512 MB of rows a chunk, in whole groups
+    chunk = max(group * 16, min(chunk, ((512 << 20) // w.row_bytes) // group * group))
     Q = dq.float()
     nq = Q.shape[0]
     best_d = torch.full((nq, k), float("inf"), device=dev)

@@ -94,6 +94,7 @@ class Workload:
     clusters: tuple = (32,)
     k: int = 10
     notes: str = ""
+    mid: tuple = ()   # encoder hidden widths after the first (H)
 
     @property
     def dtype_code(self) -> int:
@@ -129,6 +130,10 @@ WORKLOADS = {
     "u8-100m": Workload("u8-100m", 100_000_000, 128, "u8", 4096, 18.0, 10_000, 512, 24, 16, 64),
     # 1e9 uint8 x 128, b = 24
     "u8-1b": Workload("u8-1b", 1_000_000_000, 128, "u8", 16384, 18.0, 10_000, 512, 24, 16, 64),
+    # 1e7 fp32 x 1536, L2-normalised, with the paper's high-dimensional encoder
+    # shape 1536 -> 512 -> 256 -> 128 -> 64 -> 16 (four hidden layers), b = 16
+    "f32-1536": Workload("f32-1536", 10_000_000, 1536, "f32", 1024, 0.3, 10_000, 512, 16, 16, 64,
+                         mid=(256, 128, 64)),
 }
 
 
@@ -208,9 +213,17 @@ def normal(seed: int, stream: int, n: int, scale: float) -> np.ndarray:
 
 
 def encoder_weights(w: Workload, seed: int = SEED_ENCODER):
-    """Seeded encoder D -> H (ReLU) -> b with N(0, 1/fan_in) weights, zero biases.
+    """Seeded encoder D -> H (ReLU) [-> mid widths (ReLU)] -> b with
+    N(0, 1/fan_in) weights, zero biases.
 
-    Returns (W1 [H x D], b1 [H], W2 [b x H], b2 [b]) as fp32 arrays."""
+    Returns (W1 [H x D], b1 [H], W2 [b x H_last], b2 [b]) as fp32 arrays, and
+    with hidden layers after the first a fifth element ((W, b), ...) of them
+    (stream 3 + i for layer i)."""
     W1 = normal(seed, STREAM_W1, w.hidden * w.dim, 1.0 / np.sqrt(w.dim)).reshape(w.hidden, w.dim)
-    W2 = normal(seed, STREAM_W2, w.bits * w.hidden, 1.0 / np.sqrt(w.hidden)).reshape(w.bits, w.hidden)
-    return W1, np.zeros(w.hidden, np.float32), W2, np.zeros(w.bits, np.float32)
+    widths = (w.hidden,) + tuple(w.mid)
+    mid = tuple((normal(seed, 3 + i, wo * wi, 1.0 / np.sqrt(wi)).reshape(wo, wi), np.zeros(wo, np.float32))
+                for i, (wi, wo) in enumerate(zip(widths[:-1], widths[1:])))
+    hl = widths[-1]
+    W2 = normal(seed, STREAM_W2, w.bits * hl, 1.0 / np.sqrt(hl)).reshape(w.bits, hl)
+    out = (W1, np.zeros(w.hidden, np.float32), W2, np.zeros(w.bits, np.float32))
+    return out + (mid,) if mid else out

@@ -52,7 +52,7 @@ def cached_index(workload_name, tmp_root="/tmp"):
     path = os.path.join(tmp_root, f"neuroute_{w.name}_{h.hexdigest()[:16]}.nrix")
     if not os.path.exists(path):
         base = synth.base(w)
-        build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t), base,
+        build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t, mid=w.mid), base,
                     synth.encoder_weights(w), path + f".tmp{os.getpid()}")
         os.replace(path + f".tmp{os.getpid()}", path)
     return path
