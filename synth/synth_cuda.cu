@@ -143,9 +143,11 @@ int synth_mixture_cuda(int kind, uint64_t seed_rows, int M, int D, double sigma,
     mixture_u8_kernel<<<sms * 16, 256, 0, s>>>(seed_rows, M, D, sigma, row0, n, d_centres,
                                                static_cast<uint8_t *>(d_out));
   } else {
-    const int wpb = 8;
+    // warps per block: as many (up to 8) as the default 48 KB of shared memory
+    // holds rows of D doubles; the values do not depend on it
+    int wpb = (int)((48 * 1024) / ((size_t)D * sizeof(double)));
+    wpb = wpb < 1 ? 1 : (wpb > 8 ? 8 : wpb);
     const size_t smem = (size_t)wpb * D * sizeof(double);
-    if (smem > 48 * 1024) return -1;
     mixture_f32_kernel<<<sms * 8, 32 * wpb, smem, s>>>(seed_rows, M, D, sigma, row0, n, d_centres,
                                                        static_cast<float *>(d_out));
   }
