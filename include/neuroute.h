@@ -30,15 +30,20 @@
  *    bit-identical to a sequential CPU evaluation fed the same logits.
  *
  * Index file (little-endian), written by the package's builder:
- *   header 256 B: "NRIXv001", u32 version=1, u32 dtype (0 uint8, 1 fp32),
- *     u64 N (< 2^32 - 1), u32 D, H, b, K_max, t, u32 0, u64 n_clusters (< 2^31),
- *     f32 in_scale,
- *     u32 0, u64 section offsets[10], u64 file size
- *   sections (256-byte aligned): W1 f32[H][D], b1 f32[H], W2 f32[b][H],
- *     b2 f32[b], tau f32[b], bkt_off u32[2^b + 1] (code -> cluster range),
- *     cl_off u32[n_clusters + 1] (cluster -> row range), cent f32[n_clusters][b],
- *     ids u32[N] (original id of each stored row), vec (uint8|fp32)[N][D]
- *     stored in (code, cluster, id) order.
+ *   header 256 B: "NRIXv001", u32 version (1, or 2 with hidden layers after
+ *     the first), u32 dtype (0 uint8, 1 fp32), u64 N (< 2^32 - 1), u32 D, H, b,
+ *     K_max, t, u32 0, u64 n_clusters (< 2^31), f32 in_scale, u32 0,
+ *     u64 section offsets[10], u64 file size; version 2 adds at byte 152
+ *     u32 n_mid (1..7), u32 mid widths[7], u32 0, u64 offset of the eleventh
+ *     section
+ *   sections (256-byte aligned): W1 f32[H][D], b1 f32[H], W2 f32[b][H_last]
+ *     (H_last = the last hidden width), b2 f32[b], tau f32[b], bkt_off
+ *     u32[2^b + 1] (code -> cluster range), cl_off u32[n_clusters + 1]
+ *     (cluster -> row range), cent f32[n_clusters][b], ids u32[N] (original id
+ *     of each stored row), vec (uint8|fp32)[N][D] stored in (code, cluster, id)
+ *     order; version 2: the middle layers, per layer W f32[w][previous width]
+ *     then its bias f32[w]. Rows: uint8 or fp32 up to 1 KB, fp32 up to 8 KB
+ *     (D <= 2048, a multiple of 64 bytes).
  */
 #ifndef NEUROUTE_H
 #define NEUROUTE_H
