@@ -46,6 +46,7 @@ OPERATING_POINTS = {
     # the random four-hidden-layer encoder in 1536 dims tops out at Recall@10
     # 0.876 within P <= 1024 (P K_max <= 16384): the point nearest the band
     "f32-1536": dict(P=1024, C=2048, t_low=256),
+    "f32-1536-1m": dict(P=1024, C=2048, t_low=256),  # profiling proxy of f32-1536
 }
 DEFAULT_POINT = dict(P=64, C=128, t_low=4)
 CALIB_QUERIES = 10000

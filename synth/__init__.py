@@ -134,6 +134,9 @@ WORKLOADS = {
     # shape 1536 -> 512 -> 256 -> 128 -> 64 -> 16 (four hidden layers), b = 16
     "f32-1536": Workload("f32-1536", 10_000_000, 1536, "f32", 1024, 0.3, 10_000, 512, 16, 16, 64,
                          mid=(256, 128, 64)),
+    # the same at 1e6 rows (6 GB): small enough for full kernel profiles
+    "f32-1536-1m": Workload("f32-1536-1m", 1_000_000, 1536, "f32", 1024, 0.3, 10_000, 512, 16, 16, 64,
+                            mid=(256, 128, 64)),
 }
 
 
