@@ -43,8 +43,8 @@ OPERATING_POINTS = {
     "u8-100m": dict(P=1024, C=256, t_low=32),
     "u8-1b": dict(P=1024, C=1024, t_low=80, cq=0.9, cov=0.99),
     "u8-30m": dict(P=1024, C=1024, t_low=80, cq=0.9, cov=0.99),  # profiling proxy of u8-1b
-    # the random four-hidden-layer encoder in 1536 dims tops out at Recall@10
-    # 0.876 within P <= 1024 (P K_max <= 16384): the point nearest the band
+    # the random four-hidden-layer encoder in 1536 dims is a weak hash: Recall@10
+    # 0.876 at P = 1024 (sweep in the design notes)
     "f32-1536": dict(P=1024, C=2048, t_low=256),
     "f32-1536-1m": dict(P=1024, C=2048, t_low=256),  # profiling proxy of f32-1536
 }
@@ -562,6 +562,8 @@ def calibration_observations(w, ix, P, C, k, nq=CALIB_QUERIES, budget=None, bins
     t0 = time.time()
     dev = torch.device("cuda", ix.device)
     cq = torch.from_numpy(synth.calib_queries(w, nq)).to(dev)
+    # the target run's probe budget: twice the operating point's, with at most
+    # 16,384 candidate clusters a query, which bounds the calibration's cost
     cP, cC = budget or (min(4096, 2 * P, 16384 // ix.k_max), min(4096, 4 * C))
     lg = ix.encode(cq)
     targets = cal.targets_high_recall(ix, cq, lg, k, cP, cC)
@@ -702,7 +704,7 @@ def main():
         for combo in itertools.product(*(g[k] for k in names)):
             cfg = dict(zip(names, combo))
             Pp, Cc, m1 = cfg["P"], cfg["C"], cfg["m1"]
-            if Pp * ix.k_max > 16384:
+            if Pp * ix.k_max > 65536:
                 continue
             kw = {k: v for k, v in cfg.items() if k not in ("P", "C", "m1", "cq", "cov")}
             if m1 is not None:

@@ -231,7 +231,7 @@ nr_status nr_route(nr_index *ix, const float *d_logits, int64_t nq, int probe_bu
 /* Ordered cluster list C^dir U C^cent (Sec. 3.4.2) from d_logits:
  * d_clusters [nq x (probe_budget + cluster_budget)] int32 cluster indices sorted
  * by (centroid distance, cluster index), -1 padded; d_ncl [nq] their count.
- * Limits: 1 <= cluster_budget <= 4096; probe_budget * K_max <= 16384. */
+ * Limits: 1 <= cluster_budget <= 4096; probe_budget * K_max <= 65536. */
 nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int probe_budget,
                             int cluster_budget, int32_t *d_clusters, int32_t *d_ncl,
                             void *stream);
@@ -241,7 +241,7 @@ nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int
  * row sorted by (distance, id), padded with (-1, +inf) when fewer than k rows
  * were scored. For uint8 indexes distances are the exact integer sums.
  * 1 <= k <= 256, 1 <= probe_budget <= 4096, 1 <= cluster_budget <= 4096,
- * probe_budget * K_max <= 16384. The library's workspace grows on demand. */
+ * probe_budget * K_max <= 65536. The library's workspace grows on demand. */
 nr_status nr_search(nr_index *ix, const void *d_queries, int64_t nq, int k, int probe_budget,
                     int cluster_budget, int64_t *d_out_ids, float *d_out_dists, void *stream);
 

@@ -403,6 +403,46 @@ def test_select_overflow_to_global_slab(many_clusters, torch, C, m1):
     assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
 
 
+@pytest.fixture(scope="module")
+def wide(torch, tmp_path_factory):
+    """b = 12, up to 16 clusters per bucket, so that P = 2048 and 4096 give
+    probe_budget * K_max of 32,768 and 65,536 (the largest select sort)."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, base, info = build_small(tmp_path_factory.mktemp("wide"), "tiny", n=40000, bits=12,
+                                   k_max=16, t=2, name="wide")
+    w = synth.WORKLOADS["tiny"]
+    qs = synth.queries(w, 64)
+    orc = oracle.Index(path)
+    lg = orc.encode(qs)
+    return {"ix": nr.Index(path, 0), "orc": orc, "q": qs, "lg": lg, "info": info,
+            "dq": torch.from_numpy(qs).cuda(), "dl": torch.from_numpy(lg).cuda()}
+
+
+@pytest.mark.parametrize("P,C", [(2048, 4096), (4096, 1024)])
+def test_select_largest_budgets(wide, torch, P, C):
+    ix, orc = wide["ix"], wide["orc"]
+    kw = dict(t_low=4, gate_m0=0.0, gate_m1=1.0)
+    ix.set_params(**kw)
+    try:
+        cl, ncl = ix.debug_clusters(wide["dl"], P, C)
+        ids, d = ix.search_logits(wide["dq"], wide["dl"], 10, P, C)
+        st = ix.query_stats(len(wide["q"]))
+        torch.cuda.synchronize()
+    finally:
+        ix.set_params()
+    cl, ncl = cl.cpu().numpy(), ncl.cpu().numpy()
+    tau = orc.tau()
+    p = oracle.params(**kw)
+    for i in range(0, len(wide["q"]), 4):
+        codes, _, _ = oracle.probe_list(wide["lg"][i], tau, P, p)
+        L, _, _ = orc.cluster_list(wide["lg"][i], codes, C, p)
+        assert ncl[i] == len(L) and np.array_equal(cl[i, : len(L)], L), i
+    ids_o, d_o, st_o = orc.search(wide["q"], 10, P, C, p, logits=wide["lg"])
+    assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
+    assert np.array_equal(st.cpu().numpy(), st_o)
+
+
 @pytest.mark.parametrize("workload", ["tiny", "u8-10m", "f32-10m"])
 def test_encoder_large_batch(torch, tmp_path, workload):
     """Large batches (many 128-row tiles) through the tensor-core encoder, for
