@@ -22,23 +22,7 @@ constexpr int kMaxSelect = 65536;  // probe_budget * K_max (beyond 2,048: sorted
 constexpr int kMaxTopK = 256;
 constexpr size_t kChunkBudget = (size_t)4 << 30;  // workspace bytes per query chunk
 
-struct DeviceGuard {
-  int prev = -1;
-  explicit DeviceGuard(int dev) {
-    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
-    if (prev != dev) cudaSetDevice(dev);
-  }
-  ~DeviceGuard() {
-    int cur = -1;
-    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
-  }
-};
 
-nr_status cuda_status(cudaError_t e) {
-  if (e == cudaSuccess) return NR_OK;
-  if (e == cudaErrorMemoryAllocation) return NR_ERR_OOM;
-  return NR_ERR_CUDA;
-}
 
 uint32_t rd32(const unsigned char *h, int o) {
   uint32_t v;

@@ -31,23 +31,7 @@ constexpr int kMaxSample = 4096;   // sample_per_cluster
 constexpr int64_t kWarpRows = 4096;  // buckets up to this size: one warp; larger: one CTA
 constexpr int kCtaThreads = 256;
 
-struct DeviceGuard {
-  int prev = -1;
-  explicit DeviceGuard(int dev) {
-    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
-    if (prev != dev) cudaSetDevice(dev);
-  }
-  ~DeviceGuard() {
-    int cur = -1;
-    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
-  }
-};
 
-nr_status cuda_status(cudaError_t e) {
-  if (e == cudaSuccess) return NR_OK;
-  cudaGetLastError();
-  return e == cudaErrorMemoryAllocation ? NR_ERR_OOM : NR_ERR_CUDA;
-}
 
 // ---------------------------------------------------------------------------
 // Arithmetic of the build definition (identical on the host builder)

@@ -11,23 +11,7 @@
 
 namespace {
 
-struct DeviceGuard {
-  int prev = -1;
-  explicit DeviceGuard(int dev) {
-    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
-    if (prev != dev) cudaSetDevice(dev);
-  }
-  ~DeviceGuard() {
-    int cur = -1;
-    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
-  }
-};
 
-nr_status cuda_status(cudaError_t e) {
-  if (e == cudaSuccess) return NR_OK;
-  cudaGetLastError();
-  return e == cudaErrorMemoryAllocation ? NR_ERR_OOM : NR_ERR_CUDA;
-}
 
 __global__ void iota_kernel(uint32_t *v, int64_t n) {
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;

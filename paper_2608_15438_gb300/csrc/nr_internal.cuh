@@ -6,6 +6,26 @@
 
 #include "neuroute.h"
 
+// Makes `dev` the current device for a scope and restores the caller's.
+struct DeviceGuard {
+  int prev = -1;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+    if (prev != dev) cudaSetDevice(dev);
+  }
+  ~DeviceGuard() {
+    int cur = -1;
+    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+  }
+};
+
+// Library status of a CUDA result; clears the runtime's last error.
+inline nr_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return NR_OK;
+  cudaGetLastError();
+  return e == cudaErrorMemoryAllocation ? NR_ERR_OOM : NR_ERR_CUDA;
+}
+
 // Device-side check codes (first one wins; the host maps any to NR_ERR_DEVICE_CHECK)
 enum : int {
   NR_DEV_OK = 0,
