@@ -158,6 +158,7 @@ nr_status nr_index_init_device(nr_index *ix) {
     return NR_ERR_CUDA;
   }
   ix->num_sms = prop.multiProcessorCount;
+  ix->smem_optin = (int)prop.sharedMemPerBlockOptin;
   if (cudaMalloc((void **)&ix->d_err, 16) != cudaSuccess) {
     cudaGetLastError();
     ix->d_err = nullptr;
@@ -214,12 +215,19 @@ nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1
     if ((st = up((void **)&ix->WmT, t.data(), n * 4)) != NR_OK) return st;
     return NR_OK;  // the tensor-core encoder covers one hidden layer only
   }
-  // fp16 operands of the tensor-core encoder; layer 2 padded to 16 or 32 rows
+  // fp16 operands of the tensor-core encoder in its chunked operand order;
+  // layer 2 padded to 16 or 32 rows (only shapes that kernel takes)
+  if (D % 16 != 0 || H % 128 != 0 || b > 32) return NR_OK;
   const int n2 = b <= 16 ? 16 : 32;
   std::vector<__half> w1h((size_t)H * D), w2h((size_t)n2 * H, __float2half_rn(0.0f));
-  for (size_t i = 0; i < w1h.size(); ++i) w1h[i] = __float2half_rn(W1[i]);
+  for (int u = 0; u < H; ++u)
+    for (int j = 0; j < D; ++j)
+      w1h[(size_t)(u / 128) * 128 * D + nr_tc_kmajor_off(u % 128, j / 8, D / 8) / 2 + j % 8] =
+          __float2half_rn(W1[(size_t)u * D + j]);
   for (int o = 0; o < b; ++o)
-    for (int u = 0; u < H; ++u) w2h[(size_t)o * H + u] = __float2half_rn(W2[(size_t)o * H + u]);
+    for (int u = 0; u < H; ++u)
+      w2h[(size_t)(u / 128) * n2 * 128 + nr_tc_kmajor_off(o, (u % 128) / 8, 16) / 2 + u % 8] =
+          __float2half_rn(W2[(size_t)o * H + u]);
   if ((st = up(&ix->W1h, w1h.data(), w1h.size() * 2)) != NR_OK) return st;
   if ((st = up(&ix->W2h, w2h.data(), w2h.size() * 2)) != NR_OK) return st;
   return NR_OK;

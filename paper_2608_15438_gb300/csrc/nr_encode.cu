@@ -1,23 +1,30 @@
 // K1 encode: l = E(x), one hidden layer (Sec. 3.2.1):
 //   h = ReLU(s (W1 x) + b1),  l = W2 h + b2.
 //
-// Tensor-core version (tcgen05, sm_103a). One CTA of 4 warps owns 128 query
-// rows = the 128 TMEM lanes of its accumulators. Layer 1 runs in chunks of 128
-// hidden units: one thread issues tcgen05.mma (kind::f16, fp16 operands, fp32
-// accumulation in TMEM) over X [128 x D] and a W1 chunk [128 x D]; the four
-// warps read the chunk back with tcgen05.ld, apply scale, bias and ReLU, and
-// write it as fp16 into shared memory, where it becomes the A operand of the
-// layer-2 MMA that accumulates l [128 x N2] (N2 = b padded to 16 or 32) in a
-// second TMEM region across all chunks. Operands sit in shared memory in the
-// canonical K-major no-swizzle layout (8-row x 16-byte core matrices; core
-// matrices of one 8-row group consecutive along K). uint8 inputs are exact in
-// fp16; the input scale is applied to the fp32 accumulator.
+// Tensor-core version (tcgen05, sm_103a), persistent and warp-specialised:
+// one CTA per SM walks 128-row tiles (the 128 TMEM lanes of its accumulators).
+// Layer 1 runs in chunks of 128 hidden units: one thread issues tcgen05.mma
+// (kind::f16, fp16 operands, fp32 accumulation in TMEM) over the X tile and a
+// W1 chunk that a loader thread brought in by bulk async copy (a ring of three
+// chunks); eight epilogue warps read each accumulator back with tcgen05.ld,
+// apply scale, bias and ReLU and write the chunk as fp16 into shared memory,
+// where it becomes the A operand of the layer-2 MMAs that accumulate
+// l [128 x N2] (N2 = b padded to 16 or 32) against W2, which stays resident in
+// shared memory. Two layer-1 accumulators and two X tiles let the tensor pipe
+// work on the next chunk while the epilogue converts the previous one; four
+// converter warps turn the next X tile into fp16 meanwhile (uint8 inputs are
+// exact in fp16; the input scale is applied to the fp32 accumulator). Every
+// hand-off is an mbarrier: bulk-copy transaction bytes, tcgen05.commit, or
+// thread arrivals. Operands sit in shared memory in the canonical K-major
+// no-swizzle layout (nr_tc_kmajor_off); the host stores W1 and W2 in it.
 //
-// Every wait on an MMA completion barrier is bounded (1 s); on timeout the
-// kernel records NR_DEV_TIMEOUT, frees its TMEM and returns.
+// Every wait is bounded (1 s); when one expires every role stops, the CTA
+// waits (again bounded) for its own copies and MMAs in flight, records
+// NR_DEV_TIMEOUT, frees its TMEM and returns.
 //
-// Shapes the tensor-core kernel does not take (D % 16 != 0, D > 256,
-// H % 128 != 0, b > 32) run on the CUDA-core kernel below it.
+// Shapes the tensor-core kernel does not take (D % 16 != 0, D > 128,
+// H % 128 != 0, b > 32, or more shared memory than a CTA has) run on the
+// CUDA-core kernels below it.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -108,11 +115,6 @@ __device__ __forceinline__ void tc_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory");
 }
 
-// byte offset of (row r, 16-byte K chunk c) in a K-major no-swizzle tile with
-// kchunks chunks per row
-__device__ __forceinline__ uint32_t kmajor_off(int r, int c, int kchunks) {
-  return (uint32_t)((r & 7) * 16 + (r >> 3) * kchunks * 128 + c * 128);
-}
 // shared-memory matrix descriptor: start, leading (K) and stride (8-row group)
 // byte offsets, descriptor version 1, no swizzle
 __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
@@ -124,153 +126,422 @@ __host__ __device__ constexpr uint32_t mma_idesc(int M, int N) {
   return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
-constexpr int kRows = 128;  // query rows per CTA
-constexpr int kHC = 128;    // hidden units per chunk
-constexpr uint32_t kTmemCols = 256;
+// ------------------------------------------------------------ tensor-core kernel
+constexpr int kRows = 128;     // rows per tile = TMEM lanes of the accumulators
+constexpr int kHC = 128;       // hidden units per layer-1 chunk
+constexpr int kEpiWarps = 8;   // two per TMEM lane group, one column half of a chunk each
+constexpr int kConvWarps = 4;
+constexpr int kWarpMma = 0, kWarpLoad = 1, kWarpEpi = 2, kWarpConv = kWarpEpi + kEpiWarps;
+constexpr int kTcThreads = 32 * (kWarpConv + kConvWarps);  // 448
+constexpr int kEpiThreads = 32 * kEpiWarps, kConvThreads = 32 * kConvWarps;
+// TMEM columns: layer-1 accumulators at 0 and 128, layer-2 accumulators at 256 and 288
+constexpr uint32_t kTmemCols = 512;
+constexpr int kMaxStages = 3;  // W1 chunk ring
 
+struct TcBars {
+  uint64_t xfull[2], xempty[2];                    // X tiles: converters -> MMA -> converters
+  uint64_t wfull[kMaxStages], wempty[kMaxStages];  // W1 chunks: bulk copy -> MMA -> loader
+  uint64_t a1full[2], a1empty[2];                  // layer-1 accumulators: MMA -> epilogue -> MMA
+  uint64_t hfull, hempty;                          // hidden chunk operand: epilogue -> MMA -> epilogue
+  uint64_t a2full[2], a2empty[2];                  // layer-2 accumulators
+  uint64_t drain;                                  // every MMA of the CTA complete
+  uint32_t tmem_slot;
+  int abort;                                       // a wait expired: every role stops
+};
+
+// byte offsets of the shared-memory regions for a shape (host and device)
+struct TcLayout {
+  uint32_t x, w1, w2, h, b1, b2, bars, total;
+};
+__host__ __device__ inline TcLayout tc_layout(int D, int H, int n2, int stages) {
+  TcLayout L;
+  uint32_t o = 0;
+  L.x = o;  o += 2u * kRows * (uint32_t)D * 2u;              // two fp16 X tiles
+  L.w1 = o; o += (uint32_t)stages * kHC * (uint32_t)D * 2u;  // W1 chunk ring
+  L.w2 = o; o += (uint32_t)n2 * (uint32_t)H * 2u;            // all of W2, resident
+  L.h = o;  o += kRows * kHC * 2u;                           // one fp16 hidden chunk
+  L.b1 = o; o += (uint32_t)H * 4u;
+  L.b2 = o; o += 32u * 4u;
+  L.bars = o; o += (uint32_t)sizeof(TcBars);
+  L.total = o;
+  return L;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}\n" ::"r"(bar),
+               "r"(bytes)
+               : "memory");
+}
+// bulk copy global -> shared, completion counted on the barrier's transaction bytes
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+// Waits for the barrier phase of the given parity. Gives up when another role
+// has given up, or after ~1 s, which makes every role give up.
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, volatile int *abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+    if (global_ns() - t0 > 1000000000ull) {
+      *abort = 1;
+      return false;
+    }
+  }
+}
+// the same, one decision for the whole warp (all lanes wait)
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort) {
+  return __all_sync(0xffffffffu, wait_or_abort(bar, parity, abort)) != 0;
+}
+// 16 bytes of uint8 as 16 fp16 values, exactly: 0x64XX is the fp16 number 1024 + XX
+__device__ __forceinline__ void u8x16_to_f16(const uint4 v, uint4 &lo, uint4 &hi) {
+  const __half2 k1024 = __halves2half2(__ushort_as_half(0x6400), __ushort_as_half(0x6400));
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t p0 = __byte_perm(w[i], 0x64646464u, 0x4140), p1 = __byte_perm(w[i], 0x64646464u, 0x4342);
+    const __half2 h0 = __hsub2(*reinterpret_cast<const __half2 *>(&p0), k1024);
+    const __half2 h1 = __hsub2(*reinterpret_cast<const __half2 *>(&p1), k1024);
+    o[2 * i] = *reinterpret_cast<const uint32_t *>(&h0);
+    o[2 * i + 1] = *reinterpret_cast<const uint32_t *>(&h1);
+  }
+  lo = make_uint4(o[0], o[1], o[2], o[3]);
+  hi = make_uint4(o[4], o[5], o[6], o[7]);
+}
+
+// Persistent, warp-specialised: each CTA (one per SM) takes 128-row tiles
+// tile = blockIdx.x, + gridDim.x, ... and streams them through
+//   converter warps  X tile -> fp16 operand (two buffers)
+//   loader thread    W1 chunk c (128 hidden units, operand order) -> ring of `stages` by bulk copy
+//   MMA thread       layer 1 of chunk g into accumulator g % 2, then layer 2 of chunk g - 1
+//   epilogue warps   accumulator -> ReLU(s acc + b1) -> fp16 hidden chunk; after a tile's
+//                    last chunk its layer-2 accumulator + b2 -> out
+// so that the tensor pipe runs layer 1 of the next chunk while the epilogue
+// turns the previous one into the layer-2 operand. W2 stays in shared memory.
 template <int DT>
-__global__ void __launch_bounds__(128, 1)
-    encode_tc_kernel(const void *__restrict__ x, int D, int H, int b, int n2, float s,
-                     const __half *__restrict__ W1h, const float *__restrict__ b1,
-                     const __half *__restrict__ W2h, const float *__restrict__ b2, int64_t nq,
+__global__ void __launch_bounds__(kTcThreads, 1)
+    encode_tc_kernel(const void *__restrict__ x, int D, int H, int b, int n2, int stages, float s,
+                     const __half *__restrict__ W1p, const float *__restrict__ b1,
+                     const __half *__restrict__ W2p, const float *__restrict__ b2, int64_t nq,
                      float *__restrict__ out, int *err) {
   extern __shared__ __align__(1024) unsigned char smem[];
+  const TcLayout L = tc_layout(D, H, n2, stages);
+  TcBars &B = *reinterpret_cast<TcBars *>(smem + L.bars);
+  volatile int *abort = &B.abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int kx = D / 8;  // 16-byte chunks per row of X and W1
-  unsigned char *sX = smem;                            // [128][D] fp16
-  unsigned char *sW1 = sX + kRows * D * 2;             // [128][D] fp16
-  unsigned char *sH = sW1 + kHC * D * 2;               // [128][128] fp16
-  unsigned char *sW2 = sH + kRows * kHC * 2;           // [n2][128] fp16
-  float *sb1 = reinterpret_cast<float *>(sW2 + n2 * kHC * 2);  // [128]
-  uint64_t *mbar = reinterpret_cast<uint64_t *>(sb1 + kHC);
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 1);
-  const uint32_t bar = smem_u32(mbar);
-  const int64_t row0 = (int64_t)blockIdx.x * kRows;
+  const int kx = D / 8;      // 16-byte K chunks per row of X and W1
+  const int nc = H / kHC;    // layer-1 chunks per tile
+  const uint32_t x_bytes = (uint32_t)kRows * D * 2, w1_bytes = (uint32_t)kHC * D * 2;
+  const uint32_t w2_bytes = (uint32_t)n2 * kHC * 2;  // one chunk of W2
+  const int64_t ntiles = (nq + kRows - 1) / kRows;
+  const uint32_t sbase = smem_u32(smem);
+  float *sb1 = reinterpret_cast<float *>(smem + L.b1);
+  float *sb2 = reinterpret_cast<float *>(smem + L.b2);
 
-  if (warp == 0) {
-    tc_alloc(smem_u32(tmem_slot), kTmemCols);
+  if (warp == kWarpMma) {
+    tc_alloc(smem_u32(&B.tmem_slot), kTmemCols);
     tc_relinquish();
   }
   if (tid == 0) {
-    mbar_init(bar, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&B.xfull[i]), kConvThreads);
+      mbar_init(smem_u32(&B.xempty[i]), 1);
+      mbar_init(smem_u32(&B.a1full[i]), 1);
+      mbar_init(smem_u32(&B.a1empty[i]), kEpiThreads);
+      mbar_init(smem_u32(&B.a2full[i]), 1);
+      mbar_init(smem_u32(&B.a2empty[i]), kEpiThreads);
+    }
+    for (int i = 0; i < stages; ++i) {
+      mbar_init(smem_u32(&B.wfull[i]), 1);
+      mbar_init(smem_u32(&B.wempty[i]), 1);
+    }
+    mbar_init(smem_u32(&B.hfull), kEpiThreads);
+    mbar_init(smem_u32(&B.hempty), 1);
+    mbar_init(smem_u32(&B.drain), 1);
+    B.abort = 0;
     fence_mbar_init();
   }
-  // X tile to fp16 (rows past nq are zero)
-  // thread i fills row 8 (i / 8 / kx) + i % 8, chunk (i / 8) % kx: eight
-  // consecutive threads write one 128-byte core matrix (no bank conflicts)
-  for (int i = tid; i < kRows * kx; i += 128) {
-    const int c = (i >> 3) % kx, r = ((i >> 3) / kx) * 8 + (i & 7);
-    const int64_t row = row0 + r;
-    __align__(16) __half hv[8];
-    if (row < nq) {
-      if (DT == 0) {
-        const uint2 v = *reinterpret_cast<const uint2 *>(static_cast<const uint8_t *>(x) + row * D + c * 8);
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          hv[e] = __uint2half_rn((v.x >> (8 * e)) & 0xffu);
-          hv[4 + e] = __uint2half_rn((v.y >> (8 * e)) & 0xffu);
-        }
-      } else {
-        const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(x) + row * D + c * 8);
-        const float4 u = src[0], w = src[1];
-        hv[0] = __float2half_rn(u.x); hv[1] = __float2half_rn(u.y);
-        hv[2] = __float2half_rn(u.z); hv[3] = __float2half_rn(u.w);
-        hv[4] = __float2half_rn(w.x); hv[5] = __float2half_rn(w.y);
-        hv[6] = __float2half_rn(w.z); hv[7] = __float2half_rn(w.w);
-      }
-    } else {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) hv[e] = __float2half_rn(0.0f);
-    }
-    *reinterpret_cast<uint4 *>(sX + kmajor_off(r, c, kx)) = *reinterpret_cast<const uint4 *>(hv);
-  }
+  // resident operands: W2 (already in operand order) and the biases
+  for (int i = tid; i < n2 * H / 8; i += kTcThreads)
+    reinterpret_cast<uint4 *>(smem + L.w2)[i] = reinterpret_cast<const uint4 *>(W2p)[i];
+  for (int i = tid; i < H; i += kTcThreads) sb1[i] = b1[i];
+  if (tid < 32) sb2[tid] = tid < b ? b2[tid] : 0.0f;
+  fence_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  const uint32_t d1 = tmem, d2 = tmem + kHC;
-  const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
-  const int r = warp * 32 + lane;  // this thread's row = TMEM lane
-  const uint32_t idesc1 = mma_idesc(kRows, kHC), idesc2 = mma_idesc(kRows, n2);
-  uint32_t phase = 0;
-  int ok = 1;
-  for (int hc = 0; hc < H / kHC && ok; ++hc) {
-    // operands of this chunk: W1 rows [hc*128, +128), W2 columns [hc*128, +128)
-    for (int i = tid; i < kHC * kx; i += 128) {
-      const int c = (i >> 3) % kx, n = ((i >> 3) / kx) * 8 + (i & 7);
-      *reinterpret_cast<uint4 *>(sW1 + kmajor_off(n, c, kx)) =
-          *reinterpret_cast<const uint4 *>(W1h + (size_t)(hc * kHC + n) * D + c * 8);
-    }
-    for (int i = tid; i < n2 * 16; i += 128) {
-      const int c = (i >> 3) & 15, n = (i >> 7) * 8 + (i & 7);
-      *reinterpret_cast<uint4 *>(sW2 + kmajor_off(n, c, 16)) =
-          *reinterpret_cast<const uint4 *>(W2h + (size_t)n * H + hc * kHC + c * 8);
-    }
-    sb1[tid] = b1[hc * kHC + tid];
-    fence_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      for (int ks = 0; ks < D / 16; ++ks)
-        tc_mma_f16(d1, smem_desc(smem_u32(sX) + ks * 256, 128, kx * 128),
-                   smem_desc(smem_u32(sW1) + ks * 256, 128, kx * 128), idesc1, ks > 0 ? 1u : 0u);
-      tc_commit(bar);
-    }
-    ok = __syncthreads_and(mbar_wait_bounded(bar, phase));
-    phase ^= 1;
-    if (!ok) break;
-    tc_fence_after();
-    // h = ReLU(s * acc + b1) -> fp16 A operand of layer 2
-#pragma unroll 1
-    for (int cb = 0; cb < kHC; cb += 32) {
-      uint32_t v[32];
-      tc_ld32(d1 + lane_base + (uint32_t)cb, v);
-      tc_wait_ld();
-#pragma unroll
-      for (int j8 = 0; j8 < 4; ++j8) {
-        __align__(16) __half hv[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int j = cb + j8 * 8 + e;
-          const float h = __fmaf_rn(s, __uint_as_float(v[j8 * 8 + e]), sb1[j]);
-          hv[e] = __float2half_rn(h > 0.0f ? h : 0.0f);
+  const uint32_t tmem = B.tmem_slot;
+
+  if (warp == kWarpMma) {
+    if (lane == 0) {
+      const uint32_t idesc1 = mma_idesc(kRows, kHC), idesc2 = mma_idesc(kRows, n2);
+      const uint32_t sx = sbase + L.x, sw1 = sbase + L.w1, sw2 = sbase + L.w2, sh = sbase + L.h;
+      // layer 2 of chunk number gp (chunk cp of tile number ip of this CTA):
+      // hidden chunk x W2 chunk into the tile's accumulator
+      auto layer2 = [&](uint32_t gp, uint32_t ip, int cp) -> bool {
+        if (!wait_or_abort(smem_u32(&B.hfull), gp & 1u, abort)) return false;
+        if (cp == 0 && !wait_or_abort(smem_u32(&B.a2empty[ip & 1]), ((ip >> 1) & 1u) ^ 1u, abort))
+          return false;
+        tc_fence_after();
+        const uint32_t d2 = tmem + 256u + (ip & 1u) * 32u;
+        for (int ks = 0; ks < kHC / 16; ++ks)
+          tc_mma_f16(d2, smem_desc(sh + ks * 256, 128, 16 * 128),
+                     smem_desc(sw2 + (uint32_t)cp * w2_bytes + ks * 256, 128, 16 * 128), idesc2,
+                     (cp > 0 || ks > 0) ? 1u : 0u);
+        tc_commit(smem_u32(&B.hempty));
+        if (cp == nc - 1) tc_commit(smem_u32(&B.a2full[ip & 1]));
+        return true;
+      };
+      bool ok = true;
+      uint32_t g = 0, it = 0;  // chunks and tiles of this CTA so far
+      int st = 0;              // W1 ring slot of chunk g ...
+      uint32_t wpar = 0;       // ... and the parity of its fill
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+        const int xb = (int)(it & 1);
+        if (!wait_or_abort(smem_u32(&B.xfull[xb]), (it >> 1) & 1u, abort)) {
+          ok = false;
+          break;
         }
-        *reinterpret_cast<uint4 *>(sH + kmajor_off(r, (cb >> 3) + j8, 16)) =
-            *reinterpret_cast<const uint4 *>(hv);
+        for (int c = 0; c < nc; ++c, ++g) {
+          const int a = (int)(g & 1);
+          if (!wait_or_abort(smem_u32(&B.wfull[st]), wpar, abort) ||
+              !wait_or_abort(smem_u32(&B.a1empty[a]), ((g >> 1) & 1u) ^ 1u, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d1 = tmem + (uint32_t)a * kHC;
+          for (int ks = 0; ks < D / 16; ++ks)
+            tc_mma_f16(d1, smem_desc(sx + (uint32_t)xb * x_bytes + ks * 256, 128, kx * 128),
+                       smem_desc(sw1 + (uint32_t)st * w1_bytes + ks * 256, 128, kx * 128), idesc1,
+                       ks > 0 ? 1u : 0u);
+          tc_commit(smem_u32(&B.wempty[st]));
+          tc_commit(smem_u32(&B.a1full[a]));
+          if (c == nc - 1) tc_commit(smem_u32(&B.xempty[xb]));
+          if (++st == stages) {
+            st = 0;
+            wpar ^= 1u;
+          }
+          if (g > 0 && !layer2(g - 1, c > 0 ? it : it - 1, c > 0 ? c - 1 : nc - 1)) {
+            ok = false;
+            break;
+          }
+        }
+      }
+      if (ok && g > 0) layer2(g - 1, it - 1, nc - 1);
+      // every MMA of this thread completes before TMEM is freed
+      tc_commit(smem_u32(&B.drain));
+      mbar_wait_bounded(smem_u32(&B.drain), 0);
+    }
+    __syncwarp();
+  } else if (warp == kWarpLoad) {
+    if (lane == 0) {
+      int st = 0;
+      uint32_t wpar = 0, issued = 0, lastpar = 0;  // per ring slot: a copy issued, parity of the last
+      bool ok = true;
+      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x)
+        for (int c = 0; c < nc; ++c) {
+          if (!wait_or_abort(smem_u32(&B.wempty[st]), wpar ^ 1u, abort)) {
+            ok = false;
+            break;
+          }
+          mbar_expect_tx(smem_u32(&B.wfull[st]), w1_bytes);
+          bulk_g2s(sbase + L.w1 + (uint32_t)st * w1_bytes, W1p + (size_t)c * kHC * D, w1_bytes,
+                   smem_u32(&B.wfull[st]));
+          issued |= 1u << st;
+          lastpar = (lastpar & ~(1u << st)) | (wpar << st);
+          if (++st == stages) {
+            st = 0;
+            wpar ^= 1u;
+          }
+        }
+      // copies still in flight land before the CTA exits
+      for (int q = 0; q < stages; ++q)
+        if ((issued >> q) & 1u) mbar_wait_bounded(smem_u32(&B.wfull[q]), (lastpar >> q) & 1u);
+    }
+    __syncwarp();
+  } else if (warp < kWarpConv) {
+    const int lg = warp & 3;                 // TMEM lane group this warp may read
+    const int hh = (warp - kWarpEpi) >> 2;   // column half of each chunk
+    const int r = lg * 32 + lane;            // tile row = TMEM lane
+    const uint32_t lane_base = (uint32_t)(lg * 32) << 16;
+    unsigned char *sH = smem + L.h;
+    uint32_t g = 0, it = 0;
+    bool ok = true;
+    for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
+      for (int c = 0; c < nc; ++c, ++g) {
+        const int a = (int)(g & 1);
+        if (!warp_wait(smem_u32(&B.a1full[a]), (uint32_t)((g >> 1) & 1), abort)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        // h = ReLU(s acc + b1) as fp16 pairs, 32 accumulator columns at a time
+        const uint32_t col = tmem + lane_base + (uint32_t)a * kHC + (uint32_t)hh * 64u;
+        const float *bb = sb1 + c * kHC + hh * 64;
+        uint32_t hp[32];
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          float bv[32];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4 *>(&bv[4 * j]) = reinterpret_cast<const float4 *>(bb + 32 * half)[j];
+          uint32_t v[32];
+          tc_ld32(col + 32u * half, v);
+          tc_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float h0 = __fmaf_rn(s, __uint_as_float(v[2 * j]), bv[2 * j]);
+            const float h1 = __fmaf_rn(s, __uint_as_float(v[2 * j + 1]), bv[2 * j + 1]);
+            const __half2 p = __floats2half2_rn(h0 > 0.0f ? h0 : 0.0f, h1 > 0.0f ? h1 : 0.0f);
+            hp[16 * half + j] = *reinterpret_cast<const uint32_t *>(&p);
+          }
+        }
+        tc_fence_before();
+        mbar_arrive(smem_u32(&B.a1empty[a]));
+        // the previous chunk's layer-2 MMAs have read the hidden operand
+        if (!warp_wait(smem_u32(&B.hempty), (uint32_t)((g & 1) ^ 1), abort)) {
+          ok = false;
+          break;
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+          *reinterpret_cast<uint4 *>(sH + nr_tc_kmajor_off(r, hh * 8 + q, kHC / 8)) =
+              make_uint4(hp[4 * q], hp[4 * q + 1], hp[4 * q + 2], hp[4 * q + 3]);
+        fence_async_smem();
+        mbar_arrive(smem_u32(&B.hfull));
+      }
+      if (!ok) break;
+      // the tile's logits: layer-2 accumulator + b2
+      if (!warp_wait(smem_u32(&B.a2full[it & 1]), (uint32_t)((it >> 1) & 1), abort)) break;
+      tc_fence_after();
+      uint32_t o[16];
+      const bool reads = hh * 16 < n2;  // same for the whole warp
+      if (reads) {
+        tc_ld16(tmem + lane_base + 256u + (uint32_t)(it & 1) * 32u + (uint32_t)hh * 16u, o);
+        tc_wait_ld();
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&B.a2empty[it & 1]));
+      const int64_t row = tile * kRows + r;
+      if (reads && row < nq) {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int oc = hh * 16 + j;
+          if (oc < b) out[row * b + oc] = __fadd_rn(__uint_as_float(o[j]), sb2[oc]);
+        }
       }
     }
-    fence_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      for (int ks = 0; ks < kHC / 16; ++ks)
-        tc_mma_f16(d2, smem_desc(smem_u32(sH) + ks * 256, 128, 16 * 128),
-                   smem_desc(smem_u32(sW2) + ks * 256, 128, 16 * 128), idesc2,
-                   (hc > 0 || ks > 0) ? 1u : 0u);
-      tc_commit(bar);
+  } else {
+    // converters: X tile -> fp16 operand in the K-major core-matrix layout;
+    // eight consecutive threads cover eight rows of one 16-byte K chunk, so a
+    // warp's stores fill whole 128-byte core matrices
+    const int ct = tid - kWarpConv * 32;
+    // item j of this thread: row rr of the tile and piece pc of the row (16 source
+    // bytes = 2 K chunks for uint8, one K chunk of 8 floats for fp32), packed
+    // rr | pc << 8; the same for every tile
+    const int per = DT == 0 ? D / 16 : kx;  // pieces per row = items per thread (<= 8, <= 16)
+    int tab[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int k = (ct >> 3) + 16 * j;
+      tab[j] = (j < per) ? (((k / per) * 8 + (ct & 7)) | ((k % per) << 8)) : 0;
     }
-    ok = __syncthreads_and(mbar_wait_bounded(bar, phase));
-    phase ^= 1;
-    tc_fence_after();
-  }
-  if (ok) {
-    uint32_t v[32];
-    tc_ld32(d2 + lane_base, v);
-    tc_wait_ld();
-    const int64_t row = row0 + r;
-    if (row < nq)
-      for (int j = 0; j < b; ++j) out[row * b + j] = __fadd_rn(__uint_as_float(v[j]), b2[j]);
-  } else if (tid == 0) {
-    atomicCAS(err, 0, NR_DEV_TIMEOUT);
+    uint32_t it = 0;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+      const int xb = (int)(it & 1);
+      unsigned char *sX = smem + L.x + (size_t)xb * x_bytes;
+      const int64_t row0 = tile * kRows;
+      const int rows = nq - row0 < kRows ? (int)(nq - row0) : kRows;  // rows of this tile
+      bool ok = true;
+      if (DT == 0) {
+        const uint8_t *xs = static_cast<const uint8_t *>(x) + row0 * D;
+        uint4 v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int rr = tab[j] & 0xff, pc = tab[j] >> 8;
+          v[j] = make_uint4(0u, 0u, 0u, 0u);
+          if (j < per && rr < rows) v[j] = __ldg(reinterpret_cast<const uint4 *>(xs + rr * D + pc * 16));
+        }
+        ok = warp_wait(smem_u32(&B.xempty[xb]), ((it >> 1) & 1u) ^ 1u, abort);
+        if (ok) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (j >= per) break;
+            const int rr = tab[j] & 0xff, pc = tab[j] >> 8;
+            uint4 lo, hi;
+            u8x16_to_f16(v[j], lo, hi);
+            *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc, kx)) = lo;
+            *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc + 1, kx)) = hi;
+          }
+        }
+      } else {
+        const float *xs = static_cast<const float *>(x) + row0 * D;
+#pragma unroll
+        for (int j0 = 0; j0 < 16; j0 += 8) {
+          if (j0 >= per || !ok) break;
+          float4 u[8], w[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int rr = tab[j0 + j] & 0xff, pc = tab[j0 + j] >> 8;
+            u[j] = w[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            if (j0 + j < per && rr < rows) {
+              const float4 *s4 = reinterpret_cast<const float4 *>(xs + rr * D + pc * 8);
+              u[j] = __ldg(s4);
+              w[j] = __ldg(s4 + 1);
+            }
+          }
+          if (j0 == 0) ok = warp_wait(smem_u32(&B.xempty[xb]), ((it >> 1) & 1u) ^ 1u, abort);
+          if (!ok) break;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            if (j0 + j >= per) break;
+            const int rr = tab[j0 + j] & 0xff, pc = tab[j0 + j] >> 8;
+            const __half2 h0 = __floats2half2_rn(u[j].x, u[j].y), h1 = __floats2half2_rn(u[j].z, u[j].w);
+            const __half2 h2 = __floats2half2_rn(w[j].x, w[j].y), h3 = __floats2half2_rn(w[j].z, w[j].w);
+            *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, pc, kx)) =
+                make_uint4(*reinterpret_cast<const uint32_t *>(&h0), *reinterpret_cast<const uint32_t *>(&h1),
+                           *reinterpret_cast<const uint32_t *>(&h2), *reinterpret_cast<const uint32_t *>(&h3));
+          }
+        }
+      }
+      if (!ok) break;
+      fence_async_smem();
+      mbar_arrive(smem_u32(&B.xfull[xb]));
+    }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (tid == 0 && B.abort) atomicCAS(err, 0, NR_DEV_TIMEOUT);
+  if (warp == kWarpMma) {
     tc_fence_after();
     tc_dealloc(tmem, kTmemCols);
   }
+}
+
+// W1 ring depth for a shape: 3 chunks if a block's shared memory allows, else 2, else 0
+int tc_stages(int D, int H, int n2, int smem_optin) {
+  for (int st = kMaxStages; st >= 2; --st)
+    if (tc_layout(D, H, n2, st).total <= (uint32_t)smem_optin) return st;
+  return 0;
 }
 
 // ------------------------------------------------------------ CUDA-core kernel
@@ -404,24 +675,28 @@ __global__ void __launch_bounds__(kThreads)
 }  // namespace
 
 bool nr_encode_uses_tensor_cores(const nr_index *ix) {
-  return ix->W1h != nullptr && ix->D % 16 == 0 && ix->D <= 256 && ix->H % kHC == 0 && ix->b <= 32;
+  return ix->W1h != nullptr && ix->n_mid == 0 && ix->D % 16 == 0 && ix->D <= 128 &&
+         ix->H % kHC == 0 && ix->b <= 32 &&
+         tc_stages(ix->D, ix->H, ix->b <= 16 ? 16 : 32, ix->smem_optin) > 0;
 }
 
 cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
                              cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
-  if (nr_encode_uses_tensor_cores(ix)) {
+  // the tensor-core kernel reads X in 16-byte pieces
+  if (nr_encode_uses_tensor_cores(ix) && (reinterpret_cast<uintptr_t>(d_x) & 15) == 0) {
     const int n2 = ix->b <= 16 ? 16 : 32;
-    const size_t smem = (size_t)kRows * ix->D * 2 + (size_t)kHC * ix->D * 2 +
-                        (size_t)kRows * kHC * 2 + (size_t)n2 * kHC * 2 + kHC * 4 + 16;
+    const int stages = tc_stages(ix->D, ix->H, n2, ix->smem_optin);
+    const uint32_t smem = tc_layout(ix->D, ix->H, n2, stages).total;
     auto kern = ix->dtype == 0 ? encode_tc_kernel<0> : encode_tc_kernel<1>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const int64_t grid = (nq + kRows - 1) / kRows;
-    kern<<<(unsigned)grid, 128, smem, s>>>(d_x, ix->D, ix->H, ix->b, n2, ix->in_scale,
-                                           static_cast<const __half *>(ix->W1h), ix->b1,
-                                           static_cast<const __half *>(ix->W2h), ix->b2, nq,
-                                           d_logits, ix->d_err);
+    const int64_t tiles = (nq + kRows - 1) / kRows;
+    const int64_t grid = tiles < ix->num_sms ? tiles : ix->num_sms;
+    kern<<<(unsigned)grid, kTcThreads, smem, s>>>(d_x, ix->D, ix->H, ix->b, n2, stages, ix->in_scale,
+                                                  static_cast<const __half *>(ix->W1h), ix->b1,
+                                                  static_cast<const __half *>(ix->W2h), ix->b2, nq,
+                                                  d_logits, ix->d_err);
     ix->launches += 1;
     return cudaGetLastError();
   }

@@ -26,6 +26,15 @@ inline nr_status cuda_status(cudaError_t e) {
   return e == cudaErrorMemoryAllocation ? NR_ERR_OOM : NR_ERR_CUDA;
 }
 
+// Byte offset of (row r, 16-byte K chunk c) in the operand layout of the
+// tensor-core encoder: K-major without swizzle, 8-row x 16-byte core matrices,
+// the core matrices of one 8-row group consecutive along K (kchunks per row).
+// The host writes W1 and W2 in this order; the kernel stages X and the hidden
+// chunks in it.
+__host__ __device__ inline uint32_t nr_tc_kmajor_off(int r, int c, int kchunks) {
+  return (uint32_t)((r & 7) * 16 + (r >> 3) * kchunks * 128 + c * 128);
+}
+
 // Device-side check codes (first one wins; the host maps any to NR_ERR_DEVICE_CHECK)
 enum : int {
   NR_DEV_OK = 0,
@@ -54,8 +63,11 @@ struct nr_index {
   float *W1 = nullptr, *b1 = nullptr, *W2 = nullptr, *b2 = nullptr, *tau = nullptr;
   float *cent = nullptr;
   float *W1T = nullptr;  // [D][H]
-  void *W1h = nullptr;   // fp16 [H][D] (tensor-core encoder)
-  void *W2h = nullptr;   // fp16 [16 or 32][H], rows >= b zero
+  // fp16 operands of the tensor-core encoder, in chunks of 128 hidden units,
+  // each chunk in the nr_tc_kmajor_off order: W1 [128 x D] per chunk, W2
+  // [16 or 32 x 128] per chunk (rows >= b zero)
+  void *W1h = nullptr;
+  void *W2h = nullptr;
   uint32_t *bkt_off = nullptr, *cl_off = nullptr, *ids = nullptr;
   void *vec = nullptr;
   int *d_err = nullptr;
@@ -70,6 +82,7 @@ struct nr_index {
   cudaEvent_t ev[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
   int64_t launches = 0;
   int num_sms = 0;
+  int smem_optin = 0;  // shared memory a block may opt in to, bytes
 };
 
 // Per-query refinement segment: rows [row0, row0 + len) of cluster L[i]

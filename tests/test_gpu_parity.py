@@ -443,10 +443,11 @@ def test_select_largest_budgets(wide, torch, P, C):
     assert np.array_equal(st.cpu().numpy(), st_o)
 
 
-@pytest.mark.parametrize("workload", ["tiny", "u8-10m", "f32-10m"])
+@pytest.mark.parametrize("workload", ["tiny", "u8-10m", "f32-10m", "u8-1b"])
 def test_encoder_large_batch(torch, tmp_path, workload):
-    """Large batches (many 128-row tiles) through the tensor-core encoder, for
-    the three encoder shapes (H = 256, 512, 384)."""
+    """Large batches (several 128-row tiles per SM, a ragged last tile) through
+    the tensor-core encoder, for the four encoder shapes (H = 256, 512, 384,
+    512; b = 16, 20, 20, 24)."""
     from paper_2608_15438_gb300 import neuroute as nr
 
     path, _, _ = build_small(tmp_path, workload, n=20000, name="enc")
@@ -458,3 +459,38 @@ def test_encoder_large_batch(torch, tmp_path, workload):
     err = np.abs(lg - ref).max(1)
     assert np.all(err <= 1e-2 * np.abs(ref).max(1))
     assert np.median(err / np.abs(ref).max(1)) < 2e-3
+
+
+@pytest.mark.parametrize("workload", ["tiny", "f32-10m"])
+def test_encoder_tile_edges(torch, tmp_path, workload):
+    """Tile edges of the persistent tensor-core encoder: one row, a partial
+    tile, exactly one tile, one row past it, and two tiles per SM plus one row
+    (one CTA's third tile holds a single row); the same batch twice gives the
+    same bits; input rows that start 8 bytes past a 16-byte boundary take the
+    CUDA-core kernel and agree within the same tolerance."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, _, _ = build_small(tmp_path, workload, n=20000, name="enc")
+    w = synth.WORKLOADS[workload]
+    n_max = 2 * torch.cuda.get_device_properties(0).multi_processor_count * 128 + 1
+    x = synth.base(w, n_max)
+    ix, orc = nr.Index(path, 0), oracle.Index(path)
+    ref = orc.encode(x).astype(np.float64)
+    dx = torch.from_numpy(x).cuda()
+
+    def check(lg, n):
+        lg = lg.cpu().numpy().astype(np.float64)
+        assert lg.shape == (n, w.bits)
+        err = np.abs(lg - ref[:n]).max(1)
+        assert np.all(err <= 1e-2 * np.abs(ref[:n]).max(1))
+
+    for n in (1, 127, 128, 129, n_max):
+        check(ix.encode(dx[:n]), n)
+    assert torch.equal(ix.encode(dx), ix.encode(dx))
+    pad = 8 // dx.element_size()
+    buf = torch.zeros(dx.numel() + pad, dtype=dx.dtype, device="cuda")
+    shifted = buf[pad:].view(dx.shape)
+    shifted.copy_(dx)
+    assert shifted.data_ptr() % 16 == 8
+    check(ix.encode(shifted), n_max)
+    ix.close()
