@@ -131,35 +131,34 @@ constexpr int kRows = 128;     // rows per tile = TMEM lanes of the accumulators
 constexpr int kHC = 128;       // hidden units per layer-1 chunk
 constexpr int kEpiWarps = 8;   // two per TMEM lane group, one column half of a chunk each
 constexpr int kConvWarps = 4;
-constexpr int kWarpMma = 0, kWarpLoad = 1, kWarpEpi = 2, kWarpConv = kWarpEpi + kEpiWarps;
-constexpr int kTcThreads = 32 * (kWarpConv + kConvWarps);  // 448
+constexpr int kWarpMma = 0, kWarpEpi = 1, kWarpConv = kWarpEpi + kEpiWarps;
+constexpr int kTcThreads = 32 * (kWarpConv + kConvWarps);  // 416
 constexpr int kEpiThreads = 32 * kEpiWarps, kConvThreads = 32 * kConvWarps;
-// TMEM columns: layer-1 accumulators at 0 and 128, layer-2 accumulators at 256 and 288
-constexpr uint32_t kTmemCols = 512;
-constexpr int kMaxStages = 3;  // W1 chunk ring
+// TMEM columns: layer-1 accumulators at 0 and 128, layer-2 accumulators at 256
+// and 288, the hidden chunk as the fp16 A operand of layer 2 (two values a
+// column) at 320 and 384
+constexpr uint32_t kTmemCols = 512, kTmemAcc2 = 256, kTmemHid = 320;
 
 struct TcBars {
-  uint64_t xfull[2], xempty[2];                    // X tiles: converters -> MMA -> converters
-  uint64_t wfull[kMaxStages], wempty[kMaxStages];  // W1 chunks: bulk copy -> MMA -> loader
-  uint64_t a1full[2], a1empty[2];                  // layer-1 accumulators: MMA -> epilogue -> MMA
-  uint64_t hfull, hempty;                          // hidden chunk operand: epilogue -> MMA -> epilogue
-  uint64_t a2full[2], a2empty[2];                  // layer-2 accumulators
-  uint64_t drain;                                  // every MMA of the CTA complete
+  uint64_t xfull[2], xempty[2];    // X tiles: converters -> MMA -> converters
+  uint64_t a1full[2], a1empty[2];  // layer-1 accumulators: MMA -> epilogue -> MMA
+  uint64_t hfull[2], hempty[2];    // hidden chunks in TMEM: epilogue -> MMA -> epilogue
+  uint64_t a2full[2], a2empty[2];  // layer-2 accumulators
+  uint64_t drain;                  // every MMA of the CTA complete
   uint32_t tmem_slot;
-  int abort;                                       // a wait expired: every role stops
+  int abort;                       // a wait expired: every role stops
 };
 
-// byte offsets of the shared-memory regions for a shape (host and device)
+// byte offsets of the shared-memory regions for a shape with nxb X buffers
 struct TcLayout {
-  uint32_t x, w1, w2, h, b1, b2, bars, total;
+  uint32_t x, w1, w2, b1, b2, bars, total;
 };
-__host__ __device__ inline TcLayout tc_layout(int D, int H, int n2, int stages) {
+__host__ __device__ inline TcLayout tc_layout(int D, int H, int n2, int nxb) {
   TcLayout L;
   uint32_t o = 0;
-  L.x = o;  o += 2u * kRows * (uint32_t)D * 2u;              // two fp16 X tiles
-  L.w1 = o; o += (uint32_t)stages * kHC * (uint32_t)D * 2u;  // W1 chunk ring
-  L.w2 = o; o += (uint32_t)n2 * (uint32_t)H * 2u;            // all of W2, resident
-  L.h = o;  o += kRows * kHC * 2u;                           // one fp16 hidden chunk
+  L.x = o;  o += (uint32_t)nxb * kRows * (uint32_t)D * 2u;  // fp16 X tiles
+  L.w1 = o; o += (uint32_t)H * (uint32_t)D * 2u;            // all of W1, resident
+  L.w2 = o; o += (uint32_t)n2 * (uint32_t)H * 2u;           // all of W2, resident
   L.b1 = o; o += (uint32_t)H * 4u;
   L.b2 = o; o += 32u * 4u;
   L.bars = o; o += (uint32_t)sizeof(TcBars);
@@ -171,16 +170,13 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.shared::cta.b64 st, [%0];\n}\n" ::"r"(bar)
                : "memory");
 }
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("{\n .reg .b64 st;\n mbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}\n" ::"r"(bar),
-               "r"(bytes)
-               : "memory");
-}
-// bulk copy global -> shared, completion counted on the barrier's transaction bytes
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+// layer-2 MMA with A read from TMEM (a_tmem: its first column), B from shared memory
+__device__ __forceinline__ void tc_mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
   asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
-      "l"(src), "r"(bytes), "r"(bar)
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 __device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&r)[16]) {
@@ -191,6 +187,21 @@ __device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
+}
+__device__ __forceinline__ void tc_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,"
+      "%25,%26,%27,%28,%29,%30,%31,%32};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tc_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
 }
 // Waits for the barrier phase of the given parity. Gives up when another role
 // has given up, or after ~1 s, which makes every role give up.
@@ -227,23 +238,24 @@ __device__ __forceinline__ void u8x16_to_f16(const uint4 v, uint4 &lo, uint4 &hi
   hi = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
-// Persistent, warp-specialised: each CTA (one per SM) takes 128-row tiles
-// tile = blockIdx.x, + gridDim.x, ... and streams them through
-//   converter warps  X tile -> fp16 operand (two buffers)
-//   loader thread    W1 chunk c (128 hidden units, operand order) -> ring of `stages` by bulk copy
-//   MMA thread       layer 1 of chunk g into accumulator g % 2, then layer 2 of chunk g - 1
-//   epilogue warps   accumulator -> ReLU(s acc + b1) -> fp16 hidden chunk; after a tile's
-//                    last chunk its layer-2 accumulator + b2 -> out
+// Persistent, warp-specialised: each CTA (one per SM) keeps W1 and W2 in
+// shared memory and takes 128-row tiles tile = blockIdx.x, + gridDim.x, ...:
+//   converter warps  X tile -> fp16 operand (nxb = 2 buffers, or 1 for wide shapes)
+//   MMA thread       layer 1 of chunk g (128 hidden units) into accumulator g % 2,
+//                    then layer 2 of chunk g - 1 with its A operand in TMEM
+//   epilogue warps   accumulator -> ReLU(s acc + b1) -> fp16 hidden chunk in TMEM
+//                    (buffer g % 2); after a tile's last chunk its layer-2
+//                    accumulator + b2 -> out
 // so that the tensor pipe runs layer 1 of the next chunk while the epilogue
-// turns the previous one into the layer-2 operand. W2 stays in shared memory.
+// turns the previous one into the layer-2 operand.
 template <int DT>
 __global__ void __launch_bounds__(kTcThreads, 1)
-    encode_tc_kernel(const void *__restrict__ x, int D, int H, int b, int n2, int stages, float s,
+    encode_tc_kernel(const void *__restrict__ x, int D, int H, int b, int n2, int nxb, int vec_out, float s,
                      const __half *__restrict__ W1p, const float *__restrict__ b1,
                      const __half *__restrict__ W2p, const float *__restrict__ b2, int64_t nq,
                      float *__restrict__ out, int *err) {
   extern __shared__ __align__(1024) unsigned char smem[];
-  const TcLayout L = tc_layout(D, H, n2, stages);
+  const TcLayout L = tc_layout(D, H, n2, nxb);
   TcBars &B = *reinterpret_cast<TcBars *>(smem + L.bars);
   volatile int *abort = &B.abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -266,22 +278,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(smem_u32(&B.xempty[i]), 1);
       mbar_init(smem_u32(&B.a1full[i]), 1);
       mbar_init(smem_u32(&B.a1empty[i]), kEpiThreads);
+      mbar_init(smem_u32(&B.hfull[i]), kEpiThreads);
+      mbar_init(smem_u32(&B.hempty[i]), 1);
       mbar_init(smem_u32(&B.a2full[i]), 1);
       mbar_init(smem_u32(&B.a2empty[i]), kEpiThreads);
     }
-    for (int i = 0; i < stages; ++i) {
-      mbar_init(smem_u32(&B.wfull[i]), 1);
-      mbar_init(smem_u32(&B.wempty[i]), 1);
-    }
-    mbar_init(smem_u32(&B.hfull), kEpiThreads);
-    mbar_init(smem_u32(&B.hempty), 1);
     mbar_init(smem_u32(&B.drain), 1);
     B.abort = 0;
     fence_mbar_init();
   }
-  // resident operands: W2 (already in operand order) and the biases
-  for (int i = tid; i < n2 * H / 8; i += kTcThreads)
-    reinterpret_cast<uint4 *>(smem + L.w2)[i] = reinterpret_cast<const uint4 *>(W2p)[i];
+  // resident operands: W1 and W2 (already in operand order) and the biases
+  {
+    const uint4 *w1 = reinterpret_cast<const uint4 *>(W1p), *w2 = reinterpret_cast<const uint4 *>(W2p);
+    uint4 *d1 = reinterpret_cast<uint4 *>(smem + L.w1), *d2 = reinterpret_cast<uint4 *>(smem + L.w2);
+    const int n1 = H * D / 8, n2v = n2 * H / 8;
+    for (int i = tid; i < n1; i += kTcThreads) d1[i] = __ldg(w1 + i);
+    for (int i = tid; i < n2v; i += kTcThreads) d2[i] = __ldg(w2 + i);
+  }
   for (int i = tid; i < H; i += kTcThreads) sb1[i] = b1[i];
   if (tid < 32) sb2[tid] = tid < b ? b2[tid] : 0.0f;
   fence_async_smem();
@@ -293,37 +306,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (warp == kWarpMma) {
     if (lane == 0) {
       const uint32_t idesc1 = mma_idesc(kRows, kHC), idesc2 = mma_idesc(kRows, n2);
-      const uint32_t sx = sbase + L.x, sw1 = sbase + L.w1, sw2 = sbase + L.w2, sh = sbase + L.h;
+      const uint32_t sx = sbase + L.x, sw1 = sbase + L.w1, sw2 = sbase + L.w2;
       // layer 2 of chunk number gp (chunk cp of tile number ip of this CTA):
-      // hidden chunk x W2 chunk into the tile's accumulator
+      // hidden chunk (TMEM) x W2 chunk into the tile's accumulator
       auto layer2 = [&](uint32_t gp, uint32_t ip, int cp) -> bool {
-        if (!wait_or_abort(smem_u32(&B.hfull), gp & 1u, abort)) return false;
+        const int hb = (int)(gp & 1);
+        if (!wait_or_abort(smem_u32(&B.hfull[hb]), (gp >> 1) & 1u, abort)) return false;
         if (cp == 0 && !wait_or_abort(smem_u32(&B.a2empty[ip & 1]), ((ip >> 1) & 1u) ^ 1u, abort))
           return false;
         tc_fence_after();
-        const uint32_t d2 = tmem + 256u + (ip & 1u) * 32u;
+        const uint32_t d2 = tmem + kTmemAcc2 + (ip & 1u) * 32u;
+        const uint32_t ah = tmem + kTmemHid + (uint32_t)hb * (kHC / 2);
         for (int ks = 0; ks < kHC / 16; ++ks)
-          tc_mma_f16(d2, smem_desc(sh + ks * 256, 128, 16 * 128),
-                     smem_desc(sw2 + (uint32_t)cp * w2_bytes + ks * 256, 128, 16 * 128), idesc2,
-                     (cp > 0 || ks > 0) ? 1u : 0u);
-        tc_commit(smem_u32(&B.hempty));
+          tc_mma_f16_ts(d2, ah + (uint32_t)ks * 8u,
+                        smem_desc(sw2 + (uint32_t)cp * w2_bytes + ks * 256, 128, 16 * 128), idesc2,
+                        (cp > 0 || ks > 0) ? 1u : 0u);
+        tc_commit(smem_u32(&B.hempty[hb]));
         if (cp == nc - 1) tc_commit(smem_u32(&B.a2full[ip & 1]));
         return true;
       };
       bool ok = true;
       uint32_t g = 0, it = 0;  // chunks and tiles of this CTA so far
-      int st = 0;              // W1 ring slot of chunk g ...
-      uint32_t wpar = 0;       // ... and the parity of its fill
       for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
-        const int xb = (int)(it & 1);
-        if (!wait_or_abort(smem_u32(&B.xfull[xb]), (it >> 1) & 1u, abort)) {
+        const int xb = nxb == 2 ? (int)(it & 1) : 0;
+        const uint32_t xpar = (nxb == 2 ? it >> 1 : it) & 1u;
+        if (!wait_or_abort(smem_u32(&B.xfull[xb]), xpar, abort)) {
           ok = false;
           break;
         }
         for (int c = 0; c < nc; ++c, ++g) {
           const int a = (int)(g & 1);
-          if (!wait_or_abort(smem_u32(&B.wfull[st]), wpar, abort) ||
-              !wait_or_abort(smem_u32(&B.a1empty[a]), ((g >> 1) & 1u) ^ 1u, abort)) {
+          if (!wait_or_abort(smem_u32(&B.a1empty[a]), ((g >> 1) & 1u) ^ 1u, abort)) {
             ok = false;
             break;
           }
@@ -331,15 +344,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           const uint32_t d1 = tmem + (uint32_t)a * kHC;
           for (int ks = 0; ks < D / 16; ++ks)
             tc_mma_f16(d1, smem_desc(sx + (uint32_t)xb * x_bytes + ks * 256, 128, kx * 128),
-                       smem_desc(sw1 + (uint32_t)st * w1_bytes + ks * 256, 128, kx * 128), idesc1,
+                       smem_desc(sw1 + (uint32_t)c * w1_bytes + ks * 256, 128, kx * 128), idesc1,
                        ks > 0 ? 1u : 0u);
-          tc_commit(smem_u32(&B.wempty[st]));
           tc_commit(smem_u32(&B.a1full[a]));
           if (c == nc - 1) tc_commit(smem_u32(&B.xempty[xb]));
-          if (++st == stages) {
-            st = 0;
-            wpar ^= 1u;
-          }
           if (g > 0 && !layer2(g - 1, c > 0 ? it : it - 1, c > 0 ? c - 1 : nc - 1)) {
             ok = false;
             break;
@@ -352,44 +360,54 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_wait_bounded(smem_u32(&B.drain), 0);
     }
     __syncwarp();
-  } else if (warp == kWarpLoad) {
-    if (lane == 0) {
-      int st = 0;
-      uint32_t wpar = 0, issued = 0, lastpar = 0;  // per ring slot: a copy issued, parity of the last
-      bool ok = true;
-      for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x)
-        for (int c = 0; c < nc; ++c) {
-          if (!wait_or_abort(smem_u32(&B.wempty[st]), wpar ^ 1u, abort)) {
-            ok = false;
-            break;
-          }
-          mbar_expect_tx(smem_u32(&B.wfull[st]), w1_bytes);
-          bulk_g2s(sbase + L.w1 + (uint32_t)st * w1_bytes, W1p + (size_t)c * kHC * D, w1_bytes,
-                   smem_u32(&B.wfull[st]));
-          issued |= 1u << st;
-          lastpar = (lastpar & ~(1u << st)) | (wpar << st);
-          if (++st == stages) {
-            st = 0;
-            wpar ^= 1u;
-          }
-        }
-      // copies still in flight land before the CTA exits
-      for (int q = 0; q < stages; ++q)
-        if ((issued >> q) & 1u) mbar_wait_bounded(smem_u32(&B.wfull[q]), (lastpar >> q) & 1u);
-    }
-    __syncwarp();
   } else if (warp < kWarpConv) {
-    const int lg = warp & 3;                 // TMEM lane group this warp may read
+    const int lg = warp & 3;                 // TMEM lane group this warp may access
     const int hh = (warp - kWarpEpi) >> 2;   // column half of each chunk
     const int r = lg * 32 + lane;            // tile row = TMEM lane
     const uint32_t lane_base = (uint32_t)(lg * 32) << 16;
-    unsigned char *sH = smem + L.h;
+    const __half2 zero2 = __float2half2_rn(0.0f);
+    // logits of tile number ip (global tile t): layer-2 accumulator + b2 -> out,
+    // 16 columns a thread (its row, its column half), as float4 where aligned
+    auto logits = [&](uint32_t ip, int64_t t) -> bool {
+      if (!warp_wait(smem_u32(&B.a2full[ip & 1]), (ip >> 1) & 1u, abort)) return false;
+      tc_fence_after();
+      uint32_t o[16];
+      const bool reads = hh * 16 < n2;  // same for the whole warp
+      if (reads) {
+        tc_ld16(tmem + lane_base + kTmemAcc2 + (ip & 1u) * 32u + (uint32_t)hh * 16u, o);
+        tc_wait_ld();
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&B.a2empty[ip & 1]));
+      const int64_t row = t * kRows + r;
+      const int ncol = b - hh * 16 < 16 ? b - hh * 16 : 16;
+      if (reads && row < nq) {
+        float *dst = out + row * b + hh * 16;
+        const float *bias = sb2 + hh * 16;
+        if (vec_out) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (4 * q < ncol)
+              *reinterpret_cast<float4 *>(dst + 4 * q) =
+                  make_float4(__fadd_rn(__uint_as_float(o[4 * q]), bias[4 * q]),
+                              __fadd_rn(__uint_as_float(o[4 * q + 1]), bias[4 * q + 1]),
+                              __fadd_rn(__uint_as_float(o[4 * q + 2]), bias[4 * q + 2]),
+                              __fadd_rn(__uint_as_float(o[4 * q + 3]), bias[4 * q + 3]));
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            if (j < ncol) dst[j] = __fadd_rn(__uint_as_float(o[j]), bias[j]);
+        }
+      }
+      return true;
+    };
     uint32_t g = 0, it = 0;
+    int64_t last_tile = 0;
     bool ok = true;
     for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
       for (int c = 0; c < nc; ++c, ++g) {
         const int a = (int)(g & 1);
-        if (!warp_wait(smem_u32(&B.a1full[a]), (uint32_t)((g >> 1) & 1), abort)) {
+        if (!warp_wait(smem_u32(&B.a1full[a]), (g >> 1) & 1u, abort)) {
           ok = false;
           break;
         }
@@ -411,63 +429,51 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           for (int j = 0; j < 16; ++j) {
             const float h0 = __fmaf_rn(s, __uint_as_float(v[2 * j]), bv[2 * j]);
             const float h1 = __fmaf_rn(s, __uint_as_float(v[2 * j + 1]), bv[2 * j + 1]);
-            const __half2 p = __floats2half2_rn(h0 > 0.0f ? h0 : 0.0f, h1 > 0.0f ? h1 : 0.0f);
+            const __half2 p = __hmax2(__floats2half2_rn(h0, h1), zero2);
             hp[16 * half + j] = *reinterpret_cast<const uint32_t *>(&p);
           }
         }
         tc_fence_before();
         mbar_arrive(smem_u32(&B.a1empty[a]));
-        // the previous chunk's layer-2 MMAs have read the hidden operand
-        if (!warp_wait(smem_u32(&B.hempty), (uint32_t)((g & 1) ^ 1), abort)) {
+        // the layer-2 MMAs of chunk g - 2 have read this hidden buffer
+        if (!warp_wait(smem_u32(&B.hempty[a]), ((g >> 1) & 1u) ^ 1u, abort)) {
           ok = false;
           break;
         }
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          *reinterpret_cast<uint4 *>(sH + nr_tc_kmajor_off(r, hh * 8 + q, kHC / 8)) =
-              make_uint4(hp[4 * q], hp[4 * q + 1], hp[4 * q + 2], hp[4 * q + 3]);
-        fence_async_smem();
-        mbar_arrive(smem_u32(&B.hfull));
-      }
-      if (!ok) break;
-      // the tile's logits: layer-2 accumulator + b2
-      if (!warp_wait(smem_u32(&B.a2full[it & 1]), (uint32_t)((it >> 1) & 1), abort)) break;
-      tc_fence_after();
-      uint32_t o[16];
-      const bool reads = hh * 16 < n2;  // same for the whole warp
-      if (reads) {
-        tc_ld16(tmem + lane_base + 256u + (uint32_t)(it & 1) * 32u + (uint32_t)hh * 16u, o);
-        tc_wait_ld();
-      }
-      tc_fence_before();
-      mbar_arrive(smem_u32(&B.a2empty[it & 1]));
-      const int64_t row = tile * kRows + r;
-      if (reads && row < nq) {
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int oc = hh * 16 + j;
-          if (oc < b) out[row * b + oc] = __fadd_rn(__uint_as_float(o[j]), sb2[oc]);
+        tc_fence_after();
+        tc_st32(tmem + lane_base + kTmemHid + (uint32_t)a * (kHC / 2) + (uint32_t)hh * 32u, hp);
+        tc_wait_st();
+        tc_fence_before();
+        mbar_arrive(smem_u32(&B.hfull[a]));
+        // the previous tile's logits, once this tile's first chunk is on its way
+        if (c == 0 && it > 0 && !logits(it - 1, last_tile)) {
+          ok = false;
+          break;
         }
       }
+      last_tile = tile;
+      if (!ok) break;
     }
+    if (ok && it > 0) ok = logits(it - 1, last_tile);
   } else {
     // converters: X tile -> fp16 operand in the K-major core-matrix layout;
     // eight consecutive threads cover eight rows of one 16-byte K chunk, so a
     // warp's stores fill whole 128-byte core matrices
     const int ct = tid - kWarpConv * 32;
     // item j of this thread: row rr of the tile and piece pc of the row (16 source
-    // bytes = 2 K chunks for uint8, one K chunk of 8 floats for fp32), packed
-    // rr | pc << 8; the same for every tile
+    // bytes = 2 K chunks for uint8, one K chunk of 8 floats for fp32), the same
+    // for every tile; k / per by a 16-bit reciprocal, exact for k < 256, per <= 16
     const int per = DT == 0 ? D / 16 : kx;  // pieces per row = items per thread (<= 8, <= 16)
-    int tab[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const int k = (ct >> 3) + 16 * j;
-      tab[j] = (j < per) ? (((k / per) * 8 + (ct & 7)) | ((k % per) << 8)) : 0;
-    }
+    const uint32_t inv = (65536u + (uint32_t)per - 1u) / (uint32_t)per;
+    auto item = [&](int j, int &rr, int &pc) {
+      const uint32_t k = (uint32_t)(ct >> 3) + 16u * (uint32_t)j, q = (k * inv) >> 16;
+      pc = (int)(k - q * (uint32_t)per);
+      rr = (int)q * 8 + (ct & 7);
+    };
     uint32_t it = 0;
     for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-      const int xb = (int)(it & 1);
+      const int xb = nxb == 2 ? (int)(it & 1) : 0;
+      const uint32_t xpar = ((nxb == 2 ? it >> 1 : it) & 1u) ^ 1u;  // previous use of the buffer
       unsigned char *sX = smem + L.x + (size_t)xb * x_bytes;
       const int64_t row0 = tile * kRows;
       const int rows = nq - row0 < kRows ? (int)(nq - row0) : kRows;  // rows of this tile
@@ -477,16 +483,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         uint4 v[8];
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          const int rr = tab[j] & 0xff, pc = tab[j] >> 8;
+          int rr, pc;
+          item(j, rr, pc);
           v[j] = make_uint4(0u, 0u, 0u, 0u);
           if (j < per && rr < rows) v[j] = __ldg(reinterpret_cast<const uint4 *>(xs + rr * D + pc * 16));
         }
-        ok = warp_wait(smem_u32(&B.xempty[xb]), ((it >> 1) & 1u) ^ 1u, abort);
+        ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort);
         if (ok) {
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             if (j >= per) break;
-            const int rr = tab[j] & 0xff, pc = tab[j] >> 8;
+            int rr, pc;
+            item(j, rr, pc);
             uint4 lo, hi;
             u8x16_to_f16(v[j], lo, hi);
             *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc, kx)) = lo;
@@ -501,7 +509,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           float4 u[8], w[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            const int rr = tab[j0 + j] & 0xff, pc = tab[j0 + j] >> 8;
+            int rr, pc;
+            item(j0 + j, rr, pc);
             u[j] = w[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
             if (j0 + j < per && rr < rows) {
               const float4 *s4 = reinterpret_cast<const float4 *>(xs + rr * D + pc * 8);
@@ -509,12 +518,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               w[j] = __ldg(s4 + 1);
             }
           }
-          if (j0 == 0) ok = warp_wait(smem_u32(&B.xempty[xb]), ((it >> 1) & 1u) ^ 1u, abort);
+          if (j0 == 0) ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort);
           if (!ok) break;
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             if (j0 + j >= per) break;
-            const int rr = tab[j0 + j] & 0xff, pc = tab[j0 + j] >> 8;
+            int rr, pc;
+            item(j0 + j, rr, pc);
             const __half2 h0 = __floats2half2_rn(u[j].x, u[j].y), h1 = __floats2half2_rn(u[j].z, u[j].w);
             const __half2 h2 = __floats2half2_rn(w[j].x, w[j].y), h3 = __floats2half2_rn(w[j].z, w[j].w);
             *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, pc, kx)) =
@@ -537,10 +547,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
-// W1 ring depth for a shape: 3 chunks if a block's shared memory allows, else 2, else 0
-int tc_stages(int D, int H, int n2, int smem_optin) {
-  for (int st = kMaxStages; st >= 2; --st)
-    if (tc_layout(D, H, n2, st).total <= (uint32_t)smem_optin) return st;
+// X tile buffers for a shape: 2 if a block's shared memory allows, else 1, else 0
+int tc_xbuffers(int D, int H, int n2, int smem_optin) {
+  for (int nxb = 2; nxb >= 1; --nxb)
+    if (tc_layout(D, H, n2, nxb).total <= (uint32_t)smem_optin) return nxb;
   return 0;
 }
 
@@ -677,7 +687,7 @@ __global__ void __launch_bounds__(kThreads)
 bool nr_encode_uses_tensor_cores(const nr_index *ix) {
   return ix->W1h != nullptr && ix->n_mid == 0 && ix->D % 16 == 0 && ix->D <= 128 &&
          ix->H % kHC == 0 && ix->b <= 32 &&
-         tc_stages(ix->D, ix->H, ix->b <= 16 ? 16 : 32, ix->smem_optin) > 0;
+         tc_xbuffers(ix->D, ix->H, ix->b <= 16 ? 16 : 32, ix->smem_optin) > 0;
 }
 
 cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
@@ -686,14 +696,15 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
   // the tensor-core kernel reads X in 16-byte pieces
   if (nr_encode_uses_tensor_cores(ix) && (reinterpret_cast<uintptr_t>(d_x) & 15) == 0) {
     const int n2 = ix->b <= 16 ? 16 : 32;
-    const int stages = tc_stages(ix->D, ix->H, n2, ix->smem_optin);
-    const uint32_t smem = tc_layout(ix->D, ix->H, n2, stages).total;
+    const int nxb = tc_xbuffers(ix->D, ix->H, n2, ix->smem_optin);
+    const uint32_t smem = tc_layout(ix->D, ix->H, n2, nxb).total;
     auto kern = ix->dtype == 0 ? encode_tc_kernel<0> : encode_tc_kernel<1>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t tiles = (nq + kRows - 1) / kRows;
     const int64_t grid = tiles < ix->num_sms ? tiles : ix->num_sms;
-    kern<<<(unsigned)grid, kTcThreads, smem, s>>>(d_x, ix->D, ix->H, ix->b, n2, stages, ix->in_scale,
+    const int vec_out = ix->b % 4 == 0 && (reinterpret_cast<uintptr_t>(d_logits) & 15) == 0;
+    kern<<<(unsigned)grid, kTcThreads, smem, s>>>(d_x, ix->D, ix->H, ix->b, n2, nxb, vec_out, ix->in_scale,
                                                   static_cast<const __half *>(ix->W1h), ix->b1,
                                                   static_cast<const __half *>(ix->W2h), ix->b2, nq,
                                                   d_logits, ix->d_err);
