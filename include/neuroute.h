@@ -21,9 +21,9 @@
  *    enqueue work on it and return; outputs are valid once the stream has
  *    synchronised. Argument and allocation errors are returned synchronously
  *    and enqueue nothing.
- *  - Device-side range checks never trap: a bad index in the file sets a
- *    device flag that the next call (or nr_last_stats) reports as
- *    NR_ERR_DEVICE_CHECK.
+ *  - Device-side checks never trap: a bad index in the file, or a bounded
+ *    wait inside a kernel that expires, sets a device flag that
+ *    nr_last_stats reports as NR_ERR_DEVICE_CHECK (and clears).
  *  - One handle is not safe for concurrent calls (it owns one workspace).
  *  - Float arithmetic that decides an integer (bits, probe order, the gate,
  *    top-C, top-k membership) uses a fixed operation order, so results are
@@ -64,7 +64,8 @@ typedef enum {
   NR_ERR_FORMAT = -3,       /* the index file is malformed or truncated */
   NR_ERR_OOM = -4,          /* device or host allocation failed */
   NR_ERR_CUDA = -5,         /* a CUDA runtime call failed */
-  NR_ERR_DEVICE_CHECK = -6  /* a kernel found an out-of-range index in the file */
+  NR_ERR_DEVICE_CHECK = -6  /* a kernel found an out-of-range index in the file,
+                               or a bounded wait inside a kernel expired */
 } nr_status;
 
 /* Query-time knobs. Defaults from nr_params_default().
@@ -215,9 +216,15 @@ nr_status nr_centroid_dists(nr_index *ix, const float *d_logits, int64_t nq,
 nr_status nr_set_params(nr_index *ix, const nr_params *p);
 
 /* Encoder forward (Sec. 3.2.1): d_x [nq x D] (uint8 or fp32, the index dtype)
- * -> d_logits [nq x b] fp32. h = ReLU(W1 (in_scale x) + b1), l = W2 h + b2;
- * operands fp16, accumulation fp32 (logits agree with an exact evaluation to
- * about 1e-3 of their norm). nq = 0 is a no-op. */
+ * -> d_logits [nq x b] fp32, both device, row-major and contiguous.
+ * h = ReLU(W1 (in_scale x) + b1), l = W2 h + b2. One hidden layer with
+ * D % 16 == 0, D <= 128, H % 128 == 0, b <= 32 and d_x 16-byte aligned runs on
+ * the tensor cores: operands fp16, accumulation fp32 (logits agree with an
+ * exact evaluation to about 1e-3 of their norm). Other shapes, misaligned
+ * input and encoders with more hidden layers run on CUDA cores in fp32.
+ * nq = 0 is a no-op. Asynchronous on `stream`; a device-side wait that
+ * expires sets the device flag (see nr_last_stats).
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_CUDA. */
 nr_status nr_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits, void *stream);
 
 /* Probe codes (Eq. 10 and Algorithm 1) from d_logits [nq x b]:
@@ -287,7 +294,8 @@ nr_status nr_search_static(nr_index *ix, const void *d_queries, int64_t nq, int 
 nr_status nr_query_stats(nr_index *ix, int64_t *d_stats, int64_t nq, void *stream);
 
 /* Sums over the last search call (synchronises the device). Also returns
- * NR_ERR_DEVICE_CHECK if a kernel has flagged bad index data since load. */
+ * NR_ERR_DEVICE_CHECK, and clears the flag, if a kernel has flagged bad index
+ * data or an expired wait since load or since the last such report. */
 nr_status nr_last_stats(nr_index *ix, nr_stats *out);
 
 /* Kernel time in milliseconds of the stages of the last search call
