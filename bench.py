@@ -124,6 +124,24 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(x, world, device=None):
+    """The largest of the ranks' values of x (every rank calls it; x itself
+    at world size 1): the job's time is its slowest rank's."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank, world, seconds):
+    """Whole-job throughput: the units every rank processed over the job's time."""
+    return units_per_rank * world / seconds
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -771,11 +789,9 @@ def main():
     if world > 1:
         import torch.distributed as dist
 
-        t = torch.tensor([tot_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        tot_ms = float(t.item())
         dist.barrier()
-    value = nq * args.steps * world / (tot_ms / 1e3)
+    tot_ms = max_over_ranks(tot_ms, world, dev)
+    value = job_rate(nq * args.steps, world, tot_ms / 1e3)
 
     # end to end through the host-buffer entry point (copies inside the timed region)
     hq = torch.from_numpy(qs).pin_memory()
@@ -789,7 +805,7 @@ def main():
         t = time.perf_counter()
         ix.search_host(hq, k, P, C, out=(hid, hd))
         e2e_t.append(time.perf_counter() - t)
-    e2e_v = nq * args.steps * world / sum(e2e_t)
+    e2e_v = job_rate(nq * args.steps, world, max_over_ranks(sum(e2e_t), world, dev))
 
     cand = st.candidates
     row_bytes = w.row_bytes
