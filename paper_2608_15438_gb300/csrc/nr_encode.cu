@@ -2,29 +2,32 @@
 //   h = ReLU(s (W1 x) + b1),  l = W2 h + b2.
 //
 // Tensor-core version (tcgen05, sm_103a), persistent and warp-specialised:
-// one CTA per SM walks 128-row tiles (the 128 TMEM lanes of its accumulators).
-// Layer 1 runs in chunks of 128 hidden units: one thread issues tcgen05.mma
-// (kind::f16, fp16 operands, fp32 accumulation in TMEM) over the X tile and a
-// W1 chunk that a loader thread brought in by bulk async copy (a ring of three
-// chunks); eight epilogue warps read each accumulator back with tcgen05.ld,
-// apply scale, bias and ReLU and write the chunk as fp16 into shared memory,
-// where it becomes the A operand of the layer-2 MMAs that accumulate
-// l [128 x N2] (N2 = b padded to 16 or 32) against W2, which stays resident in
-// shared memory. Two layer-1 accumulators and two X tiles let the tensor pipe
-// work on the next chunk while the epilogue converts the previous one; four
-// converter warps turn the next X tile into fp16 meanwhile (uint8 inputs are
-// exact in fp16; the input scale is applied to the fp32 accumulator). Every
-// hand-off is an mbarrier: bulk-copy transaction bytes, tcgen05.commit, or
-// thread arrivals. Operands sit in shared memory in the canonical K-major
-// no-swizzle layout (nr_tc_kmajor_off); the host stores W1 and W2 in it.
+// one CTA per SM keeps W1 and W2 in shared memory and walks 128-row tiles (the
+// 128 TMEM lanes of its accumulators). Layer 1 runs in chunks of 128 hidden
+// units: one thread issues tcgen05.mma (kind::f16, fp16 operands, fp32
+// accumulation in TMEM) over the X tile and the chunk of W1; eight epilogue
+// warps read each accumulator back with tcgen05.ld, apply scale, bias and
+// ReLU, and write the chunk as fp16 pairs back into TMEM with tcgen05.st,
+// where it is the A operand of the layer-2 MMAs that accumulate
+// l [128 x N2] (N2 = b padded to 16 or 32) against W2. Two layer-1
+// accumulators, two hidden chunks and two layer-2 accumulators let the tensor
+// pipe work on the next chunk while the epilogue converts the previous one;
+// four converter warps turn the next X tile into fp16 meanwhile (two
+// buffers where shared memory allows; uint8 inputs are exact in fp16; the
+// input scale is applied to the fp32 accumulator). A tile's logits are
+// stored after the next tile's first chunk, when its layer-2 MMAs are done.
+// Every hand-off is an mbarrier (tcgen05.commit, or thread arrivals). Shared
+// memory operands sit in the canonical K-major no-swizzle layout
+// (nr_tc_kmajor_off), in which the host stores W1 and W2.
 //
 // Every wait is bounded (1 s); when one expires every role stops, the CTA
-// waits (again bounded) for its own copies and MMAs in flight, records
-// NR_DEV_TIMEOUT, frees its TMEM and returns.
+// waits (again bounded) for its MMAs in flight, records NR_DEV_TIMEOUT, frees
+// its TMEM and returns.
 //
-// Shapes the tensor-core kernel does not take (D % 16 != 0, D > 128,
-// H % 128 != 0, b > 32, or more shared memory than a CTA has) run on the
-// CUDA-core kernels below it.
+// What the tensor-core kernel does not take (D % 16 != 0, D > 128,
+// H % 128 != 0, b > 32, W1 and W2 too large for a CTA's shared memory, input
+// rows not 16-byte aligned) runs on the CUDA-core kernels below it, and so
+// do encoders with more hidden layers.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -244,13 +247,15 @@ __device__ __forceinline__ void u8x16_to_f16(const uint4 v, uint4 &lo, uint4 &hi
 //   MMA thread       layer 1 of chunk g (128 hidden units) into accumulator g % 2,
 //                    then layer 2 of chunk g - 1 with its A operand in TMEM
 //   epilogue warps   accumulator -> ReLU(s acc + b1) -> fp16 hidden chunk in TMEM
-//                    (buffer g % 2); after a tile's last chunk its layer-2
-//                    accumulator + b2 -> out
+//                    (buffer g % 2); after the next tile's first chunk, the
+//                    tile's layer-2 accumulator + b2 -> out (float4 stores if
+//                    vec_out: b % 4 == 0 and out 16-byte aligned)
 // so that the tensor pipe runs layer 1 of the next chunk while the epilogue
 // turns the previous one into the layer-2 operand.
 template <int DT>
 __global__ void __launch_bounds__(kTcThreads, 1)
-    encode_tc_kernel(const void *__restrict__ x, int D, int H, int b, int n2, int nxb, int vec_out, float s,
+    encode_tc_kernel(const void *__restrict__ x, int D, int H, int b, int n2, int nxb, int vec_out,
+                     float s,
                      const __half *__restrict__ W1p, const float *__restrict__ b1,
                      const __half *__restrict__ W2p, const float *__restrict__ b2, int64_t nq,
                      float *__restrict__ out, int *err) {
