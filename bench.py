@@ -340,11 +340,13 @@ def ground_truth(torch, base_t, q_t, k, dtype):
 
 
 def recall_at(found, truth, k=10):
+    """Recall@k (Sec. 4.4): |R & G| / min(k, |G|) over the unique valid ids of
+    the first k found (R) and true (G) neighbours, averaged over queries."""
     r = []
     for f, g in zip(found, truth):
-        g = set(int(v) for v in g[:k])
+        g = set(int(v) for v in g[:k] if v >= 0)
         f = set(int(v) for v in f[:k] if v >= 0)
-        r.append(len(f & g) / min(k, len(g)))
+        r.append(len(f & g) / min(k, len(g)) if g else 1.0)
     return float(np.mean(r))
 
 

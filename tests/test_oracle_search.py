@@ -72,6 +72,21 @@ def test_recall_definition():
     assert recall_at_k(found, truth, 3) == pytest.approx((2 / 3 + 1 / 2) / 2)
 
 
+def test_benchmark_recall_is_the_definition():
+    """The recall the benchmark reports is the definition above, -1 padding
+    and queries without true neighbours included."""
+    import bench
+
+    truth = np.array([[1, 2, 3], [4, 5, -1], [-1, -1, -1]])
+    found = np.array([[3, 9, 1], [5, 7, 8], [1, -1, -1]])
+    assert bench.recall_at(found, truth, 3) == pytest.approx((2 / 3 + 1 / 2 + 1) / 3)
+    rng = np.random.default_rng(5)
+    for _ in range(20):
+        t = rng.integers(-1, 30, (50, 10))
+        f = rng.integers(-1, 30, (50, 10))
+        assert bench.recall_at(f, t, 10) == recall_at_k(f, t, 10)
+
+
 def test_tiny_invariants(tiny_index):
     ix = oracle.Index(tiny_index["path"])
     qs = tiny_index["queries"][:200]
