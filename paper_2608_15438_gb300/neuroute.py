@@ -129,6 +129,28 @@ def _ptr(t):
     return ctypes.c_void_p(t.data_ptr())
 
 
+def _arg(t, name, dtype, shape, device):
+    """Checks a tensor argument against what the C ABI reads or writes through
+    its pointer (dtype, row-major contiguous shape, the index's GPU or the
+    host for device None) and returns it; a mismatch raises before any call."""
+    import torch
+
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch.Tensor, got {type(t).__name__}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    if t.dim() != len(shape) or any(w is not None and v != w for v, w in zip(t.shape, shape)):
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, expected {shape}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous (row-major)")
+    if device is None:
+        if t.is_cuda:
+            raise ValueError(f"{name}: expected a host tensor")
+    elif not t.is_cuda or t.device.index != device:
+        raise ValueError(f"{name}: expected a tensor on cuda:{device}, got {t.device}")
+    return t
+
+
 def _stream(stream):
     import torch
 
@@ -192,7 +214,8 @@ class Index:
         clusters in the bucket), (-1, -1, -1, 0) for an unknown id."""
         import torch
 
-        ids = ids.reshape(-1).to(torch.int64).contiguous()
+        ids = _arg(ids.reshape(-1).to(torch.int64).contiguous(), "ids", torch.int64, (None,),
+                   self.device)
         out = torch.empty((ids.numel(), 4), dtype=torch.int32, device=self._dev())
         _check("nr_index_locate", lib().nr_index_locate(self.h, _ptr(ids), ids.numel(), _ptr(out),
                                                         _stream(stream)))
@@ -203,8 +226,10 @@ class Index:
         (nr_centroid_dists): fp32 [nq x m], +inf for -1 pads."""
         import torch
 
-        clusters = clusters.to(torch.int32).contiguous()
+        clusters = _arg(clusters.to(torch.int32).contiguous(), "clusters", torch.int32,
+                        (None, None), self.device)
         nq, m = clusters.shape
+        self._logits(logits, nq)
         out = torch.empty((nq, m), dtype=torch.float32, device=self._dev())
         _check("nr_centroid_dists", lib().nr_centroid_dists(self.h, _ptr(logits), nq, _ptr(clusters), m,
                                                             _ptr(out), _stream(stream)))
@@ -221,9 +246,30 @@ class Index:
 
         return torch.device("cuda", self.device)
 
+    def _rows(self, x, name="queries", device=-1):
+        """[n x D] rows of the index dtype on this index's GPU (device -1) or the host (None)."""
+        import torch
+
+        dt = torch.uint8 if self.dtype_code == 0 else torch.float32
+        return _arg(x, name, dt, (None, self.D), self.device if device == -1 else device)
+
+    def _logits(self, lg, nq=None):
+        import torch
+
+        return _arg(lg, "logits", torch.float32, (nq, self.b), self.device)
+
+    def _outs(self, out, nq, k, device=-1):
+        import torch
+
+        dev = self.device if device == -1 else device
+        ids, d = out
+        return (_arg(ids, "out ids", torch.int64, (nq, k), dev),
+                _arg(d, "out dists", torch.float32, (nq, k), dev))
+
     def encode(self, x, stream=None):
         import torch
 
+        x = self._rows(x, "x")
         out = torch.empty((x.shape[0], self.b), dtype=torch.float32, device=self._dev())
         _check("nr_encode", lib().nr_encode(self.h, _ptr(x), x.shape[0], _ptr(out), _stream(stream)))
         return out
@@ -231,6 +277,7 @@ class Index:
     def route(self, logits, P, stream=None):
         import torch
 
+        logits = self._logits(logits)
         nq = logits.shape[0]
         codes = torch.empty((nq, P), dtype=torch.int32, device=self._dev())
         nprobe = torch.empty(nq, dtype=torch.int32, device=self._dev())
@@ -241,6 +288,7 @@ class Index:
     def debug_clusters(self, logits, P, C, stream=None):
         import torch
 
+        logits = self._logits(logits)
         nq = logits.shape[0]
         cl = torch.empty((nq, P + C), dtype=torch.int32, device=self._dev())
         ncl = torch.empty(nq, dtype=torch.int32, device=self._dev())
@@ -255,15 +303,16 @@ class Index:
                 torch.empty((nq, k), dtype=torch.float32, device=self._dev()))
 
     def search(self, queries, k, P, C, out=None, stream=None):
-        nq = queries.shape[0]
-        ids, d = out if out is not None else self._outputs(nq, k)
+        nq = self._rows(queries).shape[0]
+        ids, d = self._outs(out, nq, k) if out is not None else self._outputs(nq, k)
         _check("nr_search", lib().nr_search(self.h, _ptr(queries), nq, k, P, C, _ptr(ids), _ptr(d),
                                             _stream(stream)))
         return ids, d
 
     def search_logits(self, queries, logits, k, P, C, out=None, stream=None):
-        nq = queries.shape[0]
-        ids, d = out if out is not None else self._outputs(nq, k)
+        nq = self._rows(queries).shape[0]
+        self._logits(logits, nq)
+        ids, d = self._outs(out, nq, k) if out is not None else self._outputs(nq, k)
         _check("nr_search_logits", lib().nr_search_logits(self.h, _ptr(queries), _ptr(logits), nq, k,
                                                           P, C, _ptr(ids), _ptr(d), _stream(stream)))
         return ids, d
@@ -272,10 +321,10 @@ class Index:
         """queries, and the outputs, are host tensors (pinned for full bandwidth)."""
         import torch
 
-        nq = queries.shape[0]
+        nq = self._rows(queries, device=None).shape[0]
         if out is None:
             out = (torch.empty((nq, k), dtype=torch.int64), torch.empty((nq, k), dtype=torch.float32))
-        ids, d = out
+        ids, d = self._outs(out, nq, k, device=None)
         _check("nr_search_host", lib().nr_search_host(self.h, _ptr(queries), nq, k, P, C, _ptr(ids),
                                                       _ptr(d), _stream(stream)))
         return ids, d
@@ -283,8 +332,8 @@ class Index:
     def search_static(self, queries, k, P, C, out=None, stream=None):
         """nr_search without any allocation inside the call: scratch comes from
         the library's fixed 32 MiB device array (see include/neuroute.h)."""
-        nq = queries.shape[0]
-        ids, d = out if out is not None else self._outputs(nq, k)
+        nq = self._rows(queries).shape[0]
+        ids, d = self._outs(out, nq, k) if out is not None else self._outputs(nq, k)
         _check("nr_search_static", lib().nr_search_static(self.h, _ptr(queries), nq, k, P, C,
                                                           _ptr(ids), _ptr(d), _stream(stream)))
         return ids, d
