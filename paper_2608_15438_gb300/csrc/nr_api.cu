@@ -22,8 +22,6 @@ constexpr int kMaxSelect = 65536;  // probe_budget * K_max (beyond 2,048: sorted
 constexpr int kMaxTopK = 256;
 constexpr size_t kChunkBudget = (size_t)4 << 30;  // workspace bytes per query chunk
 
-
-
 uint32_t rd32(const unsigned char *h, int o) {
   uint32_t v;
   memcpy(&v, h + o, 4);
@@ -142,14 +140,12 @@ struct nr_index_full {
 
 static nr_index_ext *ext_of(nr_index *ix) { return &reinterpret_cast<nr_index_full *>(ix)->ext; }
 
-
 nr_index *nr_index_alloc() {
   auto *full = new (std::nothrow) nr_index_full();
   if (!full) return nullptr;
   nr_params_default(&full->ix.params);
   return &full->ix;
 }
-
 
 nr_status nr_index_init_device(nr_index *ix) {
   cudaDeviceProp prop;

@@ -31,8 +31,6 @@ constexpr int kMaxSample = 4096;   // sample_per_cluster
 constexpr int64_t kWarpRows = 4096;  // buckets up to this size: one warp; larger: one CTA
 constexpr int kCtaThreads = 256;
 
-
-
 // ---------------------------------------------------------------------------
 // Arithmetic of the build definition (identical on the host builder)
 // ---------------------------------------------------------------------------

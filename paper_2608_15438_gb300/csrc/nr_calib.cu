@@ -11,8 +11,6 @@
 
 namespace {
 
-
-
 __global__ void iota_kernel(uint32_t *v, int64_t n) {
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (int64_t)gridDim.x * blockDim.x)
