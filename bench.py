@@ -49,6 +49,7 @@ OPERATING_POINTS = {
     "f32-1536-1m": dict(P=2048, C=2048, t_low=256),  # profiling proxy of f32-1536
 }
 DEFAULT_POINT = dict(P=64, C=128, t_low=4)
+NOMINAL_HBM_GBS = 7900.0  # GB300 HBM3e, nominal
 CALIB_QUERIES = 10000
 CALIB_BINS = 16
 
@@ -818,6 +819,10 @@ def main():
     achieved = cand * row_bytes / n_ref / (refine_avg_ms / 1e3) / 1e9
     peaks, peak_src = measured_peaks()
     traffic = traffic_from_profile(w.name, P, C, cand * row_bytes, n_ref)
+    # select per launch: centroid rows of every scored cluster and the
+    # directory pair of every probe
+    sel_bytes = (st.scored * w.bits * 4 + st.probes * 8) / n_ref
+    sel_avg_ms = stage_ms["select"] / args.steps / n_ref
     out = {
         "metric": METRIC,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
@@ -837,10 +842,23 @@ def main():
                    "parallelism": f"replicas x{world} (queries sharded, no collective)"},
         "roofline": {"kernel": "nr_refine", "bound": "hbm", "achieved": achieved,
                      "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
-                     "frac": achieved / peaks.get("hbm_gbs"), "peak_source": peak_src,
+                     "frac": achieved / peaks.get("hbm_gbs"),
+                     "peak_source": f"{peak_src} hbm_gbs (a device copy's read + write bytes per "
+                                    "second); the scan reads, so it can exceed it",
+                     "frac_of_nominal": achieved / NOMINAL_HBM_GBS,
                      "traffic": traffic,
                      "algorithmic_bytes_per_launch": cand * row_bytes / n_ref,
                      "avg_launch_ms": refine_avg_ms, "launches_per_step": n_ref},
+        # the centroid stage's own roofline (Sec. 3.5's C_q b floats a query
+        # plus one directory pair per probe): latency-bound gathers
+        "roofline_select": {"kernel": "nr_select", "bound": "hbm",
+                            "achieved": sel_bytes / (sel_avg_ms / 1e3) / 1e9 if sel_avg_ms > 0 else None,
+                            "peak": peaks.get("hbm_gbs"), "unit": "GB/s",
+                            "frac": (sel_bytes / (sel_avg_ms / 1e3) / 1e9 / peaks.get("hbm_gbs")
+                                     if sel_avg_ms > 0 else None),
+                            "peak_source": peak_src, "algorithmic_bytes_per_launch": sel_bytes,
+                            "clusters_scored_per_query": st.scored / nq,
+                            "avg_launch_ms": sel_avg_ms, "launches_per_step": n_ref},
         "stage_ms_per_step": {kk: v / args.steps for kk, v in stage_ms.items()},
         "e2e": {"value": e2e_v, "unit": "queries/s", "h2d_bytes_per_step": nq * row_bytes,
                 "d2h_bytes_per_step": nq * k * 12},

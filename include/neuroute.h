@@ -148,6 +148,7 @@ typedef struct {
   int64_t rounds;     /* refinement rounds run */
   int64_t clusters;   /* |C^dir U C^cent| */
   int64_t probes;     /* probe codes generated */
+  int64_t scored;     /* clusters whose centroid distance was evaluated */
 } nr_stats;
 
 /* Status name, static storage. */
@@ -156,7 +157,9 @@ const char *nr_status_string(nr_status s);
 /* Fill *p with the defaults above. */
 nr_status nr_params_default(nr_params *p);
 
-/* Load an index file into device memory on `device` (CUDA ordinal).
+/* Load an index file into device memory on `device` (CUDA ordinal): the
+ * encoder and thresholds (Sec. 3.2.1, 3.2.3), the bucket directory and the
+ * bucket-local clusters over the stored rows (Sec. 3.3).
  * Errors: NR_ERR_IO, NR_ERR_FORMAT (bad magic, sizes, truncation; b must be in
  * [1, 24]; a row must be a multiple of 16 bytes and at most 1024 bytes),
  * NR_ERR_OOM, NR_ERR_CUDA. On success *out owns all device memory of the
@@ -243,7 +246,9 @@ nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int
                             int cluster_budget, int32_t *d_clusters, int32_t *d_ncl,
                             void *stream);
 
-/* Whole query path: d_queries [nq x D] (index dtype) -> d_out_ids [nq x k]
+/* Whole query path (the k-NN problem of Sec. 3.1, answered by the retrieval
+ * of Sec. 3.4: encode, Eq. 10, Algorithm 1, Sec. 3.3 lookup, Algorithm 2,
+ * exact refinement): d_queries [nq x D] (index dtype) -> d_out_ids [nq x k]
  * int64 original ids and d_out_dists [nq x k] fp32 squared L2 distances, each
  * row sorted by (distance, id), padded with (-1, +inf) when fewer than k rows
  * were scored. For uint8 indexes distances are the exact integer sums.
@@ -253,12 +258,12 @@ nr_status nr_search(nr_index *ix, const void *d_queries, int64_t nq, int k, int 
                     int cluster_budget, int64_t *d_out_ids, float *d_out_dists, void *stream);
 
 /* As nr_search, with the logits supplied by the caller (d_logits [nq x b]);
- * the encoder is not run. */
+ * the encoder (Sec. 3.2.1) is not run, every later step of Sec. 3.4 is. */
 nr_status nr_search_logits(nr_index *ix, const void *d_queries, const float *d_logits, int64_t nq,
                            int k, int probe_budget, int cluster_budget, int64_t *d_out_ids,
                            float *d_out_dists, void *stream);
 
-/* As nr_search with HOST buffers: h_queries [nq x D] is copied to the device,
+/* As nr_search (Sec. 3.4) with HOST buffers: h_queries [nq x D] is copied to the device,
  * the search runs, and h_out_ids / h_out_dists are copied back; the call
  * returns after the stream has synchronised. Pinned host memory gives full
  * copy bandwidth; pageable memory works. */
@@ -273,13 +278,20 @@ nr_status nr_search_host(nr_index *ix, const void *h_queries, int64_t nq, int k,
  * code running under a device-memory budget owned by a host framework or an
  * inference server, and latency-critical loops in which cudaMalloc / cudaFree
  * (which can synchronise the device) are not acceptable. The paper has no
- * counterpart; results are identical to nr_search.
- * Limit: a call needs about nq * (4b + 4P + 12(P + C) + 48) bytes, plus
- * nq * 12 * P * K_max bytes when P * K_max exceeds 2048 (each buffer rounded up
- * to 256 bytes); larger requests return NR_ERR_INVALID_ARG without enqueuing
- * work, so split the batch.
+ * counterpart; the kernels, their order and their results are nr_search's.
+ * Arguments are checked as nr_search checks them (the same budgets, k, batch
+ * size and sequential-stage limits, NR_ERR_INVALID_ARG otherwise).
+ * Size limit: with S = the smallest power of two >= probe_budget * K_max, a
+ * call needs nq * (4 b + 4 P + 12 (P + C) + 56) bytes, plus nq * 12 S bytes
+ * when S > 2048 (select's global sort slabs), each of its eleven buffers
+ * rounded up to 256 bytes; a request beyond 32 MiB returns NR_ERR_INVALID_ARG
+ * without enqueuing work. Splitting the batch brings nq down; a single query
+ * needs about 12 S bytes, so every budget nr_search accepts (S <= 65536,
+ * 768 KiB) fits for small enough batches.
  * The first call on a device looks up the array's device address with that
- * device made current; make that first call before any stream capture.
+ * device made current and keeps it for the life of the process; make that
+ * first call before any stream capture, and do not use the library across a
+ * device reset (cudaDeviceReset), which would leave the kept address stale.
  * All calls share the one array and it keeps the last call's contents: two
  * calls whose work overlaps on the GPU (different streams, or different
  * indexes on the same device) race and corrupt each other; serialise them.
@@ -289,8 +301,10 @@ nr_status nr_search_static(nr_index *ix, const void *d_queries, int64_t nq, int 
                            int cluster_budget, int64_t *d_out_ids, float *d_out_dists,
                            void *stream);
 
-/* Per-query statistics of the last search call: d_stats [nq x 4] int64 =
- * (candidates, rounds, clusters, probes). Enqueued on `stream`. */
+/* Per-query statistics of the last search call: d_stats [nq x 5] int64 =
+ * (candidates, rounds, |C^dir U C^cent|, probes, clusters scored), the last
+ * being the number of centroid distances evaluated (Sec. 3.5's C_q).
+ * Enqueued on `stream`. */
 nr_status nr_query_stats(nr_index *ix, int64_t *d_stats, int64_t nq, void *stream);
 
 /* Sums over the last search call (synchronises the device). Also returns

@@ -60,9 +60,10 @@ def lib():
         L.or_probe_order_allsubsets.restype = i32
         L.or_probe_list.argtypes = [i32, vp, vp, i32, ctypes.POINTER(Params), vp, vp, vp]
         L.or_probe_list.restype = i32
-        L.or_cluster_list.argtypes = [vp, vp, vp, i32, i32, ctypes.POINTER(Params), vp, vp, vp]
+        L.or_cluster_list.argtypes = [vp, vp, vp, i32, i32, ctypes.POINTER(Params), vp, vp, vp,
+                                      vp]
         L.or_cluster_list_seq.argtypes = [vp, vp, vp, vp, i32, i32, ctypes.POINTER(Params), vp, vp,
-                                          vp, vp]
+                                          vp, vp, vp]
         L.or_cluster_list_seq.restype = i32
         L.or_cluster_list.restype = i32
         L.or_refine_stream.argtypes = [i32, i32, vp, vp, vp, i64, i32, ctypes.POINTER(Params),
@@ -169,14 +170,16 @@ class Index:
         dL = np.empty(len(codes) + C, np.float32)
         ndir = np.zeros(1, np.int32)
         n = lib().or_cluster_list(self.h, logit.ctypes.data, codes.ctypes.data, len(codes), C,
-                                  ctypes.byref(p), L.ctypes.data, dL.ctypes.data, ndir.ctypes.data)
+                                  ctypes.byref(p), L.ctypes.data, dL.ctypes.data, ndir.ctypes.data,
+                                  None)
         if n < 0:
             raise RuntimeError("oracle: out-of-range index in file")
         return L[:n].copy(), dL[:n].copy(), int(ndir[0])
 
-    def cluster_list_seq(self, logit, codes, scores, C, p: Params):
+    def cluster_list_seq(self, logit, codes, scores, C, p: Params, with_scored=False):
         """The sequential centroid stage (Algorithm 2): returns (L, dL, n_dir,
-        n_batches)."""
+        n_batches), and the number of centroid distances evaluated after them
+        when with_scored."""
         logit = np.ascontiguousarray(logit, np.float32)
         codes = np.ascontiguousarray(codes, np.uint32)
         scores = np.ascontiguousarray(scores, np.float32)
@@ -184,13 +187,15 @@ class Index:
         dL = np.empty(len(codes) + C, np.float32)
         ndir = np.zeros(1, np.int32)
         nbat = np.zeros(1, np.int32)
+        nsc = np.zeros(1, np.int64)
         n = lib().or_cluster_list_seq(self.h, logit.ctypes.data, codes.ctypes.data,
                                       scores.ctypes.data, len(codes), C, ctypes.byref(p),
                                       L.ctypes.data, dL.ctypes.data, ndir.ctypes.data,
-                                      nbat.ctypes.data)
+                                      nbat.ctypes.data, nsc.ctypes.data)
         if n < 0:
             raise RuntimeError("oracle: out-of-range index in file")
-        return L[:n].copy(), dL[:n].copy(), int(ndir[0]), int(nbat[0])
+        out = (L[:n].copy(), dL[:n].copy(), int(ndir[0]), int(nbat[0]))
+        return out + (int(nsc[0]),) if with_scored else out
 
     def probe_list(self, logit, P, p: Params):
         """(codes, keys) of one query's probe list against this index (the
@@ -213,7 +218,7 @@ class Index:
         nq = queries.shape[0]
         ids = np.empty((nq, k), np.int64)
         d = np.empty((nq, k), np.float32)
-        st = np.empty((nq, 4), np.int64)
+        st = np.empty((nq, 5), np.int64)  # candidates, rounds, |L|, probes, distances evaluated
         lg = None if logits is None else np.ascontiguousarray(logits, np.float32)
         rc = lib().or_search(self.h, queries.ctypes.data, _p(lg), nq, k, P, C, ctypes.byref(p),
                              ids.ctypes.data, d.ctypes.data, st.ctypes.data,

@@ -443,7 +443,7 @@ static bool dc_less(const std::pair<float, int64_t> &a, const std::pair<float, i
 
 extern "C" int or_cluster_list(const or_index *ix, const float *logit, const uint32_t *codes,
                                int nprobe, int C, const or_params *p, int32_t *L, float *dL,
-                               int32_t *n_dir) {
+                               int32_t *n_dir, int64_t *n_scored) {
   const int b = ix->b;
   const uint64_t nbuckets = (uint64_t)1 << b;
   std::vector<std::pair<float, int64_t>> dir, cand;
@@ -477,6 +477,8 @@ extern "C" int or_cluster_list(const or_index *ix, const float *logit, const uin
     if (dL) dL[i] = all[i].first;
   }
   if (n_dir) *n_dir = (int32_t)dir.size();
+  // every cluster of every probed bucket had its centroid distance evaluated
+  if (n_scored) *n_scored = (int64_t)(dir.size() + cand.size());
   return (int)all.size();
 }
 
@@ -486,7 +488,8 @@ extern "C" int or_cluster_list(const or_index *ix, const float *logit, const uin
 // heap kept under the gate, the heap/front update counts and the stop test.
 extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const uint32_t *codes,
                                    const float *score, int nprobe, int C, const or_params *p,
-                                   int32_t *L, float *dL, int32_t *n_dir, int32_t *n_batches) {
+                                   int32_t *L, float *dL, int32_t *n_dir, int32_t *n_batches,
+                                   int64_t *n_scored) {
   const int b = ix->b;
   const uint64_t nbuckets = (uint64_t)1 << b;
   const int nbins = p->n_bins > 1 ? p->n_bins : 1;
@@ -502,6 +505,7 @@ extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const
   std::vector<std::pair<float, int64_t>> dir, H;
   float dmin = kInf;
   int b_proc = 0, t_low = 0, batches = 0;
+  int64_t batch_clusters = 0;  // clusters of the batches processed
   bool stop = false;
   int i = 0;
   while (i < nprobe && !stop) {
@@ -526,6 +530,7 @@ extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const
       std::vector<std::pair<float, int64_t>> batch;
       for (size_t t = s0; t < s1; ++t)
         batch.push_back({centroid_distance(logit, &ix->cent[(size_t)cz[t] * b], b), cz[t]});
+      batch_clusters += (int64_t)batch.size();
       for (auto &e : batch) dmin = std::min(dmin, e.first);
       float theta = kInf, front_th = kInf;
       if (!gate_off) {
@@ -566,6 +571,8 @@ extern "C" int or_cluster_list_seq(const or_index *ix, const float *logit, const
   }
   if (n_dir) *n_dir = (int32_t)dir.size();
   if (n_batches) *n_batches = batches;
+  // distances evaluated: C^dir of every bin entered, and the batches processed
+  if (n_scored) *n_scored = (int64_t)dir.size() + batch_clusters;
   return (int)out.size();
 }
 
@@ -702,6 +709,7 @@ extern "C" int or_search(const or_index *ix, const void *queries, const float *l
     int np = or_probe_list_index(ix, lg.data(), P, p, codes.data(), keys.data());
     std::vector<int32_t> L((size_t)np + (size_t)C);
     int nl;
+    int64_t scored = 0;
     if (p->cent_mode == 1) {
       std::vector<float> score((size_t)np);  // summed deviation of each probe's flip set
       for (int t = 0; t < np; ++t) {
@@ -709,9 +717,10 @@ extern "C" int or_search(const or_index *ix, const void *queries, const float *l
         memcpy(&score[t], &cb, 4);
       }
       nl = or_cluster_list_seq(ix, lg.data(), codes.data(), score.data(), np, C, p, L.data(),
-                               nullptr, nullptr, nullptr);
+                               nullptr, nullptr, nullptr, &scored);
     } else {
-      nl = or_cluster_list(ix, lg.data(), codes.data(), np, C, p, L.data(), nullptr, nullptr);
+      nl = or_cluster_list(ix, lg.data(), codes.data(), np, C, p, L.data(), nullptr, nullptr,
+                           &scored);
     }
     if (nl < 0) {
       bad = 1;
@@ -743,10 +752,12 @@ extern "C" int or_search(const or_index *ix, const void *queries, const float *l
     int64_t st[2] = {0, 0};
     refine_rounds(ix->dtype, D, q, n, row_at, k, p, out_ids + (size_t)qi * k, out_d + (size_t)qi * k, st);
     if (stats) {
-      stats[(size_t)qi * 4 + 0] = st[0];
-      stats[(size_t)qi * 4 + 1] = st[1];
-      stats[(size_t)qi * 4 + 2] = nl;
-      stats[(size_t)qi * 4 + 3] = np;
+      int64_t *row = stats + (size_t)qi * 5;
+      row[0] = st[0];
+      row[1] = st[1];
+      row[2] = nl;
+      row[3] = np;
+      row[4] = scored;
     }
   });
   return bad ? -1 : 0;

@@ -135,9 +135,12 @@ int or_probe_list_index(const or_index *ix, const float *logit, int P, const or_
 
 /* Ordered cluster list L = C^dir U C^cent of one query. L has room for
  * nprobe + C entries; dL (optional) gets each entry's centroid distance.
- * n_dir (optional) gets |C^dir|. Returns |L|, or -1 on an out-of-range index. */
+ * n_dir (optional) gets |C^dir|; n_scored (optional) the number of centroid
+ * distances evaluated (every cluster of every probed bucket). Returns |L|, or
+ * -1 on an out-of-range index. */
 int or_cluster_list(const or_index *ix, const float *logit, const uint32_t *codes, int nprobe,
-                    int C, const or_params *p, int32_t *L, float *dL, int32_t *n_dir);
+                    int C, const or_params *p, int32_t *L, float *dL, int32_t *n_dir,
+                    int64_t *n_scored);
 
 /* The sequential centroid stage (Algorithm 2) of one query: probes in order
  * with scores score[i] (the summed deviation of their flip set), binned by
@@ -149,10 +152,12 @@ int or_cluster_list(const or_index *ix, const float *logit, const uint32_t *code
  * d <= d_min + c_alpha_front M(d_min); stop when |H| = C, at least b_min bins
  * were entered and c_t_low consecutive batches had updates < c_u_min and
  * front < c_f_min. L = C^dir U H in (d, c) order. n_batches (optional) gets
- * the batches processed. Returns |L|, or -1 on an out-of-range index. */
+ * the batches processed, n_scored (optional) the centroid distances evaluated
+ * (C^dir of the bins entered plus the clusters of the batches processed).
+ * Returns |L|, or -1 on an out-of-range index. */
 int or_cluster_list_seq(const or_index *ix, const float *logit, const uint32_t *codes,
                         const float *score, int nprobe, int C, const or_params *p, int32_t *L,
-                        float *dL, int32_t *n_dir, int32_t *n_batches);
+                        float *dL, int32_t *n_dir, int32_t *n_batches, int64_t *n_scored);
 
 /* The gate margin M(x) of the parameters p (linear, or the calibrated curve). */
 float or_gate_margin(const or_params *p, float x);
@@ -169,8 +174,9 @@ void or_refine_stream(int dtype, int D, const void *q, const void *rows, const u
                       int64_t *stats);
 
 /* Whole search. logits may be NULL (then computed by or_encode).
- * out_ids/out_d [nq x k]; stats (optional) [nq x 4] = candidates scored, rounds,
- * |L|, probes. Returns 0, or -1 on an out-of-range index in the file. */
+ * out_ids/out_d [nq x k]; stats (optional) [nq x 5] = candidates scored, rounds,
+ * |L|, probes, centroid distances evaluated. Returns 0, or -1 on an
+ * out-of-range index in the file. */
 int or_search(const or_index *ix, const void *queries, const float *logits, int64_t nq, int k,
               int P, int C, const or_params *p, int64_t *out_ids, float *out_d, int64_t *stats,
               int nthreads);

@@ -545,6 +545,17 @@ nr_status write_nrix(const nr_index *ix, int64_t N, int64_t n_cl, const void *co
 
 }  // namespace
 
+nr_status nr_check_budgets(const nr_index *ix, int64_t nq, int k, int P, int C) {
+  if (nq < 0 || P < 1 || P > kMaxProbe || C < 1 || C > kMaxClusterBudget) return NR_ERR_INVALID_ARG;
+  if ((int64_t)P * ix->K_max > kMaxSelect) return NR_ERR_INVALID_ARG;
+  if (k < 1 || k > kMaxTopK || nq > ((int64_t)1 << 31) - 1) return NR_ERR_INVALID_ARG;
+  // the sequential centroid stage sorts C^dir in one block and keeps H in
+  // shared memory
+  if (ix->params.cent_mode == 1 && (P > 2048 || nr_select_smem_bytes(ix, P, C) > (size_t)220 * 1024))
+    return NR_ERR_INVALID_ARG;
+  return NR_OK;
+}
+
 extern "C" {
 
 nr_status nr_index_save(nr_index *ix, const char *path) {
@@ -704,22 +715,12 @@ nr_status nr_route(nr_index *ix, const float *d_logits, int64_t nq, int probe_bu
                                      (cudaStream_t)stream));
 }
 
-static nr_status check_budgets(const nr_index *ix, int64_t nq, int k, int P, int C) {
-  if (nq < 0 || P < 1 || P > kMaxProbe || C < 1 || C > kMaxClusterBudget) return NR_ERR_INVALID_ARG;
-  if ((int64_t)P * ix->K_max > kMaxSelect) return NR_ERR_INVALID_ARG;
-  if (k < 1 || k > kMaxTopK || nq > ((int64_t)1 << 31) - 1) return NR_ERR_INVALID_ARG;
-  // the sequential centroid stage sorts C^dir in one block and keeps H in
-  // shared memory
-  if (ix->params.cent_mode == 1 && (P > 2048 || nr_select_smem_bytes(ix, P, C) > (size_t)220 * 1024))
-    return NR_ERR_INVALID_ARG;
-  return NR_OK;
-}
 
 nr_status nr_debug_clusters(nr_index *ix, const float *d_logits, int64_t nq, int probe_budget,
                             int cluster_budget, int32_t *d_clusters, int32_t *d_ncl,
                             void *stream) {
   if (!ix) return NR_ERR_INVALID_ARG;
-  nr_status st = check_budgets(ix, nq, 1, probe_budget, cluster_budget);
+  nr_status st = nr_check_budgets(ix, nq, 1, probe_budget, cluster_budget);
   if (st != NR_OK) return st;
   if (nq == 0) return NR_OK;
   if (!d_logits || !d_clusters || !d_ncl) return NR_ERR_INVALID_ARG;
@@ -760,7 +761,7 @@ static nr_status ensure_pipe(nr_index *ix) {
 
 static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logits_in, int64_t nq,
                              int k, int P, int C, int64_t *d_ids, float *d_d, cudaStream_t s) {
-  nr_status st = check_budgets(ix, nq, k, P, C);
+  nr_status st = nr_check_budgets(ix, nq, k, P, C);
   if (st != NR_OK) return st;
   // chunks of qc queries: as many as the workspace budget allows, or
   // pipe_chunk when pipelined (refinement of chunk i on stream b while stream
@@ -777,7 +778,7 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
   const size_t slot_bytes = align256(l.total);
   // workspace: [per-query stats][one query counter per buffer][chunk buffers]
   const size_t stats_off = 0;
-  const size_t cnt_off = align256(stats_off + (size_t)nq * 4 * 8);
+  const size_t cnt_off = align256(stats_off + (size_t)nq * NR_QSTATS * 8);
   const size_t chunk_off = align256(cnt_off + 16 * (size_t)slots);
   if ((st = ensure_ws(ix, chunk_off + slot_bytes * (size_t)slots)) != NR_OK) return st;
   if (pipe && (st = ensure_pipe(ix)) != NR_OK) return st;
@@ -837,7 +838,7 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
     ev = tstart(2, sa);
     e = nr_launch_select(ix, lg, (uint32_t *)(cw + l.codes), (int32_t *)(cw + l.nprobe), n, P, C,
                          (int32_t *)(cw + l.L), (int32_t *)(cw + l.nL), (nr_seg *)(cw + l.seg),
-                         (uint32_t *)(cw + l.slen), stats + q0 * 4,
+                         (uint32_t *)(cw + l.slen), stats + q0 * NR_QSTATS,
                          nr_select_slab_bytes(P, ix->K_max) ? cw + l.slab : nullptr, sa);
     tend(ev, sa);
     if (e != cudaSuccess) break;
@@ -848,7 +849,7 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
     }
     ev = tstart(3, sb);
     e = nr_launch_refine(ix, qp, n, k, P + C, (nr_seg *)(cw + l.seg), (int32_t *)(cw + l.nL),
-                         (uint32_t *)(cw + l.slen), d_ids + q0 * k, d_d + q0 * k, stats + q0 * 4,
+                         (uint32_t *)(cw + l.slen), d_ids + q0 * k, d_d + q0 * k, stats + q0 * NR_QSTATS,
                          counter, (int32_t *)(cw + l.perm), sb);
     tend(ev, sb);
     if (pipe && e == cudaSuccess) e = cudaEventRecord(ps.ref[slot], sb);
@@ -870,7 +871,7 @@ nr_status nr_search(nr_index *ix, const void *d_queries, int64_t nq, int k, int 
   if (!ix) return NR_ERR_INVALID_ARG;
   if (nq > 0 && (!d_queries || !d_out_ids || !d_out_dists)) return NR_ERR_INVALID_ARG;
   DeviceGuard g(ix->device);
-  if (nq == 0) return check_budgets(ix, nq, k, probe_budget, cluster_budget);
+  if (nq == 0) return nr_check_budgets(ix, nq, k, probe_budget, cluster_budget);
   return search_impl(ix, d_queries, nullptr, nq, k, probe_budget, cluster_budget, d_out_ids,
                      d_out_dists, (cudaStream_t)stream);
 }
@@ -881,7 +882,7 @@ nr_status nr_search_logits(nr_index *ix, const void *d_queries, const float *d_l
   if (!ix) return NR_ERR_INVALID_ARG;
   if (nq > 0 && (!d_queries || !d_logits || !d_out_ids || !d_out_dists)) return NR_ERR_INVALID_ARG;
   DeviceGuard g(ix->device);
-  if (nq == 0) return check_budgets(ix, nq, k, probe_budget, cluster_budget);
+  if (nq == 0) return nr_check_budgets(ix, nq, k, probe_budget, cluster_budget);
   return search_impl(ix, d_queries, d_logits, nq, k, probe_budget, cluster_budget, d_out_ids,
                      d_out_dists, (cudaStream_t)stream);
 }
@@ -890,7 +891,7 @@ nr_status nr_search_host(nr_index *ix, const void *h_queries, int64_t nq, int k,
                          int cluster_budget, int64_t *h_out_ids, float *h_out_dists,
                          void *stream) {
   if (!ix) return NR_ERR_INVALID_ARG;
-  nr_status st = check_budgets(ix, nq, k, probe_budget, cluster_budget);
+  nr_status st = nr_check_budgets(ix, nq, k, probe_budget, cluster_budget);
   if (st != NR_OK) return st;
   if (nq == 0) return NR_OK;
   if (!h_queries || !h_out_ids || !h_out_dists) return NR_ERR_INVALID_ARG;
@@ -934,7 +935,7 @@ nr_status nr_query_stats(nr_index *ix, int64_t *d_stats, int64_t nq, void *strea
     return NR_ERR_INVALID_ARG;
   if (nq == 0) return NR_OK;
   DeviceGuard g(ix->device);
-  return cuda_status(cudaMemcpyAsync(d_stats, ix->d_stats, (size_t)nq * 4 * 8,
+  return cuda_status(cudaMemcpyAsync(d_stats, ix->d_stats, (size_t)nq * NR_QSTATS * 8,
                                      cudaMemcpyDeviceToDevice, (cudaStream_t)stream));
 }
 
@@ -946,14 +947,16 @@ nr_status nr_last_stats(nr_index *ix, nr_stats *out) {
   if (e != cudaSuccess) return cuda_status(e);
   out->nq = ix->last_nq;
   if (ix->last_nq > 0 && ix->d_stats) {
-    std::vector<int64_t> h((size_t)ix->last_nq * 4);
+    std::vector<int64_t> h((size_t)ix->last_nq * NR_QSTATS);
     e = cudaMemcpy(h.data(), ix->d_stats, h.size() * 8, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_status(e);
     for (int64_t i = 0; i < ix->last_nq; ++i) {
-      out->candidates += h[(size_t)i * 4 + 0];
-      out->rounds += h[(size_t)i * 4 + 1];
-      out->clusters += h[(size_t)i * 4 + 2];
-      out->probes += h[(size_t)i * 4 + 3];
+      const int64_t *r = &h[(size_t)i * NR_QSTATS];
+      out->candidates += r[0];
+      out->rounds += r[1];
+      out->clusters += r[2];
+      out->probes += r[3];
+      out->scored += r[4];
     }
   }
   int flag = 0;

@@ -6,12 +6,14 @@
 
 #include "neuroute.h"
 
-// Makes `dev` the current device for a scope and restores the caller's.
+// Makes `dev` the current device for a scope and restores the caller's;
+// ok tells whether `dev` could be made current.
 struct DeviceGuard {
   int prev = -1;
+  bool ok = true;
   explicit DeviceGuard(int dev) {
     if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
-    if (prev != dev) cudaSetDevice(dev);
+    if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
   }
   ~DeviceGuard() {
     int cur = -1;
@@ -84,6 +86,15 @@ struct nr_index {
   int num_sms = 0;
   int smem_optin = 0;  // shared memory a block may opt in to, bytes
 };
+
+// Per-query statistics, int64 each: candidates, rounds, |L|, probes, clusters
+// scored (centroid distances evaluated).
+constexpr int NR_QSTATS = 5;
+
+// Argument and size checks shared by every search entry point (budgets, k,
+// batch size, and the sequential centroid stage's limits); NR_OK or
+// NR_ERR_INVALID_ARG.
+nr_status nr_check_budgets(const nr_index *ix, int64_t nq, int k, int P, int C);
 
 // Per-query refinement segment: rows [row0, row0 + len) of cluster L[i]
 // start at stream position pos.

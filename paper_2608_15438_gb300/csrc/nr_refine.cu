@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(TR, MINB) refine_kernel(RefineArgs a) {
       reinterpret_cast<uint4 *>(m.sq)[c] = reinterpret_cast<const uint4 *>(a.q + q * a.row_bytes)[c];
     nrq::refine_block<DT, TR, STAGES, CPR>(a.rf, m, a.slen[q], a.nL[q], a.seg + (size_t)q * a.Lmax,
                                            a.out_ids + q * k, a.out_d + q * k,
-                                           a.stats ? a.stats + q * 4 : nullptr);
+                                           a.stats ? a.stats + q * NR_QSTATS : nullptr);
   }
 }
 
@@ -111,7 +111,7 @@ __global__ void __launch_bounds__(TR, MINB) refine_split_kernel(RefineArgs a) {
       reinterpret_cast<uint4 *>(m.sq)[c] = reinterpret_cast<const uint4 *>(a.q + q * a.row_bytes)[c];
     nrq::refine_block_split<TR, STAGES, KCC>(a.rf, m, a.slen[q], a.nL[q],
                                              a.seg + (size_t)q * a.Lmax, a.out_ids + q * k,
-                                             a.out_d + q * k, a.stats ? a.stats + q * 4 : nullptr);
+                                             a.out_d + q * k, a.stats ? a.stats + q * NR_QSTATS : nullptr);
   }
 }
 

@@ -45,21 +45,23 @@ __global__ void __launch_bounds__(kThreads, MODE == 0 ? 6 : 1)
   if (tid < sp.b) slog[tid] = logits[(size_t)q * sp.b + tid];
   __syncthreads();
   uint32_t total = 0;
+  int scored = 0;
   unsigned char *qslab = slab ? slab + (size_t)q * slab_bytes : nullptr;
   const int nl =
       MODE == 1
           ? nrq::select_block_seq(sp, slog, codes + (size_t)q * sp.P, np, scratch, warp_sums, sred,
                                   seg + (size_t)q * Lmax, L ? L + (size_t)q * Lmax : nullptr, Lmax,
-                                  &total)
+                                  &total, &scored)
           : nrq::select_block(sp, slog, codes + (size_t)q * sp.P, np, scratch, qslab, warp_sums,
                               sred, seg + (size_t)q * Lmax, L ? L + (size_t)q * Lmax : nullptr,
-                              Lmax, &total);
+                              Lmax, &total, &scored);
   if (tid == 0) {
     nL[q] = nl;
     slen[q] = total;
     if (stats) {
-      stats[(size_t)q * 4 + 2] = nl;
-      stats[(size_t)q * 4 + 3] = np;
+      stats[(size_t)q * NR_QSTATS + 2] = nl;
+      stats[(size_t)q * NR_QSTATS + 3] = np;
+      stats[(size_t)q * NR_QSTATS + 4] = scored;
     }
   }
 }

@@ -13,7 +13,9 @@
 // is loaded, on every GPU that loads it. Host code cannot use the array's
 // name as a device address (on the host it only names a stand-in), so the
 // device address is looked up with cudaGetSymbolAddress once per device, on
-// the first call made on that device, with that device current.
+// the first call made on that device, with that device current, and kept for
+// the life of the process: a device reset (cudaDeviceReset) after that call
+// leaves the kept address stale, so the library must not be used across one.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -51,19 +53,6 @@ nr_status scratch_address(int device, void **out) {
   return NR_OK;
 }
 
-struct CurrentDevice {
-  int prev = -1;
-  bool ok = false;
-  explicit CurrentDevice(int dev) {
-    if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
-    ok = (prev == dev) || cudaSetDevice(dev) == cudaSuccess;
-  }
-  ~CurrentDevice() {
-    int cur = -1;
-    if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
-  }
-};
-
 }  // namespace
 
 extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64_t nq, int k,
@@ -71,13 +60,17 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
                                       float *d_out_dists, void *stream) {
   if (!ix) return NR_ERR_INVALID_ARG;
   const int P = probe_budget, C = cluster_budget;
-  if (nq < 0 || k < 1 || k > 256 || P < 1 || P > 4096 || C < 1 || C > 4096 ||
-      (int64_t)P * ix->K_max > 16384)
-    return NR_ERR_INVALID_ARG;
+  // the checks of every other search entry point (budgets, k, batch size,
+  // the sequential centroid stage's limits)
+  nr_status st = nr_check_budgets(ix, nq, k, P, C);
+  if (st != NR_OK) return st;
   if (nq == 0) return NR_OK;
   if (!d_queries || !d_out_ids || !d_out_dists) return NR_ERR_INVALID_ARG;
   // scratch layout: logits, codes, probe counts, cluster lists and their
-  // counts, segments, stream lengths, per-query stats, the query counter
+  // counts, segments, stream lengths, the refinement order, per-query stats,
+  // select's global sort slabs, the query counter. nq < 2^31 and every
+  // per-query size is bounded (P, C <= 4096, b <= 24, the slab <= 768 KiB),
+  // so no product below overflows size_t.
   const size_t Lmax = (size_t)P + (size_t)C, q = (size_t)nq;
   size_t o = 0;
   const size_t o_logits = o; o = up256(o + q * ix->b * 4);
@@ -87,15 +80,16 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   const size_t o_nL = o;     o = up256(o + q * 4);
   const size_t o_seg = o;    o = up256(o + q * Lmax * sizeof(nr_seg));
   const size_t o_slen = o;   o = up256(o + q * 4);
-  const size_t o_stats = o;  o = up256(o + q * 4 * 8);
+  const size_t o_perm = o;   o = up256(o + q * 4);
+  const size_t o_stats = o;  o = up256(o + q * NR_QSTATS * 8);
   const size_t slab_q = nr_select_slab_bytes(P, ix->K_max);
   const size_t o_slab = o;   o = up256(o + q * slab_q);
   const size_t o_count = o;  o = up256(o + 16);
   if (o > NR_STATIC_SCRATCH_BYTES) return NR_ERR_INVALID_ARG;  // request too large for the array
-  CurrentDevice cd(ix->device);
-  if (!cd.ok) return NR_ERR_CUDA;
+  DeviceGuard g(ix->device);
+  if (!g.ok) return NR_ERR_CUDA;
   void *base = nullptr;
-  nr_status st = scratch_address(ix->device, &base);
+  st = scratch_address(ix->device, &base);
   if (st != NR_OK) return st;
   char *w = static_cast<char *>(base);
   cudaStream_t s = (cudaStream_t)stream;
@@ -113,11 +107,10 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   if (e == cudaSuccess)
     e = nr_launch_refine(ix, d_queries, nq, k, (int)Lmax, (nr_seg *)(w + o_seg),
                          (int32_t *)(w + o_nL), (uint32_t *)(w + o_slen), d_out_ids, d_out_dists,
-                         stats, (unsigned int *)(w + o_count), nullptr, s);
+                         stats, (unsigned int *)(w + o_count), (int32_t *)(w + o_perm), s);
   // statistics of this call are read from the array by nr_last_stats / nr_query_stats
   ix->d_stats = stats;
   ix->last_nq = nq;
   ix->timed_last = false;
-  if (e == cudaSuccess) return NR_OK;
-  return e == cudaErrorMemoryAllocation ? NR_ERR_OOM : NR_ERR_CUDA;
+  return cuda_status(e);
 }

@@ -209,7 +209,8 @@ __device__ __forceinline__ int select_tail_smem(const SelectParams &sp, uint64_t
 // One query: codes[0..np) -> the kept clusters C^dir U C^cent in (d, cluster)
 // order and their refinement segments. Writes seg[i] = (first row, stream
 // position) for i < nl, and L[i] (cluster index, -1 padded to Lmax) when L is
-// not null. slog: the query's b logits in shared memory; scratch:
+// not null; *n_scored = the number of centroid distances evaluated (every
+// cluster of every probed bucket). slog: the query's b logits in shared memory; scratch:
 // select_scratch_bytes(P, K_max) bytes of shared memory; slab: this query's
 // select_slab_bytes(P, K_max) bytes of global memory (null when that is 0);
 // warp_sums: 32 ints; sred: 2 unsigned. Returns nl; *total = stream length.
@@ -225,7 +226,8 @@ __device__ __forceinline__ int select_tail_smem(const SelectParams &sp, uint64_t
 __device__ __forceinline__ int select_block(const SelectParams &sp, const float *slog,
                                             const uint32_t *codes, int np, unsigned char *scratch,
                                             unsigned char *slab, int *warp_sums, unsigned *sred,
-                                            nr_seg *seg, int32_t *L, int Lmax, uint32_t *total) {
+                                            nr_seg *seg, int32_t *L, int Lmax, uint32_t *total,
+                                            int *n_scored) {
   const int tid = threadIdx.x, nt = blockDim.x;
   const int S_smem = select_smem_cap(sp.P, sp.K_max);
   const int S_full = select_sort_cap(sp.P, sp.K_max);
@@ -278,6 +280,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   }
   __syncthreads();
   int M = block_exclusive_scan(cnt, np, warp_sums);
+  *n_scored = M;  // every cluster of every probed bucket gets its distance
   // One pass over the candidates. C^dir keys are collected from the back of
   // the key array; the other clusters from the front when they are within the
   // gate of the running d_min. That gate is never tighter than the final one
@@ -531,7 +534,8 @@ __device__ __forceinline__ void sort_padded(uint64_t *k, int n) {
 __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const float *slog,
                                                 const uint32_t *codes, int np, unsigned char *seq,
                                                 int *warp_sums, unsigned *sred, nr_seg *seg,
-                                                int32_t *L, int Lmax, uint32_t *total) {
+                                                int32_t *L, int Lmax, uint32_t *total,
+                                                int *n_scored) {
   const int tid = threadIdx.x, nt = blockDim.x;
   const int C = sp.C, B = sp.b_batch, b = sp.b;
   uint64_t *Hb0 = reinterpret_cast<uint64_t *>(seq);
@@ -610,7 +614,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
   __syncthreads();
   const bool gate_off = sp.gate_off;
   float dmin = __int_as_float(0x7f800000);
-  int hN = 0, t_low = 0, b_proc = 0;
+  int hN = 0, t_low = 0, b_proc = 0, nbat = 0;  // nbat: clusters of the batches processed
   bool stop = false;
   uint64_t *H = Hb0, *Hn = Hb1;
   int i = 0;
@@ -634,6 +638,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
     const int sa = nsoff[i], sb = nsoff[j];
     for (int x = sa; x < sb && !stop; x += B) {
       const int nb = sb - x < B ? sb - x : B;
+      nbat += nb;
       if (tid == 0) sred[0] = 0xffffffffu;
       __syncthreads();
       for (int t = tid; t < nb; t += nt) {
@@ -714,6 +719,7 @@ __device__ __forceinline__ int select_block_seq(const SelectParams &sp, const fl
   // L = C^dir U H in (d, c) order, with the clusters' segments
   __syncthreads();
   const int nd = (int)st[1];
+  *n_scored = nd + nbat;  // C^dir of the bins entered and the batches processed
   sort_padded(dirk, nd);
   const int n = nd + hN;
   const int Q = (n + nt - 1) / nt;

@@ -49,7 +49,7 @@ class Params(ctypes.Structure):
 
 class Stats(ctypes.Structure):
     _fields_ = [("nq", ctypes.c_int64), ("candidates", ctypes.c_int64), ("rounds", ctypes.c_int64),
-                ("clusters", ctypes.c_int64), ("probes", ctypes.c_int64)]
+                ("clusters", ctypes.c_int64), ("probes", ctypes.c_int64), ("scored", ctypes.c_int64)]
 
 
 def lib():
@@ -341,7 +341,8 @@ class Index:
     def query_stats(self, nq, stream=None):
         import torch
 
-        st = torch.empty((nq, 4), dtype=torch.int64, device=self._dev())
+        # per query: candidates, rounds, |L|, probes, centroid distances evaluated
+        st = torch.empty((nq, 5), dtype=torch.int64, device=self._dev())
         _check("nr_query_stats", lib().nr_query_stats(self.h, _ptr(st), nq, _stream(stream)))
         return st
 

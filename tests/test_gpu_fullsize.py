@@ -63,13 +63,14 @@ def test_full_batch_sampled_parity(name):
     ix.close()
 
 
-def test_1b_sampled_parity():
-    """1e9 uint8 vectors, index built on the GPU, the whole 10,000-query batch in
-    one nr_search_logits call at the benchmark's operating point; 100 sampled
-    queries checked against the oracle, which answers them from the sub-index
-    of the buckets its own probe lists name (its own logits too). End to end
-    (GPU encoder), Recall@10 on the sample agrees with the oracle's within
-    0.002 against exact k-NN."""
+@pytest.mark.parametrize("name,sample_n", [("u8-100m", 200), ("u8-1b", 100)])
+def test_gpu_built_sampled_parity(name, sample_n):
+    """1e8 and 1e9 uint8 vectors, index built on the GPU, the whole
+    10,000-query batch in one nr_search_logits call at the benchmark's
+    operating point; sample_n sampled queries checked against the oracle,
+    which answers them from the sub-index of the buckets its own probe lists
+    name (its own logits too). End to end (GPU encoder), Recall@10 on the
+    sample agrees with the oracle's within 0.002 against exact k-NN."""
     torch = need_cuda()
     import os
     import tempfile
@@ -78,12 +79,12 @@ def test_1b_sampled_parity():
     from paper_2608_15438_gb300 import neuroute as nr
 
     torch.cuda.empty_cache()
-    w = synth.WORKLOADS["u8-1b"]
-    op = bench.OPERATING_POINTS["u8-1b"]
+    w = synth.WORKLOADS[name]
+    op = bench.OPERATING_POINTS[name]
     P, C = op["P"], op["C"]
     dev = torch.device("cuda", 0)
     ix, _ = bench.gpu_index(w, torch, nr, dev)
-    kw = bench.op_params(w, ix)       # the calibrated gate and S_max, fitted on this index
+    kw = bench.op_params(w, ix)       # a calibrated gate and S_max are fitted on this index
     qs = synth.queries(w)
     lg = oracle.encode_weights(synth.encoder_weights(w), w.in_scale, qs)
     dq = torch.from_numpy(qs).cuda()
@@ -92,7 +93,7 @@ def test_1b_sampled_parity():
     st = ix.query_stats(w.nq)
     torch.cuda.synchronize()
     ids, d, st = ids.cpu().numpy(), d.cpu().numpy(), st.cpu().numpy()
-    sample = np.linspace(0, w.nq - 1, 100).astype(np.int64)
+    sample = np.linspace(0, w.nq - 1, sample_n).astype(np.int64)
     p = oracle.params(**bench.method_kw(kw))
     with tempfile.TemporaryDirectory() as td:
         sub = os.path.join(td, "sub.nrix")
@@ -111,3 +112,44 @@ def test_1b_sampled_parity():
     r_orc = recall(ids_oe, truth)
     assert abs(r_gpu - r_orc) <= 0.002 + 1e-12, (r_gpu, r_orc)
     ix.close()
+    del ix
+    torch.cuda.empty_cache()
+
+
+def test_ground_truth_1e8_against_oracle_bruteforce():
+    """The benchmark's ground truth over 1e8 uint8 rows regenerated on the GPU
+    (bench.ground_truth_rows: TF32 matmul, exact for uint8, with the group
+    pre-selection) equals the oracle's brute-force k-NN on 200 queries: the
+    oracle scans the same rows drawn by the host generator, chunk by chunk,
+    and the chunks' exact top-k lists are merged by (distance, id)."""
+    torch = need_cuda()
+    import bench
+
+    w = synth.WORKLOADS["u8-100m"]
+    k, nq = 10, 200
+    qs = synth.queries(w, nq)
+    dev = torch.device("cuda", 0)
+    got = bench.ground_truth_rows(torch, w, torch.from_numpy(qs).to(dev), k, dev)
+    best_i = np.full((nq, k), -1, np.int64)
+    best_d = np.full((nq, k), np.inf)
+    got_d = np.full((nq, k), -1, np.int64)
+    chunk = 10_000_000
+    for r0 in range(0, w.n, chunk):
+        m = min(chunk, w.n - r0)
+        X = synth.mixture(w, synth.SEED_DATA, r0, m)
+        ci, cd = oracle.bruteforce(X, qs, k)
+        ai = np.concatenate([best_i, ci + r0], 1)
+        ad = np.concatenate([best_d, cd.astype(np.float64)], 1)
+        for qi in range(nq):
+            o = np.lexsort((ai[qi], ad[qi]))[:k]
+            best_i[qi], best_d[qi] = ai[qi][o], ad[qi][o]
+        # the distance of each GPU-found id, from the rows of this chunk
+        inside = (got >= r0) & (got < r0 + m)
+        if inside.any():
+            qq, kk = np.nonzero(inside)
+            rows = X[got[qq, kk] - r0].astype(np.int64)
+            got_d[qq, kk] = ((rows - qs[qq].astype(np.int64)) ** 2).sum(1)
+        del X
+    assert np.all(got_d >= 0)
+    # the same distances at every rank (ids may differ only among equal distances)
+    assert np.array_equal(np.sort(got_d, 1), best_d.astype(np.int64))

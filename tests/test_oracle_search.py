@@ -119,11 +119,13 @@ def test_tiny_invariants(tiny_index):
             idmap = ix.ids()
         member_ids = set(int(idmap[r]) for r in rows)
         assert set(ids[i][valid].tolist()) <= member_ids
-        # every cluster of a probed bucket is accounted for
+        # every cluster of a probed bucket is accounted for, and each had its
+        # centroid distance evaluated (the fifth statistic)
         allc = set()
         for u in codes:
             allc.update(range(bkt[u], bkt[u + 1]))
         assert set(L.tolist()) <= allc
+        assert st[i, 4] == len(allc) == int((bkt[codes.astype(np.int64) + 1] - bkt[codes]).sum())
 
 
 def test_tiny_recall_grows_with_budget(tiny_index):

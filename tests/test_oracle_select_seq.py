@@ -42,26 +42,29 @@ BASE = dict(cent_mode=1, s_max=1.0, n_bins=2, b_batch=2, b_min=2, c_t_low=1, c_u
             c_alpha_front=0.5, gate_m0=0.0, gate_m1=1.0)
 
 
-@pytest.mark.parametrize("kw,C,want_L,want_d,want_batches", [
+# want_scored: centroid distances evaluated = the C^dir cluster 2 of bin 1 plus
+# the clusters of the batches processed ([0, 1], [3, 4], [5, 6], [7, 8], then [9])
+@pytest.mark.parametrize("kw,C,want_L,want_d,want_batches,want_scored", [
     # bin 0: batch [0, 1]: d_min 1, theta 2, H = {0}. bin 1: C^dir {2};
     # [3, 4]: d_min 0.25, theta 0.5 evicts 0, H = {3}; [5, 6]: H = {3, 5}, full;
     # [7, 8]: nothing within 0.5 -> low, t_low 1, H full, 2 bins -> stop before [9]
-    (dict(), 2, [3, 5, 2], [0.25, 0.25, 9.0], 4),
+    (dict(), 2, [3, 5, 2], [0.25, 0.25, 9.0], 4, 1 + 8),
     # no early stop: [9]: d_min 0.0625, theta 0.125 evicts 3 and 5, H = {9}
-    (dict(c_t_low=0), 2, [9, 2], [0.0625, 9.0], 5),
+    (dict(c_t_low=0), 2, [9, 2], [0.0625, 9.0], 5, 1 + 9),
     # B_min = 3 bins is never reached: no stop
-    (dict(b_min=3), 2, [9, 2], [0.0625, 9.0], 5),
+    (dict(b_min=3), 2, [9, 2], [0.0625, 9.0], 5, 1 + 9),
     # C = 3: the heap is never full, no stop
-    (dict(), 3, [9, 2], [0.0625, 9.0], 5),
+    (dict(), 3, [9, 2], [0.0625, 9.0], 5, 1 + 9),
     # gate off: H keeps the C smallest of everything seen: (0.0625, 9), (0.25, 3)
-    (dict(gate_m0=float("inf"), c_t_low=0), 2, [9, 3, 2], [0.0625, 0.25, 9.0], 5),
+    (dict(gate_m0=float("inf"), c_t_low=0), 2, [9, 3, 2], [0.0625, 0.25, 9.0], 5, 1 + 9),
 ])
-def test_hand_worked_sequence(tmp_path, kw, C, want_L, want_d, want_batches):
+def test_hand_worked_sequence(tmp_path, kw, C, want_L, want_d, want_batches, want_scored):
     ix = hand_index(tmp_path)
     logit, codes, scores = hand_probes()
-    L, dL, ndir, nb = ix.cluster_list_seq(logit, codes, scores, C, oracle.params(**{**BASE, **kw}))
+    L, dL, ndir, nb, nsc = ix.cluster_list_seq(logit, codes, scores, C,
+                                               oracle.params(**{**BASE, **kw}), with_scored=True)
     assert list(L) == want_L and list(dL) == want_d
-    assert ndir == 1 and nb == want_batches
+    assert ndir == 1 and nb == want_batches and nsc == want_scored
 
 
 def test_order_independent_stage_without_stop_equals_mode_0(tmp_path):

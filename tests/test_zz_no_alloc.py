@@ -58,4 +58,42 @@ def test_static_scratch_search_matches_workspace_search(tmp_path):
                             ctypes.c_void_p(out_i.data_ptr()), ctypes.c_void_p(out_d.data_ptr()),
                             stream)
     assert st == -1  # NR_ERR_INVALID_ARG
+    # the arguments are checked as nr_search checks them: the sequential
+    # centroid stage refuses probe budgets above 2048 on both entry points
+    ix.set_params(cent_mode=1)
+    args = (ix.h, ctypes.c_void_p(dq.data_ptr()), 4, k, 3000, 64, ctypes.c_void_p(out_i.data_ptr()),
+            ctypes.c_void_p(out_d.data_ptr()), stream)
+    assert L.nr_search_static(*args) == -1
+    assert L.nr_search(*args) == -1
+    ix.close()
+
+
+def test_static_scratch_search_global_sort_slabs(tmp_path):
+    """Budgets whose candidate clusters exceed shared memory (P * K_max up to
+    65,536, sorted in global slabs inside the fixed array) give nr_search's
+    results too."""
+    torch = need_cuda()
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    path, _, _ = build_small(tmp_path, "tiny", n=30000, bits=12, k_max=16, t=4, name="slab")
+    ix = nr.Index(path, 0)
+    assert ix.k_max == 16
+    w = synth.WORKLOADS["tiny"]
+    dq = torch.from_numpy(synth.queries(w, 24)).cuda()
+    k, P, C = 10, 4096, 256
+    ref_ids, ref_d = ix.search(dq, k, P, C)
+    ref_st = ix.query_stats(dq.shape[0])
+    torch.cuda.synchronize()
+    L = nr.lib()
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    for _ in range(2):
+        ids = torch.full((dq.shape[0], k), -7, dtype=torch.int64, device="cuda")
+        d = torch.full((dq.shape[0], k), -7.0, dtype=torch.float32, device="cuda")
+        st = L.nr_search_static(ix.h, ctypes.c_void_p(dq.data_ptr()), dq.shape[0], k, P, C,
+                                ctypes.c_void_p(ids.data_ptr()), ctypes.c_void_p(d.data_ptr()),
+                                stream)
+        assert st == nr.NR_OK
+        torch.cuda.synchronize()
+        assert torch.equal(ids, ref_ids) and torch.equal(d, ref_d)
+        assert torch.equal(ix.query_stats(dq.shape[0]), ref_st)
     ix.close()
