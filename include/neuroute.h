@@ -318,6 +318,19 @@ nr_status nr_last_stats(nr_index *ix, nr_stats *out);
 nr_status nr_enable_timing(nr_index *ix, int on);
 nr_status nr_last_timing(nr_index *ix, float *ms);
 
+/* Measurement utility, not part of the search: the rate at which the GPU
+ * `device` reads rows at random. n rows of row_bytes (a multiple of 16, at
+ * most 1024) at well-mixed pseudo-random indices below `rows` are read from a
+ * rows x row_bytes array, one row per thread, with L2 evicted before each of
+ * reps runs; *h_gbs = row bytes read per second of the best run, in GB/s.
+ * It bounds a kernel whose bytes are random row gathers, as the centroid
+ * stage's are (Sec. 3.5: C_q centroid rows a query), the way the copy
+ * bandwidth bounds a stream. Allocates rows * row_bytes + 4 n + 512 MiB of
+ * device memory for the call and frees it; synchronous.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_OOM, NR_ERR_CUDA. */
+nr_status nr_measure_gather(int device, int64_t rows, int row_bytes, int64_t n, int reps,
+                            double *h_gbs);
+
 /* Number of kernels the library launched since load (all entry points). */
 int64_t nr_kernel_launches(const nr_index *ix);
 

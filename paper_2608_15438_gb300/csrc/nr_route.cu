@@ -1,7 +1,7 @@
 // K2 route: binarisation (Eq. 10), deviation scores (Sec. 3.2.3) and the
 // probe list of Algorithm 1: one block per query by threshold enumeration
-// (nrq::route_block) for probe budgets up to 1024 without the R_max filter,
-// else one warp per query (nrq::route_warp).
+// (nrq::route_block) without the R_max filter or the non-empty budget, else
+// one warp per query (nrq::route_warp).
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -24,7 +24,6 @@ __global__ void route_kernel(nrq::RouteParams rp, const float *__restrict__ logi
 }
 
 // One 128-thread block per query: the threshold enumeration (route_block).
-template <int E>
 __global__ void __launch_bounds__(nrq::kRouteThreads) route_block_kernel(
     nrq::RouteParams rp, const float *__restrict__ logits, int64_t nq, uint32_t *__restrict__ codes,
     int32_t *__restrict__ nprobe) {
@@ -32,21 +31,9 @@ __global__ void __launch_bounds__(nrq::kRouteThreads) route_block_kernel(
   const int64_t q = blockIdx.x;
   if (q >= nq) return;
   uint32_t *out = codes + (size_t)q * rp.P;
-  const int n = nrq::route_block<E>(rp, logits + q * rp.b, smem, out);
+  const int n = nrq::route_block(rp, logits + q * rp.b, smem, out);
   for (int t = n + (int)threadIdx.x; t < rp.P; t += nrq::kRouteThreads) out[t] = 0xffffffffu;
   if (threadIdx.x == 0) nprobe[q] = n;
-}
-
-template <int E>
-cudaError_t launch_route_block(const nrq::RouteParams &rp, const float *d_logits, int64_t nq,
-                               uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
-  const size_t smem = nrq::route_block_bytes(E, rp.P);
-  cudaError_t e = cudaFuncSetAttribute(route_block_kernel<E>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  route_block_kernel<E><<<(unsigned)nq, nrq::kRouteThreads, smem, s>>>(rp, d_logits, nq, d_codes,
-                                                                       d_nprobe);
-  return cudaGetLastError();
 }
 
 }  // namespace
@@ -72,21 +59,15 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
   const nrq::RouteParams rpb = nr_route_params(ix, P);  // before the launch configuration
-  if (ix->params.r_max <= 0 && !ix->params.nonempty_budget) {  // threshold enumeration (P <= 1024)
-    cudaError_t e = cudaSuccess;
-    bool done = true;
-    switch (nrq::route_block_e(P)) {
-      case 1: e = launch_route_block<1>(rpb, d_logits, nq, d_codes, d_nprobe, s); break;
-      case 2: e = launch_route_block<2>(rpb, d_logits, nq, d_codes, d_nprobe, s); break;
-      case 4: e = launch_route_block<4>(rpb, d_logits, nq, d_codes, d_nprobe, s); break;
-      case 8: e = launch_route_block<8>(rpb, d_logits, nq, d_codes, d_nprobe, s); break;
-      case 16: e = launch_route_block<16>(rpb, d_logits, nq, d_codes, d_nprobe, s); break;
-      default: done = false;
-    }
-    if (done) {
-      ix->launches += 1;
-      return e;
-    }
+  if (ix->params.r_max <= 0 && !ix->params.nonempty_budget) {  // threshold enumeration
+    const size_t smem = nrq::route_block_bytes(P);
+    cudaError_t e = cudaFuncSetAttribute(route_block_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    route_block_kernel<<<(unsigned)nq, nrq::kRouteThreads, smem, s>>>(rpb, d_logits, nq, d_codes,
+                                                                       d_nprobe);
+    ix->launches += 1;
+    return cudaGetLastError();
   }
   const size_t per_warp = nr_route_heap_bytes(rpb.Q);
   // warps per block: the choice that packs the most warps into an SM's

@@ -195,68 +195,78 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
 // query. The flip sets with cost <= T form a subtree of the tree above (costs
 // never decrease along an edge), so for any T with at least P - 1 of them, the
 // first P - 1 sets in key order are the P - 1 smallest keys of that subtree:
-// enumerate it breadth first, sort it, keep the front. T comes from counting
+// enumerate it breadth first, order it, keep the front. T comes from counting
 // subsets by cost on a grid of kRouteBins steps D over [0, T_range], T_range
 // the cost of ranks {0..m-1} with 2^m >= P (its 2^m - 1 subsets cost no more,
 // so the P - 1-th set does not either): each deviation rounded up to
 // s_r = floor(delta_r / D) + 1 steps, the number of subsets with sum of steps
 // <= c is a dynamic program over the ranks, and every such subset costs at most
 // c D in exact arithmetic, below c D (1 + 2^-16) after fp32 rounding. The
-// smallest c whose count reaches P (the empty set included) gives T. Keys,
-// ties and codes are those of route_warp; a subtree larger than the capacity,
-// the R_max filter, or P above 1024 take route_warp (warp 0 of the block).
+// smallest c whose count reaches P (the empty set included) gives T.
+//
+// The subtree's keys are ordered by a bucket sort: kRouteBuckets buckets over
+// [0, largest cost] by a monotone map of the cost (a key in a lower bucket
+// costs less, so buckets keep key order), a histogram and scan give each
+// bucket's range, and a key's rank is its bucket's start plus the number of
+// smaller keys in its bucket. Keys are distinct (distinct rank masks), so the
+// ranks are a permutation and the first P - 1 of them are the listed sets.
+// Keys, ties and codes are those of route_warp; the R_max filter, a subtree
+// beyond the capacity of 2P keys, or a bucket above kRouteBucketMax keys take
+// route_warp (warp 0 of the block).
 constexpr int kRouteThreads = 128;
 constexpr int kRouteBins = 512;
 constexpr int kRouteDp = kRouteBins + 32;  // sums of rounded-up steps overshoot by < 1 per rank
+constexpr int kRouteBuckets = 1024;        // <= 2 kRouteDp: the histogram reuses the count arrays
+constexpr int kRouteBucketMax = 64;
 
-// Keys a thread holds in the final sort: the smallest power of two E with
-// 128 E >= 2 P, or 0 when P > 1024 (route_warp only).
-__host__ __device__ inline int route_block_e(int P) {
-  int E = 1;
-  while (E * kRouteThreads < 2 * P && E < 16) E <<= 1;
-  return E * kRouteThreads >= 2 * P ? E : 0;
+// Subtree capacity for probe budget P: 2P keys, a whole number of block strides.
+__host__ __device__ inline int route_cap(int P) {
+  const int c = 2 * P;
+  return c <= kRouteThreads ? kRouteThreads : (c + kRouteThreads - 1) / kRouteThreads * kRouteThreads;
 }
 
 struct RouteSmem {
-  uint64_t *keys;   // subtree keys, then the sort's padded runs; or route_warp's heap
-  float *costp;     // per subtree key: its cost without the largest rank
-  uint32_t *dp;     // two count arrays of kRouteDp
+  uint64_t *keys;   // subtree keys; or route_warp's heap
+  float *costp;     // per subtree key: its cost without the largest rank; then the bucket order
+  uint32_t *dp;     // two count arrays of kRouteDp; then the bucket histogram
+  uint32_t *flip;   // [3][256]: bit mask of the ranks in each byte of a rank mask
   float *ssd;       // deviation of rank r
   int *bitidx;      // bit index of rank r
-  int *ctl;         // [0] tail, [1] chosen bin, [2] u0, [3] route_warp's count
+  int *ctl;         // [0] tail, [1] chosen bin, [2] u0, [3] route_warp's count, [4] largest
+                    // cost bits, [5] largest bucket
 };
 
-__host__ __device__ inline size_t route_region_bytes(int E, int P) {
-  const size_t sort = (size_t)(E * kRouteThreads + (E * kRouteThreads) / 16) * 8;
+__host__ __device__ inline size_t route_region_bytes(int P) {
+  const size_t keys = (size_t)route_cap(P) * 8;
   const size_t heap = route_heap_bytes(P);  // route_warp with Q = P
-  return ((sort > heap ? sort : heap) + 15) & ~(size_t)15;
+  return ((keys > heap ? keys : heap) + 15) & ~(size_t)15;
 }
 
-__host__ __device__ inline size_t route_block_bytes(int E, int P) {
-  return route_region_bytes(E, P) + (size_t)E * kRouteThreads * 4 + (size_t)2 * kRouteDp * 4 +
-         32 * 4 + 32 * 4 + 16 * 4;
+__host__ __device__ inline size_t route_block_bytes(int P) {
+  return route_region_bytes(P) + (size_t)route_cap(P) * 4 + (size_t)2 * kRouteDp * 4 +
+         (size_t)3 * 256 * 4 + 32 * 4 + 32 * 4 + 16 * 4;
 }
 
-__device__ __forceinline__ RouteSmem route_carve(unsigned char *base, int E, int P) {
+__device__ __forceinline__ RouteSmem route_carve(unsigned char *base, int P) {
   RouteSmem m;
   m.keys = reinterpret_cast<uint64_t *>(base);
-  m.costp = reinterpret_cast<float *>(base + route_region_bytes(E, P));
-  m.dp = reinterpret_cast<uint32_t *>(m.costp + E * kRouteThreads);
-  m.ssd = reinterpret_cast<float *>(m.dp + 2 * kRouteDp);
+  m.costp = reinterpret_cast<float *>(base + route_region_bytes(P));
+  m.dp = reinterpret_cast<uint32_t *>(m.costp + route_cap(P));
+  m.flip = m.dp + 2 * kRouteDp;
+  m.ssd = reinterpret_cast<float *>(m.flip + 3 * 256);
   m.bitidx = reinterpret_cast<int *>(m.ssd + 32);
   m.ctl = m.bitidx + 32;
   return m;
 }
 
 // Writes codes[0..n) (any address space) and returns n, uniform in the block.
-// Called by the whole 128-thread block; smem: route_block_bytes(E, P) bytes.
-template <int E>
+// Called by the whole 128-thread block; smem: route_block_bytes(P) bytes.
 __device__ __forceinline__ int route_block(const RouteParams &rp, const float *__restrict__ logit,
                                            unsigned char *smem, uint32_t *codes) {
-  constexpr int cap = E * kRouteThreads;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = rp.b, bsel = rp.bsel, P = rp.P;
-  const RouteSmem m = route_carve(smem, E, P);
+  const int cap = route_cap(P);
+  const RouteSmem m = route_carve(smem, P);
   if (warp == 0) {  // deviations, base code and ranks (Eq. 10, Sec. 3.2.3)
     float dj = __int_as_float(0x7f800000);
     bool bit = false;
@@ -280,10 +290,20 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
       m.ctl[0] = 0;
       m.ctl[1] = -1;
       m.ctl[2] = (int)u0;
+      m.ctl[4] = 0;
+      m.ctl[5] = 0;
     }
   }
   __syncthreads();
   const uint32_t u0 = (uint32_t)m.ctl[2];
+  // flip[t][v] = the bits of the ranks 8t + i, i in v (ApplyFlips by bytes)
+  for (int e = tid; e < 3 * 256; e += kRouteThreads) {
+    const int t = e >> 8, v = e & 255;
+    uint32_t f = 0;
+    for (int i = 0; i < 8; ++i)
+      if (((v >> i) & 1) && 8 * t + i < b) f |= 1u << m.bitidx[8 * t + i];
+    m.flip[e] = f;
+  }
   bool use_heap = rp.rmax > 0;
   float T = __int_as_float(0x7f800000);  // the whole tree
   const bool none = P <= 1 || bsel < 1;
@@ -408,6 +428,33 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
     }
     if (tail > cap) use_heap = true;  // uniform: every thread read the same tail
   }
+  int *order = reinterpret_cast<int *>(m.costp);  // bucket order of the keys
+  uint32_t *hist = m.dp;                           // kRouteBuckets counts, then bucket ends
+  float scale = 0.0f;
+  if (!use_heap && tail > 0) {
+    // bucket histogram over [0, largest cost]; costs are non-negative, so
+    // their bits order as their values
+    for (int i = tid; i < kRouteBuckets; i += kRouteThreads) hist[i] = 0u;
+    uint32_t cmax = 0u;
+    for (int i = tid; i < tail; i += kRouteThreads) cmax = max(cmax, (uint32_t)(m.keys[i] >> 32));
+    cmax = __reduce_max_sync(kFull, cmax);
+    if (lane == 0) atomicMax(reinterpret_cast<unsigned *>(&m.ctl[4]), cmax);
+    __syncthreads();
+    const float top = __uint_as_float((uint32_t)m.ctl[4]);
+    if (top > 0.0f && top < __int_as_float(0x7f800000))
+      scale = __fdiv_rn((float)kRouteBuckets, top);
+    for (int i = tid; i < tail; i += kRouteThreads) {
+      const float cost = __uint_as_float((uint32_t)(m.keys[i] >> 32));
+      atomicAdd(&hist[min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale))], 1u);
+    }
+    __syncthreads();
+    uint32_t bmax = 0u;
+    for (int i = tid; i < kRouteBuckets; i += kRouteThreads) bmax = max(bmax, hist[i]);
+    bmax = __reduce_max_sync(kFull, bmax);
+    if (lane == 0) atomicMax(reinterpret_cast<unsigned *>(&m.ctl[5]), bmax);
+    __syncthreads();
+    if (m.ctl[5] > kRouteBucketMax) use_heap = true;  // uniform
+  }
   if (use_heap) {
     __syncthreads();
     if (warp == 0) {
@@ -417,18 +464,56 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
     __syncthreads();
     return m.ctl[3];
   }
-  const int nout = min(P - 1, tail);
-  uint64_t r[E];
-  merge_sort_regs<E>(m.keys, tail, r);
   if (tid == 0) codes[0] = u0;
+  const int nout = min(P - 1, tail);
+  if (tail == 0) return 1;
+  // bucket ranges: an exclusive scan of the histogram (kRouteBuckets / 128
+  // buckets a thread), then a scatter in which each key takes the next slot
+  // of its bucket, leaving hist[z] = the end of bucket z
+  {
+    constexpr int per = kRouteBuckets / kRouteThreads;
+    uint32_t loc[per], sum = 0;
 #pragma unroll
-  for (int e = 0; e < E; ++e) {
-    const int i = tid * E + e;
-    if (i < nout) {
-      uint32_t flips = 0;
-      for (uint32_t mk = (uint32_t)r[e] & 0xffffffu; mk; mk &= mk - 1)
-        flips |= 1u << m.bitidx[__ffs(mk) - 1];
-      codes[1 + i] = u0 ^ flips;
+    for (int e = 0; e < per; ++e) {
+      loc[e] = hist[tid * per + e];
+      sum += loc[e];
+    }
+    uint32_t incl = sum;
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t v = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += v;
+    }
+    uint32_t *wsum = reinterpret_cast<uint32_t *>(m.ctl + 8);  // 4 warp totals
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    uint32_t run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += wsum[w];
+#pragma unroll
+    for (int e = 0; e < per; ++e) {
+      hist[tid * per + e] = run;
+      run += loc[e];
+    }
+    __syncthreads();
+  }
+  for (int i = tid; i < tail; i += kRouteThreads) {
+    const float cost = __uint_as_float((uint32_t)(m.keys[i] >> 32));
+    const int z = min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale));
+    order[atomicAdd(&hist[z], 1u)] = i;
+  }
+  __syncthreads();
+  // rank of each key = its bucket's start + the smaller keys of its bucket;
+  // the first P - 1 become codes u0 XOR flips
+  for (int i = tid; i < tail; i += kRouteThreads) {
+    const uint64_t key = m.keys[i];
+    const float cost = __uint_as_float((uint32_t)(key >> 32));
+    const int z = min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale));
+    const int lo = z > 0 ? (int)hist[z - 1] : 0, hi = (int)hist[z];
+    int r = lo;
+    for (int j = lo; j < hi; ++j) r += m.keys[order[j]] < key ? 1 : 0;
+    if (r < nout) {
+      const uint32_t mk = (uint32_t)key & 0xffffffu;
+      const uint32_t flips = m.flip[mk & 255] | m.flip[256 + ((mk >> 8) & 255)] | m.flip[512 + (mk >> 16)];
+      codes[1 + r] = u0 ^ flips;
     }
   }
   return 1 + nout;

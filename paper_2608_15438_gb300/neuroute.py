@@ -25,7 +25,8 @@ EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_f
            "nr_enable_timing", "nr_last_timing", "nr_kernel_launches", "nr_search_static",
            "nr_index_save", "nr_index_extract", "nr_index_thresholds", "nr_index_locate",
            "nr_centroid_dists", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
-           "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free"]
+           "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free",
+           "nr_measure_gather"]
 
 
 class NRError(RuntimeError):
@@ -76,6 +77,7 @@ def lib():
         L.nr_search_static.argtypes = [vp, vp, i64, i32, i32, i32, vp, vp, vp]
         L.nr_query_stats.argtypes = [vp, vp, i64, vp]
         L.nr_last_stats.argtypes = [vp, ctypes.POINTER(Stats)]
+        L.nr_measure_gather.argtypes = [i32, i64, i32, i64, i32, ctypes.POINTER(ctypes.c_double)]
         L.nr_enable_timing.argtypes = [vp, i32]
         L.nr_last_timing.argtypes = [vp, vp]
         L.nr_kernel_launches.argtypes = [vp]
@@ -123,6 +125,14 @@ def params(**kw) -> Params:
             raise KeyError(k)
         setattr(p, k, v)
     return p
+
+
+def measure_gather(device, rows, row_bytes, n=20_000_000, reps=5) -> float:
+    """GB/s at which the GPU reads rows at random (nr_measure_gather)."""
+    v = ctypes.c_double()
+    _check("nr_measure_gather", lib().nr_measure_gather(int(device), int(rows), int(row_bytes),
+                                                        int(n), int(reps), ctypes.byref(v)))
+    return v.value
 
 
 def _ptr(t):

@@ -67,14 +67,15 @@ def test_route_filters_bit_exact(tiny, torch, kw):
         assert np.array_equal(codes[i, : len(exp)], exp)
 
 
-@pytest.mark.parametrize("P", [2, 63, 64, 65, 128, 129, 256, 257, 512, 513, 777, 1024, 1025])
+@pytest.mark.parametrize("P", [2, 63, 64, 65, 128, 129, 256, 257, 512, 513, 777, 1024, 1025, 1536,
+                               2047, 2048, 2049, 4095, 4096])
 @pytest.mark.parametrize("kind", ["encoded", "ties"])
 def test_route_threshold_enumeration_bit_exact(tiny, torch, P, kind):
-    """Probe budgets up to 1024 take the block-wide threshold enumeration
-    (each capacity of its final sort and both sides of every boundary), 1025
-    the heap; logits on a grid of 1/8 around tau give deviations with many
-    ties and zeros, whose subtrees often outgrow the capacity (the block then
-    falls back to the heap)."""
+    """Every probe budget takes the block-wide threshold enumeration (both
+    sides of each multiple of the block's stride in the subtree capacity of 2P
+    keys); logits on a grid of 1/8 around tau give deviations with many ties
+    and zeros, whose subtrees often outgrow the capacity or crowd one cost
+    bucket of the final ordering (the block then falls back to the heap)."""
     ix, orc = tiny["ix"], tiny["orc"]
     tau = orc.tau()
     lg = tiny["lg"][:200]
