@@ -1,7 +1,7 @@
 // K2 route: binarisation (Eq. 10), deviation scores (Sec. 3.2.3) and the
 // probe list of Algorithm 1: one block per query by threshold enumeration
-// (nrq::route_block) without the R_max filter or the non-empty budget, else
-// one warp per query (nrq::route_warp).
+// (nrq::route_block) without the R_max filter, else one warp per query
+// (nrq::route_warp).
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -59,8 +59,8 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s) {
   if (nq <= 0) return cudaSuccess;
   const nrq::RouteParams rpb = nr_route_params(ix, P);  // before the launch configuration
-  if (ix->params.r_max <= 0 && !ix->params.nonempty_budget) {  // threshold enumeration
-    const size_t smem = nrq::route_block_bytes(P);
+  if (ix->params.r_max <= 0) {  // threshold enumeration
+    const size_t smem = nrq::route_block_bytes(P, rpb.nonempty, rpb.Q);
     cudaError_t e = cudaFuncSetAttribute(route_block_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

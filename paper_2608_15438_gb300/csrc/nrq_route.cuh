@@ -193,65 +193,84 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
 // ============================================================== route_block
 // The same probe list by a threshold enumeration, one 128-thread block per
 // query. The flip sets with cost <= T form a subtree of the tree above (costs
-// never decrease along an edge), so for any T with at least P - 1 of them, the
-// first P - 1 sets in key order are the P - 1 smallest keys of that subtree:
+// never decrease along an edge), so for any T with at least N - 1 of them, the
+// first N - 1 sets in key order are the N - 1 smallest keys of that subtree:
 // enumerate it breadth first, order it, keep the front. T comes from counting
 // subsets by cost on a grid of kRouteBins steps D over [0, T_range], T_range
-// the cost of ranks {0..m-1} with 2^m >= P (its 2^m - 1 subsets cost no more,
-// so the P - 1-th set does not either): each deviation rounded up to
+// the cost of ranks {0..m-1} with 2^m >= N (its 2^m - 1 subsets cost no more,
+// so the N - 1-th set does not either): each deviation rounded up to
 // s_r = floor(delta_r / D) + 1 steps, the number of subsets with sum of steps
 // <= c is a dynamic program over the ranks, and every such subset costs at most
 // c D in exact arithmetic, below c D (1 + 2^-16) after fp32 rounding. The
-// smallest c whose count reaches P (the empty set included) gives T.
+// smallest c whose count reaches N (the empty set included) gives T.
 //
 // The subtree's keys are ordered by a bucket sort: kRouteBuckets buckets over
 // [0, largest cost] by a monotone map of the cost (a key in a lower bucket
 // costs less, so buckets keep key order), a histogram and scan give each
 // bucket's range, and a key's rank is its bucket's start plus the number of
 // smaller keys in its bucket. Keys are distinct (distinct rank masks), so the
-// ranks are a permutation and the first P - 1 of them are the listed sets.
-// Keys, ties and codes are those of route_warp; the R_max filter, a subtree
-// beyond the capacity of 2P keys, or a bucket above kRouteBucketMax keys take
-// route_warp (warp 0 of the block).
+// ranks are a permutation.
+//
+// Plain budget: N = P, and the first P - 1 ranks become the codes after the
+// base code. Non-empty budget: N = min(Q, 2P, 4096) flip sets (the base code
+// included) are enumerated; the bucket occupancy of each of the first
+// min(N, Q) in key order is looked up (all lookups in flight at once), and a
+// scan over them in rank order lists the first P non-empty codes. When that
+// prefix holds fewer than P non-empty codes while more flip sets may be
+// examined (fewer than Q examined, and sets above T remain), the block takes
+// route_warp instead. Keys, ties and codes are those of route_warp; the R_max
+// filter, a subtree beyond its capacity of 2N keys, or a bucket above
+// kRouteBucketMax keys take route_warp too (warp 0 of the block).
 constexpr int kRouteThreads = 128;
 constexpr int kRouteBins = 512;
 constexpr int kRouteDp = kRouteBins + 32;  // sums of rounded-up steps overshoot by < 1 per rank
 constexpr int kRouteBuckets = 1024;        // <= 2 kRouteDp: the histogram reuses the count arrays
 constexpr int kRouteBucketMax = 64;
+constexpr int kRouteNonemptyMax = 4096;    // flip sets a block enumerates for the non-empty budget
 
-// Subtree capacity for probe budget P: 2P keys, a whole number of block strides.
-__host__ __device__ inline int route_cap(int P) {
-  const int c = 2 * P;
+// Flip sets (the base code included) the block enumerates.
+__host__ __device__ inline int route_enum_target(int P, int nonempty, int Q) {
+  if (!nonempty) return P;
+  int n = 2 * P < Q ? 2 * P : Q;
+  return n < kRouteNonemptyMax ? n : kRouteNonemptyMax;
+}
+// Subtree capacity for an enumeration of N: 2N keys, a whole number of block strides.
+__host__ __device__ inline int route_cap(int N) {
+  const int c = 2 * N;
   return c <= kRouteThreads ? kRouteThreads : (c + kRouteThreads - 1) / kRouteThreads * kRouteThreads;
 }
 
 struct RouteSmem {
   uint64_t *keys;   // subtree keys; or route_warp's heap
   float *costp;     // per subtree key: its cost without the largest rank; then the bucket order
+  uint32_t *rc;     // non-empty budget: code of rank r | occupied << 31
   uint32_t *dp;     // two count arrays of kRouteDp; then the bucket histogram
   uint32_t *flip;   // [3][256]: bit mask of the ranks in each byte of a rank mask
   float *ssd;       // deviation of rank r
   int *bitidx;      // bit index of rank r
   int *ctl;         // [0] tail, [1] chosen bin, [2] u0, [3] route_warp's count, [4] largest
-                    // cost bits, [5] largest bucket
+                    // cost bits, [5] largest bucket, [6] base code occupied, [8..11] warp totals
 };
 
-__host__ __device__ inline size_t route_region_bytes(int P) {
-  const size_t keys = (size_t)route_cap(P) * 8;
-  const size_t heap = route_heap_bytes(P);  // route_warp with Q = P
+__host__ __device__ inline size_t route_region_bytes(int N, int Q) {
+  const size_t keys = (size_t)route_cap(N) * 8;
+  const size_t heap = route_heap_bytes(Q);
   return ((keys > heap ? keys : heap) + 15) & ~(size_t)15;
 }
 
-__host__ __device__ inline size_t route_block_bytes(int P) {
-  return route_region_bytes(P) + (size_t)route_cap(P) * 4 + (size_t)2 * kRouteDp * 4 +
-         (size_t)3 * 256 * 4 + 32 * 4 + 32 * 4 + 16 * 4;
+// Shared memory of route_block for probe budget P (Q: route_warp's limit).
+__host__ __device__ inline size_t route_block_bytes(int P, int nonempty, int Q) {
+  const int N = route_enum_target(P, nonempty, Q);
+  return route_region_bytes(N, Q) + (size_t)route_cap(N) * 4 * (nonempty ? 2 : 1) +
+         (size_t)2 * kRouteDp * 4 + (size_t)3 * 256 * 4 + 32 * 4 + 32 * 4 + 16 * 4;
 }
 
-__device__ __forceinline__ RouteSmem route_carve(unsigned char *base, int P) {
+__device__ __forceinline__ RouteSmem route_carve(unsigned char *base, int N, int Q, int nonempty) {
   RouteSmem m;
   m.keys = reinterpret_cast<uint64_t *>(base);
-  m.costp = reinterpret_cast<float *>(base + route_region_bytes(P));
-  m.dp = reinterpret_cast<uint32_t *>(m.costp + route_cap(P));
+  m.costp = reinterpret_cast<float *>(base + route_region_bytes(N, Q));
+  m.rc = reinterpret_cast<uint32_t *>(m.costp + route_cap(N));
+  m.dp = m.rc + (nonempty ? route_cap(N) : 0);
   m.flip = m.dp + 2 * kRouteDp;
   m.ssd = reinterpret_cast<float *>(m.flip + 3 * 256);
   m.bitidx = reinterpret_cast<int *>(m.ssd + 32);
@@ -259,14 +278,20 @@ __device__ __forceinline__ RouteSmem route_carve(unsigned char *base, int P) {
   return m;
 }
 
+// Whether bucket `code` holds a cluster.
+__device__ __forceinline__ bool route_occupied(const RouteParams &rp, uint32_t code) {
+  return __ldg(&rp.bkt_off[code + 1]) != __ldg(&rp.bkt_off[code]);
+}
+
 // Writes codes[0..n) (any address space) and returns n, uniform in the block.
-// Called by the whole 128-thread block; smem: route_block_bytes(P) bytes.
+// Called by the whole 128-thread block; smem: route_block_bytes(P, nonempty, Q) bytes.
 __device__ __forceinline__ int route_block(const RouteParams &rp, const float *__restrict__ logit,
                                            unsigned char *smem, uint32_t *codes) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int b = rp.b, bsel = rp.bsel, P = rp.P;
-  const int cap = route_cap(P);
-  const RouteSmem m = route_carve(smem, P);
+  const int N = route_enum_target(P, rp.nonempty, rp.Q);
+  const int cap = route_cap(N);
+  const RouteSmem m = route_carve(smem, N, rp.Q, rp.nonempty);
   if (warp == 0) {  // deviations, base code and ranks (Eq. 10, Sec. 3.2.3)
     float dj = __int_as_float(0x7f800000);
     bool bit = false;
@@ -292,6 +317,7 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
       m.ctl[2] = (int)u0;
       m.ctl[4] = 0;
       m.ctl[5] = 0;
+      m.ctl[6] = rp.nonempty ? (route_occupied(rp, u0) ? 1 : 0) : 1;
     }
   }
   __syncthreads();
@@ -306,10 +332,10 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
   }
   bool use_heap = rp.rmax > 0;
   float T = __int_as_float(0x7f800000);  // the whole tree
-  const bool none = P <= 1 || bsel < 1;
-  if (!use_heap && !none && P - 1 < (1 << bsel) - 1) {
+  const bool none = N <= 1 || bsel < 1;
+  if (!use_heap && !none && N - 1 < (1 << bsel) - 1) {
     int mr = 0;
-    while ((1 << mr) < P) ++mr;  // mr <= bsel here
+    while ((1 << mr) < N) ++mr;  // mr <= bsel here
     float thi = 0.0f;
     for (int r = 0; r < mr; ++r) thi = __fadd_rn(thi, m.ssd[r]);
     const float trange = fminf(thi, rp.smax);
@@ -333,7 +359,7 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
         d0 = d1;
         d1 = t;
       }
-      if (warp == 0) {  // smallest c with count(sum of steps <= c) >= P
+      if (warp == 0) {  // smallest c with count(sum of steps <= c) >= N
         constexpr int per = kRouteDp / 32;
         uint32_t loc = 0;
         for (int i = 0; i < per; ++i) loc += d0[lane * per + i];
@@ -342,7 +368,7 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
           const uint32_t v = __shfl_up_sync(kFull, incl, o);
           if (lane >= o) incl += v;
         }
-        const unsigned hit = __ballot_sync(kFull, incl >= (uint32_t)P);
+        const unsigned hit = __ballot_sync(kFull, incl >= (uint32_t)N);
         if (hit) {
           const int src = __ffs(hit) - 1;
           if (lane == src) {
@@ -350,7 +376,7 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
             int c = lane * per;
             for (;; ++c) {
               run += d0[c];
-              if (run >= (uint32_t)P) break;
+              if (run >= (uint32_t)N) break;
             }
             m.ctl[1] = c;
           }
@@ -455,68 +481,106 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
     __syncthreads();
     if (m.ctl[5] > kRouteBucketMax) use_heap = true;  // uniform
   }
-  if (use_heap) {
-    __syncthreads();
-    if (warp == 0) {
-      const int n = route_warp(rp, logit, reinterpret_cast<unsigned char *>(m.keys), codes);
-      if (lane == 0) m.ctl[3] = n;
-    }
-    __syncthreads();
-    return m.ctl[3];
-  }
-  if (tid == 0) codes[0] = u0;
-  const int nout = min(P - 1, tail);
-  if (tail == 0) return 1;
-  // bucket ranges: an exclusive scan of the histogram (kRouteBuckets / 128
-  // buckets a thread), then a scatter in which each key takes the next slot
-  // of its bucket, leaving hist[z] = the end of bucket z
-  {
-    constexpr int per = kRouteBuckets / kRouteThreads;
-    uint32_t loc[per], sum = 0;
+  int nlist = 0;  // codes listed (uniform)
+  if (!use_heap) {
+    if (tail > 0) {
+      // bucket ranges: an exclusive scan of the histogram (kRouteBuckets /
+      // 128 buckets a thread), then a scatter in which each key takes the
+      // next slot of its bucket, leaving hist[z] = the end of bucket z
+      constexpr int per = kRouteBuckets / kRouteThreads;
+      uint32_t loc[per], sum = 0;
 #pragma unroll
-    for (int e = 0; e < per; ++e) {
-      loc[e] = hist[tid * per + e];
-      sum += loc[e];
+      for (int e = 0; e < per; ++e) {
+        loc[e] = hist[tid * per + e];
+        sum += loc[e];
+      }
+      uint32_t incl = sum;
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t v = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += v;
+      }
+      uint32_t *wsum = reinterpret_cast<uint32_t *>(m.ctl + 8);  // 4 warp totals
+      if (lane == 31) wsum[warp] = incl;
+      __syncthreads();
+      uint32_t run = incl - sum;
+      for (int w = 0; w < warp; ++w) run += wsum[w];
+#pragma unroll
+      for (int e = 0; e < per; ++e) {
+        hist[tid * per + e] = run;
+        run += loc[e];
+      }
+      __syncthreads();
+      for (int i = tid; i < tail; i += kRouteThreads) {
+        const float cost = __uint_as_float((uint32_t)(m.keys[i] >> 32));
+        const int z = min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale));
+        order[atomicAdd(&hist[z], 1u)] = i;
+      }
+      __syncthreads();
     }
-    uint32_t incl = sum;
+    // rank of each key = its bucket's start + the smaller keys of its bucket;
+    // its code is u0 XOR the flips of its rank mask
+    const int nexam = rp.nonempty ? min(tail, rp.Q - 1) : min(tail, P - 1);
+    for (int i = tid; i < tail; i += kRouteThreads) {
+      const uint64_t key = m.keys[i];
+      const float cost = __uint_as_float((uint32_t)(key >> 32));
+      const int z = min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale));
+      const int lo = z > 0 ? (int)hist[z - 1] : 0, hi = (int)hist[z];
+      int r = lo;
+      for (int j = lo; j < hi; ++j) r += m.keys[order[j]] < key ? 1 : 0;
+      if (r < nexam) {
+        const uint32_t mk = (uint32_t)key & 0xffffffu;
+        const uint32_t code =
+            u0 ^ (m.flip[mk & 255] | m.flip[256 + ((mk >> 8) & 255)] | m.flip[512 + (mk >> 16)]);
+        if (rp.nonempty) m.rc[r] = code | (route_occupied(rp, code) ? 0x80000000u : 0u);
+        else codes[1 + r] = code;
+      }
+    }
+    if (!rp.nonempty) {
+      if (tid == 0) codes[0] = u0;
+      return 1 + nexam;
+    }
+    // non-empty budget: the non-empty codes of ranks [0, nexam) in rank
+    // order, after the base code when it is non-empty
+    __syncthreads();
+    const int base_ne = m.ctl[6];
+    const int per = (nexam + kRouteThreads - 1) / kRouteThreads;
+    const int r0 = min(nexam, tid * per), r1 = min(nexam, r0 + per);
+    int cnt = 0;
+    for (int r = r0; r < r1; ++r) cnt += (int)(m.rc[r] >> 31);
+    int incl = cnt;
     for (int o = 1; o < 32; o <<= 1) {
-      const uint32_t v = __shfl_up_sync(kFull, incl, o);
+      const int v = __shfl_up_sync(kFull, incl, o);
       if (lane >= o) incl += v;
     }
-    uint32_t *wsum = reinterpret_cast<uint32_t *>(m.ctl + 8);  // 4 warp totals
+    int *wsum = m.ctl + 8;
+    __syncthreads();  // the warp totals of the scan above are read
     if (lane == 31) wsum[warp] = incl;
     __syncthreads();
-    uint32_t run = incl - sum;
-    for (int w = 0; w < warp; ++w) run += wsum[w];
-#pragma unroll
-    for (int e = 0; e < per; ++e) {
-      hist[tid * per + e] = run;
-      run += loc[e];
+    int before = incl - cnt, total = 0;
+    for (int w = 0; w < 4; ++w) {
+      before += w < warp ? wsum[w] : 0;
+      total += wsum[w];
     }
-    __syncthreads();
-  }
-  for (int i = tid; i < tail; i += kRouteThreads) {
-    const float cost = __uint_as_float((uint32_t)(m.keys[i] >> 32));
-    const int z = min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale));
-    order[atomicAdd(&hist[z], 1u)] = i;
+    // fewer than P non-empty codes, fewer than Q flip sets examined and sets
+    // above the enumerated cost left: the heap continues where this stopped
+    const bool complete = tail >= rp.Q - 1 || !(T < rp.smax);
+    if (base_ne + total >= P || complete) {
+      if (tid == 0 && base_ne) codes[0] = u0;
+      int pos = base_ne + before;
+      for (int r = r0; r < r1 && pos < P; ++r)
+        if (m.rc[r] >> 31) codes[pos++] = m.rc[r] & 0x7fffffffu;
+      return min(P, base_ne + total);
+    }
+    use_heap = true;  // uniform
   }
   __syncthreads();
-  // rank of each key = its bucket's start + the smaller keys of its bucket;
-  // the first P - 1 become codes u0 XOR flips
-  for (int i = tid; i < tail; i += kRouteThreads) {
-    const uint64_t key = m.keys[i];
-    const float cost = __uint_as_float((uint32_t)(key >> 32));
-    const int z = min(kRouteBuckets - 1, (int)__fmul_rn(cost, scale));
-    const int lo = z > 0 ? (int)hist[z - 1] : 0, hi = (int)hist[z];
-    int r = lo;
-    for (int j = lo; j < hi; ++j) r += m.keys[order[j]] < key ? 1 : 0;
-    if (r < nout) {
-      const uint32_t mk = (uint32_t)key & 0xffffffu;
-      const uint32_t flips = m.flip[mk & 255] | m.flip[256 + ((mk >> 8) & 255)] | m.flip[512 + (mk >> 16)];
-      codes[1 + r] = u0 ^ flips;
-    }
+  if (warp == 0) {
+    const int n = route_warp(rp, logit, reinterpret_cast<unsigned char *>(m.keys), codes);
+    if (lane == 0) m.ctl[3] = n;
   }
-  return 1 + nout;
+  __syncthreads();
+  nlist = m.ctl[3];
+  return nlist;
 }
 
 }  // namespace nrq

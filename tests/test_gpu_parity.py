@@ -112,16 +112,25 @@ def test_route_threshold_filters_bit_exact(tiny, torch, kw, P):
         assert np.array_equal(codes[i, : len(exp)], exp), i
 
 
-@pytest.mark.parametrize("P", [1, 8, 100, 1024, 4096])
-@pytest.mark.parametrize("kw", [dict(), dict(s_max=0.3), dict(l_sel=9, r_max=3)])
+@pytest.mark.parametrize("P", [1, 2, 8, 100, 500, 1024, 2048, 4096])
+@pytest.mark.parametrize("kw", [dict(), dict(s_max=0.3), dict(s_max=0.05), dict(l_sel=9, r_max=3),
+                                dict(l_sel=6), "ties"])
 def test_route_nonempty_budget_bit_exact(tiny, torch, P, kw):
     """The non-empty budget (D3 variant) skips empty buckets without spending
     the budget, examining at most 4 P flip sets (the tiny index has many
-    empty buckets)."""
+    empty buckets, so the block's first enumeration of 2 P sets often holds
+    too few non-empty ones and the heap continues; small S_max and L_sel
+    exhaust the admissible sets first; tied deviations crowd cost buckets)."""
     ix, orc = tiny["ix"], tiny["orc"]
+    lg = tiny["lg"][:100]
+    if kw == "ties":
+        rng = np.random.default_rng(P)
+        tau = orc.tau()
+        lg = (tau[None, :] + rng.integers(-3, 4, lg.shape) / 8).astype(np.float32)
+        kw = dict()
     ix.set_params(nonempty_budget=1, **kw)
     try:
-        codes, nprobe = ix.route(tiny["dl"][:100], P)
+        codes, nprobe = ix.route(torch.from_numpy(lg).cuda(), P)
     finally:
         ix.set_params()
     codes = codes.cpu().numpy().view(np.uint32)
@@ -129,7 +138,7 @@ def test_route_nonempty_budget_bit_exact(tiny, torch, P, kw):
     p = oracle.params(nonempty_budget=1, **kw)
     bkt = orc.bkt_off()
     for i in range(100):
-        exp, _ = orc.probe_list(tiny["lg"][i], P, p)
+        exp, _ = orc.probe_list(lg[i], P, p)
         assert nprobe[i] == len(exp), i
         assert np.array_equal(codes[i, : len(exp)], exp), i
         assert np.all(codes[i, len(exp):] == 0xFFFFFFFF)
