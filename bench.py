@@ -56,6 +56,17 @@ CALIB_BINS = 16
 
 EXEC_KEYS = ("pipe_chunk", "refine_ctas")  # nr_params fields that change no result
 
+# encoder weights of the run: the workload's seeded weights, or a trained
+# encoder's (--weights, written by paper_2608_15438_gb300.train)
+ENCODER = {"weights": None, "source": "seeded N(0, 1/fan_in)"}
+
+
+def workload_weights(w):
+    """The encoder weights the run indexes and queries with."""
+    import synth
+
+    return ENCODER["weights"] if ENCODER["weights"] is not None else synth.encoder_weights(w)
+
 
 def method_kw(kw):
     """The parameters of the method itself (the oracle's), without the
@@ -105,6 +116,9 @@ def parse():
     ap.add_argument("--encode", type=int, default=0,
                     help="time only the tensor-core encoder over this many base vectors")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--weights", default=None,
+                    help="encoder weights (.npz from paper_2608_15438_gb300.train) instead of the "
+                         "workload's seeded ones")
     ap.add_argument("--calibrate", type=int, default=0,
                     help="calibrate M(x) and S_max on this many held-out queries (Sec. 3.4; "
                          "default 10,000 when the operating point is calibrated); grid keys "
@@ -214,6 +228,9 @@ def index_path(w):
     h = hashlib.sha256(repr(w).encode())
     for f in ("synth/synth.c", "paper_2608_15438_gb300/builder/nrbuild.cpp"):
         h.update(open(os.path.join(ROOT, f), "rb").read())
+    if ENCODER["weights"] is not None:
+        for a in ENCODER["weights"][:4]:
+            h.update(np.ascontiguousarray(a).tobytes())
     return os.path.join(tempfile.gettempdir(), f"neuroute_{w.name}_{h.hexdigest()[:16]}.nrix")
 
 
@@ -224,7 +241,7 @@ def build_or_load_index(w, path, rank, world):
     if rank == 0 and not os.path.exists(path):
         base = synth.base(w)
         info = build_index(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t, mid=w.mid), base,
-                           synth.encoder_weights(w), path + ".tmp")
+                           workload_weights(w), path + ".tmp")
         os.replace(path + ".tmp", path)
         del base
     if world > 1:
@@ -243,7 +260,7 @@ def gpu_index(w, torch, nr, dev):
     d = dev.index or 0
     gen = synth.DeviceRows(w, synth.SEED_DATA, device=d)
     bd = nr.Builder(config(w.dtype, w.dim, w.hidden, w.bits, w.k_max, w.t, mid=w.mid), w.n,
-                    synth.encoder_weights(w), d)
+                    workload_weights(w), d)
     chunk = min(w.n, (4 << 30) // w.row_bytes)
     buf = torch.empty((chunk, w.dim), dtype=torch.uint8 if w.dtype == "u8" else torch.float32,
                       device=dev)
@@ -316,7 +333,7 @@ def oracle_subindex(w, ix, qs, P, kw, path):
     import oracle
     import synth
 
-    lg = oracle.encode_weights(synth.encoder_weights(w), w.in_scale, qs)
+    lg = oracle.encode_weights(workload_weights(w), w.in_scale, qs)
     tau = ix.thresholds()
     p = oracle.params(**method_kw(kw))
     codes = np.concatenate([oracle.probe_list(lg[i], tau, P, p)[0] for i in range(len(qs))])
@@ -629,6 +646,11 @@ def main():
     import synth
 
     w = synth.WORKLOADS[args.workload]
+    if args.weights:
+        from paper_2608_15438_gb300 import train
+
+        ENCODER["weights"] = train.load_weights(args.weights)
+        ENCODER["source"] = f"trained with L_sim ({os.path.basename(args.weights)})"
     rank, world, local = dist_env()
     if world > 1:
         import torch.distributed as dist
@@ -833,7 +855,8 @@ def main():
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "u8" if w.dtype == "u8" else "f32", "data": "synthetic",
         "config": {"workload": w.name, "N": w.n, "D": w.dim, "nq": nq, "k": k, "bits": w.bits,
-                   "hidden": w.hidden, "K_max": w.k_max, "P": P, "C": C, "t_low": t_low,
+                   "hidden": w.hidden, "K_max": w.k_max, "encoder": ENCODER["source"],
+                   "P": P, "C": C, "t_low": t_low,
                    "gate_m1": kw.get("gate_m1"), "gate_curve": kw.get("gate_curve"),
                    "s_max": kw.get("s_max"),
                    "calibration": (None if cq is None and cov is None else
