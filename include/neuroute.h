@@ -137,6 +137,13 @@ typedef struct {
    * probe_budget flip sets examined, the base code included. 0 (default):
    * probe_budget counts codes, empty buckets included. */
   int nonempty_budget;  /* 0 or 1; default 0 */
+  /* Execution only: the limit of the tensor-core encoder's bounded hand-off
+   * waits. 0 (default): 1 s; > 0: that many microseconds (at most 60 s);
+   * < 0: a wait whose phase is not complete when first tested expires at
+   * once, which exercises the failure path (the kernel stops, drains its
+   * issued MMAs under its own 1 s bound, frees its tensor memory and sets the
+   * device flag that nr_last_stats reports as NR_ERR_DEVICE_CHECK). */
+  int wait_limit_us;
 } nr_params;
 
 #define NR_NONEMPTY_SCAN 4

@@ -98,6 +98,7 @@ nr_status check_params(const nr_params *p) {
     return NR_ERR_INVALID_ARG;
   if (p->pipe_chunk < 0 || p->refine_ctas < 0 || p->refine_ctas > 32) return NR_ERR_INVALID_ARG;
   if (p->nonempty_budget != 0 && p->nonempty_budget != 1) return NR_ERR_INVALID_ARG;
+  if (p->wait_limit_us > 60000000) return NR_ERR_INVALID_ARG;
   if (p->gate_n != 0) {
     if (p->gate_n < 2 || p->gate_n > 16) return NR_ERR_INVALID_ARG;
     for (int i = 0; i < p->gate_n; ++i) {
@@ -270,6 +271,7 @@ nr_status nr_params_default(nr_params *p) {
   p->pipe_chunk = 0;
   p->refine_ctas = 0;
   p->nonempty_budget = 0;
+  p->wait_limit_us = 0;
   return NR_OK;
 }
 

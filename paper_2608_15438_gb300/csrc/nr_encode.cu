@@ -20,8 +20,9 @@
 // memory operands sit in the canonical K-major no-swizzle layout
 // (nr_tc_kmajor_off), in which the host stores W1 and W2.
 //
-// Every wait is bounded (1 s); when one expires every role stops, the CTA
-// waits (again bounded) for its MMAs in flight, records NR_DEV_TIMEOUT, frees
+// Every hand-off wait is bounded (1 s, or the limit nr_params.wait_limit_us
+// sets); when one expires every role stops, the CTA waits for its MMAs in
+// flight (bounded by 1 s whatever the limit), records NR_DEV_TIMEOUT, frees
 // its TMEM and returns.
 //
 // What the tensor-core kernel does not take (D % 16 != 0, D > 128,
@@ -206,23 +207,41 @@ __device__ __forceinline__ void tc_st32(uint32_t taddr, const uint32_t (&r)[32])
 __device__ __forceinline__ void tc_wait_st() {
   asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory");
 }
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t phase) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(phase)
+      : "memory");
+  return ok != 0;
+}
 // Waits for the barrier phase of the given parity. Gives up when another role
-// has given up, or after ~1 s, which makes every role give up.
-__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, volatile int *abort) {
+// has given up, or after wait_ns nanoseconds, which makes every role give up;
+// wait_ns < 0: gives up unless the phase is complete when first tested.
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, volatile int *abort,
+                                              int64_t wait_ns) {
+  if (wait_ns < 0) {
+    if (mbar_test_wait(bar, parity)) return true;
+    *abort = 1;
+    return false;
+  }
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (global_ns() - t0 > 1000000000ull) {
+    if (global_ns() - t0 > (uint64_t)wait_ns) {
       *abort = 1;
       return false;
     }
   }
 }
 // the same, one decision for the whole warp (all lanes wait)
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort) {
-  return __all_sync(0xffffffffu, wait_or_abort(bar, parity, abort)) != 0;
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int *abort,
+                                          int64_t wait_ns) {
+  return __all_sync(0xffffffffu, wait_or_abort(bar, parity, abort, wait_ns)) != 0;
 }
 // 16 bytes of uint8 as 16 fp16 values, exactly: 0x64XX is the fp16 number 1024 + XX
 __device__ __forceinline__ void u8x16_to_f16(const uint4 v, uint4 &lo, uint4 &hi) {
@@ -258,7 +277,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                      float s,
                      const __half *__restrict__ W1p, const float *__restrict__ b1,
                      const __half *__restrict__ W2p, const float *__restrict__ b2, int64_t nq,
-                     float *__restrict__ out, int *err) {
+                     float *__restrict__ out, int *err, int64_t wait_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   const TcLayout L = tc_layout(D, H, n2, nxb);
   TcBars &B = *reinterpret_cast<TcBars *>(smem + L.bars);
@@ -316,8 +335,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       // hidden chunk (TMEM) x W2 chunk into the tile's accumulator
       auto layer2 = [&](uint32_t gp, uint32_t ip, int cp) -> bool {
         const int hb = (int)(gp & 1);
-        if (!wait_or_abort(smem_u32(&B.hfull[hb]), (gp >> 1) & 1u, abort)) return false;
-        if (cp == 0 && !wait_or_abort(smem_u32(&B.a2empty[ip & 1]), ((ip >> 1) & 1u) ^ 1u, abort))
+        if (!wait_or_abort(smem_u32(&B.hfull[hb]), (gp >> 1) & 1u, abort, wait_ns)) return false;
+        if (cp == 0 && !wait_or_abort(smem_u32(&B.a2empty[ip & 1]), ((ip >> 1) & 1u) ^ 1u, abort, wait_ns))
           return false;
         tc_fence_after();
         const uint32_t d2 = tmem + kTmemAcc2 + (ip & 1u) * 32u;
@@ -335,13 +354,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
         const int xb = nxb == 2 ? (int)(it & 1) : 0;
         const uint32_t xpar = (nxb == 2 ? it >> 1 : it) & 1u;
-        if (!wait_or_abort(smem_u32(&B.xfull[xb]), xpar, abort)) {
+        if (!wait_or_abort(smem_u32(&B.xfull[xb]), xpar, abort, wait_ns)) {
           ok = false;
           break;
         }
         for (int c = 0; c < nc; ++c, ++g) {
           const int a = (int)(g & 1);
-          if (!wait_or_abort(smem_u32(&B.a1empty[a]), ((g >> 1) & 1u) ^ 1u, abort)) {
+          if (!wait_or_abort(smem_u32(&B.a1empty[a]), ((g >> 1) & 1u) ^ 1u, abort, wait_ns)) {
             ok = false;
             break;
           }
@@ -374,7 +393,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // logits of tile number ip (global tile t): layer-2 accumulator + b2 -> out,
     // 16 columns a thread (its row, its column half), as float4 where aligned
     auto logits = [&](uint32_t ip, int64_t t) -> bool {
-      if (!warp_wait(smem_u32(&B.a2full[ip & 1]), (ip >> 1) & 1u, abort)) return false;
+      if (!warp_wait(smem_u32(&B.a2full[ip & 1]), (ip >> 1) & 1u, abort, wait_ns)) return false;
       tc_fence_after();
       uint32_t o[16];
       const bool reads = hh * 16 < n2;  // same for the whole warp
@@ -412,7 +431,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     for (int64_t tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x, ++it) {
       for (int c = 0; c < nc; ++c, ++g) {
         const int a = (int)(g & 1);
-        if (!warp_wait(smem_u32(&B.a1full[a]), (g >> 1) & 1u, abort)) {
+        if (!warp_wait(smem_u32(&B.a1full[a]), (g >> 1) & 1u, abort, wait_ns)) {
           ok = false;
           break;
         }
@@ -441,7 +460,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         tc_fence_before();
         mbar_arrive(smem_u32(&B.a1empty[a]));
         // the layer-2 MMAs of chunk g - 2 have read this hidden buffer
-        if (!warp_wait(smem_u32(&B.hempty[a]), ((g >> 1) & 1u) ^ 1u, abort)) {
+        if (!warp_wait(smem_u32(&B.hempty[a]), ((g >> 1) & 1u) ^ 1u, abort, wait_ns)) {
           ok = false;
           break;
         }
@@ -493,7 +512,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           v[j] = make_uint4(0u, 0u, 0u, 0u);
           if (j < per && rr < rows) v[j] = __ldg(reinterpret_cast<const uint4 *>(xs + rr * D + pc * 16));
         }
-        ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort);
+        ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort, wait_ns);
         if (ok) {
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -523,7 +542,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
               w[j] = __ldg(s4 + 1);
             }
           }
-          if (j0 == 0) ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort);
+          if (j0 == 0) ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort, wait_ns);
           if (!ok) break;
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
@@ -709,10 +728,14 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
     const int64_t tiles = (nq + kRows - 1) / kRows;
     const int64_t grid = tiles < ix->num_sms ? tiles : ix->num_sms;
     const int vec_out = ix->b % 4 == 0 && (reinterpret_cast<uintptr_t>(d_logits) & 15) == 0;
+    // the roles' hand-off waits: 1 s by default; the drain of issued MMAs
+    // before TMEM is freed keeps its own 1 s bound whatever this is
+    const int wl = ix->params.wait_limit_us;
+    const int64_t wait_ns = wl == 0 ? (int64_t)1000000000 : wl > 0 ? (int64_t)wl * 1000 : (int64_t)-1;
     kern<<<(unsigned)grid, kTcThreads, smem, s>>>(d_x, ix->D, ix->H, ix->b, n2, nxb, vec_out, ix->in_scale,
                                                   static_cast<const __half *>(ix->W1h), ix->b1,
                                                   static_cast<const __half *>(ix->W2h), ix->b2, nq,
-                                                  d_logits, ix->d_err);
+                                                  d_logits, ix->d_err, wait_ns);
     ix->launches += 1;
     return cudaGetLastError();
   }

@@ -45,7 +45,8 @@ class Params(ctypes.Structure):
                 ("c_f_min", ctypes.c_int), ("c_alpha_front", ctypes.c_float),
                 ("gate_n", ctypes.c_int), ("gate_x", ctypes.c_float * 16),
                 ("gate_y", ctypes.c_float * 16), ("pipe_chunk", ctypes.c_int),
-                ("refine_ctas", ctypes.c_int), ("nonempty_budget", ctypes.c_int)]
+                ("refine_ctas", ctypes.c_int), ("nonempty_budget", ctypes.c_int),
+                ("wait_limit_us", ctypes.c_int)]
 
 
 class Stats(ctypes.Structure):

@@ -504,3 +504,39 @@ def test_encoder_tile_edges(torch, tmp_path, workload):
     assert shifted.data_ptr() % 16 == 8
     check(ix.encode(shifted), n_max)
     ix.close()
+
+
+def test_encoder_wait_expiry_is_flagged_and_the_context_stays_usable(tiny, torch):
+    """With wait_limit_us < 0 every hand-off wait of the tensor-core encoder
+    that is not already complete when first tested expires: the kernel stops,
+    drains its issued MMAs (under its own 1 s bound), frees its tensor memory
+    and sets the device flag, which nr_last_stats reports as
+    NR_ERR_DEVICE_CHECK and clears. With the default limit the next call
+    encodes correctly on the same context."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    ix = tiny["ix"]
+    # the tensor-core kernel's shapes (D % 16 == 0, D <= 128, H % 128 == 0, b <= 32)
+    assert ix.D % 16 == 0 and ix.D <= 128 and ix.H % 128 == 0 and ix.b <= 32
+    ix.set_params(wait_limit_us=-1)
+    try:
+        ix.encode(tiny["dq"])
+        torch.cuda.synchronize()
+        with pytest.raises(nr.NRError) as e:
+            ix.last_stats()
+        assert e.value.status == -6  # NR_ERR_DEVICE_CHECK
+    finally:
+        ix.set_params()
+    ix.last_stats()  # the flag was cleared
+    lg = ix.encode(tiny["dq"]).cpu().numpy()
+    ref = tiny["lg"]
+    assert np.all(np.abs(lg - ref).max(1) <= 1e-2 * np.abs(ref).max(1))
+    ix.last_stats()
+    # a limit longer than any hand-off changes nothing
+    ix.set_params(wait_limit_us=2_000_000)
+    try:
+        lg2 = ix.encode(tiny["dq"]).cpu().numpy()
+        ix.last_stats()
+    finally:
+        ix.set_params()
+    assert np.array_equal(lg2, lg)
