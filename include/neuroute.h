@@ -221,6 +221,64 @@ nr_status nr_index_locate(nr_index *ix, const int64_t *d_ids, int64_t n, int32_t
 nr_status nr_centroid_dists(nr_index *ix, const float *d_logits, int64_t nq,
                             const int32_t *d_clusters, int m, float *d_out, void *stream);
 
+/* Calibration of the gate margin M and the bucket-score cutoff S_max from
+ * held-out queries (Sec. 3.4: both are fitted on where a query's true
+ * neighbours lie). Definitions, for a query with logits l, base code u0 and
+ * deviations delta_j = |l_j - tau_j| ranked by (delta_j, j):
+ *   score of bucket code u = the fp32 sum of delta over the ranks whose bit
+ *     differs between u and u0, in ascending rank (Algorithm 1's cost);
+ *   x = the smallest centroid distance over every cluster of the target
+ *     buckets that hold two or more clusters (single-cluster buckets bypass
+ *     the gate); y = the largest distance of such a target's own cluster,
+ *     minus x (fp32); both NaN without such a target;
+ *   S_max = the pair scores (NaN skipped) sorted, the entry at position
+ *     ceil(coverage m) - 1 (clamped to [0, m - 1]);
+ *   M = the queries with an x sorted by (x, y) in B = min(n_bins, n)
+ *     equal-frequency bins [floor(i n / B), floor((i + 1) n / B)), a bin's
+ *     point (x at its lower-median position, its y at sorted position
+ *     ceil(q m) - 1), equal x merged (larger y), the y's running maximum; a
+ *     single point (x0, y0) becomes (x0, y0), (next float above x0, y0).
+ * Distances are the select kernel's fmaf chain. */
+
+/* Scores of bucket codes: d_logits [nq x b] fp32, d_tau [b], d_codes
+ * [nq x k] int32 (negative: none) -> d_scores [nq x k] fp32 (NaN for none);
+ * all device, asynchronous on `stream`. 1 <= b <= 31.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_CUDA. */
+nr_status nr_bucket_scores(const float *d_logits, const float *d_tau, int b, const int32_t *d_codes,
+                           int64_t nq, int k, float *d_scores, void *stream);
+
+/* Observations of nq calibration queries (device logits [nq x b]) with their
+ * targets d_targets [nq x k] (device int64 row ids, -1 = none; typically
+ * their top-k from a high-recall search): d_scores [nq x k] (NaN where the
+ * target is not stored), d_x [nq], d_y [nq], all device fp32. Allocates
+ * O(nq k) device scratch; synchronous on `stream`. nq k < 2^31.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_OOM, NR_ERR_CUDA. */
+nr_status nr_calib_observe(nr_index *ix, const float *d_logits, const int64_t *d_targets, int64_t nq,
+                           int k, float *d_scores, float *d_x, float *d_y, void *stream);
+
+/* S_max from host scores [nq x k] at `coverage`; *pair_coverage = the
+ * fraction of scores at or below it, *query_coverage = the fraction of the
+ * queries with a score whose scores all are; *s_max = NaN (and both 0) when
+ * no score is given. Host only. Errors: NR_ERR_INVALID_ARG. */
+nr_status nr_calib_fit_s_max(const float *h_scores, int64_t nq, int k, double coverage,
+                             float *s_max, double *pair_coverage, double *query_coverage);
+
+/* The margin curve from host x, y [n] (NaN x skipped) at quantile q with
+ * 1 <= n_bins <= 16 bins: *gate_n points (0 without observations, else 2..16)
+ * in gate_x, gate_y [16]. Host only. Errors: NR_ERR_INVALID_ARG. */
+nr_status nr_calib_fit_gate(const float *h_x, const float *h_y, int64_t n, int n_bins, double q,
+                            int *gate_n, float *gate_x, float *gate_y);
+
+/* All of the above: observations of the targets, S_max at `coverage` and the
+ * curve at `quantile` written into *p (s_max, gate_n, gate_x, gate_y; the
+ * other fields untouched; a fit without data leaves its fields as they
+ * were); info (may be NULL) [3] = pair coverage, query coverage, queries with
+ * an x. Pass *p to nr_set_params to search with them. Synchronous.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_OOM, NR_ERR_CUDA. */
+nr_status nr_calibrate(nr_index *ix, const float *d_logits, const int64_t *d_targets, int64_t nq,
+                       int k, int n_bins, double quantile, double coverage, nr_params *p,
+                       double *info, void *stream);
+
 /* Validate and set the query-time knobs (p = NULL restores the defaults).
  * NR_ERR_INVALID_ARG if a field is out of range. */
 nr_status nr_set_params(nr_index *ix, const nr_params *p);

@@ -24,37 +24,35 @@ y); the curve is the running maximum of the y's, the smallest non-decreasing
 curve on or above every bin's quantile. A single point (x0, y0) gives the
 flat curve through (x0, y0) and (next float above x0, y0).
 
-Locations and centroid distances come from the library (nr_index_locate,
-nr_centroid_dists); the scores and the fits are host arithmetic on at most a
-few hundred thousand numbers, done once per index.
+Every step runs in the library (nr_calib_observe, nr_calib_fit_s_max,
+nr_calib_fit_gate: the observations on the GPU, the fits on the host); this
+module only marshals arguments.
 """
 from __future__ import annotations
 
-import math
+import ctypes
 
 import numpy as np
 
 from . import neuroute as nr
 
 
-def bucket_scores(logits: np.ndarray, tau: np.ndarray, codes: np.ndarray) -> np.ndarray:
+def bucket_scores(logits, tau, codes, stream=None) -> np.ndarray:
     """Cost of bucket codes[q, t] for query q (fp32 [nq x k]); nan where the
-    code is negative."""
-    logits = np.asarray(logits, np.float32)
-    tau = np.asarray(tau, np.float32)
-    codes = np.asarray(codes, np.int64)
-    nq, b = logits.shape
-    delta = np.abs(logits - tau[None, :])
-    u0 = ((logits >= tau[None, :]).astype(np.int64) << np.arange(b, dtype=np.int64)).sum(axis=1)
-    ranks = np.argsort(delta, axis=1, kind="stable")          # ties: lower bit first
-    diff = codes ^ u0[:, None]
-    rows = np.arange(nq)
-    s = np.zeros(codes.shape, np.float32)
-    for r in range(b):
-        j = ranks[:, r]
-        flip = ((diff >> j[:, None]) & 1).astype(bool)
-        s = np.where(flip, s + delta[rows, j][:, None], s)
-    return np.where(codes >= 0, s, np.float32(np.nan)).astype(np.float32)
+    code is negative (nr_bucket_scores on the GPU)."""
+    import torch
+
+    dev = torch.device("cuda", torch.cuda.current_device())
+    lg = torch.as_tensor(np.asarray(logits, np.float32), device=dev).contiguous()
+    tu = torch.as_tensor(np.asarray(tau, np.float32), device=dev).contiguous()
+    cd = torch.as_tensor(np.asarray(codes, np.int64).astype(np.int32), device=dev).contiguous()
+    nq, b = lg.shape
+    k = cd.shape[1]
+    out = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    st = nr.lib().nr_bucket_scores(nr._ptr(lg), nr._ptr(tu), b, nr._ptr(cd), nq, k, nr._ptr(out),
+                                   nr._stream(stream))
+    nr._check("nr_bucket_scores", st)
+    return out.cpu().numpy()
 
 
 def observations(ix: "nr.Index", logits, targets, stream=None):
@@ -63,42 +61,34 @@ def observations(ix: "nr.Index", logits, targets, stream=None):
     import torch
 
     nq, k = targets.shape
-    loc = ix.locate(targets, stream).view(nq, k, 4)
-    loc_h = loc.cpu().numpy()
-    lg = logits.cpu().numpy()
-    found = loc_h[..., 0] >= 0
-    scores = bucket_scores(lg, ix.thresholds(), np.where(found, loc_h[..., 1], -1))
-    gated = found & (loc_h[..., 3] >= 2)
-    j = np.arange(ix.k_max, dtype=np.int32)
-    members = np.where(gated[..., None] & (j < loc_h[..., 3:4]), loc_h[..., 2:3] + j, -1)
     dev = logits.device
-    d_all = ix.centroid_dists(logits, torch.from_numpy(members.reshape(nq, -1)).to(dev), stream)
-    d_own = ix.centroid_dists(logits, torch.from_numpy(np.where(gated, loc_h[..., 0], -1)).to(dev),
-                              stream)
-    d_all, d_own = d_all.cpu().numpy(), d_own.cpu().numpy()
-    has = gated.any(axis=1)
-    x = d_all.min(axis=1)
-    far = np.where(gated, d_own, np.float32(-np.inf)).max(axis=1)
-    with np.errstate(invalid="ignore"):  # queries without a gated target: -inf - inf
-        y = (far - x).astype(np.float32)
-    nan = np.float32(np.nan)
-    return scores, np.where(has, x, nan).astype(np.float32), np.where(has, y, nan).astype(np.float32)
+    lg = nr._arg(logits, "logits", torch.float32, (nq, ix.b), ix.device)
+    tg = nr._arg(targets, "targets", torch.int64, (nq, k), ix.device)
+    sc = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    x = torch.empty(nq, dtype=torch.float32, device=dev)
+    y = torch.empty(nq, dtype=torch.float32, device=dev)
+    st = nr.lib().nr_calib_observe(ix.h, nr._ptr(lg), nr._ptr(tg), nq, k, nr._ptr(sc), nr._ptr(x),
+                                   nr._ptr(y), nr._stream(stream))
+    nr._check("nr_calib_observe", st)
+    return sc.cpu().numpy(), x.cpu().numpy(), y.cpu().numpy()
 
 
 def fit_s_max(scores, coverage: float):
     """(S_max, fraction of target pairs covered, fraction of queries whose
     every target is covered); (None, 0, 0) without scores."""
-    scores = np.asarray(scores, np.float32)
-    valid = ~np.isnan(scores)
-    flat = np.sort(scores[valid])
-    m = flat.size
-    if m == 0:
+    scores = np.ascontiguousarray(np.asarray(scores, np.float32))
+    if scores.size == 0:
         return None, 0.0, 0.0
-    t = flat[min(m - 1, max(0, math.ceil(coverage * m) - 1))]
-    pairs = int((flat <= t).sum()) / m
-    has = valid.any(axis=1)
-    worst = np.where(valid, scores, np.float32(-np.inf)).max(axis=1)
-    return np.float32(t), pairs, int((worst[has] <= t).sum()) / int(has.sum())
+    scores = scores.reshape(len(scores), -1)
+    t = ctypes.c_float()
+    pc, qc = ctypes.c_double(), ctypes.c_double()
+    st = nr.lib().nr_calib_fit_s_max(scores.ctypes.data, scores.shape[0], max(1, scores.shape[1]),
+                                     float(coverage), ctypes.byref(t), ctypes.byref(pc),
+                                     ctypes.byref(qc))
+    nr._check("nr_calib_fit_s_max", st)
+    if np.isnan(t.value):
+        return None, 0.0, 0.0
+    return np.float32(t.value), pc.value, qc.value
 
 
 def fit_gate(x, y, n_bins: int = 16, q: float = 0.95):
@@ -106,32 +96,16 @@ def fit_gate(x, y, n_bins: int = 16, q: float = 0.95):
     observations."""
     if not 1 <= n_bins <= 16:
         raise ValueError("n_bins: 1..16")
-    x, y = np.asarray(x, np.float32), np.asarray(y, np.float32)
-    keep = ~np.isnan(x)
-    x, y = x[keep], y[keep]
-    n = x.size
-    if n == 0:
+    x = np.ascontiguousarray(x, np.float32)
+    y = np.ascontiguousarray(y, np.float32)
+    n = ctypes.c_int()
+    gx, gy = np.zeros(16, np.float32), np.zeros(16, np.float32)
+    st = nr.lib().nr_calib_fit_gate(x.ctypes.data, y.ctypes.data, x.size, int(n_bins), float(q),
+                                    ctypes.byref(n), gx.ctypes.data, gy.ctypes.data)
+    nr._check("nr_calib_fit_gate", st)
+    if n.value == 0:
         return None
-    order = np.lexsort((y, x))
-    x, y = x[order], y[order]
-    B = min(n_bins, n)
-    px, py = [], []
-    for i in range(B):
-        lo, hi = i * n // B, (i + 1) * n // B
-        m = hi - lo
-        xm = x[lo + (m - 1) // 2]
-        yq = np.sort(y[lo:hi])[min(m - 1, max(0, math.ceil(q * m) - 1))]
-        if px and px[-1] == xm:
-            py[-1] = max(py[-1], yq)
-        else:
-            px.append(xm)
-            py.append(yq)
-    ys = np.maximum.accumulate(np.array(py, np.float32))
-    xs = np.array(px, np.float32)
-    if xs.size == 1:
-        xs = np.array([xs[0], np.nextafter(xs[0], np.float32(np.inf))], np.float32)
-        ys = np.array([ys[0], ys[0]], np.float32)
-    return tuple(float(v) for v in xs), tuple(float(v) for v in ys)
+    return tuple(float(v) for v in gx[:n.value]), tuple(float(v) for v in gy[:n.value])
 
 
 def targets_high_recall(ix: "nr.Index", queries, logits, k: int, P: int, C: int, stream=None):

@@ -26,7 +26,8 @@ EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_f
            "nr_index_save", "nr_index_extract", "nr_index_thresholds", "nr_index_locate",
            "nr_centroid_dists", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
            "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free",
-           "nr_measure_gather"]
+           "nr_measure_gather", "nr_bucket_scores", "nr_calib_observe", "nr_calib_fit_s_max",
+           "nr_calib_fit_gate", "nr_calibrate"]
 
 
 class NRError(RuntimeError):
@@ -79,6 +80,13 @@ def lib():
         L.nr_query_stats.argtypes = [vp, vp, i64, vp]
         L.nr_last_stats.argtypes = [vp, ctypes.POINTER(Stats)]
         L.nr_measure_gather.argtypes = [i32, i64, i32, i64, i32, ctypes.POINTER(ctypes.c_double)]
+        dp, fp = ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_float)
+        L.nr_bucket_scores.argtypes = [vp, vp, i32, vp, i64, i32, vp, vp]
+        L.nr_calib_observe.argtypes = [vp, vp, vp, i64, i32, vp, vp, vp, vp]
+        L.nr_calib_fit_s_max.argtypes = [vp, i64, i32, ctypes.c_double, fp, dp, dp]
+        L.nr_calib_fit_gate.argtypes = [vp, vp, i64, i32, ctypes.c_double, ctypes.POINTER(i32), vp, vp]
+        L.nr_calibrate.argtypes = [vp, vp, vp, i64, i32, i32, ctypes.c_double, ctypes.c_double,
+                                   ctypes.POINTER(Params), vp, vp]
         L.nr_enable_timing.argtypes = [vp, i32]
         L.nr_last_timing.argtypes = [vp, vp]
         L.nr_kernel_launches.argtypes = [vp]

@@ -94,6 +94,22 @@ def test_calibration_matches_oracle(tiny, torch):
     assert np.array_equal(np.array(res["gate_curve"][0], np.float32), np.array(xs, np.float32))
     assert np.array_equal(np.array(res["gate_curve"][1], np.float32), np.array(ys, np.float32))
     assert (res["s_max"], res["pair_coverage"], res["query_coverage"]) == oc.fit_s_max(scores, 0.95)
+    # the whole calibration in one library call (nr_calibrate) writes the same
+    # curve and cutoff into the search parameters
+    import ctypes
+
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    p = nr.params(t_low=7)
+    info = np.zeros(3, np.float64)
+    assert nr.lib().nr_calibrate(ix.h, nr._ptr(lg), nr._ptr(targets), lg.shape[0], 10, 8, 0.9, 0.95,
+                                 ctypes.byref(p), info.ctypes.data, nr._stream(None)) == 0
+    assert p.gate_n == len(xs) and p.t_low == 7
+    assert np.array_equal(np.array(p.gate_x[:p.gate_n], np.float32), np.array(xs, np.float32))
+    assert np.array_equal(np.array(p.gate_y[:p.gate_n], np.float32), np.array(ys, np.float32))
+    s_o, pc_o, qc_o = oc.fit_s_max(scores, 0.95)
+    assert np.float32(p.s_max) == s_o and info[0] == pc_o and info[1] == qc_o
+    assert info[2] == res["n_gated"]
     # the fitted curve is a valid gate and keeps the search near the targets
     ix.set_params(gate_curve=res["gate_curve"], t_low=0)
     try:
@@ -120,3 +136,25 @@ def test_argument_checks(tiny, torch):
     assert lib.nr_centroid_dists(ix.h, ctypes.c_void_p(lg.data_ptr()), 2, ctypes.c_void_p(cl.data_ptr()),
                                  -1, None, None) == -1
     assert lib.nr_centroid_dists(ix.h, ctypes.c_void_p(lg.data_ptr()), 2, None, 3, None, None) == -1
+
+
+@pytest.mark.parametrize("b", [2, 8, 16, 24])
+def test_bucket_scores_match_oracle(torch, b):
+    rng = np.random.default_rng(b)
+    nq, k = 40, 12
+    # dyadic logits on a coarse grid: many equal deviations and logits on tau
+    logits = (rng.integers(-8, 9, (nq, b)) / 4).astype(np.float32)
+    tau = (rng.integers(-2, 3, b) / 4).astype(np.float32)
+    if b >= 8:
+        logits[: nq // 2] = rng.normal(0, 1, (nq // 2, b)).astype(np.float32)
+    codes = rng.integers(0, 1 << b, (nq, k)).astype(np.int64)
+    codes[rng.random((nq, k)) < 0.1] = -1
+    from paper_2608_15438_gb300 import calibrate as pc
+
+    got = pc.bucket_scores(logits, tau, codes)
+    for q in range(nq):
+        for t in range(k):
+            if codes[q, t] < 0:
+                assert np.isnan(got[q, t])
+            else:
+                assert got[q, t] == oc.bucket_score(logits[q], tau, int(codes[q, t])), (q, t)
