@@ -385,10 +385,10 @@ def traffic_from_profile(workload, P, C, algorithmic_bytes, launches=1):
     path = os.path.join(ROOT, "profiles", "refine_traffic.json")
     try:
         rec = json.load(open(path))
-        if rec.get("sources_sha256") != refine_sources_digest():
-            return None
         e = rec.get("captures", {}).get(f"{workload}/P{P}/C{C}")
-        if e is None or e.get("launches", 1) != launches:
+        if e is None or e.get("sources_sha256") != refine_sources_digest():
+            return None
+        if e.get("launches", 1) != launches:
             return None
         if e.get("algorithmic_bytes_per_launch") * launches != algorithmic_bytes:
             return None
@@ -847,7 +847,8 @@ def main():
     sel_avg_ms = stage_ms["select"] / args.steps / n_ref
     sel_gbs = sel_bytes / (sel_avg_ms / 1e3) / 1e9 if sel_avg_ms > 0 else None
     # the random-row read rate of this GPU over an array of the centroids' shape
-    gather_gbs = nr.measure_gather(local, max(1 << 20, ix.n_clusters), w.bits * 4)
+    # (rows of 4b bytes rounded up to 16, the granule of the measurement)
+    gather_gbs = nr.measure_gather(local, max(1 << 20, ix.n_clusters), (w.bits * 4 + 15) // 16 * 16)
     out = {
         "metric": METRIC,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
@@ -883,9 +884,10 @@ def main():
                             "achieved": sel_gbs, "peak": gather_gbs, "unit": "GB/s",
                             "frac": (sel_gbs / gather_gbs if sel_gbs and gather_gbs else None),
                             "frac_of_copy": (sel_gbs / peaks.get("hbm_gbs") if sel_gbs else None),
-                            "peak_source": f"measured in this run: random {w.bits * 4}-byte row "
-                                           "reads, 2e7 rows at random from an n_clusters x 4b-byte "
-                                           "array, L2 flushed (nr_measure_gather)",
+                            "peak_source": f"measured in this run: random "
+                                           f"{(w.bits * 4 + 15) // 16 * 16}-byte row reads, 2e7 rows "
+                                           "at random from an n_clusters-row array, L2 flushed "
+                                           "(nr_measure_gather)",
                             "algorithmic_bytes_per_launch": sel_bytes,
                             "clusters_scored_per_query": st.scored / nq,
                             "avg_launch_ms": sel_avg_ms, "launches_per_step": n_ref},
