@@ -439,23 +439,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         // h = ReLU(s acc + b1) as fp16 pairs, 32 accumulator columns at a time
         const uint32_t col = tmem + lane_base + (uint32_t)a * kHC + (uint32_t)hh * 64u;
         const float *bb = sb1 + c * kHC + hh * 64;
+        // both 32-column loads in flight before one wait
+        uint32_t v[64];
+        tc_ld32(col, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
+        tc_ld32(col + 32u, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
+        tc_wait_ld();
         uint32_t hp[32];
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          float bv[32];
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            *reinterpret_cast<float4 *>(&bv[4 * j]) = reinterpret_cast<const float4 *>(bb + 32 * half)[j];
-          uint32_t v[32];
-          tc_ld32(col + 32u * half, v);
-          tc_wait_ld();
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float h0 = __fmaf_rn(s, __uint_as_float(v[2 * j]), bv[2 * j]);
-            const float h1 = __fmaf_rn(s, __uint_as_float(v[2 * j + 1]), bv[2 * j + 1]);
-            const __half2 p = __hmax2(__floats2half2_rn(h0, h1), zero2);
-            hp[16 * half + j] = *reinterpret_cast<const uint32_t *>(&p);
-          }
+        for (int j4 = 0; j4 < 16; ++j4) {
+          const float4 bq = reinterpret_cast<const float4 *>(bb)[j4];
+          const float h0 = __fmaf_rn(s, __uint_as_float(v[4 * j4]), bq.x);
+          const float h1 = __fmaf_rn(s, __uint_as_float(v[4 * j4 + 1]), bq.y);
+          const float h2 = __fmaf_rn(s, __uint_as_float(v[4 * j4 + 2]), bq.z);
+          const float h3 = __fmaf_rn(s, __uint_as_float(v[4 * j4 + 3]), bq.w);
+          const __half2 p0 = __hmax2(__floats2half2_rn(h0, h1), zero2);
+          const __half2 p1 = __hmax2(__floats2half2_rn(h2, h3), zero2);
+          hp[2 * j4] = *reinterpret_cast<const uint32_t *>(&p0);
+          hp[2 * j4 + 1] = *reinterpret_cast<const uint32_t *>(&p1);
         }
         tc_fence_before();
         mbar_arrive(smem_u32(&B.a1empty[a]));

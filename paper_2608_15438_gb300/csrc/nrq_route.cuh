@@ -222,9 +222,11 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
 // filter, a subtree beyond its capacity of 2N keys, or a bucket above
 // kRouteBucketMax keys take route_warp too (warp 0 of the block).
 constexpr int kRouteThreads = 128;
-constexpr int kRouteBins = 512;
+constexpr int kRouteBins = 480;
 constexpr int kRouteDp = kRouteBins + 32;  // sums of rounded-up steps overshoot by < 1 per rank
 constexpr int kRouteBuckets = 1024;        // <= 2 kRouteDp: the histogram reuses the count arrays
+static_assert(kRouteBuckets <= 2 * kRouteDp, "the bucket histogram must fit the count arrays");
+static_assert(kRouteDp % 32 == 0, "the count scan gives each lane kRouteDp / 32 bins");
 constexpr int kRouteBucketMax = 64;
 constexpr int kRouteNonemptyMax = 4096;    // flip sets a block enumerates for the non-empty budget
 
@@ -342,9 +344,9 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
     if (!(trange > 0.0f)) {
       T = trange;
     } else {
-      // step D = T_range / 512 (exact in fp32); s_r = floor(q + 0.001) + 1 with
-      // q = delta_r / D rounded, whose error (< 1e-4 for q below 544) the 0.001
-      // covers, so s_r D >= delta_r exactly
+      // step D = T_range / kRouteBins (rounded); s_r = floor(q + 0.001) + 1
+      // with q = delta_r / D rounded, whose error (< 1e-4 for q below
+      // kRouteDp) the 0.001 covers, so s_r D >= delta_r exactly
       const float step = __fdiv_rn(trange, (float)kRouteBins);
       uint32_t *d0 = m.dp, *d1 = m.dp + kRouteDp;
       for (int c = tid; c < kRouteDp; c += kRouteThreads) d0[c] = c == 0 ? 1u : 0u;
