@@ -50,7 +50,7 @@ Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   l.nL = o;     o = align256(o + (size_t)qc * 4);
   l.seg = o;    o = align256(o + (size_t)qc * Lmax * sizeof(nr_seg));
   l.slen = o;   o = align256(o + (size_t)qc * 4);
-  l.slab = o;   o = align256(o + (size_t)qc * nr_select_slab_bytes(P, ix->K_max));
+  l.slab = o;   o = align256(o + nr_select_slab_total(qc, P, ix->K_max));
   l.perm = o;   o = align256(o + (size_t)qc * 4);
   l.total = o;
   return l;

@@ -136,6 +136,9 @@ cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int
 size_t nr_select_smem_bytes(const nr_index *ix, int P, int C);
 // global scratch per query that select needs for probe budget P (0: none)
 size_t nr_select_slab_bytes(int P, int K_max);
+// the global scratch of a select launch over nq queries: their slabs and the
+// list of the queries deferred to its overflow kernel (0: none needed)
+size_t nr_select_slab_total(int64_t nq, int P, int K_max);
 cudaError_t nr_launch_select(nr_index *ix, const float *d_logits, const uint32_t *d_codes,
                              const int32_t *d_nprobe, int64_t nq, int P, int C, int32_t *d_L,
                              int32_t *d_nL, nr_seg *d_seg, uint32_t *d_slen, int64_t *d_stats,

@@ -83,7 +83,7 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   const size_t o_perm = o;   o = up256(o + q * 4);
   const size_t o_stats = o;  o = up256(o + q * NR_QSTATS * 8);
   const size_t slab_q = nr_select_slab_bytes(P, ix->K_max);
-  const size_t o_slab = o;   o = up256(o + q * slab_q);
+  const size_t o_slab = o;   o = up256(o + nr_select_slab_total((int64_t)q, P, ix->K_max));
   const size_t o_count = o;  o = up256(o + 16);
   if (o > NR_STATIC_SCRATCH_BYTES) return NR_ERR_INVALID_ARG;  // request too large for the array
   DeviceGuard g(ix->device);

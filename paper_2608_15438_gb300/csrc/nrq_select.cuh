@@ -216,16 +216,17 @@ __device__ __forceinline__ int select_tail_smem(const SelectParams &sp, uint64_t
 // cluster of every probed bucket). slog: the query's b logits in shared memory; scratch:
 // select_scratch_bytes(P, K_max) bytes of shared memory; slab: this query's
 // select_slab_bytes(P, K_max) bytes of global memory (null when that is 0);
-// warp_sums: 32 ints; sred: 2 unsigned. Returns nl; *total = stream length.
-// Whole block calls.
+// warp_sums: 32 ints; sred: 2 unsigned. Returns nl (*total = stream length),
+// or -1 when the query is deferred to the overflow kernel. Whole block calls.
 //
 // The keys to sort (C^dir and the gate's survivors) are collected straight
 // into shared memory: one pass over the candidate clusters computes their
 // distances, keeps the single-cluster buckets' and takes d_min over the rest;
 // a second pass recomputes the others' distances and keeps those within the
-// gate. Only when they do not fit does the query fall back to sorting all its
-// candidate keys in the global slab. Both give the same keys, and the sort
-// orders them by exact value.
+// gate. Only when they do not fit are the query's candidate keys written to
+// its global slab and the query deferred (returns -1) to the overflow
+// kernel, whose blocks sort more keys in shared memory. Both give the same
+// keys, and the sort orders them by exact value.
 __device__ __forceinline__ int select_block(const SelectParams &sp, const float *slog,
                                             const uint32_t *codes, int np, unsigned char *scratch,
                                             unsigned char *slab, int *warp_sums, unsigned *sred,
@@ -290,6 +291,9 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   // when theta(x) = x + M(x) does not decrease with x: for m1 >= 0
   // (x + fmaf(m1, x, m0)) and for a calibrated curve (non-decreasing y, each
   // segment held within its end values).
+  // Without the gate every candidate is kept: more than fit in shared memory
+  // go straight to the slab (one distance pass instead of two)
+  const bool direct = sp.gate_off && M > S_smem && slab != nullptr;
   if (tid == 0) sred[2] = 0u;  // keys collected from the front
   __syncthreads();
   const float m1 = sp.m1;
@@ -299,7 +303,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   // or one contiguous run of slots a thread, measured slower at 1e9 rows:
   // these random row reads run at the GPU's random-sector rate already.)
   int pi = tid < M ? slot_probe(cnt, np, tid) : 0;
-  for (int s = tid; s < M; s += nt) {
+  for (int s = tid; s < (direct ? 0 : M); s += nt) {
     const uint32_t c = (uint32_t)(c0s[pi] + (s - cnt[pi]));
     const bool single = (pi + 1 < np ? cnt[pi + 1] : M) - cnt[pi] == 1;  // C^dir
     const int sn = s + nt;
@@ -336,7 +340,7 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     theta = __fadd_rn(dmin, gate_margin(sp, dmin));  // theta = d_min + M(d_min)
   }
   const int nA = (int)sred[1], nB = (int)sred[2];
-  int Mk = nA + nB;
+  int Mk = direct ? S_smem + 1 : nA + nB;
   if (Mk <= S_smem) {
     // keep the front keys within the final gate, compacted toward the front
     // (a key never moves up, and each chunk reads before it writes), then move
@@ -386,35 +390,49 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
     Mk = S_smem + 1;  // does not fit: the slab path below
   }
   if (Mk <= S_smem) return select_tail_smem(sp, keys, Mk, warp_sums, seg, L, Lmax, total);
-  int Sn = 1;
-  int *ints = ibuf;
-  {
-    // more keys than shared memory holds: all candidate keys in the global slab
-    // (slab is present: without it M <= S_full = S_smem)
-    while (Sn < M) Sn <<= 1;
-    if (slab == nullptr || Sn > S_full) {
-      if (tid == 0) set_err(sp.err, NR_DEV_TOO_MANY);
-      *total = 0;
-      return 0;
-    }
-    keys = reinterpret_cast<uint64_t *>(slab);
-    ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
-    for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
-      const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
-      for (int j = 0; j < n; ++j) keys[o + j] = ((uint64_t)(uint32_t)(c0s[i] + j) << 1) | (n == 1 ? 1u : 0u);
-    }
-    __syncthreads();
-    for (int s = tid; s < M; s += nt) {
-      const uint64_t kc = keys[s];
-      const uint32_t c = key_cluster(kc);
-      const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
-      const bool keep = key_single(kc) || d <= theta;
-      keys[s] = keep ? tagged_key(d, c, key_single(kc)) : kEmpty;
-    }
-    for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
-    __syncthreads();
-    bitonic_sort(keys, Sn);
+  // more keys than shared memory holds: every candidate key goes to the
+  // query's global slab (tagged, or kEmpty where the gate drops it), and the
+  // query is finished by select_overflow_block in a kernel of its own, whose
+  // blocks hold more keys (returns -1: deferred)
+  if (slab == nullptr || M > S_full) {
+    if (tid == 0) set_err(sp.err, NR_DEV_TOO_MANY);
+    *total = 0;
+    return 0;
   }
+  uint64_t *gk = reinterpret_cast<uint64_t *>(slab);
+  for (int i = tid; i < np; i += nt) {  // each probe fills its clusters' slots
+    const int o = cnt[i], n = (i + 1 < np ? cnt[i + 1] : M) - o;
+    for (int j = 0; j < n; ++j) gk[o + j] = ((uint64_t)(uint32_t)(c0s[i] + j) << 1) | (n == 1 ? 1u : 0u);
+  }
+  __syncthreads();
+  for (int s = tid; s < M; s += nt) {
+    const uint64_t kc = gk[s];
+    const uint32_t c = key_cluster(kc);
+    const float d = centroid_dist(sp.cent + (size_t)c * sp.b, slog, sp.b);
+    const bool keep = key_single(kc) || d <= theta;
+    gk[s] = keep ? tagged_key(d, c, key_single(kc)) : kEmpty;
+  }
+  __syncthreads();
+  *total = 0;
+  return -1;
+}
+
+// The kept list of a deferred query from its slab keys[0..M) (tagged keys
+// or kEmpty) by a bitonic network over the slab itself: C^dir and the first
+// C others in key order, their segments and (L not null) clusters. For
+// queries whose kept keys exceed the overflow block's shared memory.
+__device__ __noinline__ int select_slab_finish(const SelectParams &sp, unsigned char *slab, int M,
+                                               int *warp_sums, nr_seg *seg, int32_t *L, int Lmax,
+                                               uint32_t *total) {
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int S_full = select_sort_cap(sp.P, sp.K_max);
+  int Sn = 1;
+  while (Sn < M) Sn <<= 1;
+  uint64_t *keys = reinterpret_cast<uint64_t *>(slab);
+  int *ints = reinterpret_cast<int *>(slab + (size_t)S_full * 8);
+  for (int s = M + tid; s < Sn; s += nt) keys[s] = kEmpty;
+  __syncthreads();
+  bitonic_sort(keys, Sn);
   // keep C^dir and the first C survivors in key order
   int *keep = ints;  // [Sn]
   for (int s = tid; s < Sn; s += nt) {
@@ -459,6 +477,113 @@ __device__ __forceinline__ int select_block(const SelectParams &sp, const float 
   __syncthreads();
   *total = (uint32_t)tot;
   return nl;
+}
+
+// Keys a block of the overflow kernel sorts in shared memory (its merge sort
+// runs of 16 keys a thread over kSelOvfThreads threads), and the buckets of
+// its preselection histogram.
+constexpr int kSelOvfThreads = 512;
+constexpr int kSelOvfKeys = 16 * kSelOvfThreads;
+constexpr int kSelOvfBuckets = 2048;
+__host__ __device__ inline size_t select_overflow_smem_bytes() {
+  return (size_t)select_smem_keys(kSelOvfKeys) * 8 + (size_t)kSelOvfBuckets * 4 + 32 * 4 + 32;
+}
+
+// A deferred query, from its slab keys[0..M) (tagged keys, or kEmpty where
+// the gate dropped a cluster). Only the C^dir keys and the C smallest others
+// can be in the list, so the others are preselected first: a histogram of
+// their distances' float bits (non-negative floats order as their bits) over
+// [lo, hi] in kSelOvfBuckets buckets (a key in a lower bucket is smaller),
+// and z* the bucket in which the count of others reaches C. Every other key
+// in a bucket above z* has at least C smaller others, so it cannot be kept;
+// the C^dir keys and the others up to bucket z* are collected into shared
+// memory in any order, and the list is made from them exactly as
+// select_tail_smem makes it (sort order, top-C, segments). When the
+// collection exceeds kSelOvfKeys, select_slab_finish sorts the whole slab.
+// skeys: select_smem_keys(kSelOvfKeys) keys and hist: kSelOvfBuckets uints of
+// shared memory; sctl: 4 unsigned. Whole block (kSelOvfThreads threads) calls.
+__device__ __forceinline__ int select_overflow_block(const SelectParams &sp, unsigned char *slab,
+                                                     int M, uint64_t *skeys, uint32_t *hist,
+                                                     unsigned *sctl, int *warp_sums, nr_seg *seg,
+                                                     int32_t *L, int Lmax, uint32_t *total) {
+  const int tid = threadIdx.x, nt = blockDim.x, lane = tid & 31;
+  const uint64_t *gk = reinterpret_cast<const uint64_t *>(slab);
+  for (int z = tid; z < kSelOvfBuckets; z += nt) hist[z] = 0u;
+  if (tid == 0) {
+    sctl[0] = 0u;           // keys collected
+    sctl[1] = 0xffffffffu;  // smallest distance bits of the others
+    sctl[2] = 0u;           // largest
+    sctl[3] = 0u;           // the others
+  }
+  __syncthreads();
+  uint32_t lo = 0xffffffffu, hi = 0u, no = 0u;
+  for (int s = tid; s < M; s += nt) {
+    const uint64_t k = gk[s];
+    if (k == kEmpty || key_single(k)) continue;
+    const uint32_t db = (uint32_t)(k >> 32);
+    lo = min(lo, db);
+    hi = max(hi, db);
+    ++no;
+  }
+  lo = __reduce_min_sync(kFull, lo);
+  hi = __reduce_max_sync(kFull, hi);
+  no = __reduce_add_sync(kFull, no);
+  if (lane == 0) {
+    atomicMin(&sctl[1], lo);
+    atomicMax(&sctl[2], hi);
+    atomicAdd(&sctl[3], no);
+  }
+  __syncthreads();
+  lo = sctl[1];
+  hi = sctl[2];
+  const uint32_t n_other = sctl[3];
+  int shift = 0;
+  if (hi >= lo)
+    while (((hi - lo) >> shift) >= (uint32_t)kSelOvfBuckets) ++shift;
+  uint32_t zs = kSelOvfBuckets - 1;  // every other key kept
+  if (n_other > (uint32_t)sp.C) {
+    for (int s = tid; s < M; s += nt) {
+      const uint64_t k = gk[s];
+      if (k == kEmpty || key_single(k)) continue;
+      atomicAdd(&hist[((uint32_t)(k >> 32) - lo) >> shift], 1u);
+    }
+    __syncthreads();
+    if (tid < 32) {  // the bucket in which the running count reaches C
+      constexpr int per = kSelOvfBuckets / 32;
+      uint32_t loc = 0;
+      for (int e = 0; e < per; ++e) loc += hist[lane * per + e];
+      uint32_t incl = loc;
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t v = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += v;
+      }
+      const unsigned hit = __ballot_sync(kFull, incl >= (uint32_t)sp.C);
+      const int src = __ffs(hit) - 1;  // hit != 0: the total exceeds C
+      if (lane == src) {
+        uint32_t run = incl - loc;
+        int z = lane * per;
+        for (;; ++z) {
+          run += hist[z];
+          if (run >= (uint32_t)sp.C) break;
+        }
+        sctl[1] = (unsigned)z;
+      }
+    }
+    __syncthreads();
+    zs = sctl[1];
+  }
+  for (int s = tid; s < M; s += nt) {
+    const uint64_t k = gk[s];
+    if (k == kEmpty) continue;
+    if (!key_single(k) && (((uint32_t)(k >> 32) - lo) >> shift) > zs) continue;
+    const unsigned pos = atomicAdd(&sctl[0], 1u);
+    if (pos < (unsigned)kSelOvfKeys) skeys[pos] = k;
+  }
+  __syncthreads();
+  const int n = (int)sctl[0];
+  __syncthreads();  // every thread has read the count
+  if (n <= kSelOvfKeys) return select_tail_smem(sp, skeys, n, warp_sums, seg, L, Lmax, total);
+  return select_slab_finish(sp, slab, M, warp_sums, seg, L, Lmax, total);
 }
 
 // ============================================================== select, mode 1

@@ -413,6 +413,47 @@ def test_select_overflow_to_global_slab(many_clusters, torch, C, m1):
     assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
 
 
+@pytest.mark.parametrize("C,m1", [(64, None), (4096, None), (64, 1.0)])
+def test_select_overflow_tied_distances(torch, tmp_path, C, m1):
+    """Every bucket of a 12-bit index holds 16 clusters with the same centroid,
+    so the 65,536 candidate distances of an all-probing query tie: the
+    overflow kernel's preselection cannot thin them out, and the list comes
+    from the bitonic sort of the whole slab, ties broken by cluster index
+    (and, with the gate on, every cluster sits exactly at d_min)."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    b, K = 12, 16
+    ncl = (1 << b) * K
+    rng = np.random.default_rng(5)
+    vec = rng.integers(0, 256, (ncl, 16)).astype(np.uint8)
+    path = str(tmp_path / "tied.nrix")
+    write_nrix(path, vec, np.arange(ncl), np.arange(0, ncl + 1, K), np.arange(ncl + 1),
+               np.full((ncl, b), 0.25, np.float32), np.zeros(b), np.zeros((16, 16)), np.zeros(16),
+               np.zeros((b, 16)), np.zeros(b), K_max=K)
+    ix = nr.Index(path, 0)
+    orc = oracle.Index(path)
+    lg = rng.normal(0, 1, (4, b)).astype(np.float32)
+    q = rng.integers(0, 256, (4, 16)).astype(np.uint8)
+    kw = {} if m1 is None else dict(gate_m0=0.0, gate_m1=m1)
+    ix.set_params(**kw)
+    try:
+        cl, ncl_q = ix.debug_clusters(torch.from_numpy(lg).cuda(), 1 << b, C)
+        ids, d = ix.search_logits(torch.from_numpy(q).cuda(), torch.from_numpy(lg).cuda(), 10,
+                                  1 << b, C)
+        torch.cuda.synchronize()
+    finally:
+        ix.set_params()
+    p = oracle.params(**kw)
+    cl, ncl_q = cl.cpu().numpy(), ncl_q.cpu().numpy()
+    for i in range(4):
+        codes, _, _ = oracle.probe_list(lg[i], orc.tau(), 1 << b, p)
+        L, _, _ = orc.cluster_list(lg[i], codes, C, p)
+        assert ncl_q[i] == len(L) == C and np.array_equal(cl[i, :C], L), i
+    ids_o, d_o, _ = orc.search(q, 10, 1 << b, C, p, logits=lg)
+    assert np.array_equal(ids.cpu().numpy(), ids_o) and np.array_equal(d.cpu().numpy(), d_o)
+    ix.close()
+
+
 @pytest.fixture(scope="module")
 def wide(torch, tmp_path_factory):
     """b = 12, up to 16 clusters per bucket, so that P = 2048 and 4096 give
