@@ -583,7 +583,8 @@ def encode_bench(args, w, torch, nr, dev):
     b.record(stream)
     torch.cuda.synchronize()
     ms = a.elapsed_time(b) / args.steps
-    flops = 2.0 * args.encode * (w.dim * w.hidden + w.hidden * w.bits)
+    dims = [w.dim, w.hidden, *getattr(w, "mid", ()), w.bits]
+    flops = 2.0 * args.encode * sum(a * c for a, c in zip(dims[:-1], dims[1:]))
     peaks, src = measured_peaks()
     tf = flops / (ms / 1e3) / 1e12
     print(json.dumps({"metric": "encoder TFLOP/s (fp16 tensor cores, fp32 accumulate)", "value": tf,
@@ -591,7 +592,7 @@ def encode_bench(args, w, torch, nr, dev):
                       "roofline": {"bound": "tensor", "achieved": tf, "peak": peaks.get("bf16_tflops"),
                                    "unit": "TFLOP/s", "frac": tf / peaks.get("bf16_tflops"),
                                    "peak_source": src + " bf16 dense (fp16 dense runs at the same nominal rate)"},
-                      "config": {"workload": w.name, "D": w.dim, "H": w.hidden, "b": w.bits}}), flush=True)
+                      "config": {"workload": w.name, "layers": dims}}), flush=True)
     return 0
 
 

@@ -285,13 +285,18 @@ nr_status nr_set_params(nr_index *ix, const nr_params *p);
 
 /* Encoder forward (Sec. 3.2.1): d_x [nq x D] (uint8 or fp32, the index dtype)
  * -> d_logits [nq x b] fp32, both device, row-major and contiguous.
- * h = ReLU(W1 (in_scale x) + b1), l = W2 h + b2. One hidden layer with
- * D % 16 == 0, D <= 128, H % 128 == 0, b <= 32 and d_x 16-byte aligned runs on
- * the tensor cores: operands fp16, accumulation fp32 (logits agree with an
- * exact evaluation to about 1e-3 of their norm). Other shapes, misaligned
- * input and encoders with more hidden layers run on CUDA cores in fp32.
- * nq = 0 is a no-op. Asynchronous on `stream`; a device-side wait that
- * expires sets the device flag (see nr_last_stats).
+ * h = ReLU(W1 (in_scale x) + b1), l = W2 h + b2 (with hidden layers after
+ * the first, each h' = ReLU(W h + b) in turn). With d_x 16-byte aligned these
+ * run on the tensor cores, operands fp16 (fp32 inputs and hidden activations
+ * rounded to fp16, so magnitudes beyond 65504 do not fit), accumulation fp32
+ * (logits agree with an exact evaluation to about 1e-3 of their norm): one
+ * hidden layer with D % 16 == 0, D <= 128, H % 128 == 0, b <= 32, fused in one
+ * kernel; several hidden layers with D and every hidden width multiples of
+ * 64, layer by layer, each layer's activations in a scratch buffer the index
+ * keeps (grown on demand: the first call of a larger batch, up to 2^18 rows,
+ * allocates and synchronises the device). Other shapes and misaligned input
+ * run on CUDA cores in fp32. nq = 0 is a no-op. Asynchronous on `stream`; a
+ * device-side wait that expires sets the device flag (see nr_last_stats).
  * Errors: NR_ERR_INVALID_ARG, NR_ERR_CUDA. */
 nr_status nr_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits, void *stream);
 

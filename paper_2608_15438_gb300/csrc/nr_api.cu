@@ -37,7 +37,7 @@ size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 // Per-chunk workspace layout of a search over qc queries.
 struct Layout {
-  size_t logits, codes, nprobe, L, nL, seg, slen, slab, perm, total;
+  size_t logits, codes, nprobe, L, nL, seg, slen, slab, perm, enc, total;
 };
 Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   Layout l;
@@ -52,6 +52,7 @@ Layout chunk_layout(const nr_index *ix, int64_t qc, int P, int C) {
   l.slen = o;   o = align256(o + (size_t)qc * 4);
   l.slab = o;   o = align256(o + nr_select_slab_total(qc, P, ix->K_max));
   l.perm = o;   o = align256(o + (size_t)qc * 4);
+  l.enc = o;    o = align256(o + nr_encode_scratch_bytes(ix, qc));
   l.total = o;
   return l;
 }
@@ -210,7 +211,48 @@ nr_status nr_index_upload_encoder(nr_index *ix, const float *W1, const float *b1
     }
     if ((st = up((void **)&ix->Wm, Wm, n * 4)) != NR_OK) return st;
     if ((st = up((void **)&ix->WmT, t.data(), n * 4)) != NR_OK) return st;
-    return NR_OK;  // the tensor-core encoder covers one hidden layer only
+    // the tensor-core layers: every K a multiple of 64, every hidden width a
+    // multiple of 64, b <= 256 (padded to a multiple of 16)
+    bool tc = D % 64 == 0 && H % 64 == 0 && b <= 256;
+    for (int l = 0; l < ix->n_mid; ++l) tc = tc && ix->mid_w[l] % 64 == 0;
+    if (!tc) return NR_OK;
+    const int L = ix->n_mid + 2;
+    std::vector<int> Kl(L), Nl(L);
+    std::vector<const float *> Wsrc(L);
+    Kl[0] = D, Nl[0] = H, Wsrc[0] = W1;
+    size_t o2 = 0;
+    for (int l = 0, prev = H; l < ix->n_mid; prev = ix->mid_w[l], ++l) {
+      Kl[l + 1] = prev, Nl[l + 1] = ix->mid_w[l], Wsrc[l + 1] = Wm + o2;
+      o2 += (size_t)ix->mid_w[l] * prev + ix->mid_w[l];
+    }
+    Kl[L - 1] = HL, Nl[L - 1] = b, Wsrc[L - 1] = W2;
+    size_t total = 0;
+    for (int l = 0; l < L; ++l) {
+      const int Np = (Nl[l] + 15) / 16 * 16;
+      int nt = 16;  // the largest multiple of 16 that divides Np, at most 256
+      for (int c = 256; c >= 16; c -= 16)
+        if (Np % c == 0) {
+          nt = c;
+          break;
+        }
+      ix->ly_nt[l] = nt;
+      ix->ly_off[l] = total;
+      total += (size_t)Np * Kl[l];
+    }
+    std::vector<__half> wl(total, __float2half_rn(0.0f));
+    for (int l = 0; l < L; ++l) {
+      const int K = Kl[l], N = Nl[l], nt = ix->ly_nt[l], nks = K / 64;
+      for (int r = 0; r < N; ++r)
+        for (int k = 0; k < K; ++k) {
+          const int ct = r / nt, rr = r % nt, ks = k / 64, kk = k % 64;
+          const size_t at = ix->ly_off[l] + ((size_t)ct * nks + ks) * nt * 64 +
+                            nr_tc_kmajor_off(rr, kk / 8, 8) / 2 + kk % 8;
+          wl[at] = __float2half_rn(Wsrc[l][(size_t)r * K + k]);
+        }
+    }
+    if ((st = up(&ix->Wl, wl.data(), wl.size() * 2)) != NR_OK) return st;
+    ix->n_ly = L;
+    return NR_OK;
   }
   // fp16 operands of the tensor-core encoder in its chunked operand order;
   // layer 2 padded to 16 or 32 rows (only shapes that kernel takes)
@@ -293,7 +335,7 @@ void nr_index_free(nr_index *ix) {
   if (ps.a) cudaStreamDestroy(ps.a);
   if (ps.b) cudaStreamDestroy(ps.b);
   void *ptrs[] = {ix->W1, ix->b1, ix->W2, ix->b2, ix->Wm, ix->WmT, ix->tau, ix->cent, ix->W1T, ix->W1h, ix->W2h, ix->bkt_off,
-                  ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->io};
+                  ix->cl_off, ix->ids, ix->vec, ix->d_err, ix->ws, e->io, ix->Wl, ix->enc_ws};
   for (void *p : ptrs)
     if (p) cudaFree(p);
   delete reinterpret_cast<nr_index_full *>(ix);
@@ -829,7 +871,7 @@ static nr_status search_impl(nr_index *ix, const void *d_q, const float *d_logit
     size_t ev;
     if (!d_logits_in) {
       ev = tstart(0, sa);
-      e = nr_launch_encode(ix, qp, n, (float *)(cw + l.logits), sa);
+      e = nr_launch_encode(ix, qp, n, (float *)(cw + l.logits), sa, cw + l.enc);
       tend(ev, sa);
       if (e != cudaSuccess) break;
     }

@@ -571,6 +571,262 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
 }
 
+// ------------------------------------------------------------ one layer on tensor cores
+// Encoders with hidden layers after the first run layer by layer, each layer
+// y = act(s x W^T + b) as a persistent tensor-core GEMM: a CTA takes
+// (128-row tile, Nt-column tile) items; four producer warps stage 64-wide K
+// slices of x (converted to fp16: uint8 exactly, fp32 rounded) and of W
+// (stored in fp16 as column tiles x K slices, each slice in the K-major
+// core-matrix order) into a ring of kLyStages shared-memory stages; one
+// thread issues four tcgen05.mma (K = 16 each) a slice into one of two TMEM
+// accumulators; four epilogue warps (one per TMEM lane group) read it back,
+// apply s, the bias and ReLU (hidden layers) and write fp16 activations, or
+// fp32 logits for the last layer. Waits are bounded as in the kernel above.
+constexpr int kLyKs = 64;        // K elements a slice
+constexpr int kLyStages = 3;
+constexpr int kLyEpiWarps = 4, kLyProdWarps = 4;
+constexpr int kLyWarpEpi = 1, kLyWarpProd = kLyWarpEpi + kLyEpiWarps;
+constexpr int kLyThreads = 32 * (kLyWarpProd + kLyProdWarps);  // 288
+constexpr int kLyProdThreads = 32 * kLyProdWarps, kLyEpiThreads = 32 * kLyEpiWarps;
+
+struct LyBars {
+  uint64_t full[kLyStages], empty[kLyStages];
+  uint64_t accfull[2], accempty[2];
+  uint64_t drain;
+  uint32_t tmem_slot;
+  int abort;
+};
+
+__host__ __device__ inline uint32_t ly_stage_bytes(int Nt) { return (uint32_t)(kRows + Nt) * kLyKs * 2u; }
+__host__ __device__ inline uint32_t ly_smem_bytes(int Nt) {
+  return kLyStages * ly_stage_bytes(Nt) + (uint32_t)sizeof(LyBars);
+}
+// TMEM columns of the two accumulators: a power of two of at least 32
+__host__ __device__ inline uint32_t ly_tmem_cols(int Nt) {
+  uint32_t c = 32;
+  while (c < 2u * (uint32_t)Nt) c <<= 1;
+  return c;
+}
+
+__device__ __forceinline__ void tc_alloc_n(uint32_t slot, uint32_t ncols) { tc_alloc(slot, ncols); }
+
+// XT: the input's type (0 uint8, 1 fp32, 2 fp16); YF: 1 fp32 output (the
+// logits, no activation), 0 fp16 output with ReLU. x [n x K], y [n x N]
+// row-major; W: (Npad / Nt) column tiles x (K / 64) slices of Nt x 64.
+template <int XT, int YF>
+__global__ void __launch_bounds__(kLyThreads, 1)
+    encode_layer_kernel(const void *__restrict__ x, int K, int N, int Nt, int Npad, float s,
+                        const __half *__restrict__ Wp, const float *__restrict__ bias, int64_t n,
+                        void *__restrict__ y, int *err, int64_t wait_ns) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  const uint32_t stage_b = ly_stage_bytes(Nt);
+  LyBars &B = *reinterpret_cast<LyBars *>(smem + kLyStages * stage_b);
+  volatile int *abort = &B.abort;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nks = K / kLyKs;                       // slices an item
+  const int nct = Npad / Nt;                       // column tiles
+  const int64_t nrt = (n + kRows - 1) / kRows;     // row tiles
+  const int64_t items = nrt * nct;
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t tcols = ly_tmem_cols(Nt);
+  if (warp == 0) {
+    tc_alloc_n(smem_u32(&B.tmem_slot), tcols);
+    tc_relinquish();
+  }
+  if (tid == 0) {
+    for (int i = 0; i < kLyStages; ++i) {
+      mbar_init(smem_u32(&B.full[i]), kLyProdThreads);
+      mbar_init(smem_u32(&B.empty[i]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&B.accfull[i]), 1);
+      mbar_init(smem_u32(&B.accempty[i]), kLyEpiThreads);
+    }
+    mbar_init(smem_u32(&B.drain), 1);
+    B.abort = 0;
+    fence_mbar_init();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = B.tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {  // the MMA thread
+      const uint32_t idesc = mma_idesc(kRows, Nt);
+      uint32_t g = 0, it = 0;  // slices and items of this CTA so far
+      bool ok = true;
+      for (int64_t item = blockIdx.x; item < items && ok; item += gridDim.x, ++it) {
+        const uint32_t a = it & 1u;
+        if (!wait_or_abort(smem_u32(&B.accempty[a]), ((it >> 1) & 1u) ^ 1u, abort, wait_ns)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + a * (uint32_t)Nt;
+        for (int ks = 0; ks < nks; ++ks, ++g) {
+          const uint32_t st = g % kLyStages;
+          if (!wait_or_abort(smem_u32(&B.full[st]), (g / kLyStages) & 1u, abort, wait_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sx = sbase + st * stage_b, sw = sx + (uint32_t)kRows * kLyKs * 2u;
+          for (int k = 0; k < kLyKs / 16; ++k)
+            tc_mma_f16(d, smem_desc(sx + (uint32_t)k * 256u, 128, 8 * 128),
+                       smem_desc(sw + (uint32_t)k * 256u, 128, 8 * 128), idesc,
+                       (ks > 0 || k > 0) ? 1u : 0u);
+          tc_commit(smem_u32(&B.empty[st]));
+        }
+        if (!ok) break;
+        tc_commit(smem_u32(&B.accfull[a]));
+      }
+      // every MMA of this thread completes before TMEM is freed
+      tc_commit(smem_u32(&B.drain));
+      mbar_wait_bounded(smem_u32(&B.drain), 0);
+    }
+    __syncwarp();
+  } else if (warp < kLyWarpProd) {  // epilogue: one TMEM lane group a warp
+    const int lg = warp & 3;
+    const uint32_t lane_base = (uint32_t)(lg * 32) << 16;
+    uint32_t it = 0;
+    for (int64_t item = blockIdx.x; item < items; item += gridDim.x, ++it) {
+      const uint32_t a = it & 1u;
+      if (!warp_wait(smem_u32(&B.accfull[a]), (it >> 1) & 1u, abort, wait_ns)) break;
+      tc_fence_after();
+      const int64_t rt = item / nct;
+      const int c0 = (int)(item % nct) * Nt;
+      const int64_t row = rt * kRows + lg * 32 + lane;
+      for (int cc = 0; cc < Nt; cc += 32) {
+        uint32_t v[32];
+        if (Nt - cc >= 32) {
+          tc_ld32(tmem + lane_base + a * (uint32_t)Nt + (uint32_t)cc, v);
+        } else {
+          uint32_t w16[16];
+          tc_ld16(tmem + lane_base + a * (uint32_t)Nt + (uint32_t)cc, w16);
+#pragma unroll
+          for (int j = 0; j < 16; ++j) v[j] = w16[j];
+        }
+        tc_wait_ld();
+        const int ncol = min(32, Nt - cc);
+        if (row < n) {
+          if (YF) {
+            float *dst = static_cast<float *>(y) + row * N;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const int col = c0 + cc + j;
+              if (j < ncol && col < N) dst[col] = __fmaf_rn(s, __uint_as_float(v[j]), bias[col]);
+            }
+          } else {
+            // hidden widths are multiples of 64: every column of the tile exists
+            __half *dst = static_cast<__half *>(y) + row * N + c0 + cc;
+            uint32_t hp[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const int col = c0 + cc + (2 * j < ncol ? 2 * j : 0);
+              const float h0 = __fmaf_rn(s, __uint_as_float(v[2 * j]), bias[col]);
+              const float h1 = __fmaf_rn(s, __uint_as_float(v[2 * j + 1]), bias[col + 1]);
+              const __half2 p = __hmax2(__floats2half2_rn(h0, h1), __float2half2_rn(0.0f));
+              hp[j] = *reinterpret_cast<const uint32_t *>(&p);
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if (8 * q < ncol)
+                reinterpret_cast<uint4 *>(dst)[q] = make_uint4(hp[4 * q], hp[4 * q + 1], hp[4 * q + 2], hp[4 * q + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(smem_u32(&B.accempty[a]));
+    }
+  } else {  // producers: x and W slices into the stage ring
+    const int ct = tid - kLyWarpProd * 32;
+    uint32_t g = 0;
+    for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+      const int64_t rt = item / nct;
+      const int ctile = (int)(item % nct);
+      const int64_t row0 = rt * kRows;
+      const int rows = n - row0 < kRows ? (int)(n - row0) : kRows;
+      const uint4 *wt = reinterpret_cast<const uint4 *>(Wp) + (size_t)ctile * nks * Nt * 8;
+      bool ok = true;
+      for (int ks = 0; ks < nks; ++ks, ++g) {
+        const uint32_t st = g % kLyStages;
+        unsigned char *sx = smem + st * stage_b;
+        unsigned char *sw = sx + kRows * kLyKs * 2;
+        // the slice's loads first, then the wait for its stage
+        uint4 xv[8];
+        if (XT == 2) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {  // 128 rows x 8 chunks of 8 fp16
+            const int k = ct + kLyProdThreads * j, r = k >> 3, c = k & 7;
+            xv[j] = make_uint4(0u, 0u, 0u, 0u);
+            if (r < rows)
+              xv[j] = __ldg(reinterpret_cast<const uint4 *>(static_cast<const __half *>(x) +
+                                                            (row0 + r) * K + ks * kLyKs) + c);
+          }
+        } else if (XT == 1) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int k = ct + kLyProdThreads * j, r = k >> 3, c = k & 7;
+            float4 u = make_float4(0.f, 0.f, 0.f, 0.f), w = u;
+            if (r < rows) {
+              const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(x) +
+                                                                   (row0 + r) * K + ks * kLyKs) + 2 * c;
+              u = __ldg(src);
+              w = __ldg(src + 1);
+            }
+            const __half2 h0 = __floats2half2_rn(u.x, u.y), h1 = __floats2half2_rn(u.z, u.w);
+            const __half2 h2 = __floats2half2_rn(w.x, w.y), h3 = __floats2half2_rn(w.z, w.w);
+            xv[j] = make_uint4(*reinterpret_cast<const uint32_t *>(&h0), *reinterpret_cast<const uint32_t *>(&h1),
+                               *reinterpret_cast<const uint32_t *>(&h2), *reinterpret_cast<const uint32_t *>(&h3));
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {  // 128 rows x 4 pieces of 16 uint8
+            const int k = ct + kLyProdThreads * j, r = k >> 2, c = k & 3;
+            uint4 v = make_uint4(0u, 0u, 0u, 0u);
+            if (r < rows)
+              v = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint8_t *>(x) +
+                                                        (row0 + r) * K + ks * kLyKs) + c);
+            u8x16_to_f16(v, xv[2 * j], xv[2 * j + 1]);
+          }
+        }
+        if (!warp_wait(smem_u32(&B.empty[st]), ((g / kLyStages) & 1u) ^ 1u, abort, wait_ns)) {
+          ok = false;
+          break;
+        }
+        if (XT == 0) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int k = ct + kLyProdThreads * j, r = k >> 2, c = k & 3;
+            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, 2 * c, 8)) = xv[2 * j];
+            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, 2 * c + 1, 8)) = xv[2 * j + 1];
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int k = ct + kLyProdThreads * j, r = k >> 3, c = k & 7;
+            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, c, 8)) = xv[j];
+          }
+        }
+        const uint4 *ws = wt + (size_t)ks * Nt * 8;  // the W slice, already in operand order
+        for (int i = ct; i < Nt * 8; i += kLyProdThreads)
+          reinterpret_cast<uint4 *>(sw)[i] = __ldg(ws + i);
+        fence_async_smem();
+        mbar_arrive(smem_u32(&B.full[st]));
+      }
+      if (!ok) break;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (tid == 0 && B.abort) atomicCAS(err, 0, NR_DEV_TIMEOUT);
+  if (warp == 0) {
+    tc_fence_after();
+    tc_dealloc(tmem, tcols);
+  }
+}
+
 // X tile buffers for a shape: 2 if a block's shared memory allows, else 1, else 0
 int tc_xbuffers(int D, int H, int n2, int smem_optin) {
   for (int nxb = 2; nxb >= 1; --nxb)
@@ -709,14 +965,108 @@ __global__ void __launch_bounds__(kThreads)
 }  // namespace
 
 bool nr_encode_uses_tensor_cores(const nr_index *ix) {
+  if (ix->n_ly > 0) return true;
   return ix->W1h != nullptr && ix->n_mid == 0 && ix->D % 16 == 0 && ix->D <= 128 &&
          ix->H % kHC == 0 && ix->b <= 32 &&
          tc_xbuffers(ix->D, ix->H, ix->b <= 16 ? 16 : 32, ix->smem_optin) > 0;
 }
 
+// rows a layer-by-layer encode runs at once (its activation scratch: two
+// buffers of rows x the widest hidden layer, fp16)
+constexpr int64_t kEncRowBlock = (int64_t)1 << 18;
+
+static int enc_max_hidden(const nr_index *ix) {
+  int m = ix->H;
+  for (int l = 0; l < ix->n_mid; ++l) m = ix->mid_w[l] > m ? ix->mid_w[l] : m;
+  return m;
+}
+
+size_t nr_encode_scratch_bytes(const nr_index *ix, int64_t n) {
+  if (ix->n_ly == 0 || n <= 0) return 0;
+  const int64_t rows = n < kEncRowBlock ? n : kEncRowBlock;
+  return ((size_t)rows * enc_max_hidden(ix) * 2 + 255) / 256 * 256 * 2;
+}
+
+template <int XT, int YF>
+static cudaError_t launch_layer(nr_index *ix, const void *x, int K, int N, int l, float sc,
+                                const float *bias, int64_t n, void *y, int64_t wait_ns,
+                                cudaStream_t s) {
+  const int nt = ix->ly_nt[l], Np = (N + 15) / 16 * 16;
+  uint32_t smem = ly_smem_bytes(nt);
+  // accumulators wider than half of TMEM: one CTA an SM (a second would
+  // stall in its TMEM allocation until the first ends)
+  if (ly_tmem_cols(nt) > 256 && smem <= (uint32_t)ix->smem_optin / 2)
+    smem = (uint32_t)ix->smem_optin / 2 + 1024;
+  auto kern = encode_layer_kernel<XT, YF>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int64_t items = (n + kRows - 1) / kRows * (Np / nt);
+  const int64_t grid = items < ix->num_sms ? items : ix->num_sms;
+  kern<<<(unsigned)grid, kLyThreads, smem, s>>>(x, K, N, nt, Np, sc,
+                                                static_cast<const __half *>(ix->Wl) + ix->ly_off[l],
+                                                bias, n, y, ix->d_err, wait_ns);
+  ix->launches += 1;
+  return cudaGetLastError();
+}
+
+// An encoder with hidden layers after the first, layer by layer on tensor
+// cores, in row blocks of kEncRowBlock (activations in scratch).
+static cudaError_t encode_layers(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
+                                 cudaStream_t s, void *scratch, int64_t wait_ns) {
+  const int L = ix->n_ly;
+  const size_t half = nr_encode_scratch_bytes(ix, nq) / 2;
+  __half *act[2] = {static_cast<__half *>(scratch),
+                    reinterpret_cast<__half *>(static_cast<char *>(scratch) + half)};
+  const size_t esz = ix->dtype == 0 ? 1 : 4;
+  for (int64_t r0 = 0; r0 < nq; r0 += kEncRowBlock) {
+    const int64_t n = nq - r0 < kEncRowBlock ? nq - r0 : kEncRowBlock;
+    const void *x = static_cast<const char *>(d_x) + (size_t)r0 * ix->D * esz;
+    cudaError_t e = ix->dtype == 0
+                        ? launch_layer<0, 0>(ix, x, ix->D, ix->H, 0, ix->in_scale, ix->b1, n, act[0],
+                                             wait_ns, s)
+                        : launch_layer<1, 0>(ix, x, ix->D, ix->H, 0, ix->in_scale, ix->b1, n, act[0],
+                                             wait_ns, s);
+    if (e != cudaSuccess) return e;
+    size_t o = 0;  // the middle layers' weights then bias, as the file stores them
+    int prev = ix->H;
+    for (int l = 0; l < ix->n_mid; ++l) {
+      const int w = ix->mid_w[l];
+      const float *bias = ix->Wm + o + (size_t)w * prev;
+      e = launch_layer<2, 0>(ix, act[l & 1], prev, w, l + 1, 1.0f, bias, n, act[(l + 1) & 1], wait_ns,
+                             s);
+      if (e != cudaSuccess) return e;
+      o += (size_t)w * prev + w;
+      prev = w;
+    }
+    e = launch_layer<2, 1>(ix, act[ix->n_mid & 1], prev, ix->b, L - 1, 1.0f, ix->b2, n,
+                           d_logits + (size_t)r0 * ix->b, wait_ns, s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
 cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
-                             cudaStream_t s) {
+                             cudaStream_t s, void *scratch) {
   if (nq <= 0) return cudaSuccess;
+  const int wl = ix->params.wait_limit_us;
+  const int64_t wait_ns = wl == 0 ? (int64_t)1000000000 : wl > 0 ? (int64_t)wl * 1000 : (int64_t)-1;
+  if (ix->n_ly > 0 && (reinterpret_cast<uintptr_t>(d_x) & 15) == 0) {
+    if (!scratch) {  // the index's own scratch, grown on demand
+      const size_t need = nr_encode_scratch_bytes(ix, nq);
+      if (ix->enc_ws_cap < need) {
+        cudaError_t e = cudaDeviceSynchronize();  // earlier encodes may still read it
+        if (e != cudaSuccess) return e;
+        if (ix->enc_ws) cudaFree(ix->enc_ws);
+        ix->enc_ws = nullptr;
+        ix->enc_ws_cap = 0;
+        e = cudaMalloc(&ix->enc_ws, need);
+        if (e != cudaSuccess) return e;
+        ix->enc_ws_cap = need;
+      }
+      scratch = ix->enc_ws;
+    }
+    return encode_layers(ix, d_x, nq, d_logits, s, scratch, wait_ns);
+  }
   // the tensor-core kernel reads X in 16-byte pieces
   if (nr_encode_uses_tensor_cores(ix) && (reinterpret_cast<uintptr_t>(d_x) & 15) == 0) {
     const int n2 = ix->b <= 16 ? 16 : 32;
@@ -728,10 +1078,8 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
     const int64_t tiles = (nq + kRows - 1) / kRows;
     const int64_t grid = tiles < ix->num_sms ? tiles : ix->num_sms;
     const int vec_out = ix->b % 4 == 0 && (reinterpret_cast<uintptr_t>(d_logits) & 15) == 0;
-    // the roles' hand-off waits: 1 s by default; the drain of issued MMAs
-    // before TMEM is freed keeps its own 1 s bound whatever this is
-    const int wl = ix->params.wait_limit_us;
-    const int64_t wait_ns = wl == 0 ? (int64_t)1000000000 : wl > 0 ? (int64_t)wl * 1000 : (int64_t)-1;
+    // the roles' hand-off waits: wait_ns (1 s by default); the drain of
+    // issued MMAs before TMEM is freed keeps its own 1 s bound whatever this is
     kern<<<(unsigned)grid, kTcThreads, smem, s>>>(d_x, ix->D, ix->H, ix->b, n2, nxb, vec_out, ix->in_scale,
                                                   static_cast<const __half *>(ix->W1h), ix->b1,
                                                   static_cast<const __half *>(ix->W2h), ix->b2, nq,

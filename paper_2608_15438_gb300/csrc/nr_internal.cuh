@@ -70,6 +70,17 @@ struct nr_index {
   // [16 or 32 x 128] per chunk (rows >= b zero)
   void *W1h = nullptr;
   void *W2h = nullptr;
+  // encoders with hidden layers after the first, on tensor cores layer by
+  // layer: every layer's fp16 weights in (column tile, 64-wide K slice)
+  // blocks in the nr_tc_kmajor_off order (n_ly = 0: such an encoder runs on
+  // CUDA cores); the activation scratch of nr_encode and the index build,
+  // grown on demand
+  int n_ly = 0;
+  size_t ly_off[9] = {};  // element offset of layer l's weights in Wl
+  int ly_nt[9] = {};      // its column tile (a multiple of 16, at most 256)
+  void *Wl = nullptr;
+  void *enc_ws = nullptr;
+  size_t enc_ws_cap = 0;
   uint32_t *bkt_off = nullptr, *cl_off = nullptr, *ids = nullptr;
   void *vec = nullptr;
   int *d_err = nullptr;
@@ -127,8 +138,13 @@ size_t nr_mid_floats(const nr_index *ix);
 
 // kernel launchers (each returns cudaGetLastError() after the launch)
 bool nr_encode_uses_tensor_cores(const nr_index *ix);
+// device scratch an encode of n rows needs (the activations of an encoder
+// with several hidden layers on tensor cores), 0 when none
+size_t nr_encode_scratch_bytes(const nr_index *ix, int64_t n);
+// scratch: nr_encode_scratch_bytes(ix, nq) bytes, or null to use (and grow,
+// synchronising the device) the index's own
 cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d_logits,
-                             cudaStream_t s);
+                             cudaStream_t s, void *scratch = nullptr);
 cudaError_t nr_launch_route(nr_index *ix, const float *d_logits, int64_t nq, int P,
                             uint32_t *d_codes, int32_t *d_nprobe, cudaStream_t s);
 // dynamic shared memory of the select kernel for budgets (P, C) under the

@@ -68,7 +68,8 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   if (!d_queries || !d_out_ids || !d_out_dists) return NR_ERR_INVALID_ARG;
   // scratch layout: logits, codes, probe counts, cluster lists and their
   // counts, segments, stream lengths, the refinement order, per-query stats,
-  // select's global sort slabs, the query counter. nq < 2^31 and every
+  // select's global sort slabs, the query counter, the activations of an
+  // encoder with several hidden layers. nq < 2^31 and every
   // per-query size is bounded (P, C <= 4096, b <= 24, the slab <= 768 KiB),
   // so no product below overflows size_t.
   const size_t Lmax = (size_t)P + (size_t)C, q = (size_t)nq;
@@ -85,6 +86,7 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   const size_t slab_q = nr_select_slab_bytes(P, ix->K_max);
   const size_t o_slab = o;   o = up256(o + nr_select_slab_total((int64_t)q, P, ix->K_max));
   const size_t o_count = o;  o = up256(o + 16);
+  const size_t o_enc = o;    o = up256(o + nr_encode_scratch_bytes(ix, (int64_t)q));
   if (o > NR_STATIC_SCRATCH_BYTES) return NR_ERR_INVALID_ARG;  // request too large for the array
   DeviceGuard g(ix->device);
   if (!g.ok) return NR_ERR_CUDA;
@@ -97,7 +99,7 @@ extern "C" nr_status nr_search_static(nr_index *ix, const void *d_queries, int64
   int64_t *stats = (int64_t *)(w + o_stats);
   // every buffer below is fully written before it is read, except the
   // refine kernel's query counter, which its launcher clears on the stream
-  cudaError_t e = nr_launch_encode(ix, d_queries, nq, logits, s);
+  cudaError_t e = nr_launch_encode(ix, d_queries, nq, logits, s, w + o_enc);
   if (e == cudaSuccess)
     e = nr_launch_route(ix, logits, nq, P, (uint32_t *)(w + o_codes), (int32_t *)(w + o_nprobe), s);
   if (e == cudaSuccess)
