@@ -25,10 +25,10 @@
 // flight (bounded by 1 s whatever the limit), records NR_DEV_TIMEOUT, frees
 // its TMEM and returns.
 //
-// What the tensor-core kernel does not take (D % 16 != 0, D > 128,
-// H % 128 != 0, b > 32, W1 and W2 too large for a CTA's shared memory, input
-// rows not 16-byte aligned) runs on the CUDA-core kernels below it, and so
-// do encoders with more hidden layers.
+// Encoders with hidden layers after the first run layer by layer on a second
+// tensor-core kernel (encode_layer_kernel). What neither takes (shapes
+// outside their limits, input rows not 16-byte aligned) runs on the
+// CUDA-core kernels at the end of the file.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -574,30 +574,42 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // ------------------------------------------------------------ one layer on tensor cores
 // Encoders with hidden layers after the first run layer by layer, each layer
 // y = act(s x W^T + b) as a persistent tensor-core GEMM: a CTA takes
-// (128-row tile, Nt-column tile) items; four producer warps stage 64-wide K
-// slices of x (converted to fp16: uint8 exactly, fp32 rounded) and of W
-// (stored in fp16 as column tiles x K slices, each slice in the K-major
-// core-matrix order) into a ring of kLyStages shared-memory stages; one
-// thread issues four tcgen05.mma (K = 16 each) a slice into one of two TMEM
-// accumulators; four epilogue warps (one per TMEM lane group) read it back,
-// apply s, the bias and ReLU (hidden layers) and write fp16 activations, or
-// fp32 logits for the last layer. Waits are bounded as in the kernel above.
+// (128-row tile, Nt-column tile) items; producers fill a ring of kLyStages
+// shared-memory stages with 64-wide K slices of x and of W; one thread issues
+// four tcgen05.mma (K = 16 each) a slice into one of two TMEM accumulators;
+// four epilogue warps (one per TMEM lane group) read it back, apply s, the
+// bias and ReLU (hidden layers) and write fp16 activations, or fp32 logits
+// for the last layer.
+//
+// W sits in global memory as (Npad / Nt) column tiles x (K / 64) slices of
+// Nt x 64 fp16 in the K-major core-matrix order (the host writes it so at
+// load), and hidden activations are written in the same order, as 128-row
+// tiles x 64-column slices of 16 KB: every slice of either operand is one
+// contiguous block, fetched by one bulk copy (cp.async.bulk, completing on
+// an mbarrier by its byte count). The first layer's input (uint8 or fp32
+// rows) goes through the producer warps' registers, converted to fp16
+// (uint8 exactly, fp32 rounded); the first producer thread fetches W.
+// Waits are bounded as in the kernel above; a CTA that gives up first waits
+// (bounded) for the bulk copies it issued.
 constexpr int kLyKs = 64;        // K elements a slice
 constexpr int kLyStages = 3;
-constexpr int kLyEpiWarps = 4, kLyProdWarps = 4;
+constexpr int kLyEpiWarps = 4, kLyProdWarps = 4;  // a producer group
 constexpr int kLyWarpEpi = 1, kLyWarpProd = kLyWarpEpi + kLyEpiWarps;
-constexpr int kLyThreads = 32 * (kLyWarpProd + kLyProdWarps);  // 288
+constexpr int kLyThreads = 32 * (kLyWarpProd + 2 * kLyProdWarps);  // 416
 constexpr int kLyProdThreads = 32 * kLyProdWarps, kLyEpiThreads = 32 * kLyEpiWarps;
+constexpr uint32_t kLyXSlice = (uint32_t)kRows * kLyKs * 2u;    // 16 KB of fp16
 
 struct LyBars {
-  uint64_t full[kLyStages], empty[kLyStages];
+  uint64_t xfull[kLyStages];  // x stored by the producer threads (first layer)
+  uint64_t tfull[2][kLyStages];  // a producer group's bulk copies into the stage landed
+  uint64_t empty[kLyStages];
   uint64_t accfull[2], accempty[2];
   uint64_t drain;
   uint32_t tmem_slot;
   int abort;
 };
 
-__host__ __device__ inline uint32_t ly_stage_bytes(int Nt) { return (uint32_t)(kRows + Nt) * kLyKs * 2u; }
+__host__ __device__ inline uint32_t ly_stage_bytes(int Nt) { return kLyXSlice + (uint32_t)Nt * kLyKs * 2u; }
 __host__ __device__ inline uint32_t ly_smem_bytes(int Nt) {
   return kLyStages * ly_stage_bytes(Nt) + (uint32_t)sizeof(LyBars);
 }
@@ -608,11 +620,21 @@ __host__ __device__ inline uint32_t ly_tmem_cols(int Nt) {
   return c;
 }
 
-__device__ __forceinline__ void tc_alloc_n(uint32_t slot, uint32_t ncols) { tc_alloc(slot, ncols); }
+__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+// bulk copy global -> this CTA's shared memory, completing on `bar` by bytes
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
 
-// XT: the input's type (0 uint8, 1 fp32, 2 fp16); YF: 1 fp32 output (the
-// logits, no activation), 0 fp16 output with ReLU. x [n x K], y [n x N]
-// row-major; W: (Npad / Nt) column tiles x (K / 64) slices of Nt x 64.
+// XT: the input's type (0 uint8 rows, 1 fp32 rows, 2 fp16 activations in
+// operand order); YF: 1 fp32 output rows (the logits, no activation), 0 fp16
+// activations in operand order with ReLU. x [n x K], y [n x N].
 template <int XT, int YF>
 __global__ void __launch_bounds__(kLyThreads, 1)
     encode_layer_kernel(const void *__restrict__ x, int K, int N, int Nt, int Npad, float s,
@@ -629,13 +651,16 @@ __global__ void __launch_bounds__(kLyThreads, 1)
   const int64_t items = nrt * nct;
   const uint32_t sbase = smem_u32(smem);
   const uint32_t tcols = ly_tmem_cols(Nt);
+  const uint32_t wbytes = (uint32_t)Nt * kLyKs * 2u;
   if (warp == 0) {
-    tc_alloc_n(smem_u32(&B.tmem_slot), tcols);
+    tc_alloc(smem_u32(&B.tmem_slot), tcols);
     tc_relinquish();
   }
   if (tid == 0) {
     for (int i = 0; i < kLyStages; ++i) {
-      mbar_init(smem_u32(&B.full[i]), kLyProdThreads);
+      mbar_init(smem_u32(&B.xfull[i]), kLyProdThreads);
+      mbar_init(smem_u32(&B.tfull[0][i]), 1);
+      mbar_init(smem_u32(&B.tfull[1][i]), 1);
       mbar_init(smem_u32(&B.empty[i]), 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -665,13 +690,18 @@ __global__ void __launch_bounds__(kLyThreads, 1)
         tc_fence_after();
         const uint32_t d = tmem + a * (uint32_t)Nt;
         for (int ks = 0; ks < nks; ++ks, ++g) {
-          const uint32_t st = g % kLyStages;
-          if (!wait_or_abort(smem_u32(&B.full[st]), (g / kLyStages) & 1u, abort, wait_ns)) {
+          const uint32_t st = g % kLyStages, ph = (g / kLyStages) & 1u;
+          // the copies of slice g: group g % 2 (XT 0 / 1: that group's phases
+          // on the stage are slices g, g + 6, ...), or group 0 (XT 2)
+          const uint32_t tb = XT == 2 ? smem_u32(&B.tfull[0][st]) : smem_u32(&B.tfull[g & 1u][st]);
+          const uint32_t tph = XT == 2 ? ph : (g / (2 * kLyStages)) & 1u;
+          if (!wait_or_abort(tb, tph, abort, wait_ns) ||
+              (XT != 2 && !wait_or_abort(smem_u32(&B.xfull[st]), ph, abort, wait_ns))) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sx = sbase + st * stage_b, sw = sx + (uint32_t)kRows * kLyKs * 2u;
+          const uint32_t sx = sbase + st * stage_b, sw = sx + kLyXSlice;
           for (int k = 0; k < kLyKs / 16; ++k)
             tc_mma_f16(d, smem_desc(sx + (uint32_t)k * 256u, 128, 8 * 128),
                        smem_desc(sw + (uint32_t)k * 256u, 128, 8 * 128), idesc,
@@ -689,6 +719,7 @@ __global__ void __launch_bounds__(kLyThreads, 1)
   } else if (warp < kLyWarpProd) {  // epilogue: one TMEM lane group a warp
     const int lg = warp & 3;
     const uint32_t lane_base = (uint32_t)(lg * 32) << 16;
+    const int r = lg * 32 + lane;  // the row in the tile
     uint32_t it = 0;
     for (int64_t item = blockIdx.x; item < items; item += gridDim.x, ++it) {
       const uint32_t a = it & 1u;
@@ -696,7 +727,7 @@ __global__ void __launch_bounds__(kLyThreads, 1)
       tc_fence_after();
       const int64_t rt = item / nct;
       const int c0 = (int)(item % nct) * Nt;
-      const int64_t row = rt * kRows + lg * 32 + lane;
+      const int64_t row = rt * kRows + r;
       for (int cc = 0; cc < Nt; cc += 32) {
         uint32_t v[32];
         if (Nt - cc >= 32) {
@@ -718,21 +749,25 @@ __global__ void __launch_bounds__(kLyThreads, 1)
               if (j < ncol && col < N) dst[col] = __fmaf_rn(s, __uint_as_float(v[j]), bias[col]);
             }
           } else {
-            // hidden widths are multiples of 64: every column of the tile exists
-            __half *dst = static_cast<__half *>(y) + row * N + c0 + cc;
-            uint32_t hp[16];
+            // hidden widths are multiples of 64: every column of the tile
+            // exists; 8 columns (16 bytes) go to their core-matrix row
+            __half *tile = static_cast<__half *>(y) + (size_t)rt * N * kRows;
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const int col = c0 + cc + (2 * j < ncol ? 2 * j : 0);
-              const float h0 = __fmaf_rn(s, __uint_as_float(v[2 * j]), bias[col]);
-              const float h1 = __fmaf_rn(s, __uint_as_float(v[2 * j + 1]), bias[col + 1]);
-              const __half2 p = __hmax2(__floats2half2_rn(h0, h1), __float2half2_rn(0.0f));
-              hp[j] = *reinterpret_cast<const uint32_t *>(&p);
+            for (int q = 0; q < 4; ++q) {
+              if (8 * q >= ncol) break;
+              const int col = c0 + cc + 8 * q;
+              uint32_t hp[4];
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                const float h0 = __fmaf_rn(s, __uint_as_float(v[8 * q + 2 * j]), bias[col + 2 * j]);
+                const float h1 = __fmaf_rn(s, __uint_as_float(v[8 * q + 2 * j + 1]), bias[col + 2 * j + 1]);
+                const __half2 p = __hmax2(__floats2half2_rn(h0, h1), __float2half2_rn(0.0f));
+                hp[j] = *reinterpret_cast<const uint32_t *>(&p);
+              }
+              __half *dst = tile + (size_t)(col >> 6) * (kRows * kLyKs) +
+                            nr_tc_kmajor_off(r, (col & 63) >> 3, 8) / 2;
+              *reinterpret_cast<uint4 *>(dst) = make_uint4(hp[0], hp[1], hp[2], hp[3]);
             }
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-              if (8 * q < ncol)
-                reinterpret_cast<uint4 *>(dst)[q] = make_uint4(hp[4 * q], hp[4 * q + 1], hp[4 * q + 2], hp[4 * q + 3]);
           }
         }
       }
@@ -740,82 +775,108 @@ __global__ void __launch_bounds__(kLyThreads, 1)
       mbar_arrive(smem_u32(&B.accempty[a]));
     }
   } else {  // producers: x and W slices into the stage ring
-    const int ct = tid - kLyWarpProd * 32;
+    const int grp = (warp - kLyWarpProd) / kLyProdWarps;  // XT 0 / 1: two groups
+    const int ct = tid - kLyWarpProd * 32 - grp * kLyProdThreads;
+    const bool lead = ct == 0;  // issues the bulk copies (of its group's slices)
     uint32_t g = 0;
-    for (int64_t item = blockIdx.x; item < items; item += gridDim.x) {
+    bool ok = true;
+    for (int64_t item = blockIdx.x; item < items && ok; item += gridDim.x) {
       const int64_t rt = item / nct;
       const int ctile = (int)(item % nct);
       const int64_t row0 = rt * kRows;
       const int rows = n - row0 < kRows ? (int)(n - row0) : kRows;
-      const uint4 *wt = reinterpret_cast<const uint4 *>(Wp) + (size_t)ctile * nks * Nt * 8;
-      bool ok = true;
+      const char *wt = reinterpret_cast<const char *>(Wp) + (size_t)ctile * nks * wbytes;
       for (int ks = 0; ks < nks; ++ks, ++g) {
-        const uint32_t st = g % kLyStages;
+        const uint32_t st = g % kLyStages, ph = ((g / kLyStages) & 1u) ^ 1u;
         unsigned char *sx = smem + st * stage_b;
-        unsigned char *sw = sx + kRows * kLyKs * 2;
-        // the slice's loads first, then the wait for its stage
-        uint4 xv[8];
-        if (XT == 2) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {  // 128 rows x 8 chunks of 8 fp16
-            const int k = ct + kLyProdThreads * j, r = k >> 3, c = k & 7;
-            xv[j] = make_uint4(0u, 0u, 0u, 0u);
-            if (r < rows)
-              xv[j] = __ldg(reinterpret_cast<const uint4 *>(static_cast<const __half *>(x) +
-                                                            (row0 + r) * K + ks * kLyKs) + c);
+        if (XT == 2) {  // both operands by bulk copy, from one thread
+          if (!lead || grp != 0) continue;
+          if (!wait_or_abort(smem_u32(&B.empty[st]), ph, abort, wait_ns)) {
+            ok = false;
+            break;
           }
-        } else if (XT == 1) {
+          const uint32_t bar = smem_u32(&B.tfull[0][st]);
+          mbar_arrive_tx(bar, kLyXSlice + wbytes);
+          bulk_g2s(sbase + st * stage_b,
+                   static_cast<const char *>(x) + ((size_t)rt * nks + ks) * kLyXSlice, kLyXSlice, bar);
+          bulk_g2s(sbase + st * stage_b + kLyXSlice, wt + (size_t)ks * wbytes, wbytes, bar);
+          continue;
+        }
+        // group grp takes the slices g with g % 2 == grp: two slices' loads
+        // in flight. Warp pw of the group takes rows 32 pw .. 32 pw + 31; in
+        // each load a lane reads row 8 i + lane % 8 of them, so that a warp
+        // touches 8 rows (8 cache lines) and every 8 lanes store 8 different
+        // rows of one chunk (different banks in the core-matrix layout)
+        if ((g & 1u) != (uint32_t)grp) continue;
+        const int pw = ct >> 5, rl = lane & 7, q = lane >> 3;
+        uint4 xv[8];
+        if (XT == 1) {
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int k = ct + kLyProdThreads * j, r = k >> 3, c = k & 7;
-            float4 u = make_float4(0.f, 0.f, 0.f, 0.f), w = u;
-            if (r < rows) {
-              const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(x) +
-                                                                   (row0 + r) * K + ks * kLyKs) + 2 * c;
-              u = __ldg(src);
-              w = __ldg(src + 1);
+          for (int i = 0; i < 4; ++i) {
+            const int r = pw * 32 + 8 * i + rl;
+            const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(x) +
+                                                                 (row0 + r) * K + ks * kLyKs);
+#pragma unroll
+            for (int jj = 0; jj < 2; ++jj) {  // chunk q + 4 jj: 8 fp32 values
+              float4 u = make_float4(0.f, 0.f, 0.f, 0.f), w = u;
+              if (r < rows) {
+                u = __ldg(src + 2 * (q + 4 * jj));
+                w = __ldg(src + 2 * (q + 4 * jj) + 1);
+              }
+              const __half2 h0 = __floats2half2_rn(u.x, u.y), h1 = __floats2half2_rn(u.z, u.w);
+              const __half2 h2 = __floats2half2_rn(w.x, w.y), h3 = __floats2half2_rn(w.z, w.w);
+              xv[2 * i + jj] = make_uint4(*reinterpret_cast<const uint32_t *>(&h0),
+                                          *reinterpret_cast<const uint32_t *>(&h1),
+                                          *reinterpret_cast<const uint32_t *>(&h2),
+                                          *reinterpret_cast<const uint32_t *>(&h3));
             }
-            const __half2 h0 = __floats2half2_rn(u.x, u.y), h1 = __floats2half2_rn(u.z, u.w);
-            const __half2 h2 = __floats2half2_rn(w.x, w.y), h3 = __floats2half2_rn(w.z, w.w);
-            xv[j] = make_uint4(*reinterpret_cast<const uint32_t *>(&h0), *reinterpret_cast<const uint32_t *>(&h1),
-                               *reinterpret_cast<const uint32_t *>(&h2), *reinterpret_cast<const uint32_t *>(&h3));
           }
         } else {
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {  // 128 rows x 4 pieces of 16 uint8
-            const int k = ct + kLyProdThreads * j, r = k >> 2, c = k & 3;
+          for (int i = 0; i < 4; ++i) {  // 16 uint8 values (piece q) -> chunks 2q, 2q + 1
+            const int r = pw * 32 + 8 * i + rl;
             uint4 v = make_uint4(0u, 0u, 0u, 0u);
             if (r < rows)
-              v = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint8_t *>(x) +
-                                                        (row0 + r) * K + ks * kLyKs) + c);
-            u8x16_to_f16(v, xv[2 * j], xv[2 * j + 1]);
+              v = __ldg(reinterpret_cast<const uint4 *>(static_cast<const uint8_t *>(x) + (row0 + r) * K +
+                                                        ks * kLyKs) + q);
+            u8x16_to_f16(v, xv[2 * i], xv[2 * i + 1]);
           }
         }
-        if (!warp_wait(smem_u32(&B.empty[st]), ((g / kLyStages) & 1u) ^ 1u, abort, wait_ns)) {
+        if (!warp_wait(smem_u32(&B.empty[st]), ph, abort, wait_ns)) {
           ok = false;
           break;
         }
-        if (XT == 0) {
+        if (lead) {
+          const uint32_t bar = smem_u32(&B.tfull[grp][st]);
+          mbar_arrive_tx(bar, wbytes);
+          bulk_g2s(sbase + st * stage_b + kLyXSlice, wt + (size_t)ks * wbytes, wbytes, bar);
+        }
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int k = ct + kLyProdThreads * j, r = k >> 2, c = k & 3;
-            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, 2 * c, 8)) = xv[2 * j];
-            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, 2 * c + 1, 8)) = xv[2 * j + 1];
-          }
-        } else {
+        for (int i = 0; i < 4; ++i) {
+          const int r = pw * 32 + 8 * i + rl;
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const int k = ct + kLyProdThreads * j, r = k >> 3, c = k & 7;
-            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, c, 8)) = xv[j];
+          for (int jj = 0; jj < 2; ++jj) {
+            const int c = XT == 1 ? q + 4 * jj : 2 * q + jj;
+            *reinterpret_cast<uint4 *>(sx + nr_tc_kmajor_off(r, c, 8)) = xv[2 * i + jj];
           }
         }
-        const uint4 *ws = wt + (size_t)ks * Nt * 8;  // the W slice, already in operand order
-        for (int i = ct; i < Nt * 8; i += kLyProdThreads)
-          reinterpret_cast<uint4 *>(sw)[i] = __ldg(ws + i);
         fence_async_smem();
-        mbar_arrive(smem_u32(&B.full[st]));
+        mbar_arrive(smem_u32(&B.xfull[st]));
       }
-      if (!ok) break;
+    }
+    // the bulk copies it issued land before the CTA ends, even if a role
+    // gave up: the latest phase of each of its barriers (XT 2: slices
+    // g - 3 .. g - 1, all group 0's; else its slices among g - 6 .. g - 1)
+    if (lead) {
+      if (XT == 2) {
+        if (grp == 0)
+          for (uint32_t i = g > (uint32_t)kLyStages ? g - kLyStages : 0u; i < g; ++i)
+            mbar_wait_bounded(smem_u32(&B.tfull[0][i % kLyStages]), (i / kLyStages) & 1u);
+      } else {
+        for (uint32_t i = g > 2u * kLyStages ? g - 2u * kLyStages : 0u; i < g; ++i)
+          if ((i & 1u) == (uint32_t)grp)
+            mbar_wait_bounded(smem_u32(&B.tfull[grp][i % kLyStages]), (i / (2 * kLyStages)) & 1u);
+      }
     }
   }
   tc_fence_before();
@@ -983,7 +1044,8 @@ static int enc_max_hidden(const nr_index *ix) {
 
 size_t nr_encode_scratch_bytes(const nr_index *ix, int64_t n) {
   if (ix->n_ly == 0 || n <= 0) return 0;
-  const int64_t rows = n < kEncRowBlock ? n : kEncRowBlock;
+  // whole 128-row tiles: the bulk copies of a ragged last tile stay in the buffer
+  const int64_t rows = ((n < kEncRowBlock ? n : kEncRowBlock) + kRows - 1) / kRows * kRows;
   return ((size_t)rows * enc_max_hidden(ix) * 2 + 255) / 256 * 256 * 2;
 }
 

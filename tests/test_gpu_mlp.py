@@ -136,3 +136,30 @@ def test_gpu_build_same_bytes_and_save_extract(built, torch, tmp_path):
     assert np.allclose(tau, np.sort(logits, axis=0)[(base.shape[0] - 1) // 2], atol=1e-3)
     ix.close()
     ix2.close()
+
+
+def test_layer_kernel_wait_expiry_is_flagged(built, torch):
+    """The per-layer tensor-core encoder (D and every hidden width multiples
+    of 64) under wait_limit_us < 0: every hand-off wait not complete when
+    first tested gives up, the kernel waits for its bulk copies and MMAs in
+    flight, frees its tensor memory and sets the device flag
+    (NR_ERR_DEVICE_CHECK); the next encode on the same context is right."""
+    from paper_2608_15438_gb300 import neuroute as nr
+
+    ix, cfg = built["ix"], built["cfg"]
+    if cfg.D % 64 or cfg.H % 64 or any(w % 64 for w in cfg.mid_w[: cfg.n_mid]):
+        pytest.skip("shape of the CUDA-core encoder")
+    q = torch.from_numpy(built["q"]).cuda()
+    ix.set_params(wait_limit_us=-1)
+    try:
+        ix.encode(q)
+        torch.cuda.synchronize()
+        with pytest.raises(nr.NRError) as e:
+            ix.last_stats()
+        assert e.value.status == -6  # NR_ERR_DEVICE_CHECK
+    finally:
+        ix.set_params()
+    ix.last_stats()
+    lg = ix.encode(q).cpu().numpy()
+    ref = built["orc"].encode(built["q"])
+    assert np.all(np.abs(lg - ref).max(1) <= 1e-2 * np.abs(ref).max(1))
