@@ -29,9 +29,11 @@
 // tensor-core kernel (encode_layer_kernel). What neither takes (shapes
 // outside their limits, input rows not 16-byte aligned) runs on the
 // CUDA-core kernels at the end of the file.
+#include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+#include <string.h>
 
 #include "nr_internal.cuh"
 
@@ -593,9 +595,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // (bounded) for the bulk copies it issued.
 constexpr int kLyKs = 64;        // K elements a slice
 constexpr int kLyStages = 3;
+constexpr int kLyRawMax = 4;     // raw fp32 stages (first layer), at most
+constexpr uint32_t kLyRawStage = (uint32_t)kRows * kLyKs * 4u;  // 32 KB: two 16 KB boxes
 constexpr int kLyEpiWarps = 4, kLyProdWarps = 4;  // a producer group
 constexpr int kLyWarpEpi = 1, kLyWarpProd = kLyWarpEpi + kLyEpiWarps;
-constexpr int kLyThreads = 32 * (kLyWarpProd + 2 * kLyProdWarps);  // 416
+constexpr int kLyWarpTma = kLyWarpProd + 2 * kLyProdWarps;
+constexpr int kLyThreads = 32 * (kLyWarpTma + 1);  // 448
 constexpr int kLyProdThreads = 32 * kLyProdWarps, kLyEpiThreads = 32 * kLyEpiWarps;
 constexpr uint32_t kLyXSlice = (uint32_t)kRows * kLyKs * 2u;    // 16 KB of fp16
 
@@ -603,6 +608,7 @@ struct LyBars {
   uint64_t xfull[kLyStages];  // x stored by the producer threads (first layer)
   uint64_t tfull[2][kLyStages];  // a producer group's bulk copies into the stage landed
   uint64_t empty[kLyStages];
+  uint64_t rawfull[kLyRawMax], rawempty[kLyRawMax];  // fp32 rows by tensor copy (first layer)
   uint64_t accfull[2], accempty[2];
   uint64_t drain;
   uint32_t tmem_slot;
@@ -610,8 +616,11 @@ struct LyBars {
 };
 
 __host__ __device__ inline uint32_t ly_stage_bytes(int Nt) { return kLyXSlice + (uint32_t)Nt * kLyKs * 2u; }
-__host__ __device__ inline uint32_t ly_smem_bytes(int Nt) {
-  return kLyStages * ly_stage_bytes(Nt) + (uint32_t)sizeof(LyBars);
+// operand stages, the bars, then (fp32 first layer) nraw raw stages from the
+// next 1024-byte boundary (the 128-byte swizzle's alignment)
+__host__ __device__ inline uint32_t ly_smem_bytes(int Nt, int nraw) {
+  return kLyStages * ly_stage_bytes(Nt) + (uint32_t)sizeof(LyBars) +
+         (nraw > 0 ? 1024u + (uint32_t)nraw * kLyRawStage : 0u);
 }
 // TMEM columns of the two accumulators: a power of two of at least 32
 __host__ __device__ inline uint32_t ly_tmem_cols(int Nt) {
@@ -623,6 +632,14 @@ __host__ __device__ inline uint32_t ly_tmem_cols(int Nt) {
 __device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(bar), "r"(bytes)
                : "memory");
+}
+// 2D tensor copy global -> this CTA's shared memory (box of the tensor map at
+// element coordinates (c0, c1)), completing on `bar` by bytes
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *tm, int c0, int c1, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];\n" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
 }
 // bulk copy global -> this CTA's shared memory, completing on `bar` by bytes
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
@@ -639,10 +656,15 @@ template <int XT, int YF>
 __global__ void __launch_bounds__(kLyThreads, 1)
     encode_layer_kernel(const void *__restrict__ x, int K, int N, int Nt, int Npad, float s,
                         const __half *__restrict__ Wp, const float *__restrict__ bias, int64_t n,
-                        void *__restrict__ y, int *err, int64_t wait_ns) {
+                        void *__restrict__ y, int nraw, const __grid_constant__ CUtensorMap tmx,
+                        int *err, int64_t wait_ns) {
   extern __shared__ __align__(1024) unsigned char smem[];
   const uint32_t stage_b = ly_stage_bytes(Nt);
   LyBars &B = *reinterpret_cast<LyBars *>(smem + kLyStages * stage_b);
+  // raw stages (XT 1): nraw x 32 KB from the first 1024-byte boundary after the bars
+  const uint32_t raw_s =
+      (smem_u32(smem) + kLyStages * stage_b + (uint32_t)sizeof(LyBars) + 1023u) & ~1023u;
+  const unsigned char *raw = smem + (raw_s - smem_u32(smem));
   volatile int *abort = &B.abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nks = K / kLyKs;                       // slices an item
@@ -663,6 +685,10 @@ __global__ void __launch_bounds__(kLyThreads, 1)
       mbar_init(smem_u32(&B.tfull[1][i]), 1);
       mbar_init(smem_u32(&B.empty[i]), 1);
     }
+    for (int i = 0; i < kLyRawMax; ++i) {
+      mbar_init(smem_u32(&B.rawfull[i]), 1);
+      mbar_init(smem_u32(&B.rawempty[i]), kLyProdThreads);
+    }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&B.accfull[i]), 1);
       mbar_init(smem_u32(&B.accempty[i]), kLyEpiThreads);
@@ -676,7 +702,34 @@ __global__ void __launch_bounds__(kLyThreads, 1)
   tc_fence_after();
   const uint32_t tmem = B.tmem_slot;
 
-  if (warp == 0) {
+  if (warp == kLyWarpTma) {
+    // fp32 first layer: lane 0 fetches each slice's 128 rows x 64 values by
+    // two tensor copies (boxes of 32 values x 128 rows, 128-byte swizzle;
+    // rows past n read as zeros) into raw stage g % nraw
+    if (XT == 1 && lane == 0) {
+      uint32_t g = 0;
+      bool ok = true;
+      for (int64_t item = blockIdx.x; item < items && ok; item += gridDim.x) {
+        const int row0 = (int)(item / nct * kRows);
+        for (int ks = 0; ks < nks; ++ks, ++g) {
+          const uint32_t rs = g % (uint32_t)nraw;
+          if (!wait_or_abort(smem_u32(&B.rawempty[rs]), ((g / (uint32_t)nraw) & 1u) ^ 1u, abort, wait_ns)) {
+            ok = false;
+            break;
+          }
+          const uint32_t bar = smem_u32(&B.rawfull[rs]), dst = raw_s + rs * kLyRawStage;
+          mbar_arrive_tx(bar, kLyRawStage);
+          tma_load_2d(dst, &tmx, ks * kLyKs, row0, bar);
+          tma_load_2d(dst + kLyRawStage / 2, &tmx, ks * kLyKs + kLyKs / 2, row0, bar);
+        }
+      }
+      // the copies issued (the last on each stage are among the last nraw) land
+      // before the CTA ends, even if a role gave up
+      for (uint32_t i = g > (uint32_t)nraw ? g - nraw : 0u; i < g; ++i)
+        mbar_wait_bounded(smem_u32(&B.rawfull[i % nraw]), (i / nraw) & 1u);
+    }
+    __syncwarp();
+  } else if (warp == 0) {
     if (lane == 0) {  // the MMA thread
       const uint32_t idesc = mma_idesc(kRows, Nt);
       uint32_t g = 0, it = 0;  // slices and items of this CTA so far
@@ -774,7 +827,7 @@ __global__ void __launch_bounds__(kLyThreads, 1)
       tc_fence_before();
       mbar_arrive(smem_u32(&B.accempty[a]));
     }
-  } else {  // producers: x and W slices into the stage ring
+  } else if (warp < kLyWarpTma) {  // producers: x and W slices into the stage ring
     const int grp = (warp - kLyWarpProd) / kLyProdWarps;  // XT 0 / 1: two groups
     const int ct = tid - kLyWarpProd * 32 - grp * kLyProdThreads;
     const bool lead = ct == 0;  // issues the bulk copies (of its group's slices)
@@ -811,18 +864,23 @@ __global__ void __launch_bounds__(kLyThreads, 1)
         const int pw = ct >> 5, rl = lane & 7, q = lane >> 3;
         uint4 xv[8];
         if (XT == 1) {
+          // from raw stage g % nraw: value column 8 c + 4 h of row r sits in
+          // box c / 4, 16-byte piece (2 (c % 4) + h) ^ (r % 8) of the row's
+          // 128 bytes (the swizzle; 8 lanes read 8 rows, different banks)
+          const uint32_t rs = g % (uint32_t)nraw;
+          if (!warp_wait(smem_u32(&B.rawfull[rs]), (g / (uint32_t)nraw) & 1u, abort, wait_ns)) {
+            ok = false;
+            break;
+          }
+          const unsigned char *rst = raw + rs * kLyRawStage;
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             const int r = pw * 32 + 8 * i + rl;
-            const float4 *src = reinterpret_cast<const float4 *>(static_cast<const float *>(x) +
-                                                                 (row0 + r) * K + ks * kLyKs);
 #pragma unroll
-            for (int jj = 0; jj < 2; ++jj) {  // chunk q + 4 jj: 8 fp32 values
-              float4 u = make_float4(0.f, 0.f, 0.f, 0.f), w = u;
-              if (r < rows) {
-                u = __ldg(src + 2 * (q + 4 * jj));
-                w = __ldg(src + 2 * (q + 4 * jj) + 1);
-              }
+            for (int jj = 0; jj < 2; ++jj) {  // chunk q + 4 jj: box jj, pieces 2q, 2q + 1
+              const unsigned char *row = rst + jj * (kLyRawStage / 2) + r * 128;
+              const float4 u = *reinterpret_cast<const float4 *>(row + (((2 * q) ^ (r & 7)) << 4));
+              const float4 w = *reinterpret_cast<const float4 *>(row + (((2 * q + 1) ^ (r & 7)) << 4));
               const __half2 h0 = __floats2half2_rn(u.x, u.y), h1 = __floats2half2_rn(u.z, u.w);
               const __half2 h2 = __floats2half2_rn(w.x, w.y), h3 = __floats2half2_rn(w.z, w.w);
               xv[2 * i + jj] = make_uint4(*reinterpret_cast<const uint32_t *>(&h0),
@@ -831,6 +889,7 @@ __global__ void __launch_bounds__(kLyThreads, 1)
                                           *reinterpret_cast<const uint32_t *>(&h3));
             }
           }
+          mbar_arrive(smem_u32(&B.rawempty[rs]));
         } else {
 #pragma unroll
           for (int i = 0; i < 4; ++i) {  // 16 uint8 values (piece q) -> chunks 2q, 2q + 1
@@ -1054,7 +1113,25 @@ static cudaError_t launch_layer(nr_index *ix, const void *x, int K, int N, int l
                                 const float *bias, int64_t n, void *y, int64_t wait_ns,
                                 cudaStream_t s) {
   const int nt = ix->ly_nt[l], Np = (N + 15) / 16 * 16;
-  uint32_t smem = ly_smem_bytes(nt);
+  // fp32 first layer: raw stages for the tensor copies, as many as fit (<= 4)
+  int nraw = 0;
+  CUtensorMap tm;
+  memset(&tm, 0, sizeof(tm));
+  if (XT == 1) {
+    nraw = kLyRawMax;
+    while (nraw > 1 && ly_smem_bytes(nt, nraw) > (uint32_t)ix->smem_optin) --nraw;
+    if (ly_smem_bytes(nt, nraw) > (uint32_t)ix->smem_optin) return cudaErrorInvalidConfiguration;
+    // x [n rows x K] fp32: boxes of 32 values x 128 rows, 128-byte swizzle
+    const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)n};
+    const cuuint64_t strides[1] = {(cuuint64_t)K * 4u};
+    const cuuint32_t box[2] = {(cuuint32_t)(kLyKs / 2), (cuuint32_t)kRows}, es[2] = {1u, 1u};
+    if (cuTensorMapEncodeTiled(&tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void *>(x), dims,
+                               strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  uint32_t smem = ly_smem_bytes(nt, nraw);
   // accumulators wider than half of TMEM: one CTA an SM (a second would
   // stall in its TMEM allocation until the first ends)
   if (ly_tmem_cols(nt) > 256 && smem <= (uint32_t)ix->smem_optin / 2)
@@ -1066,7 +1143,7 @@ static cudaError_t launch_layer(nr_index *ix, const void *x, int K, int N, int l
   const int64_t grid = items < ix->num_sms ? items : ix->num_sms;
   kern<<<(unsigned)grid, kLyThreads, smem, s>>>(x, K, N, nt, Np, sc,
                                                 static_cast<const __half *>(ix->Wl) + ix->ly_off[l],
-                                                bias, n, y, ix->d_err, wait_ns);
+                                                bias, n, y, nraw, tm, ix->d_err, wait_ns);
   ix->launches += 1;
   return cudaGetLastError();
 }

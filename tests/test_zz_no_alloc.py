@@ -97,3 +97,35 @@ def test_static_scratch_search_global_sort_slabs(tmp_path):
         assert torch.equal(ids, ref_ids) and torch.equal(d, ref_d)
         assert torch.equal(ix.query_stats(dq.shape[0]), ref_st)
     ix.close()
+
+
+def test_static_scratch_search_multi_layer_encoder(tmp_path):
+    """An index whose encoder has hidden layers after the first: the layer
+    activations of its tensor-core encoder also live in the fixed array, and
+    the results are nr_search's (fp32 distances by the same fmaf chain)."""
+    torch = need_cuda()
+    from paper_2608_15438_gb300 import neuroute as nr
+    from paper_2608_15438_gb300.builder import build_index, config
+    from test_gpu_mlp import mlp_case
+
+    base, q, weights, widths, b = mlp_case(512, (256, 128, 64), 12, 12_000)
+    cfg = config("f32", base.shape[1], widths[0], b, 4, 16, mid=widths[1:])
+    path = str(tmp_path / "mlp.nrix")
+    build_index(cfg, base, weights, path)
+    ix = nr.Index(path, 0)
+    dq = torch.from_numpy(q).cuda()
+    k, P, C = 10, 32, 64
+    ref_ids, ref_d = ix.search(dq, k, P, C)
+    torch.cuda.synchronize()
+    L = nr.lib()
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    for _ in range(2):
+        ids = torch.full((dq.shape[0], k), -7, dtype=torch.int64, device="cuda")
+        d = torch.full((dq.shape[0], k), -7.0, dtype=torch.float32, device="cuda")
+        st = L.nr_search_static(ix.h, ctypes.c_void_p(dq.data_ptr()), dq.shape[0], k, P, C,
+                                ctypes.c_void_p(ids.data_ptr()), ctypes.c_void_p(d.data_ptr()),
+                                stream)
+        assert st == nr.NR_OK
+        torch.cuda.synchronize()
+        assert torch.equal(ids, ref_ids) and torch.equal(d, ref_d)
+    ix.close()
