@@ -595,6 +595,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // (bounded) for the bulk copies it issued.
 constexpr int kLyKs = 64;        // K elements a slice
 constexpr int kLyStages = 3;
+// slices g and g + kLyPeriod use the same stage and the same producer group
+constexpr int kLyPeriod = kLyStages % 2 == 0 ? kLyStages : 2 * kLyStages;
 constexpr int kLyRawMax = 4;     // raw fp32 stages (first layer), at most
 constexpr uint32_t kLyRawStage = (uint32_t)kRows * kLyKs * 4u;  // 32 KB: two 16 KB boxes
 constexpr int kLyEpiWarps = 4, kLyProdWarps = 4;  // a producer group
@@ -745,9 +747,9 @@ __global__ void __launch_bounds__(kLyThreads, 1)
         for (int ks = 0; ks < nks; ++ks, ++g) {
           const uint32_t st = g % kLyStages, ph = (g / kLyStages) & 1u;
           // the copies of slice g: group g % 2 (XT 0 / 1: that group's phases
-          // on the stage are slices g, g + 6, ...), or group 0 (XT 2)
+          // on the stage are slices g, g + kLyPeriod, ...), or group 0 (XT 2)
           const uint32_t tb = XT == 2 ? smem_u32(&B.tfull[0][st]) : smem_u32(&B.tfull[g & 1u][st]);
-          const uint32_t tph = XT == 2 ? ph : (g / (2 * kLyStages)) & 1u;
+          const uint32_t tph = XT == 2 ? ph : (g / kLyPeriod) & 1u;
           if (!wait_or_abort(tb, tph, abort, wait_ns) ||
               (XT != 2 && !wait_or_abort(smem_u32(&B.xfull[st]), ph, abort, wait_ns))) {
             ok = false;
@@ -925,16 +927,17 @@ __global__ void __launch_bounds__(kLyThreads, 1)
     }
     // the bulk copies it issued land before the CTA ends, even if a role
     // gave up: the latest phase of each of its barriers (XT 2: slices
-    // g - 3 .. g - 1, all group 0's; else its slices among g - 6 .. g - 1)
+    // g - kLyStages .. g - 1, all group 0's; else its slices among
+    // g - kLyPeriod .. g - 1)
     if (lead) {
       if (XT == 2) {
         if (grp == 0)
           for (uint32_t i = g > (uint32_t)kLyStages ? g - kLyStages : 0u; i < g; ++i)
             mbar_wait_bounded(smem_u32(&B.tfull[0][i % kLyStages]), (i / kLyStages) & 1u);
       } else {
-        for (uint32_t i = g > 2u * kLyStages ? g - 2u * kLyStages : 0u; i < g; ++i)
+        for (uint32_t i = g > (uint32_t)kLyPeriod ? g - kLyPeriod : 0u; i < g; ++i)
           if ((i & 1u) == (uint32_t)grp)
-            mbar_wait_bounded(smem_u32(&B.tfull[grp][i % kLyStages]), (i / (2 * kLyStages)) & 1u);
+            mbar_wait_bounded(smem_u32(&B.tfull[grp][i % kLyStages]), (i / kLyPeriod) & 1u);
       }
     }
   }
