@@ -30,6 +30,7 @@
 // outside their limits, input rows not 16-byte aligned) runs on the
 // CUDA-core kernels at the end of the file.
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -1111,6 +1112,23 @@ size_t nr_encode_scratch_bytes(const nr_index *ix, int64_t n) {
   return ((size_t)rows * enc_max_hidden(ix) * 2 + 255) / 256 * 256 * 2;
 }
 
+// The driver's tensor-map encoder, looked up once through the runtime (so the
+// library needs no link-time dependency on the driver library).
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess) {
+      cudaGetLastError();
+      p = nullptr;
+    }
+    return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }();
+  return fn;
+}
+
 template <int XT, int YF>
 static cudaError_t launch_layer(nr_index *ix, const void *x, int K, int N, int l, float sc,
                                 const float *bias, int64_t n, void *y, int64_t wait_ns,
@@ -1128,10 +1146,11 @@ static cudaError_t launch_layer(nr_index *ix, const void *x, int K, int N, int l
     const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)n};
     const cuuint64_t strides[1] = {(cuuint64_t)K * 4u};
     const cuuint32_t box[2] = {(cuuint32_t)(kLyKs / 2), (cuuint32_t)kRows}, es[2] = {1u, 1u};
-    if (cuTensorMapEncodeTiled(&tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void *>(x), dims,
-                               strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    const PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
+    if (!encode) return cudaErrorNotSupported;
+    if (encode(&tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void *>(x), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
   uint32_t smem = ly_smem_bytes(nt, nraw);
