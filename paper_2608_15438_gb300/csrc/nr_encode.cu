@@ -589,11 +589,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // load), and hidden activations are written in the same order, as 128-row
 // tiles x 64-column slices of 16 KB: every slice of either operand is one
 // contiguous block, fetched by one bulk copy (cp.async.bulk, completing on
-// an mbarrier by its byte count). The first layer's input (uint8 or fp32
-// rows) goes through the producer warps' registers, converted to fp16
-// (uint8 exactly, fp32 rounded); the first producer thread fetches W.
-// Waits are bounded as in the kernel above; a CTA that gives up first waits
-// (bounded) for the bulk copies it issued.
+// an mbarrier by its byte count). The first layer's input is converted to
+// fp16 by two groups of four producer warps, which take alternate slices:
+// fp32 rows arrive by 2D tensor copies (cp.async.bulk.tensor, a warp of
+// their own, 128-byte swizzle) in a ring of raw stages that the producers
+// read from shared memory; uint8 rows go through the producers' registers.
+// Each group's first thread fetches W for its slices. Waits are bounded as in
+// the kernel above; a CTA that gives up first waits (bounded) for the bulk
+// and tensor copies it issued.
 constexpr int kLyKs = 64;        // K elements a slice
 constexpr int kLyStages = 3;
 // slices g and g + kLyPeriod use the same stage and the same producer group
