@@ -163,3 +163,21 @@ def test_layer_kernel_wait_expiry_is_flagged(built, torch):
     lg = ix.encode(q).cpu().numpy()
     ref = built["orc"].encode(built["q"])
     assert np.all(np.abs(lg - ref).max(1) <= 1e-2 * np.abs(ref).max(1))
+
+
+def test_encoder_across_row_blocks(built, torch):
+    """A batch longer than the layer-by-layer encoder's row block (2^18 rows,
+    the unit its activation scratch holds): rows on both sides of the block
+    boundary and in the ragged last tile agree with the oracle's forward."""
+    cfg = built["cfg"]
+    if cfg.D % 64 or cfg.H % 64 or any(w % 64 for w in cfg.mid_w[: cfg.n_mid]):
+        pytest.skip("shape of the CUDA-core encoder")
+    n = (1 << 18) + 1000 + 37
+    rng = np.random.default_rng(5)
+    q = built["q"]
+    x = q[rng.integers(0, len(q), n)] + 0.05 * rng.normal(size=(n, q.shape[1])).astype(np.float32)
+    lg = built["ix"].encode(torch.from_numpy(x).cuda()).cpu().numpy()
+    pick = np.r_[0:64, (1 << 18) - 64:(1 << 18) + 64, n - 101:n]
+    ref = built["orc"].encode(x[pick])
+    err = np.max(np.abs(lg[pick] - ref), axis=1)
+    assert np.all(err <= 1e-2 * np.max(np.abs(ref), axis=1))
