@@ -39,18 +39,27 @@ def mlp_case(D=48, widths=(64, 32, 24, 16), b=12, n=20_000, seed=1):
 # (D, hidden widths, b, rows): one hidden-layer chain per case; D = 272, 288,
 # 512 and 1536 fp32 rows (1,088 to 6,144 bytes) take the long-row refinement
 # with 4, 8 and 16 chunks a piece
-CASES = [(48, (64, 32, 24, 16), 12, 20_000), (272, (128, 64), 12, 12_000), (288, (128, 64), 12, 12_000),
-         (512, (256, 128, 64), 12, 12_000), (1536, (512, 256, 128, 64), 16, 6_000)]
+# The tensor-core layer kernel takes D = 512, 1536 and 128 (every width a
+# multiple of 64); the 704-wide layer has 176-column tiles (a 16-column
+# remainder in the epilogue, accumulators wider than half of TMEM), and the
+# uint8 case feeds its first layer through the producers' registers.
+CASES = [("f32", 48, (64, 32, 24, 16), 12, 20_000), ("f32", 272, (128, 64), 12, 12_000),
+         ("f32", 288, (128, 64), 12, 12_000), ("f32", 512, (256, 128, 64), 12, 12_000),
+         ("f32", 1536, (512, 256, 128, 64), 16, 6_000), ("f32", 128, (704, 192), 20, 8_000),
+         ("u8", 128, (256, 128), 16, 12_000)]
 
 
-@pytest.fixture(scope="module", params=CASES, ids=[f"D{c[0]}" for c in CASES])
+@pytest.fixture(scope="module", params=CASES, ids=[f"{c[0]}D{c[1]}" for c in CASES])
 def built(torch, tmp_path_factory, request):
     from paper_2608_15438_gb300 import neuroute as nr
     from paper_2608_15438_gb300.builder import build_index, config
 
-    D, widths, b, n = request.param
+    dt, D, widths, b, n = request.param
     base, q, weights, widths, b = mlp_case(D, widths, b, n)
-    cfg = config("f32", base.shape[1], widths[0], b, 4, 16, mid=widths[1:])
+    if dt == "u8":  # the same points as bytes
+        base = np.clip(np.rint(base * 400 + 128), 0, 255).astype(np.uint8)
+        q = np.clip(np.rint(q * 400 + 128), 0, 255).astype(np.uint8)
+    cfg = config(dt, base.shape[1], widths[0], b, 4, 16, mid=widths[1:])
     path = str(tmp_path_factory.mktemp("mlp") / "m.nrix")
     build_index(cfg, base, weights, path)
     return {"ix": nr.Index(path, 0), "orc": oracle.Index(path), "base": base, "q": q,
@@ -175,7 +184,11 @@ def test_encoder_across_row_blocks(built, torch):
     n = (1 << 18) + 1000 + 37
     rng = np.random.default_rng(5)
     q = built["q"]
-    x = q[rng.integers(0, len(q), n)] + 0.05 * rng.normal(size=(n, q.shape[1])).astype(np.float32)
+    if q.dtype == np.uint8:
+        x = np.clip(q[rng.integers(0, len(q), n)].astype(np.int16) + rng.integers(-3, 4, (n, q.shape[1])),
+                    0, 255).astype(np.uint8)
+    else:
+        x = q[rng.integers(0, len(q), n)] + 0.05 * rng.normal(size=(n, q.shape[1])).astype(np.float32)
     lg = built["ix"].encode(torch.from_numpy(x).cuda()).cpu().numpy()
     pick = np.r_[0:64, (1 << 18) - 64:(1 << 18) + 64, n - 101:n]
     ref = built["orc"].encode(x[pick])
