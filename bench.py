@@ -419,11 +419,24 @@ def cpu_baseline(w, path, queries, k, P, C, kw, seconds, truth=None):
     t = time.perf_counter()
     ids, _, _ = orc.search(queries[:n2], k, P, C, p, nthreads=cores)
     dt2 = time.perf_counter() - t
+    v1, n1, dt1 = one_thread_rate(orc, queries, n2, dt2, cores, k, P, C, p, seconds)
     res = {"value": n2 / dt2, "unit": "queries/s", "cores": cores, "kind": "oracle",
+           "value_1_thread": v1,
            "sample": f"first {n2} of {len(queries)} queries of {w.name}, P={P} C={C} t_low={t_low}, "
-                     f"{cores} threads, {dt2:.1f} s"}
+                     f"{cores} threads, {dt2:.1f} s; one thread: first {n1}, {dt1:.1f} s"}
     orc.close()
     return res, ids
+
+
+def one_thread_rate(orc, queries, n, dt, cores, k, P, C, p, seconds):
+    """The oracle's rate on one thread over a prefix of the timed sample sized
+    to about a quarter of `seconds` (from the all-core rate at perfect scaling)."""
+    per_q = dt * cores / max(n, 1)
+    n1 = int(min(n, max(2, 0.25 * seconds / max(per_q, 1e-9))))
+    t = time.perf_counter()
+    orc.search(queries[:n1], k, P, C, p, nthreads=1)
+    dt1 = max(time.perf_counter() - t, 1e-9)
+    return n1 / dt1, n1, dt1
 
 
 def calibrate_subindex(w, ix, queries, k, P, C, kw, seconds, path, row_budget):
@@ -466,11 +479,14 @@ def cpu_baseline_subindex(w, ix, queries, k, P, C, kw, seconds, row_budget=100_0
         for _ in range(reps):
             orc.search(queries[:n2], k, P, C, p, nthreads=cores)
         dt2 = time.perf_counter() - t
+        v1, n1, dt1 = one_thread_rate(orc, queries, n2, dt2 / reps, cores, k, P, C, p, seconds)
         orc.close()
     return {"value": n2 * reps / dt2, "unit": "queries/s", "cores": cores, "kind": "oracle",
+            "value_1_thread": v1,
             "sample": f"first {n2} of {len(queries)} queries of {w.name} (oracle encoder included), "
                       f"{reps} passes, P={P} C={C} t_low={t_low}, {cores} threads, {dt2:.1f} s, on "
-                      f"the {rows}-row sub-index of the buckets they probe"}
+                      f"the {rows}-row sub-index of the buckets they probe; one thread: first {n1}, "
+                      f"{dt1:.1f} s"}
 
 
 def run_reference(args, w, rank, world):
