@@ -873,6 +873,9 @@ def main():
     # the random-row read rate of this GPU over an array of the centroids' shape
     # (rows of 4b bytes rounded up to 16, the granule of the measurement)
     gather_gbs = nr.measure_gather(local, max(1 << 20, ix.n_clusters), (w.bits * 4 + 15) // 16 * 16)
+    # the sequential-read rate of this GPU (8 GiB, L2 flushed): the scan's
+    # bytes are reads of long runs
+    read_gbs = nr.measure_read(local)
     out = {
         "metric": METRIC,
         "value": value, "unit": "queries/s", "n_gpus": world, "steps": args.steps,
@@ -897,6 +900,9 @@ def main():
                      "peak_source": f"{peak_src} hbm_gbs (a device copy's read + write bytes per "
                                     "second); the scan reads, so it can exceed it",
                      "frac_of_nominal": achieved / NOMINAL_HBM_GBS,
+                     "stream_read_gbs": read_gbs, "frac_of_stream_read": achieved / read_gbs,
+                     "stream_read_source": "measured in this run: an 8 GiB sequential read, L2 "
+                                           "flushed, best of 5 (nr_measure_read)",
                      "traffic": traffic, "traffic_source": traffic_src,
                      "algorithmic_bytes_per_launch": cand * row_bytes / n_ref,
                      "avg_launch_ms": refine_avg_ms, "launches_per_step": n_ref},

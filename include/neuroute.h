@@ -401,6 +401,17 @@ nr_status nr_last_timing(nr_index *ix, float *ms);
 nr_status nr_measure_gather(int device, int64_t rows, int row_bytes, int64_t n, int reps,
                             double *h_gbs);
 
+/* Measurement utility, not part of the search: the rate at which the GPU
+ * `device` reads a long contiguous array (`bytes`, a multiple of 16, at least
+ * 1 MiB), sequentially, with no writes but one word a thread, L2 evicted
+ * before each of reps runs; *h_gbs = bytes read per second of the best run,
+ * in GB/s. It bounds a kernel whose bytes are reads of long runs, as the
+ * refinement's are (Sec. 3.5: the candidate rows), more tightly than the
+ * copy bandwidth, whose bytes are half writes. Allocates bytes + 512 MiB and
+ * a few MB of device memory for the call and frees it; synchronous.
+ * Errors: NR_ERR_INVALID_ARG, NR_ERR_OOM, NR_ERR_CUDA. */
+nr_status nr_measure_read(int device, int64_t bytes, int reps, double *h_gbs);
+
 /* Number of kernels the library launched since load (all entry points). */
 int64_t nr_kernel_launches(const nr_index *ix);
 

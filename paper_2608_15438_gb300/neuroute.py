@@ -26,7 +26,7 @@ EXPORTS = ["nr_status_string", "nr_params_default", "nr_index_load", "nr_index_f
            "nr_index_save", "nr_index_extract", "nr_index_thresholds", "nr_index_locate",
            "nr_centroid_dists", "nr_build_begin", "nr_build_encode", "nr_build_set_logits",
            "nr_build_finish", "nr_build_place", "nr_build_end", "nr_build_free",
-           "nr_measure_gather", "nr_bucket_scores", "nr_calib_observe", "nr_calib_fit_s_max",
+           "nr_measure_gather", "nr_measure_read", "nr_bucket_scores", "nr_calib_observe", "nr_calib_fit_s_max",
            "nr_calib_fit_gate", "nr_calibrate"]
 
 
@@ -80,6 +80,7 @@ def lib():
         L.nr_query_stats.argtypes = [vp, vp, i64, vp]
         L.nr_last_stats.argtypes = [vp, ctypes.POINTER(Stats)]
         L.nr_measure_gather.argtypes = [i32, i64, i32, i64, i32, ctypes.POINTER(ctypes.c_double)]
+        L.nr_measure_read.argtypes = [i32, i64, i32, ctypes.POINTER(ctypes.c_double)]
         dp, fp = ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_float)
         L.nr_bucket_scores.argtypes = [vp, vp, i32, vp, i64, i32, vp, vp]
         L.nr_calib_observe.argtypes = [vp, vp, vp, i64, i32, vp, vp, vp, vp]
@@ -134,6 +135,13 @@ def params(**kw) -> Params:
             raise KeyError(k)
         setattr(p, k, v)
     return p
+
+
+def measure_read(device, nbytes=8 << 30, reps=5) -> float:
+    """GB/s at which the GPU reads a long array sequentially (nr_measure_read)."""
+    v = ctypes.c_double()
+    _check("nr_measure_read", lib().nr_measure_read(int(device), int(nbytes), int(reps), ctypes.byref(v)))
+    return v.value
 
 
 def measure_gather(device, rows, row_bytes, n=20_000_000, reps=5) -> float:
