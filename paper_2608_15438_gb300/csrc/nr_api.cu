@@ -20,7 +20,7 @@ constexpr int kMaxProbe = 4096;
 constexpr int kMaxClusterBudget = 4096;
 constexpr int kMaxSelect = 65536;  // probe_budget * K_max (beyond 2,048: sorted in a global slab)
 constexpr int kMaxTopK = 256;
-constexpr size_t kChunkBudget = (size_t)4 << 30;  // workspace bytes per query chunk
+constexpr size_t kChunkBudget = (size_t)8 << 30;  // workspace bytes per query chunk
 
 uint32_t rd32(const unsigned char *h, int o) {
   uint32_t v;
