@@ -194,3 +194,22 @@ def test_encoder_across_row_blocks(built, torch):
     ref = built["orc"].encode(x[pick])
     err = np.max(np.abs(lg[pick] - ref), axis=1)
     assert np.all(err <= 1e-2 * np.max(np.abs(ref), axis=1))
+
+
+def test_encoder_misaligned_input(built, torch):
+    """Input rows that do not start on a 16-byte boundary take the CUDA-core
+    encoder (the tensor-core kernels copy 16-byte pieces); the logits agree
+    with the oracle's within the same tolerance."""
+    q = built["q"]
+    n, D = q.shape
+    esz = q.dtype.itemsize
+    tdt = torch.uint8 if q.dtype == np.uint8 else torch.float32
+    buf = torch.zeros(n * D + 16 // esz, dtype=tdt, device="cuda")
+    off = 4 // esz if esz < 4 else 1           # 4 bytes past a 16-byte boundary
+    x = buf[off:off + n * D].view(n, D)
+    x.copy_(torch.from_numpy(q).cuda())
+    assert x.data_ptr() % 16 != 0
+    lg = built["ix"].encode(x).cpu().numpy()
+    ref = built["orc"].encode(q)
+    err = np.max(np.abs(lg - ref), axis=1)
+    assert np.all(err <= 1e-2 * np.max(np.abs(ref), axis=1))
