@@ -263,6 +263,97 @@ __device__ __forceinline__ void u8x16_to_f16(const uint4 v, uint4 &lo, uint4 &hi
   hi = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
+// The converter warps' role in the tensor-core encoders: each X tile of 128
+// rows -> fp16 operand in the K-major core-matrix layout of buffer tile % nxb
+// (xempty: the buffer is free; xfull: it is written, kConvThreads arrivals).
+// ct: the thread's index among the converter threads.
+template <int DT>
+__device__ __forceinline__ void tc_convert_tiles(const void *__restrict__ x, int D, int kx, int nxb,
+                                                 int64_t nq, int64_t ntiles, uint32_t x_bytes,
+                                                 unsigned char *smem_x, uint64_t *xfull,
+                                                 uint64_t *xempty, volatile int *abort,
+                                                 int64_t wait_ns, int ct) {
+  // eight consecutive threads cover eight rows of one 16-byte K chunk, so a
+  // warp's stores fill whole 128-byte core matrices
+  // item j of this thread: row rr of the tile and piece pc of the row (16 source
+  // bytes = 2 K chunks for uint8, one K chunk of 8 floats for fp32), the same
+  // for every tile; k / per by a 16-bit reciprocal, exact for k < 256, per <= 16
+  const int per = DT == 0 ? D / 16 : kx;  // pieces per row = items per thread (<= 8, <= 16)
+  const uint32_t inv = (65536u + (uint32_t)per - 1u) / (uint32_t)per;
+  auto item = [&](int j, int &rr, int &pc) {
+    const uint32_t k = (uint32_t)(ct >> 3) + 16u * (uint32_t)j, q = (k * inv) >> 16;
+    pc = (int)(k - q * (uint32_t)per);
+    rr = (int)q * 8 + (ct & 7);
+  };
+  uint32_t it = 0;
+  for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
+    const int xb = nxb == 2 ? (int)(it & 1) : 0;
+    const uint32_t xpar = ((nxb == 2 ? it >> 1 : it) & 1u) ^ 1u;  // previous use of the buffer
+    unsigned char *sX = smem_x + (size_t)xb * x_bytes;
+    const int64_t row0 = tile * kRows;
+    const int rows = nq - row0 < kRows ? (int)(nq - row0) : kRows;  // rows of this tile
+    bool ok = true;
+    if (DT == 0) {
+      const uint8_t *xs = static_cast<const uint8_t *>(x) + row0 * D;
+      uint4 v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        int rr, pc;
+        item(j, rr, pc);
+        v[j] = make_uint4(0u, 0u, 0u, 0u);
+        if (j < per && rr < rows) v[j] = __ldg(reinterpret_cast<const uint4 *>(xs + rr * D + pc * 16));
+      }
+      ok = warp_wait(smem_u32(&xempty[xb]), xpar, abort, wait_ns);
+      if (ok) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (j >= per) break;
+          int rr, pc;
+          item(j, rr, pc);
+          uint4 lo, hi;
+          u8x16_to_f16(v[j], lo, hi);
+          *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc, kx)) = lo;
+          *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc + 1, kx)) = hi;
+        }
+      }
+    } else {
+      const float *xs = static_cast<const float *>(x) + row0 * D;
+#pragma unroll
+      for (int j0 = 0; j0 < 16; j0 += 8) {
+        if (j0 >= per || !ok) break;
+        float4 u[8], w[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          int rr, pc;
+          item(j0 + j, rr, pc);
+          u[j] = w[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+          if (j0 + j < per && rr < rows) {
+            const float4 *s4 = reinterpret_cast<const float4 *>(xs + rr * D + pc * 8);
+            u[j] = __ldg(s4);
+            w[j] = __ldg(s4 + 1);
+          }
+        }
+        if (j0 == 0) ok = warp_wait(smem_u32(&xempty[xb]), xpar, abort, wait_ns);
+        if (!ok) break;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (j0 + j >= per) break;
+          int rr, pc;
+          item(j0 + j, rr, pc);
+          const __half2 h0 = __floats2half2_rn(u[j].x, u[j].y), h1 = __floats2half2_rn(u[j].z, u[j].w);
+          const __half2 h2 = __floats2half2_rn(w[j].x, w[j].y), h3 = __floats2half2_rn(w[j].z, w[j].w);
+          *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, pc, kx)) =
+              make_uint4(*reinterpret_cast<const uint32_t *>(&h0), *reinterpret_cast<const uint32_t *>(&h1),
+                         *reinterpret_cast<const uint32_t *>(&h2), *reinterpret_cast<const uint32_t *>(&h3));
+        }
+      }
+    }
+    if (!ok) break;
+    fence_async_smem();
+    mbar_arrive(smem_u32(&xfull[xb]));
+  }
+}
+
 // Persistent, warp-specialised: each CTA (one per SM) keeps W1 and W2 in
 // shared memory and takes 128-row tiles tile = blockIdx.x, + gridDim.x, ...:
 //   converter warps  X tile -> fp16 operand (nxb = 2 buffers, or 1 for wide shapes)
@@ -483,87 +574,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     if (ok && it > 0) ok = logits(it - 1, last_tile);
   } else {
-    // converters: X tile -> fp16 operand in the K-major core-matrix layout;
-    // eight consecutive threads cover eight rows of one 16-byte K chunk, so a
-    // warp's stores fill whole 128-byte core matrices
-    const int ct = tid - kWarpConv * 32;
-    // item j of this thread: row rr of the tile and piece pc of the row (16 source
-    // bytes = 2 K chunks for uint8, one K chunk of 8 floats for fp32), the same
-    // for every tile; k / per by a 16-bit reciprocal, exact for k < 256, per <= 16
-    const int per = DT == 0 ? D / 16 : kx;  // pieces per row = items per thread (<= 8, <= 16)
-    const uint32_t inv = (65536u + (uint32_t)per - 1u) / (uint32_t)per;
-    auto item = [&](int j, int &rr, int &pc) {
-      const uint32_t k = (uint32_t)(ct >> 3) + 16u * (uint32_t)j, q = (k * inv) >> 16;
-      pc = (int)(k - q * (uint32_t)per);
-      rr = (int)q * 8 + (ct & 7);
-    };
-    uint32_t it = 0;
-    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
-      const int xb = nxb == 2 ? (int)(it & 1) : 0;
-      const uint32_t xpar = ((nxb == 2 ? it >> 1 : it) & 1u) ^ 1u;  // previous use of the buffer
-      unsigned char *sX = smem + L.x + (size_t)xb * x_bytes;
-      const int64_t row0 = tile * kRows;
-      const int rows = nq - row0 < kRows ? (int)(nq - row0) : kRows;  // rows of this tile
-      bool ok = true;
-      if (DT == 0) {
-        const uint8_t *xs = static_cast<const uint8_t *>(x) + row0 * D;
-        uint4 v[8];
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          int rr, pc;
-          item(j, rr, pc);
-          v[j] = make_uint4(0u, 0u, 0u, 0u);
-          if (j < per && rr < rows) v[j] = __ldg(reinterpret_cast<const uint4 *>(xs + rr * D + pc * 16));
-        }
-        ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort, wait_ns);
-        if (ok) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (j >= per) break;
-            int rr, pc;
-            item(j, rr, pc);
-            uint4 lo, hi;
-            u8x16_to_f16(v[j], lo, hi);
-            *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc, kx)) = lo;
-            *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, 2 * pc + 1, kx)) = hi;
-          }
-        }
-      } else {
-        const float *xs = static_cast<const float *>(x) + row0 * D;
-#pragma unroll
-        for (int j0 = 0; j0 < 16; j0 += 8) {
-          if (j0 >= per || !ok) break;
-          float4 u[8], w[8];
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            int rr, pc;
-            item(j0 + j, rr, pc);
-            u[j] = w[j] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
-            if (j0 + j < per && rr < rows) {
-              const float4 *s4 = reinterpret_cast<const float4 *>(xs + rr * D + pc * 8);
-              u[j] = __ldg(s4);
-              w[j] = __ldg(s4 + 1);
-            }
-          }
-          if (j0 == 0) ok = warp_wait(smem_u32(&B.xempty[xb]), xpar, abort, wait_ns);
-          if (!ok) break;
-#pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            if (j0 + j >= per) break;
-            int rr, pc;
-            item(j0 + j, rr, pc);
-            const __half2 h0 = __floats2half2_rn(u[j].x, u[j].y), h1 = __floats2half2_rn(u[j].z, u[j].w);
-            const __half2 h2 = __floats2half2_rn(w[j].x, w[j].y), h3 = __floats2half2_rn(w[j].z, w[j].w);
-            *reinterpret_cast<uint4 *>(sX + nr_tc_kmajor_off(rr, pc, kx)) =
-                make_uint4(*reinterpret_cast<const uint32_t *>(&h0), *reinterpret_cast<const uint32_t *>(&h1),
-                           *reinterpret_cast<const uint32_t *>(&h2), *reinterpret_cast<const uint32_t *>(&h3));
-          }
-        }
-      }
-      if (!ok) break;
-      fence_async_smem();
-      mbar_arrive(smem_u32(&B.xfull[xb]));
-    }
+    tc_convert_tiles<DT>(x, D, kx, nxb, nq, ntiles, x_bytes, smem + L.x, B.xfull, B.xempty, abort,
+                         wait_ns, tid - kWarpConv * 32);
   }
   tc_fence_before();
   __syncthreads();
@@ -1236,11 +1248,11 @@ cudaError_t nr_launch_encode(nr_index *ix, const void *d_x, int64_t nq, float *d
     const int n2 = ix->b <= 16 ? 16 : 32;
     const int nxb = tc_xbuffers(ix->D, ix->H, n2, ix->smem_optin);
     const uint32_t smem = tc_layout(ix->D, ix->H, n2, nxb).total;
+    const int64_t tiles = (nq + kRows - 1) / kRows;
+    const int64_t grid = tiles < ix->num_sms ? tiles : ix->num_sms;
     auto kern = ix->dtype == 0 ? encode_tc_kernel<0> : encode_tc_kernel<1>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = (nq + kRows - 1) / kRows;
-    const int64_t grid = tiles < ix->num_sms ? tiles : ix->num_sms;
     const int vec_out = ix->b % 4 == 0 && (reinterpret_cast<uintptr_t>(d_logits) & 15) == 0;
     // the roles' hand-off waits: wait_ns (1 s by default); the drain of
     // issued MMAs before TMEM is freed keeps its own 1 s bound whatever this is
