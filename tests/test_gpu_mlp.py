@@ -213,3 +213,15 @@ def test_encoder_misaligned_input(built, torch):
     ref = built["orc"].encode(q)
     err = np.max(np.abs(lg - ref), axis=1)
     assert np.all(err <= 1e-2 * np.max(np.abs(ref), axis=1))
+
+
+@pytest.mark.parametrize("n", [1, 5, 127, 129])
+def test_encoder_small_batches(built, torch, n):
+    """Batches smaller than one 128-row tile (and one row past it): the tile's
+    missing rows are zeros on the way in and are not written out."""
+    q = built["q"][:n]
+    lg = built["ix"].encode(torch.from_numpy(np.ascontiguousarray(q)).cuda()).cpu().numpy()
+    ref = built["orc"].encode(q)
+    assert lg.shape == ref.shape
+    err = np.max(np.abs(lg - ref), axis=1)
+    assert np.all(err <= 1e-2 * np.max(np.abs(ref), axis=1))
