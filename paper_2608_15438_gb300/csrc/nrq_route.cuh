@@ -223,6 +223,7 @@ __device__ __forceinline__ int route_warp(const RouteParams &rp, const float *__
 // kRouteBucketMax keys take route_warp too (warp 0 of the block).
 constexpr int kRouteThreads = 128;
 constexpr int kRouteBins = 480;
+constexpr int kRouteSeedRanks = 7;          // the walk starts from all subsets of ranks 0..6
 constexpr int kRouteDp = kRouteBins + 32;  // sums of rounded-up steps overshoot by < 1 per rank
 constexpr int kRouteBuckets = 1024;        // <= 2 kRouteDp: the histogram reuses the count arrays
 static_assert(kRouteBuckets <= 2 * kRouteDp, "the bucket histogram must fit the count arrays");
@@ -393,11 +394,35 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
   const float teff = fminf(T, rp.smax);
   // breadth-first enumeration of the subtree with cost <= teff
   int tail = 0;
+  // The walk starts from every non-empty subset of ranks 0 .. s7 - 1 within
+  // the threshold, one a thread (the subtree's sets of those ranks: costs
+  // never fall along an edge, so their ancestors are within it too), each
+  // cost the left-to-right sum over its ranks as the tree's additions give
+  // it; only seeds whose largest rank is s7 - 1 have children outside them.
+  const int s7 = bsel < kRouteSeedRanks ? bsel : kRouteSeedRanks;
   if (!use_heap && !none) {
-    if (tid == 0 && m.ssd[0] <= teff) {
-      m.keys[0] = pack_key(m.ssd[0], 1u, 1u);
-      m.costp[0] = 0.0f;
-      m.ctl[0] = 1;
+    {
+      uint64_t key = kEmpty;
+      float cp = 0.0f;
+      if (tid >= 1 && tid < (1 << s7)) {
+        const int mx = 31 - __clz(tid);
+        float c = 0.0f;
+        for (int r = 0; r <= mx; ++r)
+          if ((tid >> r) & 1) {
+            cp = c;
+            c = __fadd_rn(c, m.ssd[r]);
+          }
+        if (c <= teff) key = pack_key(c, (uint32_t)__popc(tid), (uint32_t)tid);
+      }
+      const unsigned bal = __ballot_sync(kFull, key != kEmpty);
+      int base = 0;
+      if (lane == 0 && bal) base = atomicAdd(&m.ctl[0], __popc(bal));
+      base = __shfl_sync(kFull, base, 0);
+      if (key != kEmpty) {
+        const int pos = base + __popc(bal & ((1u << lane) - 1u));
+        m.keys[pos] = key;  // at most 127 seeds, within the capacity
+        m.costp[pos] = cp;
+      }
     }
     __syncthreads();
     int head = 0;
@@ -414,7 +439,7 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
         const uint32_t size = ((uint32_t)key >> 24) & 0xffu;
         const float cost = __uint_as_float((uint32_t)(key >> 32));
         const int mx = 31 - __clz((int)mask);
-        if (mx + 1 < bsel) {
+        if (mx + 1 < bsel && mx + 1 >= s7) {  // children of smaller seeds are seeds
           const float sdn = m.ssd[mx + 1];
           const float c1 = __fadd_rn(cp, sdn);  // shift: rank mx -> mx + 1
           if (c1 <= teff) {
