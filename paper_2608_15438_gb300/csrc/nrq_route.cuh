@@ -350,9 +350,33 @@ __device__ __forceinline__ int route_block(const RouteParams &rp, const float *_
       // kRouteDp) the 0.001 covers, so s_r D >= delta_r exactly
       const float step = __fdiv_rn(trange, (float)kRouteBins);
       uint32_t *d0 = m.dp, *d1 = m.dp + kRouteDp;
-      for (int c = tid; c < kRouteDp; c += kRouteThreads) d0[c] = c == 0 ? 1u : 0u;
+      for (int c = tid; c < kRouteDp; c += kRouteThreads) d0[c] = 0u;
+      // the counts over the first ranks in one step: each subset of ranks
+      // 0 .. r0 - 1 (those that fit a bin, at most kRouteSeedRanks) adds one
+      // to the bin of its sum of steps, as the passes below would
+      const int rs = bsel < kRouteSeedRanks ? bsel : kRouteSeedRanks;
+      int r0 = 0, sr_seed[kRouteSeedRanks];
+#pragma unroll
+      for (int r = 0; r < kRouteSeedRanks; ++r) {
+        sr_seed[r] = 0;
+        if (r < rs && r0 == r) {
+          const float qv = __fdiv_rn(m.ssd[r], step);
+          if (qv < (float)(kRouteDp - 2)) {
+            sr_seed[r] = (int)__fadd_rn(qv, 0.001f) + 1;
+            r0 = r + 1;
+          }
+        }
+      }
       __syncthreads();
-      for (int r = 0; r < bsel; ++r) {
+      if (tid < (1 << r0)) {
+        int sum = 0;
+#pragma unroll
+        for (int r = 0; r < kRouteSeedRanks; ++r)
+          if ((tid >> r) & 1) sum += sr_seed[r];
+        if (sum < kRouteDp) atomicAdd(&d0[sum], 1u);
+      }
+      __syncthreads();
+      for (int r = r0; r < bsel; ++r) {
         const float qv = __fdiv_rn(m.ssd[r], step);
         if (!(qv < (float)(kRouteDp - 2))) break;  // this rank and all later ones fit no bin
         const int sr = (int)__fadd_rn(qv, 0.001f) + 1;
